@@ -1,0 +1,172 @@
+/*
+ * flashslice.h -- C ABI of the GB300 slice -> token mix -> deslice library.
+ *
+ * The operation is the coupling of Transolver's physics-attention sublayer
+ * with a constant token core (paper Sec. 2 "The Transolver layer" and Eq. (1);
+ * Appendix G.1 "Single-tile kernels" / "G-blocked kernels").  Per batch b and
+ * head h, with x = x_mid[b,:,h,:] (N x d), f = fx[b,:,h,:] (N x d),
+ * W = W_slice[h] (d x G), beta = bias[h] (G), tau = tau[h]:
+ *
+ *   a_ng   = (x_n . W[:,g] + beta_g) / tau           slice logits
+ *   w_ng   = exp(a_ng - lse_n),  lse_n = log sum_g exp(a_ng)
+ *   S_g    = sum_n w_ng,   U_g = sum_n w_ng f_n      (partials over points)
+ *   z_g    = U_g / (S_g + eps)                       tokens
+ *   z'_g   = sum_k M[g,k] z_k                        constant G x G mix
+ *   out_n  = sum_g w_ng z'_g                         deslice, tied weights
+ *
+ * The N x H x G weight tensor w is never written to memory: every pass
+ * recomputes it tile by tile from x_mid and the per-point statistic lse.
+ *
+ * Conventions for every entry point
+ *  - All tensor pointers are DEVICE pointers owned by the caller.  The library
+ *    never allocates, frees or synchronises (except fs_device_status, which
+ *    synchronises `stream` to read the status word).  Every call is
+ *    asynchronous on `stream` (a cudaStream_t; NULL = legacy default stream).
+ *  - Layouts are dense, row-major, contiguous:
+ *      x_mid, fx, out, dout, dx_mid, dfx : [B, N, H, d]   dtype of the shape
+ *      W_slice, dW                       : [H, d, G]      fp32
+ *      bias, dbias                       : [H, G]         fp32
+ *      tau, dtau                         : [H]            fp32
+ *      M, dM                             : [H, G, G]      fp32, M[h][g][k]
+ *      tokens, tokens_mixed, d_tokens*   : [B, H, G, d]   fp32
+ *      wsum                              : [B, H, G]      fp32
+ *      lse                               : [B, N, H]      fp32, natural log
+ *    Channel c of a point's C = H*d features is head c / d, lane c % d.
+ *  - Every pointer must be 16-byte aligned.
+ *  - `ws` is caller-owned scratch of at least fs_workspace_bytes(shape, op)
+ *    bytes (16-byte aligned).  Its first word is a device status word that
+ *    each call resets; fs_device_status reads it.
+ *  - Host-side validation fails with FS_ERR_INVALID / FS_ERR_UNSUPPORTED
+ *    before anything is launched.  Device-side problems (tau <= 0 or not
+ *    finite; a bounded wait that gave up) are written to the status word and
+ *    the affected kernel skips its work; no kernel traps.
+ *  - Results are deterministic: no floating-point atomics; partial sums over
+ *    points are reduced in a fixed order, so repeated calls on the same
+ *    device agree bit for bit.
+ *  - Supported: d in {16, 32, 64}; G in [1, 4096]; B*N*H*d < 2^40.
+ *    Precision: FS_F32 computes every product in fp32 FMA; FS_BF16 computes
+ *    the point-by-slot products on bf16 tensor cores with fp32 accumulation
+ *    (bf16 operands, the paper's "bf16" dot level, Appendix G.2 Table of dot
+ *    levels) where a tensor-core kernel exists for the shape, else in fp32.
+ */
+#ifndef FLASHSLICE_H
+#define FLASHSLICE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* fs_stream_t; /* identical to cudaStream_t */
+
+typedef enum fs_status {
+  FS_OK = 0,
+  FS_ERR_INVALID = 1,     /* null/misaligned pointer, bad size, workspace too small */
+  FS_ERR_UNSUPPORTED = 2, /* well-formed shape that no kernel implements (e.g. d = 48) */
+  FS_ERR_CUDA = 3,        /* a CUDA runtime call or kernel launch failed */
+  FS_ERR_TIMEOUT = 4,     /* device: a bounded wait gave up (status word only) */
+  FS_ERR_BAD_TAU = 5      /* device: some tau[h] <= 0 or not finite (status word only) */
+} fs_status;
+
+typedef enum fs_dtype { FS_F32 = 0, FS_BF16 = 1 } fs_dtype;
+
+typedef struct fs_shape {
+  int64_t B;     /* batch size, >= 1 */
+  int64_t N;     /* points per sample, >= 1 */
+  int32_t H;     /* heads, >= 1 */
+  int32_t d;     /* head width (value width equals it), 16, 32 or 64 */
+  int32_t G;     /* slices per head, 1..4096 */
+  int32_t dtype; /* fs_dtype of the [B,N,H,d] point tensors */
+  float eps;     /* added to the weight sums before normalising, >= 0 (paper: 1e-5) */
+} fs_shape;
+
+typedef enum fs_op {
+  FS_OP_SLICE_FWD = 0,
+  FS_OP_DESLICE_FWD = 1,
+  FS_OP_DESLICE_BWD = 2,
+  FS_OP_SLICE_BWD = 3
+} fs_op;
+
+/* Bytes of scratch `ws` that entry point `op` needs for this shape on the
+ * current device (0 for an invalid shape).  Depends on the device's SM count. */
+size_t fs_workspace_bytes(const fs_shape* s, int op);
+
+/* Slice (Sec. 2; App. G.1 "G-blocked kernels": statistics, slot-owned partial
+ * numerators and weight sums, normalisation after the partials are combined).
+ *   in : x_mid, fx [B,N,H,d]; W_slice [H,d,G]; bias [H,G]; tau [H]
+ *   out: tokens [B,H,G,d] = U/(S+eps) if finalize != 0, else the unnormalised
+ *        numerators U (for a cross-device sum before fs_slice_finalize);
+ *        wsum [B,H,G] = S; lse [B,N,H] (may be NULL: then kept in ws only). */
+fs_status fs_slice_fwd(const fs_shape* s, const void* x_mid, const void* fx,
+                       const float* W_slice, const float* bias, const float* tau,
+                       float* tokens, float* wsum, float* lse, int finalize,
+                       void* ws, size_t ws_bytes, fs_stream_t stream);
+
+/* tokens <- tokens / (wsum + eps), in place ("column normalisation after
+ * partials have been combined", App. G.1). */
+fs_status fs_slice_finalize(const fs_shape* s, float* tokens, const float* wsum,
+                            fs_stream_t stream);
+
+/* Constant token mix, the core of Eq. (1) acting on the slot index:
+ * tokens_mixed[b,h,g,:] = sum_k M[h,g,k] tokens[b,h,k,:].  Out-of-place only. */
+fs_status fs_mix(const fs_shape* s, const float* M, const float* tokens,
+                 float* tokens_mixed, fs_stream_t stream);
+
+/* Deslice with tied weights (Sec. 2; App. G.1): out[b,n,h,:] = sum_g w z'_g.
+ *   lse: statistics from fs_slice_fwd; NULL makes the call compute them first
+ *   (into ws).  out has the dtype of the shape. */
+fs_status fs_deslice_fwd(const fs_shape* s, const void* x_mid, const float* W_slice,
+                         const float* bias, const float* tau, const float* tokens_mixed,
+                         const float* lse, void* out, void* ws, size_t ws_bytes,
+                         fs_stream_t stream);
+
+/* Backward of the deslice given dout (App. G.1 "Backward uses separate
+ * point-owned and slot-owned kernels"; temperature gradient App. G.2):
+ *   d_tokens_mixed [B,H,G,d] = sum_n w_ng dout_n  (always overwritten)
+ *   dx_mid [B,N,H,d], dW [H,d,G], dbias [H,G], dtau [H]: the contribution of
+ *   the deslice weights; written if accumulate == 0, added if accumulate != 0.
+ *   lse must be the statistics of the forward pass (not NULL). */
+fs_status fs_deslice_bwd(const fs_shape* s, const void* x_mid, const float* W_slice,
+                         const float* bias, const float* tau, const float* tokens_mixed,
+                         const float* lse, const void* dout, float* d_tokens_mixed,
+                         void* dx_mid, float* dW, float* dbias, float* dtau,
+                         int accumulate, void* ws, size_t ws_bytes, fs_stream_t stream);
+
+/* Backward of the mix: d_tokens = M^T d_tokens_mixed per (b,h) (overwritten);
+ * dM [H,G,G] = sum_b d_tokens_mixed tokens^T (overwritten). */
+fs_status fs_mix_bwd(const fs_shape* s, const float* M, const float* tokens,
+                     const float* d_tokens_mixed, float* d_tokens, float* dM,
+                     fs_stream_t stream);
+
+/* Backward of the slice given d_tokens (the gradient w.r.t. the normalised
+ * tokens); tokens and wsum are the forward's normalised tokens and S.
+ *   dfx [B,N,H,d] (overwritten); dx_mid, dW, dbias, dtau: written if
+ *   accumulate == 0, added if accumulate != 0. */
+fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx,
+                       const float* W_slice, const float* bias, const float* tau,
+                       const float* tokens, const float* wsum, const float* lse,
+                       const float* d_tokens, void* dx_mid, void* dfx, float* dW,
+                       float* dbias, float* dtau, int accumulate, void* ws,
+                       size_t ws_bytes, fs_stream_t stream);
+
+/* Synchronises `stream` and returns the device status word of `ws`
+ * (FS_OK, FS_ERR_TIMEOUT or FS_ERR_BAD_TAU), or FS_ERR_CUDA. */
+fs_status fs_device_status(const void* ws, fs_stream_t stream);
+
+/* Static, human-readable name of a status code. */
+const char* fs_status_string(fs_status st);
+
+/* Kernel path the library takes for this shape: 0 = SIMT fp32 kernels,
+ * 1 = tcgen05 tensor-core kernels.  For tests and benchmarks. */
+int fs_path_for_shape(const fs_shape* s);
+
+/* Number of kernels the forward (slice + mix + deslice) launches for this shape. */
+int fs_forward_launch_count(const fs_shape* s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FLASHSLICE_H */
