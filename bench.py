@@ -1,0 +1,337 @@
+#!/usr/bin/env python
+"""Throughput of the slice -> mix -> deslice coupling on GB300 (one JSON line).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload large_g_bf16|...] [--no-cpu-baseline]
+
+A step is one pass of the whole forward hot path (fs_slice_fwd -> fs_mix ->
+fs_deslice_fwd through the C ABI) over one batch of the named synthetic
+workload, default N = 1,048,576 points, H = 8, d = 32, G = 1024, bf16
+(inputs 512 MiB each, larger than the 129 MB L2, so no flush is needed between
+steps).  Metric: Mpoints/s of the whole job (B*N points per step per rank).
+
+Multi-GPU: the workload is replicated (each rank runs its own full copy; no
+collective on the data path), so scaling is weak.  Launched with torchrun for
+N > 1; rank 0 prints the line.
+
+--impl reference times the fp64 CPU oracle (the only reference this method
+has) on the host cores, on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "slice+deslice Mpoints/s (N=1M, G=1024, bf16) and % of roofline"
+UNIT = "Mpoints/s"
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained", d["bf16_tflops"]), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+def _algorithmic(wl):
+    """Algorithmic work of one forward (per point, all heads; C = H*d):
+    flops 8*C*G (logits twice, slice accumulate, deslice apply), bytes 4*C*e
+    (slice reads x_mid and fx; deslice reads x_mid and writes out).  Each of the
+    two streaming calls carries half of both."""
+    C = wl.H * wl.d
+    e = 2 if wl.dtype == "bf16" else 4
+    P = wl.B * wl.N
+    return {"flops": 8.0 * C * wl.G * P, "bytes": 4.0 * C * e * P,
+            "flops_per_call": 4.0 * C * wl.G * P, "bytes_per_call": 2.0 * C * e * P}
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms in the background."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id=None):
+        self.path = tempfile.mktemp(prefix="fs_clocks_", suffix=".csv")
+        cmd = ["nvidia-smi", "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits", "-lms", "200"]
+        if gpu_id:
+            cmd += ["-i", str(gpu_id)]
+        try:
+            self.f = open(self.path, "w")
+            self.p = subprocess.Popen(cmd, stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.p.terminate()
+        try:
+            self.p.wait(timeout=5)
+        except Exception:
+            self.p.kill()
+        self.f.close()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+def cpu_oracle_rate(wl, target_s=12.0):
+    """The fp64 oracle as it stands, forward (slice over the sample, mix, deslice
+    of the sample) on the first n points of the workload, all heads.  Returns
+    (Mpoints/s, sample description, threads)."""
+    from oracle import flashslice_oracle as orc
+
+    def run(n):
+        t0 = time.perf_counter()
+        orc.forward(wl.x_mid[:, :n], wl.fx[:, :n], wl.W_slice, wl.bias, wl.tau, wl.M, eps=wl.eps)
+        return time.perf_counter() - t0
+
+    n = min(wl.N, 4096)
+    t = run(n)
+    n2 = int(min(wl.N, max(n, n * target_s / max(t, 1e-3))))
+    n2 = max(1024, (n2 // 1024) * 1024) if n2 >= 1024 else n2
+    t2 = run(n2)
+    threads = os.cpu_count()
+    try:
+        from threadpoolctl import threadpool_info
+
+        threads = max([i.get("num_threads", 1) for i in threadpool_info()] + [1])
+    except Exception:
+        pass
+    pts = wl.B * n2
+    desc = (f"{wl.name}: first {n2} of {wl.N} points x B={wl.B}, all {wl.H} heads, fp64 forward "
+            f"(slice over the sample, mix, deslice of the sample), {t2:.1f} s")
+    return pts / t2 / 1e6, desc, threads
+
+
+def run_reference(args):
+    """--impl reference: the fp64 CPU oracle timed on the host cores."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from oracle import flashslice_oracle as orc
+    from paper_2609_32525_gb300.workloads import make_named
+
+    wl = make_named(args.workload)
+    n = int(args.ref_points)
+    times = []
+    for i in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        orc.forward(wl.x_mid[:, :n], wl.fx[:, :n], wl.W_slice, wl.bias, wl.tau, wl.M, eps=wl.eps)
+        if i >= args.warmup:
+            times.append(time.perf_counter() - t0)
+    t = float(np.sum(times))
+    value = wl.B * n * len(times) / t / 1e6
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * t / len(times),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": wl.name, "sample_points": n, "B": wl.B, "N": wl.N,
+                                             "H": wl.H, "d": wl.d, "G": wl.G},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+                             "sample": f"first {n} points of {wl.name} per step, all heads, fp64 forward"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="large_g_bf16")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--ref-points", type=int, default=16384)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        return run_reference(args)
+
+    import torch
+    import torch.distributed as dist
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    from paper_2609_32525_gb300 import build as _build
+
+    if not os.path.exists(_build.LIB):
+        _build.build()
+    from paper_2609_32525_gb300 import flashslice as fs
+    from paper_2609_32525_gb300.workloads import make_named
+
+    wl = make_named(args.workload)
+    tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+
+    def put(a, dt):
+        return torch.from_numpy(a).to(device=dev, dtype=dt).contiguous()
+
+    x, fx = put(wl.x_mid, tdt), put(wl.fx, tdt)
+    W, b, t, M = (put(getattr(wl, k), torch.float32) for k in ("W_slice", "bias", "tau", "M"))
+    c = fs.Coupling(wl.B, wl.N, wl.H, wl.d, wl.G, tdt, wl.eps, device=dev)
+    s = c.shape
+    stream = torch.cuda.current_stream()
+
+    def step(ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        fs.fs_slice_fwd(s, x, fx, W, b, t, c.tokens, c.wsum, c.lse, True, c.ws_slice)
+        if ev is not None:
+            ev[1].record(stream)
+        fs.fs_mix(s, M, c.tokens, c.tokens_mixed)
+        if ev is not None:
+            ev[2].record(stream)
+        fs.fs_deslice_fwd(s, x, W, b, t, c.tokens_mixed, c.lse, c.out, c.ws_deslice)
+        if ev is not None:
+            ev[3].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if c.device_status() != fs.FS_OK:
+        raise RuntimeError("device status after warm-up: " + fs.status_string(c.device_status()))
+
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        pass
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(uuid)
+    time.sleep(0.3)
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        step(evs[i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    slice_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in evs]))
+    mix_ms = float(np.mean([e[1].elapsed_time(e[2]) for e in evs]))
+    desl_ms = float(np.mean([e[2].elapsed_time(e[3]) for e in evs]))
+    if world > 1:
+        tt = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    ms_per_step = total_ms / args.steps
+    value = world * wl.points / (ms_per_step * 1e-3) / 1e6
+    assert c.device_status() == fs.FS_OK
+
+    # End to end through the same C-ABI calls with host buffers: pinned host
+    # inputs copied in, the forward, the output copied back, every step.
+    hx = torch.from_numpy(wl.x_mid).to(tdt).pin_memory()
+    hf = torch.from_numpy(wl.fx).to(tdt).pin_memory()
+    hout = torch.empty(c.out.shape, dtype=tdt).pin_memory()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    x2, f2 = torch.empty_like(x), torch.empty_like(fx)
+
+    def e2e_step():
+        x2.copy_(hx, non_blocking=True)
+        f2.copy_(hf, non_blocking=True)
+        fs.fs_slice_fwd(s, x2, f2, W, b, t, c.tokens, c.wsum, c.lse, True, c.ws_slice)
+        fs.fs_mix(s, M, c.tokens, c.tokens_mixed)
+        fs.fs_deslice_fwd(s, x2, W, b, t, c.tokens_mixed, c.lse, c.out, c.ws_deslice)
+        hout.copy_(c.out, non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    e0.record(stream)
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1) / args.e2e_steps
+    if world > 1:
+        tt = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        e2e_ms = float(tt.item())
+    e2e_val = world * wl.points / (e2e_ms * 1e-3) / 1e6
+    h2d = 2 * hx.numel() * hx.element_size()
+    d2h = hout.numel() * hout.element_size()
+
+    peaks = _peaks()
+    alg = _algorithmic(wl)
+    dom_name, dom_ms = ("fs_slice_fwd", slice_ms) if slice_ms >= desl_ms else ("fs_deslice_fwd", desl_ms)
+    achieved_tf = alg["flops_per_call"] / (dom_ms * 1e-3) / 1e12
+    roof_t = max(alg["flops"] / (peaks["bf16_tflops"] * 1e12), alg["bytes"] / (peaks["hbm_gbs"] * 1e9))
+    roofline = {"bound": "tensor", "achieved": achieved_tf, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": achieved_tf / peaks["bf16_tflops"], "traffic": None, "kernel": dom_name,
+                "peak_source": peaks["source"] + " bf16 burst",
+                "frac_sustained": achieved_tf / peaks["bf16_tflops_sustained"],
+                "step_frac": roof_t / (ms_per_step * 1e-3),
+                "call_ms": {"fs_slice_fwd": slice_ms, "fs_mix": mix_ms, "fs_deslice_fwd": desl_ms},
+                "per_call_work": "4*C*G flops per point for each of slice and deslice (C=256)"}
+
+    launches = fs.forward_launch_count(s) * args.steps
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
+            "data": "synthetic (seeded; " + wl.recipe + ")",
+            "config": {"workload": wl.name, "B": wl.B, "N": wl.N, "H": wl.H, "d": wl.d, "G": wl.G,
+                       "step": "fs_slice_fwd + fs_mix + fs_deslice_fwd", "parallelism": f"replicas x{world}",
+                       "l2": "inputs 2 x %d MiB > 129 MB L2, no flush" % (hx.numel() * hx.element_size() >> 20),
+                       "path": ["simt", "tcgen05"][fs.path_for_shape(s)]},
+            "clocks": clocks, "gpu_launches": launches, "roofline": roofline,
+            "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "ms_per_step": e2e_ms}}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, desc, threads = cpu_oracle_rate(wl)
+        line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": desc}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

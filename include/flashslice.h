@@ -43,7 +43,7 @@
  *  - Results are deterministic: no floating-point atomics; partial sums over
  *    points are reduced in a fixed order, so repeated calls on the same
  *    device agree bit for bit.
- *  - Supported: d in {16, 32, 64}; G in [1, 4096]; B*N*H*d < 2^40.
+ *  - Supported: d in {16, 32, 64}; G in [1, 4096]; B*H <= 65535; B*N*H*d < 2^40.
  *    Precision: FS_F32 computes every product in fp32 FMA; FS_BF16 computes
  *    the point-by-slot products on bf16 tensor cores with fp32 accumulation
  *    (bf16 operands, the paper's "bf16" dot level, Appendix G.2 Table of dot

@@ -1,0 +1,291 @@
+// C ABI of the library: host-side validation, workspace layout, kernel dispatch.
+// Declarations and the contract of every entry point: include/flashslice.h.
+#include "fs_internal.h"
+#include "fs_tc.h"
+
+#include <cmath>
+#include <cstring>
+
+namespace fs {
+
+int num_sms() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1) return 1;
+  return n;
+}
+
+int slot_splits(const Shape& s) {
+  const int64_t gblocks = (s.G + 127) / 128;
+  const int64_t units = s.BH() * gblocks;
+  int64_t P = (2LL * num_sms() + units - 1) / units;
+  const int64_t max_by_n = (s.N + 255) / 256;
+  if (P > max_by_n) P = max_by_n;
+  if (P < 1) P = 1;
+  if (P > 1024) P = 1024;
+  return (int)P;
+}
+
+namespace {
+
+constexpr size_t kAlign = 256;
+
+bool valid_shape(const fs_shape* s) {
+  if (!s) return false;
+  if (s->B < 1 || s->N < 1 || s->H < 1 || s->d < 1 || s->G < 1) return false;
+  if (s->dtype != FS_F32 && s->dtype != FS_BF16) return false;
+  if (!(s->eps >= 0.f) || !std::isfinite(s->eps)) return false;
+  const double elems = (double)s->B * (double)s->N * (double)s->H * (double)s->d;
+  if (elems >= 1099511627776.0) return false;  // 2^40
+  return true;
+}
+
+bool supported_shape(const fs_shape* s) {
+  return (s->d == 16 || s->d == 32 || s->d == 64) && s->G <= 4096 && (int64_t)s->B * s->H <= 65535;
+}
+
+Shape to_shape(const fs_shape* s) { return Shape{s->B, s->N, s->H, s->d, s->G, s->dtype, s->eps}; }
+
+bool aligned(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Byte sizes of the regions each op places in `ws` (each 256-byte aligned).
+struct Regions {
+  size_t status, partials, stats, delta, dus, dtau_g, tc, total;
+};
+
+Regions regions(const Shape& s, int op) {
+  Regions r{};
+  const int P = slot_splits(s);
+  const size_t BHG = (size_t)s.BH() * s.G;
+  const size_t pts = (size_t)s.BH() * s.N;
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = align_up(off + bytes, kAlign);
+    return o;
+  };
+  r.status = take(sizeof(uint32_t));
+  switch (op) {
+    case FS_OP_SLICE_FWD: {
+      size_t part = (size_t)P * BHG * (s.d + 1) * sizeof(float);
+      const size_t tcb = tc_slice_partials_bytes(s);
+      if (tcb > part) part = tcb;
+      r.partials = take(part);
+      r.stats = take(pts * sizeof(float));
+      r.tc = take(tc_slice_prep_bytes(s));
+      break;
+    }
+    case FS_OP_DESLICE_FWD:
+      r.stats = take(pts * sizeof(float));
+      r.tc = take(tc_deslice_prep_bytes(s));
+      break;
+    case FS_OP_DESLICE_BWD:
+      r.delta = take(pts * sizeof(float));
+      r.partials = take((size_t)P * BHG * (2 * s.d + 2) * sizeof(float));
+      r.dtau_g = take((size_t)s.H * s.G * sizeof(float));
+      break;
+    case FS_OP_SLICE_BWD:
+      r.delta = take(pts * sizeof(float));
+      r.dus = take(BHG * (s.d + 1) * sizeof(float));
+      r.partials = take((size_t)P * BHG * (s.d + 2) * sizeof(float));
+      r.dtau_g = take((size_t)s.H * s.G * sizeof(float));
+      break;
+    default:
+      return Regions{};
+  }
+  r.total = off;
+  return r;
+}
+
+template <typename T>
+T* at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<char*>(ws) + off);
+}
+
+fs_status check_ws(const Shape& s, int op, void* ws, size_t ws_bytes) {
+  const Regions r = regions(s, op);
+  if (!ws || !aligned(ws) || ws_bytes < r.total) return FS_ERR_INVALID;
+  return FS_OK;
+}
+
+fs_status cuda_status(cudaError_t e) { return e == cudaSuccess ? FS_OK : FS_ERR_CUDA; }
+
+// Every ws-using call starts by clearing its status word.
+cudaError_t reset_status(void* ws, cudaStream_t st) { return cudaMemsetAsync(ws, 0, sizeof(uint32_t), st); }
+
+#define FS_CHECK_SHAPE(s)                               \
+  do {                                                  \
+    if (!valid_shape(s)) return FS_ERR_INVALID;         \
+    if (!supported_shape(s)) return FS_ERR_UNSUPPORTED; \
+  } while (0)
+
+#define FS_CHECK_PTR(p)                                      \
+  do {                                                       \
+    if (!(p) || !aligned(p)) return FS_ERR_INVALID;          \
+  } while (0)
+
+#define FS_CUDA(call)                                          \
+  do {                                                         \
+    cudaError_t e_ = (call);                                   \
+    if (e_ != cudaSuccess) return FS_ERR_CUDA;                 \
+  } while (0)
+
+}  // namespace
+}  // namespace fs
+
+using namespace fs;
+
+extern "C" {
+
+size_t fs_workspace_bytes(const fs_shape* s, int op) {
+  if (!valid_shape(s) || !supported_shape(s)) return 0;
+  return regions(to_shape(s), op).total;
+}
+
+const char* fs_status_string(fs_status st) {
+  switch (st) {
+    case FS_OK: return "FS_OK";
+    case FS_ERR_INVALID: return "FS_ERR_INVALID: invalid argument";
+    case FS_ERR_UNSUPPORTED: return "FS_ERR_UNSUPPORTED: shape not implemented";
+    case FS_ERR_CUDA: return "FS_ERR_CUDA: CUDA runtime or launch failure";
+    case FS_ERR_TIMEOUT: return "FS_ERR_TIMEOUT: device wait gave up";
+    case FS_ERR_BAD_TAU: return "FS_ERR_BAD_TAU: tau <= 0 or not finite";
+  }
+  return "unknown fs_status";
+}
+
+int fs_path_for_shape(const fs_shape* s) {
+  if (!valid_shape(s) || !supported_shape(s)) return -1;
+  return tc_forward_supported(to_shape(s)) ? 1 : 0;
+}
+
+int fs_forward_launch_count(const fs_shape* s) {
+  if (!valid_shape(s) || !supported_shape(s)) return -1;
+  const Shape sh = to_shape(s);
+  if (tc_forward_supported(sh)) return tc_forward_launch_count(sh) + 1;  // + mix
+  return 3 /*stats, partials, reduce*/ + 1 /*mix*/ + 1 /*deslice*/;
+}
+
+fs_status fs_slice_fwd(const fs_shape* s, const void* x_mid, const void* fx, const float* W_slice,
+                       const float* bias, const float* tau, float* tokens, float* wsum, float* lse,
+                       int finalize, void* ws, size_t ws_bytes, fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(x_mid); FS_CHECK_PTR(fx); FS_CHECK_PTR(W_slice); FS_CHECK_PTR(bias); FS_CHECK_PTR(tau);
+  FS_CHECK_PTR(tokens); FS_CHECK_PTR(wsum);
+  if (lse && !aligned(lse)) return FS_ERR_INVALID;
+  const Shape sh = to_shape(s);
+  if (fs_status e = check_ws(sh, FS_OP_SLICE_FWD, ws, ws_bytes)) return e;
+  const Regions r = regions(sh, FS_OP_SLICE_FWD);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  uint32_t* status = at<uint32_t>(ws, r.status);
+  float* lse_buf = lse ? lse : at<float>(ws, r.stats);
+  FS_CUDA(reset_status(ws, st));
+  if (tc_forward_supported(sh)) {
+    return cuda_status(tc_slice_fwd(sh, x_mid, fx, W_slice, bias, tau, tokens, wsum, lse_buf, finalize,
+                                    at<float>(ws, r.partials), at<void>(ws, r.tc), status, st));
+  }
+  const int P = slot_splits(sh);
+  float* part = at<float>(ws, r.partials);
+  FS_CUDA(simt_stats(sh, x_mid, W_slice, bias, tau, lse_buf, status, st));
+  FS_CUDA(simt_slice_partials(sh, P, x_mid, fx, W_slice, bias, tau, lse_buf, part, status, st));
+  FS_CUDA(simt_reduce_tokens(sh, P, part, tokens, wsum, finalize, st));
+  return FS_OK;
+}
+
+fs_status fs_slice_finalize(const fs_shape* s, float* tokens, const float* wsum, fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(tokens); FS_CHECK_PTR(wsum);
+  return cuda_status(simt_finalize(to_shape(s), tokens, wsum, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+fs_status fs_mix(const fs_shape* s, const float* M, const float* tokens, float* tokens_mixed,
+                 fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(M); FS_CHECK_PTR(tokens); FS_CHECK_PTR(tokens_mixed);
+  if (tokens == tokens_mixed) return FS_ERR_INVALID;
+  return cuda_status(simt_mix(to_shape(s), M, tokens, tokens_mixed, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+fs_status fs_deslice_fwd(const fs_shape* s, const void* x_mid, const float* W_slice, const float* bias,
+                         const float* tau, const float* tokens_mixed, const float* lse, void* out, void* ws,
+                         size_t ws_bytes, fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(x_mid); FS_CHECK_PTR(W_slice); FS_CHECK_PTR(bias); FS_CHECK_PTR(tau);
+  FS_CHECK_PTR(tokens_mixed); FS_CHECK_PTR(out);
+  if (lse && !aligned(lse)) return FS_ERR_INVALID;
+  const Shape sh = to_shape(s);
+  if (fs_status e = check_ws(sh, FS_OP_DESLICE_FWD, ws, ws_bytes)) return e;
+  const Regions r = regions(sh, FS_OP_DESLICE_FWD);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  uint32_t* status = at<uint32_t>(ws, r.status);
+  FS_CUDA(reset_status(ws, st));
+  const float* lse_use = lse;
+  if (!lse_use) {
+    float* buf = at<float>(ws, r.stats);
+    if (tc_forward_supported(sh)) FS_CUDA(tc_stats(sh, x_mid, W_slice, bias, tau, buf, at<void>(ws, r.tc), status, st));
+    else FS_CUDA(simt_stats(sh, x_mid, W_slice, bias, tau, buf, status, st));
+    lse_use = buf;
+  }
+  if (tc_forward_supported(sh))
+    return cuda_status(tc_deslice_fwd(sh, x_mid, W_slice, bias, tau, tokens_mixed, lse_use, out,
+                                      at<void>(ws, r.tc), status, st));
+  return cuda_status(simt_deslice(sh, x_mid, W_slice, bias, tau, tokens_mixed, lse_use, out, status, st));
+}
+
+fs_status fs_deslice_bwd(const fs_shape* s, const void* x_mid, const float* W_slice, const float* bias,
+                         const float* tau, const float* tokens_mixed, const float* lse, const void* dout,
+                         float* d_tokens_mixed, void* dx_mid, float* dW, float* dbias, float* dtau, int accumulate,
+                         void* ws, size_t ws_bytes, fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(x_mid); FS_CHECK_PTR(W_slice); FS_CHECK_PTR(bias); FS_CHECK_PTR(tau);
+  FS_CHECK_PTR(tokens_mixed); FS_CHECK_PTR(lse); FS_CHECK_PTR(dout); FS_CHECK_PTR(d_tokens_mixed);
+  FS_CHECK_PTR(dx_mid); FS_CHECK_PTR(dW); FS_CHECK_PTR(dbias); FS_CHECK_PTR(dtau);
+  const Shape sh = to_shape(s);
+  if (fs_status e = check_ws(sh, FS_OP_DESLICE_BWD, ws, ws_bytes)) return e;
+  const Regions r = regions(sh, FS_OP_DESLICE_BWD);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  FS_CUDA(reset_status(ws, st));
+  return cuda_status(simt_deslice_bwd(sh, slot_splits(sh), x_mid, W_slice, bias, tau, tokens_mixed, lse, dout,
+                                      d_tokens_mixed, dx_mid, dW, dbias, dtau, accumulate, at<float>(ws, r.delta),
+                                      at<float>(ws, r.partials), at<float>(ws, r.dtau_g),
+                                      at<uint32_t>(ws, r.status), st));
+}
+
+fs_status fs_mix_bwd(const fs_shape* s, const float* M, const float* tokens, const float* d_tokens_mixed,
+                     float* d_tokens, float* dM, fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(M); FS_CHECK_PTR(tokens); FS_CHECK_PTR(d_tokens_mixed); FS_CHECK_PTR(d_tokens); FS_CHECK_PTR(dM);
+  if (d_tokens == d_tokens_mixed) return FS_ERR_INVALID;
+  return cuda_status(simt_mix_bwd(to_shape(s), M, tokens, d_tokens_mixed, d_tokens, dM,
+                                  reinterpret_cast<cudaStream_t>(stream)));
+}
+
+fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx, const float* W_slice,
+                       const float* bias, const float* tau, const float* tokens, const float* wsum,
+                       const float* lse, const float* d_tokens, void* dx_mid, void* dfx, float* dW, float* dbias,
+                       float* dtau, int accumulate, void* ws, size_t ws_bytes, fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(x_mid); FS_CHECK_PTR(fx); FS_CHECK_PTR(W_slice); FS_CHECK_PTR(bias); FS_CHECK_PTR(tau);
+  FS_CHECK_PTR(tokens); FS_CHECK_PTR(wsum); FS_CHECK_PTR(lse); FS_CHECK_PTR(d_tokens);
+  FS_CHECK_PTR(dx_mid); FS_CHECK_PTR(dfx); FS_CHECK_PTR(dW); FS_CHECK_PTR(dbias); FS_CHECK_PTR(dtau);
+  const Shape sh = to_shape(s);
+  if (fs_status e = check_ws(sh, FS_OP_SLICE_BWD, ws, ws_bytes)) return e;
+  const Regions r = regions(sh, FS_OP_SLICE_BWD);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  FS_CUDA(reset_status(ws, st));
+  return cuda_status(simt_slice_bwd(sh, slot_splits(sh), x_mid, fx, W_slice, bias, tau, tokens, wsum, lse,
+                                    d_tokens, dx_mid, dfx, dW, dbias, dtau, accumulate, at<float>(ws, r.delta),
+                                    at<float>(ws, r.dus), at<float>(ws, r.partials), at<float>(ws, r.dtau_g),
+                                    at<uint32_t>(ws, r.status), st));
+}
+
+fs_status fs_device_status(const void* ws, fs_stream_t stream) {
+  if (!ws || !aligned(ws)) return FS_ERR_INVALID;
+  uint32_t v = 0;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&v, ws, sizeof(v), cudaMemcpyDeviceToHost, st) != cudaSuccess) return FS_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return FS_ERR_CUDA;
+  return static_cast<fs_status>(v);
+}
+
+}  // extern "C"

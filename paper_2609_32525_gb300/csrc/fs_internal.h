@@ -1,0 +1,60 @@
+// Internal declarations shared by the library's translation units (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cstdint>
+#include <cstddef>
+
+#include "flashslice.h"
+
+namespace fs {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+// Status word codes written by kernels (same values as fs_status).
+constexpr uint32_t kDevOk = 0, kDevTimeout = 4, kDevBadTau = 5;
+
+struct Shape {
+  int64_t B, N;
+  int H, d, G;
+  int dtype;
+  float eps;
+  int64_t BH() const { return B * (int64_t)H; }
+  int64_t points() const { return B * N; }
+};
+
+inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+int num_sms();
+// Number of point splits for slot-owned kernels (fixed for a shape on a device).
+int slot_splits(const Shape& s);
+
+// ---- SIMT kernels (fs_simt.cu) -------------------------------------------------
+cudaError_t simt_stats(const Shape& s, const void* x, const float* W, const float* bias,
+                       const float* tau, float* lse, uint32_t* status, cudaStream_t st);
+cudaError_t simt_slice_partials(const Shape& s, int P, const void* x, const void* f,
+                                const float* W, const float* bias, const float* tau,
+                                const float* lse, float* part, uint32_t* status, cudaStream_t st);
+cudaError_t simt_reduce_tokens(const Shape& s, int P, const float* part, float* tokens,
+                               float* wsum, int finalize, cudaStream_t st);
+cudaError_t simt_finalize(const Shape& s, float* tokens, const float* wsum, cudaStream_t st);
+cudaError_t simt_mix(const Shape& s, const float* M, const float* z, float* zp, cudaStream_t st);
+cudaError_t simt_mix_bwd(const Shape& s, const float* M, const float* z, const float* dzp,
+                         float* dz, float* dM, cudaStream_t st);
+cudaError_t simt_deslice(const Shape& s, const void* x, const float* W, const float* bias,
+                         const float* tau, const float* zp, const float* lse, void* out,
+                         uint32_t* status, cudaStream_t st);
+cudaError_t simt_deslice_bwd(const Shape& s, int P, const void* x, const float* W,
+                             const float* bias, const float* tau, const float* zp,
+                             const float* lse, const void* dout, float* dzp, void* dx,
+                             float* dW, float* db, float* dtau, int accumulate, float* delta,
+                             float* part, float* dtau_g, uint32_t* status, cudaStream_t st);
+cudaError_t simt_slice_bwd(const Shape& s, int P, const void* x, const void* f, const float* W,
+                           const float* bias, const float* tau, const float* z,
+                           const float* wsum, const float* lse, const float* dz, void* dx,
+                           void* dfx, float* dW, float* db, float* dtau, int accumulate,
+                           float* delta, float* dUS, float* part, float* dtau_g,
+                           uint32_t* status, cudaStream_t st);
+
+}  // namespace fs

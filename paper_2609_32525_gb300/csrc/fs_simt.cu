@@ -1,0 +1,751 @@
+// SIMT fp32 kernels: every step of the coupling with fp32 FMA products and fp32
+// accumulation.  They serve fp32 inputs (the paper's default "ieee" dot level,
+// Appendix G.2) and every shape the tensor-core kernels do not cover.
+//
+// Ownership follows the paper's G-blocked family (Appendix G.1): a statistics
+// pass per point; slot-owned split-N partial numerators and weight sums with a
+// fixed-order reduction afterwards; point-owned deslice; backward as
+// point-owned (input gradients, two sweeps over slots) plus slot-owned
+// (parameter and token gradients) kernels.  No float atomics anywhere.
+//
+// Logits are formed as a2 = x . (W * log2e/tau) + beta * log2e/tau, i.e. the
+// temperature-scaled logit in base-2 units, so that w = exp2(a2 - lse*log2e).
+#include "fs_internal.h"
+
+#include <cuda_bf16.h>
+#include <math_constants.h>
+
+namespace fs {
+namespace {
+
+constexpr int kThreads = 128;
+
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 v) { return __bfloat162float(v); }
+// Row of D contiguous elements -> floats (16-byte vector loads).
+template <int D>
+__device__ __forceinline__ void load_row(const float* p, float (&v)[D]) {
+  const float4* q = reinterpret_cast<const float4*>(p);
+#pragma unroll
+  for (int i = 0; i < D / 4; i++) {
+    float4 t = q[i];
+    v[4 * i] = t.x; v[4 * i + 1] = t.y; v[4 * i + 2] = t.z; v[4 * i + 3] = t.w;
+  }
+}
+template <int D>
+__device__ __forceinline__ void load_row(const __nv_bfloat16* p, float (&v)[D]) {
+  const uint4* q = reinterpret_cast<const uint4*>(p);
+#pragma unroll
+  for (int i = 0; i < D / 8; i++) {
+    uint4 t = q[i];
+    const uint32_t w[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+      v[8 * i + 2 * j] = __uint_as_float(w[j] << 16);
+      v[8 * i + 2 * j + 1] = __uint_as_float(w[j] & 0xffff0000u);
+    }
+  }
+}
+template <int D>
+__device__ __forceinline__ void store_row(float* p, const float (&v)[D]) {
+  float4* q = reinterpret_cast<float4*>(p);
+#pragma unroll
+  for (int i = 0; i < D / 4; i++) q[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+}
+template <int D>
+__device__ __forceinline__ void store_row(__nv_bfloat16* p, const float (&v)[D]) {
+  uint4* q = reinterpret_cast<uint4*>(p);
+#pragma unroll
+  for (int i = 0; i < D / 8; i++) {
+    uint32_t w[4];
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+      __nv_bfloat162 t = __floats2bfloat162_rn(v[8 * i + 2 * j], v[8 * i + 2 * j + 1]);
+      w[j] = *reinterpret_cast<uint32_t*>(&t);
+    }
+    q[i] = make_uint4(w[0], w[1], w[2], w[3]);
+  }
+}
+
+__device__ __forceinline__ void set_status(uint32_t* status, uint32_t code) {
+  if (status) atomicCAS(status, 0u, code);
+}
+
+// tau must be positive and finite; returns false (and flags the status word) otherwise.
+__device__ __forceinline__ bool tau_ok(float t, uint32_t* status) {
+  if (t > 0.f && t < CUDART_INF_F) return true;
+  if (threadIdx.x == 0) set_status(status, kDevBadTau);
+  return false;
+}
+
+__device__ __forceinline__ int64_t row_index(int64_t b, int64_t n, int h, int64_t N, int H) {
+  return (b * N + n) * H + h;
+}
+
+// Stage GC slots of W[h] (scaled by `scale`) as sW[g][k] plus the scaled bias.
+template <int D, int GC>
+__device__ __forceinline__ void stage_w(float (*sW)[D + 1], float* sB, const float* W,
+                                        const float* bias, int h, int G, int g0, float scale) {
+  for (int i = threadIdx.x; i < GC * D; i += kThreads) {
+    const int g = i % GC, k = i / GC;
+    sW[g][k] = (g0 + g < G) ? W[((int64_t)h * D + k) * G + g0 + g] * scale : 0.f;
+  }
+  for (int i = threadIdx.x; i < GC; i += kThreads)
+    sB[i] = (g0 + i < G) ? bias[(int64_t)h * G + g0 + i] * scale : 0.f;
+}
+
+// ---- statistics: lse per (point, head) ------------------------------------------
+template <int D, typename T>
+__global__ void __launch_bounds__(kThreads) k_stats(const T* __restrict__ x, const float* __restrict__ W,
+                                                     const float* __restrict__ bias,
+                                                     const float* __restrict__ tau, float* __restrict__ lse,
+                                                     int64_t N, int H, int G, uint32_t* status) {
+  constexpr int GC = 32;
+  __shared__ float sW[GC][D + 1];
+  __shared__ float sB[GC];
+  const int64_t bh = blockIdx.y;
+  const int64_t b = bh / H;
+  const int h = (int)(bh % H);
+  if (!tau_ok(tau[h], status)) return;
+  const float scale = kLog2e / tau[h];
+  const int64_t n = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  const bool valid = n < N;
+  float xr[D];
+  if (valid) load_row<D>(x + row_index(b, n, h, N, H) * D, xr);
+  else {
+#pragma unroll
+    for (int k = 0; k < D; k++) xr[k] = 0.f;
+  }
+  float m = -CUDART_INF_F, l = 0.f;
+  for (int g0 = 0; g0 < G; g0 += GC) {
+    __syncthreads();
+    stage_w<D, GC>(sW, sB, W, bias, h, G, g0, scale);
+    __syncthreads();
+    const int gn = min(GC, G - g0);
+    float a[GC];
+    float cm = -CUDART_INF_F;
+#pragma unroll
+    for (int g = 0; g < GC; g++) {
+      float s = sB[g];
+#pragma unroll
+      for (int k = 0; k < D; k++) s = fmaf(xr[k], sW[g][k], s);
+      a[g] = (g < gn) ? s : -CUDART_INF_F;
+      cm = fmaxf(cm, a[g]);
+    }
+    const float mn = fmaxf(m, cm);
+    float acc = 0.f;
+#pragma unroll
+    for (int g = 0; g < GC; g++) acc += exp2f(a[g] - mn);
+    l = l * exp2f(m - mn) + acc;
+    m = mn;
+  }
+  if (valid) lse[row_index(b, n, h, N, H)] = (m + log2f(l)) * kLn2;
+}
+
+// ---- slice: slot-owned split-N partials ------------------------------------------
+// grid (ceil(G/128), B*H, P); thread = slot.  part[p][bh][g][0..D] = (U, S).
+template <int D, typename T>
+__global__ void __launch_bounds__(kThreads) k_slice_partial(
+    const T* __restrict__ x, const T* __restrict__ f, const float* __restrict__ W,
+    const float* __restrict__ bias, const float* __restrict__ tau, const float* __restrict__ lse,
+    float* __restrict__ part, int64_t B, int64_t N, int H, int G, int64_t per_split, uint32_t* status) {
+  constexpr int PT = 32;
+  __shared__ float sx[PT][D];
+  __shared__ float sf[PT][D];
+  __shared__ float sl[PT];
+  const int g = blockIdx.x * kThreads + threadIdx.x;
+  const int64_t bh = blockIdx.y;
+  const int64_t b = bh / H;
+  const int h = (int)(bh % H);
+  const int p = blockIdx.z;
+  if (!tau_ok(tau[h], status)) return;
+  const float scale = kLog2e / tau[h];
+  float wc[D], U[D];
+  float bb = 0.f, S = 0.f;
+#pragma unroll
+  for (int k = 0; k < D; k++) {
+    wc[k] = (g < G) ? W[((int64_t)h * D + k) * G + g] * scale : 0.f;
+    U[k] = 0.f;
+  }
+  if (g < G) bb = bias[(int64_t)h * G + g] * scale;
+  const int64_t n_begin = (int64_t)p * per_split;
+  const int64_t n_end = min(N, n_begin + per_split);
+  for (int64_t n0 = n_begin; n0 < n_end; n0 += PT) {
+    __syncthreads();
+    for (int i = threadIdx.x; i < PT * D; i += kThreads) {
+      const int j = i / D, k = i % D;
+      const int64_t n = n0 + j;
+      float xv = 0.f, fv = 0.f;
+      if (n < n_end) {
+        const int64_t idx = row_index(b, n, h, N, H) * D + k;
+        xv = to_f(x[idx]);
+        fv = to_f(f[idx]);
+      }
+      sx[j][k] = xv;
+      sf[j][k] = fv;
+    }
+    for (int i = threadIdx.x; i < PT; i += kThreads) {
+      const int64_t n = n0 + i;
+      sl[i] = (n < n_end) ? lse[row_index(b, n, h, N, H)] * kLog2e : CUDART_INF_F;
+    }
+    __syncthreads();
+#pragma unroll 4
+    for (int j = 0; j < PT; j++) {
+      float a = bb;
+#pragma unroll
+      for (int k = 0; k < D; k++) a = fmaf(sx[j][k], wc[k], a);
+      const float w = exp2f(a - sl[j]);
+      S += w;
+#pragma unroll
+      for (int k = 0; k < D; k++) U[k] = fmaf(w, sf[j][k], U[k]);
+    }
+  }
+  if (g < G) {
+    float* o = part + (((int64_t)p * B * H + bh) * G + g) * (D + 1);
+#pragma unroll
+    for (int k = 0; k < D; k++) o[k] = U[k];
+    o[D] = S;
+  }
+}
+
+// Fixed-order sum of the P partials, then (optionally) the normalisation.
+__global__ void k_reduce_tokens(const float* __restrict__ part, int P, int64_t BHG, int D,
+                                float* __restrict__ tokens, float* __restrict__ wsum, int finalize,
+                                float eps) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= BHG) return;
+  float S = 0.f;
+  for (int p = 0; p < P; p++) S += part[((int64_t)p * BHG + i) * (D + 1) + D];
+  const float den = S + eps;
+  for (int c = 0; c < D; c++) {
+    float U = 0.f;
+    for (int p = 0; p < P; p++) U += part[((int64_t)p * BHG + i) * (D + 1) + c];
+    tokens[i * D + c] = finalize ? U / den : U;
+  }
+  wsum[i] = S;
+}
+
+__global__ void k_finalize(float* __restrict__ tokens, const float* __restrict__ wsum, int64_t BHG,
+                           int D, float eps) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= BHG * D) return;
+  tokens[i] = tokens[i] / (wsum[i / D] + eps);
+}
+
+// ---- mix and its backward ------------------------------------------------------------
+// zp[bh][g][c] = sum_k M[h][g][k] z[bh][k][c]; grid (ceil(G*D/256), B*H).
+__global__ void k_mix(const float* __restrict__ M, const float* __restrict__ z, float* __restrict__ zp,
+                      int H, int G, int D) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= G * D) return;
+  const int g = idx / D, c = idx % D;
+  const int64_t bh = blockIdx.y;
+  const int h = (int)(bh % H);
+  const float* Mr = M + ((int64_t)h * G + g) * G;
+  const float* zb = z + bh * G * D;
+  float s = 0.f;
+  for (int k = 0; k < G; k++) s = fmaf(Mr[k], zb[(int64_t)k * D + c], s);
+  zp[bh * G * D + idx] = s;
+}
+
+// dz[bh][k][c] = sum_g M[h][g][k] dzp[bh][g][c]
+__global__ void k_mix_bwd_dz(const float* __restrict__ M, const float* __restrict__ dzp,
+                             float* __restrict__ dz, int H, int G, int D) {
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= G * D) return;
+  const int k = idx / D, c = idx % D;
+  const int64_t bh = blockIdx.y;
+  const int h = (int)(bh % H);
+  const float* Mh = M + (int64_t)h * G * G;
+  const float* db = dzp + bh * G * D;
+  float s = 0.f;
+  for (int g = 0; g < G; g++) s = fmaf(Mh[(int64_t)g * G + k], db[(int64_t)g * D + c], s);
+  dz[bh * G * D + idx] = s;
+}
+
+// dM[h][g][k] = sum_b sum_c dzp[b,h,g,c] z[b,h,k,c]
+__global__ void k_mix_bwd_dM(const float* __restrict__ z, const float* __restrict__ dzp,
+                             float* __restrict__ dM, int64_t B, int H, int G, int D) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)H * G * G) return;
+  const int h = (int)(idx / ((int64_t)G * G));
+  const int g = (int)((idx / G) % G), k = (int)(idx % G);
+  float s = 0.f;
+  for (int64_t b = 0; b < B; b++) {
+    const float* a = dzp + ((b * H + h) * G + g) * D;
+    const float* t = z + ((b * H + h) * G + k) * D;
+    for (int c = 0; c < D; c++) s = fmaf(a[c], t[c], s);
+  }
+  dM[idx] = s;
+}
+
+// ---- deslice: point-owned ----------------------------------------------------------
+template <int D, typename T>
+__global__ void __launch_bounds__(kThreads) k_deslice(const T* __restrict__ x, const float* __restrict__ W,
+                                                       const float* __restrict__ bias,
+                                                       const float* __restrict__ tau,
+                                                       const float* __restrict__ zp,
+                                                       const float* __restrict__ lse, T* __restrict__ out,
+                                                       int64_t N, int H, int G, uint32_t* status) {
+  constexpr int GC = 32;
+  __shared__ float sW[GC][D + 1];
+  __shared__ float sZ[GC][D];
+  __shared__ float sB[GC];
+  const int64_t bh = blockIdx.y;
+  const int64_t b = bh / H;
+  const int h = (int)(bh % H);
+  if (!tau_ok(tau[h], status)) return;
+  const float scale = kLog2e / tau[h];
+  const int64_t n = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  const bool valid = n < N;
+  float xr[D], acc[D];
+#pragma unroll
+  for (int k = 0; k < D; k++) { xr[k] = 0.f; acc[k] = 0.f; }
+  float l2 = CUDART_INF_F;
+  if (valid) {
+    load_row<D>(x + row_index(b, n, h, N, H) * D, xr);
+    l2 = lse[row_index(b, n, h, N, H)] * kLog2e;
+  }
+  const float* zb = zp + bh * G * D;
+  for (int g0 = 0; g0 < G; g0 += GC) {
+    __syncthreads();
+    stage_w<D, GC>(sW, sB, W, bias, h, G, g0, scale);
+    for (int i = threadIdx.x; i < GC * D; i += kThreads) {
+      const int g = i / D, k = i % D;
+      sZ[g][k] = (g0 + g < G) ? zb[(int64_t)(g0 + g) * D + k] : 0.f;
+    }
+    __syncthreads();
+    const int gn = min(GC, G - g0);
+    for (int g = 0; g < gn; g++) {
+      float a = sB[g];
+#pragma unroll
+      for (int k = 0; k < D; k++) a = fmaf(xr[k], sW[g][k], a);
+      const float w = exp2f(a - l2);
+#pragma unroll
+      for (int k = 0; k < D; k++) acc[k] = fmaf(w, sZ[g][k], acc[k]);
+    }
+  }
+  if (valid) store_row<D>(out + row_index(b, n, h, N, H) * D, acc);
+}
+
+// ---- backward, point-owned -------------------------------------------------------------
+// Gradient w.r.t. the weights of point n at slot g:
+//   MODE 0 (deslice): dw_g = dO . z'_g
+//   MODE 1 (slice)  : dw_g = f . dU_g + dS_g      (dUS[bh][g] = (dU_g, dS_g))
+// Sweep 1 forms delta = sum_g w_g dw_g (and, for the slice, dfx = sum_g w_g dU_g);
+// sweep 2 forms dx = (1/tau) sum_g w_g (dw_g - delta) W[:,g].
+template <int D, typename T, int MODE>
+__global__ void __launch_bounds__(kThreads) k_bwd_point(
+    const T* __restrict__ x, const T* __restrict__ v /* dout (MODE 0) or fx (MODE 1) */,
+    const float* __restrict__ W, const float* __restrict__ bias, const float* __restrict__ tau,
+    const float* __restrict__ tok /* z' (MODE 0) or (dU,dS) (MODE 1) */, const float* __restrict__ lse,
+    T* __restrict__ dx, T* __restrict__ dfx, float* __restrict__ delta, int accumulate, int64_t N, int H,
+    int G, uint32_t* status) {
+  constexpr int GC = 16;
+  constexpr int TS = (MODE == 0) ? D : D + 1;  // token row stride
+  __shared__ float sW[GC][D + 1];
+  __shared__ float sT[GC][TS];
+  __shared__ float sB[GC];
+  const int64_t bh = blockIdx.y;
+  const int64_t b = bh / H;
+  const int h = (int)(bh % H);
+  if (!tau_ok(tau[h], status)) return;
+  const float scale = kLog2e / tau[h];
+  const int64_t n = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  const bool valid = n < N;
+  float xr[D], vr[D], acc[D];
+#pragma unroll
+  for (int k = 0; k < D; k++) { xr[k] = 0.f; vr[k] = 0.f; acc[k] = 0.f; }
+  float l2 = CUDART_INF_F;
+  const int64_t row = row_index(b, n, h, N, H);
+  if (valid) {
+    load_row<D>(x + row * D, xr);
+    load_row<D>(v + row * D, vr);
+    l2 = lse[row] * kLog2e;
+  }
+  const float* tb = tok + bh * G * TS;
+  float dl = 0.f;
+  for (int sweep = 0; sweep < 2; sweep++) {
+    for (int g0 = 0; g0 < G; g0 += GC) {
+      __syncthreads();
+      stage_w<D, GC>(sW, sB, W, bias, h, G, g0, scale);
+      for (int i = threadIdx.x; i < GC * TS; i += kThreads) {
+        const int g = i / TS, k = i % TS;
+        sT[g][k] = (g0 + g < G) ? tb[(int64_t)(g0 + g) * TS + k] : 0.f;
+      }
+      __syncthreads();
+      const int gn = min(GC, G - g0);
+      for (int g = 0; g < gn; g++) {
+        float a = sB[g];
+#pragma unroll
+        for (int k = 0; k < D; k++) a = fmaf(xr[k], sW[g][k], a);
+        const float w = exp2f(a - l2);
+        float dw = (MODE == 0) ? 0.f : sT[g][D];
+#pragma unroll
+        for (int k = 0; k < D; k++) dw = fmaf(vr[k], sT[g][k], dw);
+        if (sweep == 0) {
+          dl = fmaf(w, dw, dl);
+          if (MODE == 1) {
+#pragma unroll
+            for (int k = 0; k < D; k++) acc[k] = fmaf(w, sT[g][k], acc[k]);
+          }
+        } else {
+          const float da = w * (dw - dl);
+#pragma unroll
+          for (int k = 0; k < D; k++) acc[k] = fmaf(da, sW[g][k], acc[k]);
+        }
+      }
+    }
+    if (sweep == 0) {
+      if (MODE == 1 && valid) store_row<D>(dfx + row * D, acc);
+#pragma unroll
+      for (int k = 0; k < D; k++) acc[k] = 0.f;
+    }
+  }
+  if (!valid) return;
+  delta[row] = dl;
+  // acc = sum_g da_g W[:,g] * log2e/tau ; dx = sum_g da_g W[:,g] / tau = acc * ln2.
+#pragma unroll
+  for (int k = 0; k < D; k++) acc[k] *= kLn2;
+  if (accumulate) {
+    float old[D];
+    load_row<D>(dx + row * D, old);
+#pragma unroll
+    for (int k = 0; k < D; k++) acc[k] += old[k];
+  }
+  store_row<D>(dx + row * D, acc);
+}
+
+// ---- backward, slot-owned ---------------------------------------------------------------
+// grid (ceil(G/128), B*H, P); thread = slot g.  For every point n of the split:
+//   da = w (dw - delta_n);  dWa += da x_n;  dba += da;  dta += da * a_n
+//   MODE 0 also accumulates dz'_g += w dO_n.
+// part[p][bh][g][...] = (MODE 0: dz'(D)) , dWa(D), dba, dta   (un-scaled by 1/tau)
+template <int D, typename T, int MODE>
+__global__ void __launch_bounds__(kThreads) k_bwd_slot(
+    const T* __restrict__ x, const T* __restrict__ v, const float* __restrict__ W,
+    const float* __restrict__ bias, const float* __restrict__ tau, const float* __restrict__ tok,
+    const float* __restrict__ lse, const float* __restrict__ delta, float* __restrict__ part, int64_t B,
+    int64_t N, int H, int G, int64_t per_split, uint32_t* status) {
+  constexpr int PT = 32;
+  constexpr int TS = (MODE == 0) ? D : D + 1;
+  constexpr int PS = (MODE == 0) ? 2 * D + 2 : D + 2;
+  __shared__ float sx[PT][D];
+  __shared__ float sv[PT][D];
+  __shared__ float sl[PT];
+  __shared__ float sd[PT];
+  const int g = blockIdx.x * kThreads + threadIdx.x;
+  const int64_t bh = blockIdx.y;
+  const int64_t b = bh / H;
+  const int h = (int)(bh % H);
+  const int p = blockIdx.z;
+  if (!tau_ok(tau[h], status)) return;
+  const float scale = kLog2e / tau[h];
+  float wc[D], tg[D], dzp[D], dWa[D];
+  float bb = 0.f, dSg = 0.f, dba = 0.f, dta = 0.f;
+#pragma unroll
+  for (int k = 0; k < D; k++) {
+    wc[k] = (g < G) ? W[((int64_t)h * D + k) * G + g] * scale : 0.f;
+    tg[k] = (g < G) ? tok[(bh * G + g) * TS + k] : 0.f;
+    dzp[k] = 0.f;
+    dWa[k] = 0.f;
+  }
+  if (g < G) {
+    bb = bias[(int64_t)h * G + g] * scale;
+    if (MODE == 1) dSg = tok[(bh * G + g) * TS + D];
+  }
+  const int64_t n_begin = (int64_t)p * per_split;
+  const int64_t n_end = min(N, n_begin + per_split);
+  for (int64_t n0 = n_begin; n0 < n_end; n0 += PT) {
+    __syncthreads();
+    for (int i = threadIdx.x; i < PT * D; i += kThreads) {
+      const int j = i / D, k = i % D;
+      const int64_t n = n0 + j;
+      float xv = 0.f, vv = 0.f;
+      if (n < n_end) {
+        const int64_t idx = row_index(b, n, h, N, H) * D + k;
+        xv = to_f(x[idx]);
+        vv = to_f(v[idx]);
+      }
+      sx[j][k] = xv;
+      sv[j][k] = vv;
+    }
+    for (int i = threadIdx.x; i < PT; i += kThreads) {
+      const int64_t n = n0 + i;
+      const bool ok = n < n_end;
+      sl[i] = ok ? lse[row_index(b, n, h, N, H)] * kLog2e : CUDART_INF_F;
+      sd[i] = ok ? delta[row_index(b, n, h, N, H)] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll 2
+    for (int j = 0; j < PT; j++) {
+      float a = bb;
+#pragma unroll
+      for (int k = 0; k < D; k++) a = fmaf(sx[j][k], wc[k], a);
+      const float w = exp2f(a - sl[j]);
+      float dw = dSg;
+#pragma unroll
+      for (int k = 0; k < D; k++) dw = fmaf(sv[j][k], tg[k], dw);
+      const float da = w * (dw - sd[j]);
+      if (MODE == 0) {
+#pragma unroll
+        for (int k = 0; k < D; k++) dzp[k] = fmaf(w, sv[j][k], dzp[k]);
+      }
+#pragma unroll
+      for (int k = 0; k < D; k++) dWa[k] = fmaf(da, sx[j][k], dWa[k]);
+      dba += da;
+      // a is the base-2 logit; the natural logit is a * ln2 (zero for padded points: w = 0).
+      dta = fmaf(da, a * kLn2, dta);
+    }
+  }
+  if (g < G) {
+    float* o = part + (((int64_t)p * B * H + bh) * G + g) * PS;
+    int off = 0;
+    if (MODE == 0) {
+#pragma unroll
+      for (int k = 0; k < D; k++) o[k] = dzp[k];
+      off = D;
+    }
+#pragma unroll
+    for (int k = 0; k < D; k++) o[off + k] = dWa[k];
+    o[off + D] = dba;
+    o[off + D + 1] = dta;
+  }
+}
+
+// Token-gradient prep for the slice backward: dUS[bh][g] = (dz_g/(S_g+eps), -(dz_g.z_g)/(S_g+eps)).
+__global__ void k_slice_bwd_prep(const float* __restrict__ z, const float* __restrict__ wsum,
+                                 const float* __restrict__ dz, float* __restrict__ dUS, int64_t BHG, int D,
+                                 float eps) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= BHG) return;
+  const float den = wsum[i] + eps;
+  float s = 0.f;
+  for (int c = 0; c < D; c++) {
+    const float g = dz[i * D + c];
+    dUS[i * (D + 1) + c] = g / den;
+    s = fmaf(g, z[i * D + c], s);
+  }
+  dUS[i * (D + 1) + D] = -s / den;
+}
+
+// Fixed-order reduction of slot-owned backward partials over (b, p).
+// Writes (or adds) dW[h][k][g], db[h][g]; dtau_g[h][g] = per-slot dtau terms;
+// optionally d_tokens_mixed[b][h][g][c] (sum over p only).
+__global__ void k_reduce_bwd(const float* __restrict__ part, int P, int64_t B, int H, int G, int D,
+                             int PS, int has_dzp, const float* __restrict__ tau, float* __restrict__ dzp,
+                             float* __restrict__ dW, float* __restrict__ db, float* __restrict__ dtau_g,
+                             int accumulate) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)H * G) return;
+  const int h = (int)(idx / G), g = (int)(idx % G);
+  const float inv = 1.f / tau[h];
+  const int off = has_dzp ? D : 0;
+  const int64_t BH = B * H;
+  if (has_dzp) {
+    for (int64_t b = 0; b < B; b++) {
+      for (int c = 0; c < D; c++) {
+        float s = 0.f;
+        for (int p = 0; p < P; p++) s += part[(((int64_t)p * BH + b * H + h) * G + g) * PS + c];
+        dzp[((b * H + h) * G + g) * D + c] = s;
+      }
+    }
+  }
+  for (int k = 0; k <= D + 1; k++) {
+    float s = 0.f;
+    for (int64_t b = 0; b < B; b++)
+      for (int p = 0; p < P; p++) s += part[(((int64_t)p * BH + b * H + h) * G + g) * PS + off + k];
+    if (k < D) {
+      const int64_t o = ((int64_t)h * D + k) * G + g;
+      dW[o] = (accumulate ? dW[o] : 0.f) + s * inv;
+    } else if (k == D) {
+      db[idx] = (accumulate ? db[idx] : 0.f) + s * inv;
+    } else {
+      dtau_g[idx] = -s * inv;
+    }
+  }
+}
+
+// dtau[h] (+)= sum_g dtau_g[h][g], fixed-order tree within one block per head.
+__global__ void k_reduce_dtau(const float* __restrict__ dtau_g, int G, float* __restrict__ dtau,
+                              int accumulate) {
+  __shared__ float s[256];
+  const int h = blockIdx.x;
+  float v = 0.f;
+  for (int g = threadIdx.x; g < G; g += 256) v += dtau_g[(int64_t)h * G + g];
+  s[threadIdx.x] = v;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if (threadIdx.x < w) s[threadIdx.x] += s[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) dtau[h] = (accumulate ? dtau[h] : 0.f) + s[0];
+}
+
+inline dim3 point_grid(const Shape& s) {
+  return dim3((unsigned)((s.N + kThreads - 1) / kThreads), (unsigned)s.BH());
+}
+inline dim3 slot_grid(const Shape& s, int P) {
+  return dim3((unsigned)((s.G + kThreads - 1) / kThreads), (unsigned)s.BH(), (unsigned)P);
+}
+inline int64_t per_split(const Shape& s, int P) { return (s.N + P - 1) / P; }
+
+template <int D, typename T>
+cudaError_t launch_stats(const Shape& s, const void* x, const float* W, const float* bias, const float* tau,
+                         float* lse, uint32_t* status, cudaStream_t st) {
+  k_stats<D, T><<<point_grid(s), kThreads, 0, st>>>((const T*)x, W, bias, tau, lse, s.N, s.H, s.G, status);
+  return cudaGetLastError();
+}
+
+template <int D, typename T>
+cudaError_t launch_slice_partials(const Shape& s, int P, const void* x, const void* f, const float* W,
+                                  const float* bias, const float* tau, const float* lse, float* part,
+                                  uint32_t* status, cudaStream_t st) {
+  k_slice_partial<D, T><<<slot_grid(s, P), kThreads, 0, st>>>((const T*)x, (const T*)f, W, bias, tau, lse,
+                                                               part, s.B, s.N, s.H, s.G, per_split(s, P),
+                                                               status);
+  return cudaGetLastError();
+}
+
+template <int D, typename T>
+cudaError_t launch_deslice(const Shape& s, const void* x, const float* W, const float* bias, const float* tau,
+                           const float* zp, const float* lse, void* out, uint32_t* status, cudaStream_t st) {
+  k_deslice<D, T><<<point_grid(s), kThreads, 0, st>>>((const T*)x, W, bias, tau, zp, lse, (T*)out, s.N, s.H,
+                                                       s.G, status);
+  return cudaGetLastError();
+}
+
+template <int D, typename T, int MODE>
+cudaError_t launch_bwd(const Shape& s, int P, const void* x, const void* v, const float* W, const float* bias,
+                       const float* tau, const float* tok, const float* lse, void* dx, void* dfx, float* delta,
+                       float* part, int accumulate, uint32_t* status, cudaStream_t st) {
+  k_bwd_point<D, T, MODE><<<point_grid(s), kThreads, 0, st>>>((const T*)x, (const T*)v, W, bias, tau, tok, lse,
+                                                               (T*)dx, (T*)dfx, delta, accumulate, s.N, s.H,
+                                                               s.G, status);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_bwd_slot<D, T, MODE><<<slot_grid(s, P), kThreads, 0, st>>>((const T*)x, (const T*)v, W, bias, tau, tok,
+                                                                lse, delta, part, s.B, s.N, s.H, s.G,
+                                                                per_split(s, P), status);
+  return cudaGetLastError();
+}
+
+// Dispatch over (d, dtype).
+#define FS_DISPATCH(s, FN, ...)                                                        \
+  do {                                                                                 \
+    const bool bf = (s).dtype == FS_BF16;                                              \
+    switch ((s).d) {                                                                   \
+      case 16: return bf ? FN<16, __nv_bfloat16>(__VA_ARGS__) : FN<16, float>(__VA_ARGS__); \
+      case 32: return bf ? FN<32, __nv_bfloat16>(__VA_ARGS__) : FN<32, float>(__VA_ARGS__); \
+      case 64: return bf ? FN<64, __nv_bfloat16>(__VA_ARGS__) : FN<64, float>(__VA_ARGS__); \
+      default: return cudaErrorInvalidValue;                                           \
+    }                                                                                  \
+  } while (0)
+
+template <int D, typename T>
+cudaError_t launch_bwd_deslice(const Shape& s, int P, const void* x, const void* v, const float* W,
+                               const float* bias, const float* tau, const float* tok, const float* lse,
+                               void* dx, float* delta, float* part, int accumulate, uint32_t* status,
+                               cudaStream_t st) {
+  return launch_bwd<D, T, 0>(s, P, x, v, W, bias, tau, tok, lse, dx, nullptr, delta, part, accumulate, status,
+                             st);
+}
+template <int D, typename T>
+cudaError_t launch_bwd_slice(const Shape& s, int P, const void* x, const void* v, const float* W,
+                             const float* bias, const float* tau, const float* tok, const float* lse, void* dx,
+                             void* dfx, float* delta, float* part, int accumulate, uint32_t* status,
+                             cudaStream_t st) {
+  return launch_bwd<D, T, 1>(s, P, x, v, W, bias, tau, tok, lse, dx, dfx, delta, part, accumulate, status, st);
+}
+
+cudaError_t reduce_params(const Shape& s, int P, const float* part, int PS, int has_dzp, const float* tau,
+                          float* dzp, float* dW, float* db, float* dtau, float* dtau_g, int accumulate,
+                          cudaStream_t st) {
+  const int64_t HG = (int64_t)s.H * s.G;
+  k_reduce_bwd<<<(unsigned)((HG + 127) / 128), 128, 0, st>>>(part, P, s.B, s.H, s.G, s.d, PS, has_dzp, tau,
+                                                              dzp, dW, db, dtau_g, accumulate);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_reduce_dtau<<<s.H, 256, 0, st>>>(dtau_g, s.G, dtau, accumulate);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t simt_stats(const Shape& s, const void* x, const float* W, const float* bias, const float* tau,
+                       float* lse, uint32_t* status, cudaStream_t st) {
+  FS_DISPATCH(s, launch_stats, s, x, W, bias, tau, lse, status, st);
+}
+
+cudaError_t simt_slice_partials(const Shape& s, int P, const void* x, const void* f, const float* W,
+                                const float* bias, const float* tau, const float* lse, float* part,
+                                uint32_t* status, cudaStream_t st) {
+  FS_DISPATCH(s, launch_slice_partials, s, P, x, f, W, bias, tau, lse, part, status, st);
+}
+
+cudaError_t simt_reduce_tokens(const Shape& s, int P, const float* part, float* tokens, float* wsum,
+                               int finalize, cudaStream_t st) {
+  const int64_t BHG = s.BH() * s.G;
+  k_reduce_tokens<<<(unsigned)((BHG + 255) / 256), 256, 0, st>>>(part, P, BHG, s.d, tokens, wsum, finalize,
+                                                                 s.eps);
+  return cudaGetLastError();
+}
+
+cudaError_t simt_finalize(const Shape& s, float* tokens, const float* wsum, cudaStream_t st) {
+  const int64_t BHG = s.BH() * s.G;
+  k_finalize<<<(unsigned)((BHG * s.d + 255) / 256), 256, 0, st>>>(tokens, wsum, BHG, s.d, s.eps);
+  return cudaGetLastError();
+}
+
+cudaError_t simt_mix(const Shape& s, const float* M, const float* z, float* zp, cudaStream_t st) {
+  dim3 grid((unsigned)((s.G * s.d + 255) / 256), (unsigned)s.BH());
+  k_mix<<<grid, 256, 0, st>>>(M, z, zp, s.H, s.G, s.d);
+  return cudaGetLastError();
+}
+
+cudaError_t simt_mix_bwd(const Shape& s, const float* M, const float* z, const float* dzp, float* dz, float* dM,
+                         cudaStream_t st) {
+  dim3 grid((unsigned)((s.G * s.d + 255) / 256), (unsigned)s.BH());
+  k_mix_bwd_dz<<<grid, 256, 0, st>>>(M, dzp, dz, s.H, s.G, s.d);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int64_t HGG = (int64_t)s.H * s.G * s.G;
+  k_mix_bwd_dM<<<(unsigned)((HGG + 255) / 256), 256, 0, st>>>(z, dzp, dM, s.B, s.H, s.G, s.d);
+  return cudaGetLastError();
+}
+
+cudaError_t simt_deslice(const Shape& s, const void* x, const float* W, const float* bias, const float* tau,
+                         const float* zp, const float* lse, void* out, uint32_t* status, cudaStream_t st) {
+  FS_DISPATCH(s, launch_deslice, s, x, W, bias, tau, zp, lse, out, status, st);
+}
+
+cudaError_t simt_deslice_bwd(const Shape& s, int P, const void* x, const float* W, const float* bias,
+                             const float* tau, const float* zp, const float* lse, const void* dout, float* dzp,
+                             void* dx, float* dW, float* db, float* dtau, int accumulate, float* delta,
+                             float* part, float* dtau_g, uint32_t* status, cudaStream_t st) {
+  cudaError_t e = [&]() -> cudaError_t {
+    FS_DISPATCH(s, launch_bwd_deslice, s, P, x, dout, W, bias, tau, zp, lse, dx, delta, part, accumulate,
+                status, st);
+  }();
+  if (e != cudaSuccess) return e;
+  return reduce_params(s, P, part, 2 * s.d + 2, 1, tau, dzp, dW, db, dtau, dtau_g, accumulate, st);
+}
+
+cudaError_t simt_slice_bwd(const Shape& s, int P, const void* x, const void* f, const float* W,
+                           const float* bias, const float* tau, const float* z, const float* wsum,
+                           const float* lse, const float* dz, void* dx, void* dfx, float* dW, float* db,
+                           float* dtau, int accumulate, float* delta, float* dUS, float* part, float* dtau_g,
+                           uint32_t* status, cudaStream_t st) {
+  const int64_t BHG = s.BH() * s.G;
+  k_slice_bwd_prep<<<(unsigned)((BHG + 255) / 256), 256, 0, st>>>(z, wsum, dz, dUS, BHG, s.d, s.eps);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  e = [&]() -> cudaError_t {
+    FS_DISPATCH(s, launch_bwd_slice, s, P, x, f, W, bias, tau, dUS, lse, dx, dfx, delta, part, accumulate,
+                status, st);
+  }();
+  if (e != cudaSuccess) return e;
+  return reduce_params(s, P, part, s.d + 2, 0, tau, nullptr, dW, db, dtau, dtau_g, accumulate, st);
+}
+
+}  // namespace fs

@@ -1,0 +1,100 @@
+"""Host-side checks of the C-ABI library: it loads, exports every entry point the
+header declares, and validates arguments before launching anything.  No GPU:
+every call here fails validation (or only queries sizes) before any launch."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "flashslice.h")
+LIB = os.path.join(ROOT, "paper_2609_32525_gb300", "libflashslice.so")
+
+
+@pytest.fixture(scope="module")
+def fs():
+    if not os.path.exists(LIB):
+        from paper_2609_32525_gb300 import build
+
+        build.build()
+    from paper_2609_32525_gb300 import flashslice
+
+    return flashslice
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(fs_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_documented_entry_points():
+    names = declared_functions()
+    for n in ("fs_slice_fwd", "fs_mix", "fs_deslice_fwd", "fs_slice_bwd", "fs_deslice_bwd", "fs_mix_bwd",
+              "fs_slice_finalize", "fs_workspace_bytes", "fs_device_status", "fs_status_string"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(fs):
+    lib = ctypes.CDLL(LIB)
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert set(fs.EXPORTED) <= set(declared_functions())
+
+
+def test_status_strings(fs):
+    for st in range(6):
+        assert fs.status_string(st).startswith("FS_")
+    assert "unknown" in fs.status_string(99)
+
+
+def test_workspace_sizes(fs):
+    s = fs.make_shape(1, 4096, 8, 32, 32)
+    for op in range(4):
+        assert fs.workspace_bytes(s, op) >= 256
+    assert fs.workspace_bytes(fs.make_shape(1, 4096, 8, 32, 32), 99) == 0
+    assert fs.workspace_bytes(fs.make_shape(0, 4096, 8, 32, 32), 0) == 0       # invalid
+    assert fs.workspace_bytes(fs.make_shape(1, 4096, 8, 48, 32), 0) == 0       # unsupported d
+    big = fs.workspace_bytes(fs.make_shape(1, 1 << 20, 8, 32, 1024), fs.FS_OP_SLICE_FWD)
+    assert big >= (1 << 20) * 8 * 4  # at least the lse scratch
+
+
+def _call_slice(fs, shape, ptrs, ws_ptr=16, ws_bytes=1 << 30):
+    lib = fs._lib
+    P = ctypes.c_void_p
+    return lib.fs_slice_fwd(ctypes.byref(shape), *[P(p) if p else None for p in ptrs], None, 1, P(ws_ptr) if ws_ptr else None,
+                            ws_bytes, None)
+
+
+def test_validation_rejects_bad_arguments_without_launching(fs):
+    good = [16 * (i + 1) for i in range(7)]  # fake aligned addresses, never dereferenced
+    s = fs.make_shape(1, 100, 2, 32, 8)
+    # null pointer
+    assert _call_slice(fs, s, [0] + good[1:]) == fs.FS_ERR_INVALID
+    # misaligned pointer
+    assert _call_slice(fs, s, [good[0] + 4] + good[1:]) == fs.FS_ERR_INVALID
+    # bad sizes
+    for bad in (fs.make_shape(0, 100, 2, 32, 8), fs.make_shape(1, 0, 2, 32, 8), fs.make_shape(1, 100, 0, 32, 8),
+                fs.make_shape(1, 100, 2, 32, 0), fs.make_shape(1, 100, 2, 32, 8, dtype=7),
+                fs.make_shape(1, 100, 2, 32, 8, eps=-1.0), fs.make_shape(1, 100, 2, 32, 8, eps=float("nan"))):
+        assert _call_slice(fs, bad, good) == fs.FS_ERR_INVALID
+    # unsupported head width / slice count
+    assert _call_slice(fs, fs.make_shape(1, 100, 2, 48, 8), good) == fs.FS_ERR_UNSUPPORTED
+    assert _call_slice(fs, fs.make_shape(1, 100, 2, 32, 5000), good) == fs.FS_ERR_UNSUPPORTED
+    # workspace missing or too small
+    assert _call_slice(fs, s, good, ws_ptr=0) == fs.FS_ERR_INVALID
+    assert _call_slice(fs, s, good, ws_bytes=8) == fs.FS_ERR_INVALID
+
+
+def test_mix_rejects_in_place(fs):
+    s = fs.make_shape(1, 100, 2, 32, 8)
+    P = ctypes.c_void_p
+    assert fs._lib.fs_mix(ctypes.byref(s), P(16), P(32), P(32), None) == fs.FS_ERR_INVALID
+    assert fs._lib.fs_device_status(None, None) == fs.FS_ERR_INVALID
+
+
+def test_path_query(fs):
+    assert fs.path_for_shape(fs.make_shape(1, 100, 2, 48, 8)) == -1
+    assert fs.path_for_shape(fs.make_shape(1, 100, 2, 32, 8, dtype=fs.FS_F32)) == 0
+    assert fs.forward_launch_count(fs.make_shape(1, 100, 2, 32, 8)) >= 3
