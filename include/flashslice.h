@@ -30,7 +30,7 @@
  *      M, dM                             : [H, G, G]      fp32, M[h][g][k]
  *      tokens, tokens_mixed, d_tokens*   : [B, H, G, d]   fp32
  *      wsum                              : [B, H, G]      fp32
- *      lse                               : [B, N, H]      fp32, natural log
+ *      lse                               : [B, H, N]      fp32, natural log
  *    Channel c of a point's C = H*d features is head c / d, lane c % d.
  *  - Every pointer must be 16-byte aligned.
  *  - `ws` is caller-owned scratch of at least fs_workspace_bytes(shape, op)
@@ -98,7 +98,7 @@ size_t fs_workspace_bytes(const fs_shape* s, int op);
  *   in : x_mid, fx [B,N,H,d]; W_slice [H,d,G]; bias [H,G]; tau [H]
  *   out: tokens [B,H,G,d] = U/(S+eps) if finalize != 0, else the unnormalised
  *        numerators U (for a cross-device sum before fs_slice_finalize);
- *        wsum [B,H,G] = S; lse [B,N,H] (may be NULL: then kept in ws only). */
+ *        wsum [B,H,G] = S; lse [B,H,N] (may be NULL: then kept in ws only). */
 fs_status fs_slice_fwd(const fs_shape* s, const void* x_mid, const void* fx,
                        const float* W_slice, const float* bias, const float* tau,
                        float* tokens, float* wsum, float* lse, int finalize,

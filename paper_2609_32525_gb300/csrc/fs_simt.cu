@@ -139,7 +139,7 @@ __global__ void __launch_bounds__(kThreads) k_stats(const T* __restrict__ x, con
     l = l * exp2f(m - mn) + acc;
     m = mn;
   }
-  if (valid) lse[row_index(b, n, h, N, H)] = (m + log2f(l)) * kLn2;
+  if (valid) lse[bh * N + n] = (m + log2f(l)) * kLn2;
 }
 
 // ---- slice: slot-owned split-N partials ------------------------------------------
@@ -186,7 +186,7 @@ __global__ void __launch_bounds__(kThreads) k_slice_partial(
     }
     for (int i = threadIdx.x; i < PT; i += kThreads) {
       const int64_t n = n0 + i;
-      sl[i] = (n < n_end) ? lse[row_index(b, n, h, N, H)] * kLog2e : CUDART_INF_F;
+      sl[i] = (n < n_end) ? lse[bh * N + n] * kLog2e : CUDART_INF_F;
     }
     __syncthreads();
 #pragma unroll 4
@@ -304,7 +304,7 @@ __global__ void __launch_bounds__(kThreads) k_deslice(const T* __restrict__ x, c
   float l2 = CUDART_INF_F;
   if (valid) {
     load_row<D>(x + row_index(b, n, h, N, H) * D, xr);
-    l2 = lse[row_index(b, n, h, N, H)] * kLog2e;
+    l2 = lse[bh * N + n] * kLog2e;
   }
   const float* zb = zp + bh * G * D;
   for (int g0 = 0; g0 < G; g0 += GC) {
@@ -361,7 +361,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_point(
   if (valid) {
     load_row<D>(x + row * D, xr);
     load_row<D>(v + row * D, vr);
-    l2 = lse[row] * kLog2e;
+    l2 = lse[bh * N + n] * kLog2e;
   }
   const float* tb = tok + bh * G * TS;
   float dl = 0.f;
@@ -403,7 +403,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_point(
     }
   }
   if (!valid) return;
-  delta[row] = dl;
+  delta[bh * N + n] = dl;
   // acc = sum_g da_g W[:,g] * log2e/tau ; dx = sum_g da_g W[:,g] / tau = acc * ln2.
 #pragma unroll
   for (int k = 0; k < D; k++) acc[k] *= kLn2;
@@ -473,8 +473,8 @@ __global__ void __launch_bounds__(kThreads) k_bwd_slot(
     for (int i = threadIdx.x; i < PT; i += kThreads) {
       const int64_t n = n0 + i;
       const bool ok = n < n_end;
-      sl[i] = ok ? lse[row_index(b, n, h, N, H)] * kLog2e : CUDART_INF_F;
-      sd[i] = ok ? delta[row_index(b, n, h, N, H)] : 0.f;
+      sl[i] = ok ? lse[bh * N + n] * kLog2e : CUDART_INF_F;
+      sd[i] = ok ? delta[bh * N + n] : 0.f;
     }
     __syncthreads();
 #pragma unroll 2

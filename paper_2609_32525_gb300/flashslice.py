@@ -10,7 +10,7 @@ the library and fails loudly if it has not been built
 Tensor conventions (see the header for the full contract):
   x_mid, fx, out, dout, dx_mid, dfx : [B,N,H,d] float32 or bfloat16, contiguous
   W_slice [H,d,G], bias [H,G], tau [H], M [H,G,G]            float32
-  tokens, tokens_mixed, d_tokens*  [B,H,G,d], wsum [B,H,G], lse [B,N,H]  float32
+  tokens, tokens_mixed, d_tokens*  [B,H,G,d], wsum [B,H,G], lse [B,H,N]  float32
 """
 from __future__ import annotations
 
@@ -182,7 +182,7 @@ class Coupling:
         f32 = dict(dtype=torch.float32, device=device)
         self.tokens = torch.empty(B, H, G, d, **f32)
         self.wsum = torch.empty(B, H, G, **f32)
-        self.lse = torch.empty(B, N, H, **f32)
+        self.lse = torch.empty(B, H, N, **f32)
         self.tokens_mixed = torch.empty(B, H, G, d, **f32)
         self.out = torch.empty(B, N, H, d, dtype=dtype, device=device)
         self.ws_slice = workspace(self.shape, FS_OP_SLICE_FWD, device)
