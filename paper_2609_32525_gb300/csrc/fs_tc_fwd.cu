@@ -16,10 +16,11 @@
 // into two bf16 halves to keep them near fp32 accurate).  The stats pass uses
 // A = [x | 1, 1, 0, 0] and keeps a running max / sum in registers.
 //
-// CTA layout (256 threads): warp 0 issues TMA / bulk copies, warp 1 owns the
-// TMEM allocation and issues every tcgen05.mma from one lane, warps 4..7 form
-// the softmax warpgroup: thread r of it owns TMEM lane r = point r of the tile
-// (tcgen05.ld 32x32b).  Warps 2, 3 idle.  All waits are bounded (2 s): a wait
+// CTA layout (384 threads): warp 0 issues TMA / bulk copies, warp 1 owns the
+// TMEM allocation and issues every tcgen05.mma from one lane, warps 4..11 form
+// two softmax warpgroups that split the columns of every chunk: thread r of a
+// warpgroup owns TMEM lane r = point r of the tile (tcgen05.ld 32x32b), so
+// every SM sub-partition runs two softmax warps.  Warps 2, 3 idle.  All waits are bounded (2 s): a wait
 // that gives up flags FS_ERR_TIMEOUT in the status word and the CTA drains its
 // in-flight copies and MMAs, frees TMEM and exits.
 //
@@ -43,10 +44,10 @@ namespace {
 
 using namespace tc;
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 384;
 constexpr int kTile = 128;        // points per tile
 constexpr int kD = 32;            // head width of the tensor-core path
-constexpr int kSoftmaxWarp0 = 4;  // warps 4..7
+constexpr int kSoftmaxWarp0 = 4;  // warps 4..11: two softmax warpgroups
 constexpr int kStages = 3;        // x-tile pipeline depth (stats / deslice)
 constexpr int kSliceStages = 3;   // slice pipeline depth
 constexpr uint32_t kXBytes = kTile * 64;    // 128 points x 32 bf16
@@ -169,13 +170,20 @@ __device__ __forceinline__ void load_images(uint8_t* dst, const uint8_t* src, ui
 // =========================================================================================
 // Deslice: out_n = sum_g w_ng z'_g.
 // smem: [W img G*96][Z' img G*64][x stages][xe stages][barriers]
-// TMEM: S/P buffers at [0, 2*GC), O buffers at [2*GC, 2*GC + 64).
+// TMEM: three S buffers [0, 3*GC), O buffers [3*GC, 3*GC + 64).  The logits run
+// two chunks ahead of the softmax.  The two softmax warpgroups split every
+// chunk's columns: warpgroup wg reads S columns [64 wg, 64 wg + 64) and writes
+// their bf16 weights back, packed in pairs, into columns [64 wg, 64 wg + 32) of
+// the same buffer, which the P x Z' MMA reads as its A operand.
 // =========================================================================================
+constexpr int kSBuf = 3;
+
 template <int GC>
 __global__ void __launch_bounds__(kThreads, 1)
     k_deslice(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ wimg,
               const uint8_t* __restrict__ zimg, const float* __restrict__ lse, __nv_bfloat16* __restrict__ out,
               int64_t N, int H, int G, int splits, uint32_t* status) {
+  static_assert(GC == 128, "chunk width");
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t wbytes = (uint32_t)G * 96, zbytes = (uint32_t)G * 64;
@@ -189,8 +197,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* x_empty = x_full + kStages;
   uint64_t* xe_ready = x_empty + kStages;
   uint64_t* s_full = xe_ready + kStages;
-  uint64_t* p_ready = s_full + 2;
-  uint64_t* o_full = p_ready + 2;
+  uint64_t* p_ready = s_full + kSBuf;
+  uint64_t* o_full = p_ready + kSBuf;
   uint64_t* o_free = o_full + 2;
   uint64_t* drain = o_free + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
@@ -201,6 +209,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int64_t b = wk.bh / H;
   const int h = (int)(wk.bh % H);
   const int nch = G / GC;
+  constexpr uint32_t kO = kSBuf * GC;  // TMEM column base of the O buffers
 
   if (threadIdx.x == 0) {
     mbar_init(wz_full, 1);
@@ -209,11 +218,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&x_empty[s], 1);
       mbar_init(&xe_ready[s], 4);
     }
-    for (int i = 0; i < 2; i++) {
+    for (int i = 0; i < kSBuf; i++) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&p_ready[i], 4);
+      mbar_init(&p_ready[i], 8);
+    }
+    for (int i = 0; i < 2; i++) {
       mbar_init(&o_full[i], 1);
-      mbar_init(&o_free[i], 4);
+      mbar_init(&o_free[i], 8);
     }
     mbar_init(drain, 1);
     ab->flag = 0;
@@ -246,8 +257,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     // ------------------------------ MMA issuer ------------------------------
-    // One flattened sequence q = tile * nch + chunk: the logits of q+1 are issued
-    // before waiting for the softmax of q, across tile boundaries.
+    // One flattened sequence q = tile * nch + chunk; the logits of q+2 are issued
+    // before waiting for the softmax of q, across tile boundaries.  A buffer is
+    // rewritten only by an MMA issued after the P x Z' MMA that last read it, and
+    // tcgen05.mma executes in issue order.
     if (lane == 0 && wk.ntiles > 0) {
       constexpr uint32_t idesc_pv = idesc_bf16(128, kD, false, false);
       const uint32_t sw = smem_u32(s_w), swe = sw + (uint32_t)G * 64, sz = smem_u32(s_z);
@@ -261,28 +274,31 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (!mbar_wait(&x_full[s], par, ab, status) || !mbar_wait(&xe_ready[s], par, ab, status)) return false;
           tc_fence_after();
         }
-        issue_logits<GC>(tmem + (uint32_t)(qq & 1) * GC, smem_u32(s_x + s * kXBytes), smem_u32(s_xe + s * kXeBytes),
-                         sw, swe, c);
-        mma_commit(&s_full[qq & 1]);
+        const int bb = (int)(qq % kSBuf);
+        issue_logits<GC>(tmem + (uint32_t)bb * GC, smem_u32(s_x + s * kXBytes), smem_u32(s_xe + s * kXeBytes), sw,
+                         swe, c);
+        mma_commit(&s_full[bb]);
         if (c == nch - 1) mma_commit(&x_empty[s]);
         return true;
       };
-      bool ok = mbar_wait(wz_full, 0, ab, status) && logits(0);
+      bool ok = mbar_wait(wz_full, 0, ab, status) && logits(0) && (total < 2 || logits(1));
       for (int64_t q = 0; ok && q < total; q++) {
         const int64_t i = q / nch;
         const int c = (int)(q % nch);
         const int ob = (int)(i & 1);
-        if (q + 1 < total && !(ok = logits(q + 1))) break;
+        const int bb = (int)(q % kSBuf);
+        if (q + 2 < total && !(ok = logits(q + 2))) break;
         if (c == 0 && i >= 2 && !(ok = mbar_wait(&o_free[ob], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
-        if (!(ok = mbar_wait(&p_ready[q & 1], (uint32_t)((q >> 1) & 1), ab, status))) break;
+        if (!(ok = mbar_wait(&p_ready[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t tP = tmem + (uint32_t)(q & 1) * GC;
-        const uint32_t tO = tmem + 2 * GC + ob * kD;
+        const uint32_t tS = tmem + (uint32_t)bb * GC;
+        const uint32_t tO = tmem + kO + (uint32_t)ob * kD;
 #pragma unroll
         for (int k = 0; k < GC / 16; k++) {
           const int g0 = c * GC + k * 16;
           const uint32_t zaddr = sz + (uint32_t)((g0 >> 6) * 4096 + (g0 & 63) * 2);
-          mma_ts(tO, tP + (uint32_t)k * 8, sdesc(zaddr, 16, 1024, kSw128), idesc_pv, (c > 0 || k > 0) ? 1u : 0u);
+          const uint32_t tP = tS + (uint32_t)((k >> 2) * 64 + (k & 3) * 8);
+          mma_ts(tO, tP, sdesc(zaddr, 16, 1024, kSw128), idesc_pv, (c > 0 || k > 0) ? 1u : 0u);
         }
         if (c == nch - 1) mma_commit(&o_full[ob]);
       }
@@ -291,18 +307,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait(drain, 0, ab, nullptr, 2000000000ull);
     }
   } else if (warp >= kSoftmaxWarp0) {
-    // ------------------------------ softmax warpgroup ------------------------------
-    const int wq = warp - kSoftmaxWarp0;
+    // ------------------------------ softmax warpgroups ------------------------------
+    const int wg = (warp - kSoftmaxWarp0) >> 2;
+    const int wq = warp & 3;  // TMEM sub-partition of this warp
     const int r = wq * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     int64_t q = 0;
     bool ok = true;
-    // The A extra block of tile j carries -lse of its points; it is written one
-    // tile ahead so the MMA warp can run the next tile's logits early.
-    auto put_extra = [&](int64_t j) -> bool {
-      const int s = (int)(j % kStages);
+    // lse of tile j, loaded two tiles ahead of its use.
+    auto load_l2 = [&](int64_t j) -> float {
       const int64_t nn = (wk.tile0 + j) * kTile + r;
-      const float l2 = nn < N ? lse[wk.bh * N + nn] * kLog2e : 0.f;
+      return (j < wk.ntiles && nn < N) ? lse[wk.bh * N + nn] * kLog2e : 0.f;
+    };
+    // The A extra block of tile j carries -lse of its points; warpgroup 0 writes
+    // it one tile ahead so the MMA warp can run the next tile's logits early.
+    auto put_extra = [&](int64_t j, float l2) -> bool {
+      const int s = (int)(j % kStages);
       if (j >= kStages && !mbar_wait(&x_empty[s], (uint32_t)(((j / kStages) - 1) & 1), ab, status)) return false;
       write_a_extra(s_xe + s * kXeBytes, r, l2);
       fence_proxy_async_smem();
@@ -310,51 +330,68 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(&xe_ready[s]);
       return true;
     };
-    if (wk.ntiles > 0) ok = put_extra(0);
-    for (int64_t i = 0; ok && i < wk.ntiles; i++) {
-      const int64_t n = (wk.tile0 + i) * kTile + r;
-      const bool valid = n < N;
-      if (i + 1 < wk.ntiles && !(ok = put_extra(i + 1))) break;
-      for (int c = 0; c < nch; c++, q++) {
-        if (!(ok = mbar_wait(&s_full[q & 1], (uint32_t)((q >> 1) & 1), ab, status))) break;
-        tc_fence_after();
-        const uint32_t tS = tmem + lane_addr + (uint32_t)(q & 1) * GC;
-#pragma unroll 1
-        for (int part = 0; part < GC / 32; part++) {
-          uint32_t v[32];
-          tmem_ld32(tS + part * 32, v);
-          tmem_wait_ld(v);
-          uint32_t pk[16];
-#pragma unroll
-          for (int j = 0; j < 16; j++)
-            pk[j] = pack_bf16(ex2(__uint_as_float(v[2 * j])), ex2(__uint_as_float(v[2 * j + 1])));
-          tmem_st16(tS + part * 16, pk);
-        }
-        tmem_wait_st();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&p_ready[q & 1]);
-      }
-      if (!ok) break;
-      const int ob = (int)(i & 1);
-      if (!(ok = mbar_wait(&o_full[ob], (uint32_t)((i >> 1) & 1), ab, status))) break;
+    // Output of tile t: this warpgroup's 16 channels of O -> bf16 -> global.
+    auto epilogue = [&](int64_t t) -> bool {
+      const int ob = (int)(t & 1);
+      if (!mbar_wait(&o_full[ob], (uint32_t)((t >> 1) & 1), ab, status)) return false;
       tc_fence_after();
-      uint32_t o[32];
-      tmem_ld32(tmem + lane_addr + 2 * GC + ob * kD, o);
+      uint32_t o[16];
+      tmem_ld16(tmem + lane_addr + kO + (uint32_t)ob * kD + (uint32_t)wg * 16, o);
       tmem_wait_ld(o);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&o_free[ob]);
-      if (valid) {
-        uint4* dst = reinterpret_cast<uint4*>(out + ((b * N + n) * H + h) * kD);
+      const int64_t n = (wk.tile0 + t) * kTile + r;
+      if (n < N) {
+        uint4* dst = reinterpret_cast<uint4*>(out + ((b * N + n) * H + h) * kD + wg * 16);
 #pragma unroll
-        for (int j = 0; j < 4; j++)
+        for (int j = 0; j < 2; j++)
           dst[j] = make_uint4(pack_bf16(__uint_as_float(o[8 * j]), __uint_as_float(o[8 * j + 1])),
                               pack_bf16(__uint_as_float(o[8 * j + 2]), __uint_as_float(o[8 * j + 3])),
                               pack_bf16(__uint_as_float(o[8 * j + 4]), __uint_as_float(o[8 * j + 5])),
                               pack_bf16(__uint_as_float(o[8 * j + 6]), __uint_as_float(o[8 * j + 7])));
       }
+      return true;
+    };
+    float l2_next = 0.f;
+    if (wg == 0 && wk.ntiles > 0) {
+      const float l2_0 = load_l2(0);
+      l2_next = load_l2(1);
+      ok = put_extra(0, l2_0);
     }
+    for (int64_t i = 0; ok && i < wk.ntiles; i++) {
+      if (wg == 0 && i + 1 < wk.ntiles) {
+        const float l2 = l2_next;
+        l2_next = load_l2(i + 2);
+        if (!(ok = put_extra(i + 1, l2))) break;
+      }
+      for (int c = 0; c < nch; c++, q++) {
+        const int bb = (int)(q % kSBuf);
+        if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
+        tc_fence_after();
+        const uint32_t tS = tmem + lane_addr + (uint32_t)bb * GC + (uint32_t)wg * 64;
+        uint32_t v0[32], v1[32];
+        tmem_ld32(tS, v0);
+        tmem_ld32(tS + 32, v1);
+        tmem_wait_ld2(v0, v1);
+        uint32_t pk0[16], pk1[16];
+#pragma unroll
+        for (int j = 0; j < 16; j++) {
+          pk0[j] = pack_bf16(ex2(__uint_as_float(v0[2 * j])), ex2(__uint_as_float(v0[2 * j + 1])));
+          pk1[j] = pack_bf16(ex2(__uint_as_float(v1[2 * j])), ex2(__uint_as_float(v1[2 * j + 1])));
+        }
+        tmem_st16(tS, pk0);
+        tmem_st16(tS + 16, pk1);
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_ready[bb]);
+        // The output of the previous tile is drained after this tile's first chunk,
+        // when its last P x Z' MMA has long finished.
+        if (c == 0 && i > 0 && !(ok = epilogue(i - 1))) break;
+      }
+    }
+    if (ok && wk.ntiles > 0) epilogue(wk.ntiles - 1);
   }
   tc_fence_before();
   __syncthreads();
@@ -364,25 +401,31 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // =========================================================================================
 // Statistics: lse_n = log sum_g exp(a_ng)  (natural log), written to lse[bh*N + n].
-// Same logits pipeline as the deslice with A extra = [1, 1, 0, 0].
+// Same logits pipeline as the deslice with A extra = [1, 1, 0, 0].  Each
+// softmax warpgroup keeps a running (max, sum) over its half of every chunk;
+// the halves are combined through shared memory at the end of a tile.
 // =========================================================================================
 template <int GC>
 __global__ void __launch_bounds__(kThreads, 1)
     k_stats(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ wimg, float* __restrict__ lse,
             int64_t N, int H, int G, int splits, uint32_t* status) {
+  static_assert(GC == 128, "chunk width");
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t wbytes = (uint32_t)G * 96;
   uint8_t* s_w = smem;
   uint8_t* s_x = s_w + wbytes;
   uint8_t* s_xe = s_x + kStages * kXBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_xe + kStages * kXeBytes);
+  float2* s_ml = reinterpret_cast<float2*>(s_xe + kStages * kXeBytes);  // [2][128] warpgroup-1 partials
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_ml + 2 * kTile);
   uint64_t* w_full = bars;
   uint64_t* x_full = bars + 1;
   uint64_t* x_empty = x_full + kStages;
   uint64_t* s_full = x_empty + kStages;
   uint64_t* s_free = s_full + 2;
-  uint64_t* drain = s_free + 2;
+  uint64_t* ml_full = s_free + 2;   // warpgroup 1 partials written   (per tile parity)
+  uint64_t* ml_empty = ml_full + 2; // warpgroup 0 has read them
+  uint64_t* drain = ml_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
 
@@ -400,7 +443,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; i++) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_free[i], 4);
+      mbar_init(&s_free[i], 8);
+      mbar_init(&ml_full[i], 4);
+      mbar_init(&ml_empty[i], 4);
     }
     mbar_init(drain, 1);
     ab->flag = 0;
@@ -455,7 +500,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait(drain, 0, ab, nullptr, 2000000000ull);
     }
   } else if (warp >= kSoftmaxWarp0) {
-    const int wq = warp - kSoftmaxWarp0;
+    const int wg = (warp - kSoftmaxWarp0) >> 2;
+    const int wq = warp & 3;
     const int r = wq * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     int64_t q = 0;
@@ -466,30 +512,54 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int c = 0; c < nch; c++, q++) {
         if (!(ok = mbar_wait(&s_full[q & 1], (uint32_t)((q >> 1) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t tS = tmem + lane_addr + (uint32_t)(q & 1) * GC;
-#pragma unroll 1
-        for (int part = 0; part < GC / 32; part++) {
-          uint32_t v[32];
-          tmem_ld32(tS + part * 32, v);
-          tmem_wait_ld(v);
-          if (part == GC / 32 - 1) {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s_free[q & 1]);
-          }
-          float cm = __uint_as_float(v[0]);
+        const uint32_t tS = tmem + lane_addr + (uint32_t)(q & 1) * GC + (uint32_t)wg * (GC / 2);
+        uint32_t v0[32], v1[32];
+        tmem_ld32(tS, v0);
+        tmem_ld32(tS + 32, v1);
+        tmem_wait_ld2(v0, v1);
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&s_free[q & 1]);
+        // Chunk maximum as a tree of three-input maxima (short dependency chains).
+        float t[22];
 #pragma unroll
-          for (int j = 1; j < 32; j++) cm = fmaxf(cm, __uint_as_float(v[j]));
-          const float mn = fmaxf(m, cm);
-          float acc = 0.f;
-#pragma unroll
-          for (int j = 0; j < 32; j++) acc += ex2(__uint_as_float(v[j]) - mn);
-          l = l * ex2(m - mn) + acc;
-          m = mn;
+        for (int j = 0; j < 10; j++) {
+          t[j] = max3(__uint_as_float(v0[3 * j]), __uint_as_float(v0[3 * j + 1]), __uint_as_float(v0[3 * j + 2]));
+          t[10 + j] = max3(__uint_as_float(v1[3 * j]), __uint_as_float(v1[3 * j + 1]), __uint_as_float(v1[3 * j + 2]));
         }
+        t[20] = max3(__uint_as_float(v0[30]), __uint_as_float(v0[31]), __uint_as_float(v1[30]));
+        t[21] = fmaxf(__uint_as_float(v1[31]), m);
+#pragma unroll
+        for (int j = 0; j < 7; j++) t[j] = max3(t[3 * j], t[3 * j + 1], t[3 * j + 2]);
+        const float mn = max3(max3(t[0], t[1], t[2]), max3(t[3], t[4], t[5]), fmaxf(t[6], t[21]));
+        float acc[8];
+#pragma unroll
+        for (int j = 0; j < 8; j++) acc[j] = 0.f;
+#pragma unroll
+        for (int j = 0; j < 32; j++) {
+          acc[j & 7] += ex2(__uint_as_float(v0[j]) - mn);
+          acc[(j + 4) & 7] += ex2(__uint_as_float(v1[j]) - mn);
+        }
+        const float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+        l = l * ex2(m - mn) + sum;
+        m = mn;
       }
       if (!ok) break;
-      if (n < N) lse[wk.bh * N + n] = (m + log2f(l)) * kLn2;
+      const int pb = (int)(i & 1);
+      if (wg == 1) {
+        if (i >= 2 && !(ok = mbar_wait(&ml_empty[pb], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
+        s_ml[pb * kTile + r] = make_float2(m, l);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&ml_full[pb]);
+      } else {
+        if (!(ok = mbar_wait(&ml_full[pb], (uint32_t)((i >> 1) & 1), ab, status))) break;
+        const float2 o = s_ml[pb * kTile + r];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&ml_empty[pb]);
+        const float M = fmaxf(m, o.x);
+        const float L = l * ex2(m - M) + o.y * ex2(o.x - M);
+        if (n < N) lse[wk.bh * N + n] = (M + log2f(L)) * kLn2;
+      }
     }
   }
   tc_fence_before();
@@ -505,6 +575,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Writes part[p][bh][g][0..32] = (U_g, S_g).
 // smem: [W img of the range, up to 512*96][stages: x | xe | F_lo F_hi ones][E buffers 2 x 32 KB][bars]
 // TMEM: S buffers [0, 256), accumulators [256 + 48 j, ...) for M-tile j.
+// Warpgroup wg writes the E rows of slots [64 wg, 64 wg + 64) of every chunk.
 // =========================================================================================
 constexpr uint32_t kStageBytes = kXBytes + kXeBytes + 3 * kFBlock;  // 8 + 4 + 12 KB
 constexpr uint32_t kEBytes = 128 * kTile * 2;                       // 128 slots x 128 points bf16
@@ -554,8 +625,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; i++) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_free[i], 4);
-      mbar_init(&e_ready[i], 4);
+      mbar_init(&s_free[i], 8);
+      mbar_init(&e_ready[i], 8);
       mbar_init(&e_free[i], 1);
     }
     mbar_init(acc_full, 1);
@@ -649,15 +720,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_wait(drain, 0, ab, nullptr, 2000000000ull);
     }
   } else if (warp >= kSoftmaxWarp0) {
-    const int wq = warp - kSoftmaxWarp0;
+    const int wg = (warp - kSoftmaxWarp0) >> 2;
+    const int wq = warp & 3;
     const int r = wq * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     int64_t q = 0;
     bool ok = true;
-    auto put_extra = [&](int64_t j) -> bool {
-      const int s = (int)(j % kSliceStages);
+    auto load_l2 = [&](int64_t j) -> float {
       const int64_t nn = (wk.tile0 + j) * kTile + r;
-      const float l2 = nn < N ? lse[wk.bh * N + nn] * kLog2e : 0.f;
+      return (j < wk.ntiles && nn < N) ? lse[wk.bh * N + nn] * kLog2e : 0.f;
+    };
+    auto put_extra = [&](int64_t j, float l2) -> bool {
+      const int s = (int)(j % kSliceStages);
       if (j >= kSliceStages && !mbar_wait(&st_empty[s], (uint32_t)(((j / kSliceStages) - 1) & 1), ab, status))
         return false;
       write_a_extra(s_st + s * kStageBytes + kXBytes, r, l2);
@@ -666,70 +740,80 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(&xe_ready[s]);
       return true;
     };
-    if (wk.ntiles > 0) ok = put_extra(0);
+    float l2_next = 0.f;
+    if (wg == 0 && wk.ntiles > 0) {
+      const float l2_0 = load_l2(0);
+      l2_next = load_l2(1);
+      ok = put_extra(0, l2_0);
+    }
     for (int64_t i = 0; ok && i < wk.ntiles; i++) {
       const int64_t n = (wk.tile0 + i) * kTile + r;
       const bool valid = n < N;
-      if (i + 1 < wk.ntiles && !(ok = put_extra(i + 1))) break;
+      if (wg == 0 && i + 1 < wk.ntiles) {
+        const float l2 = l2_next;
+        l2_next = load_l2(i + 2);
+        if (!(ok = put_extra(i + 1, l2))) break;
+      }
       for (int c = 0; c < NCH; c++, q++) {
         if (!(ok = mbar_wait(&s_full[q & 1], (uint32_t)((q >> 1) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t tS = tmem + lane_addr + (uint32_t)(q & 1) * GC;
-        uint32_t v[128];
-#pragma unroll
-        for (int part = 0; part < 4; part++) {
-          uint32_t t[32];
-          tmem_ld32(tS + part * 32, t);
-          tmem_wait_ld(t);
-#pragma unroll
-          for (int j = 0; j < 32; j++) v[part * 32 + j] = t[j];
-        }
+        const uint32_t tS = tmem + lane_addr + (uint32_t)(q & 1) * GC + (uint32_t)wg * 64;
+        uint32_t v0[32], v1[32];
+        tmem_ld32(tS, v0);
+        tmem_ld32(tS + 32, v1);
+        tmem_wait_ld2(v0, v1);
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&s_free[q & 1]);
         // w = 2^(a2 - lse2); padded points contribute nothing.
-        uint32_t pk[64];
-#pragma unroll
-        for (int j = 0; j < 64; j++) {
-          const float e0 = valid ? ex2(__uint_as_float(v[2 * j])) : 0.f;
-          const float e1 = valid ? ex2(__uint_as_float(v[2 * j + 1])) : 0.f;
-          pk[j] = pack_bf16(e0, e1);
-        }
-        if (q >= 2 && !(ok = mbar_wait(&e_free[q & 1], (uint32_t)(((q >> 1) - 1) & 1), ab, status))) break;
-        // E[r][g] for g in [0,128): MN-major, m-block g/64 at 16 KB, k-group r/8 at 1 KB.
-        const uint32_t eb = smem_u32(s_e + (q & 1) * kEBytes) + (uint32_t)((r >> 3) * 1024 + (r & 7) * 128);
+        uint32_t pk[32];
 #pragma unroll
         for (int j = 0; j < 16; j++) {
-          const uint32_t mb = (uint32_t)(j >> 3), ch = (uint32_t)(j & 7);
-          st_shared_v4(eb + mb * 16384 + ((ch ^ (uint32_t)(r & 7)) << 4), pk[4 * j], pk[4 * j + 1], pk[4 * j + 2],
-                       pk[4 * j + 3]);
+          pk[j] = valid ? pack_bf16(ex2(__uint_as_float(v0[2 * j])), ex2(__uint_as_float(v0[2 * j + 1]))) : 0u;
+          pk[16 + j] = valid ? pack_bf16(ex2(__uint_as_float(v1[2 * j])), ex2(__uint_as_float(v1[2 * j + 1]))) : 0u;
         }
+        if (q >= 2 && !(ok = mbar_wait(&e_free[q & 1], (uint32_t)(((q >> 1) - 1) & 1), ab, status))) break;
+        // E[r][g], g in this warpgroup's 64 slots: MN-major m-block wg (16 KB apart), k-group r/8.
+        const uint32_t eb = smem_u32(s_e + (q & 1) * kEBytes) + (uint32_t)wg * 16384 +
+                            (uint32_t)((r >> 3) * 1024 + (r & 7) * 128);
+#pragma unroll
+        for (int j = 0; j < 8; j++)
+          st_shared_v4(eb + (((uint32_t)j ^ (uint32_t)(r & 7)) << 4), pk[4 * j], pk[4 * j + 1], pk[4 * j + 2],
+                       pk[4 * j + 3]);
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(&e_ready[q & 1]);
       }
     }
-    // Epilogue: the accumulators of this CTA's slot range -> partials.
+    // Epilogue: the accumulators of this CTA's slot range -> partials
+    // (warpgroup 0 the numerators U, warpgroup 1 the weight sums S).
+    const int64_t BH = gridDim.y;
     if (ok && wk.ntiles > 0 && mbar_wait(acc_full, 0, ab, status)) {
       tc_fence_after();
-      const int64_t BH = gridDim.y;
       for (int j = 0; j < NCH; j++) {
-        uint32_t u[32], sv[16];
-        tmem_ld32(tmem + lane_addr + 256 + j * 48, u);
-        tmem_ld16(tmem + lane_addr + 256 + j * 48 + 32, sv);
-        tmem_wait_ld(u, sv);
         const int g = g_base + j * GC + r;
         float* o = part + (((int64_t)blockIdx.x * BH + wk.bh) * G + g) * (kD + 1);
+        if (wg == 0) {
+          uint32_t u[32];
+          tmem_ld32(tmem + lane_addr + 256 + j * 48, u);
+          tmem_wait_ld(u);
 #pragma unroll
-        for (int k = 0; k < kD; k++) o[k] = __uint_as_float(u[k]);
-        o[kD] = __uint_as_float(sv[0]);
+          for (int k = 0; k < kD; k++) o[k] = __uint_as_float(u[k]);
+        } else {
+          uint32_t sv[16];
+          tmem_ld16(tmem + lane_addr + 256 + j * 48 + 32, sv);
+          tmem_wait_ld(sv);
+          o[kD] = __uint_as_float(sv[0]);
+        }
       }
     } else if (ok && wk.ntiles == 0) {
-      const int64_t BH = gridDim.y;
       for (int j = 0; j < NCH; j++) {
         const int g = g_base + j * GC + r;
         float* o = part + (((int64_t)blockIdx.x * BH + wk.bh) * G + g) * (kD + 1);
-        for (int k = 0; k <= kD; k++) o[k] = 0.f;
+        if (wg == 0)
+          for (int k = 0; k < kD; k++) o[k] = 0.f;
+        else
+          o[kD] = 0.f;
       }
     }
   }
@@ -789,7 +873,7 @@ int slice_ranges(const Shape& s) {
 int slice_splits(const Shape& s) { return point_splits(s, (int)(s.BH() * slice_ranges(s))); }
 
 size_t smem_deslice(int G) { return 1024 + (size_t)G * 160 + kStages * (kXBytes + kXeBytes) + 256; }
-size_t smem_stats(int G) { return 1024 + (size_t)G * 96 + kStages * (kXBytes + kXeBytes) + 256; }
+size_t smem_stats(int G) { return 1024 + (size_t)G * 96 + kStages * (kXBytes + kXeBytes) + 2 * kTile * 8 + 256; }
 size_t smem_slice() { return 1024 + (size_t)kSliceRange * 96 + kSliceStages * kStageBytes + 2 * kEBytes + 256; }
 
 template <typename K>
