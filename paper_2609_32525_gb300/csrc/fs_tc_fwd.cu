@@ -7,31 +7,40 @@
 //   k_deslice : per point, out_n = sum_g w_ng z'_g                      (point-owned)
 // w is recomputed tile by tile in every pass and never leaves the SM.
 //
-// Every pass forms the logits of a 128-point tile against a chunk of GC slots
-// with one tcgen05.mma chain (M = 128 points, N = GC slots, K = 48):
-//   A = [ x (32 bf16) | 1, 1, -lse_hi, -lse_lo, 0.. ]     (per point)
-//   B = [ W*log2e/tau (32) | beta'_hi, beta'_lo, 1, 1, 0.. ]  (per slot)
-// so the accumulator already holds a2 - lse2 = log2 of the slice weight (the
-// bias and the normaliser ride on the tensor core; lse2 and beta' are split
-// into two bf16 halves to keep them near fp32 accurate).  The stats pass uses
-// A = [x | 1, 1, 0, 0] and keeps a running max / sum in registers.
+// Logits.  A 128-point x 128-slot block of base-2 logits a2 = a * log2(e) is one
+// tcgen05.mma chain with K = 48:
+//   point side [ x (32 bf16) | 1, 1, 0 ... ]            (the last block constant)
+//   slot side  [ W*log2e/tau (32) | b'_hi, b'_lo, 0 ... ]  (b' = bias*log2e/tau in
+//                                                           two bf16 halves)
+// The point-major passes (stats, deslice) put points on the MMA's M (TMEM lane
+// = point); the slice swaps the operands, so its TMEM lane is a slot and its
+// column a point.  The normaliser lse2 is subtracted in registers (packed
+// f32x2 adds) and never written into an MMA operand: no thread writes a
+// tensor-core operand per tile (that costs a generic -> async proxy fence).
 //
-// CTA layout (384 threads): warp 0 issues TMA / bulk copies, warp 1 owns the
-// TMEM allocation and issues every tcgen05.mma from one lane, warps 4..11 form
-// two softmax warpgroups that split the columns of every chunk: thread r of a
-// warpgroup owns TMEM lane r = point r of the tile (tcgen05.ld 32x32b), so
-// every SM sub-partition runs two softmax warps.  Warps 2, 3 idle.  All waits are bounded (2 s): a wait
-// that gives up flags FS_ERR_TIMEOUT in the status word and the CTA drains its
-// in-flight copies and MMAs, frees TMEM and exits.
+// Products.  The bf16 weights are written back into the S buffer they came
+// from and feed the second MMA as its TMEM A operand: P x Z' in the deslice
+// (M = points, K = slots, N = 32 channels), E x [F | 1] in the slice (M =
+// slots, K = points, N = 48: 32 channels and a ones column for the weight sums).
+//
+// Issue.  A tcgen05.mma from one thread takes ~130 cycles before the thread can
+// issue the next, whatever N; separate warps overlap.  Warp 1 issues the logits
+// (stats: warps 1 and 2), warps 2 and 3 each issue half of every block's K-steps
+// of the product into an accumulator of their own; the two are summed in a
+// fixed order, so the result is deterministic.
+//
+// CTA (384 threads): warp 0 TMA producer, warps 1..3 MMA issuers, warps 4..11
+// two softmax warpgroups that split the columns of every block; a thread owns
+// one TMEM lane (tcgen05.ld/st 32x32b).  Every wait is bounded (2 s): a wait
+// that gives up writes FS_ERR_TIMEOUT to the status word, the CTA drains its
+// copies and MMAs, frees TMEM and exits.
 //
 // Shared-memory operand layouts (all bases 1024-byte aligned):
-//   x tile      K-major, 64 B rows, 64B swizzle (TMA)          128 x 32
-//   A extra     K-major, 32 B rows, 32B swizzle (threads)      128 x 16
-//   W' chunk    K-major, 64 B rows, 64B swizzle (prep image)    GC x 32
-//   B extra     K-major, 32 B rows, 32B swizzle (prep image)    GC x 16
-//   Z' (deslice B)  K-major rows = channels, 128 B rows, 128B swizzle
-//   E (slice A)     MN-major (slots contiguous), 128B swizzle
-//   [F | 1] (slice B)  MN-major, three 16-channel blocks, 32B swizzle (TMA)
+//   x tile          K-major, 64 B rows, 64B swizzle (TMA)        128 points x 32
+//   constant extra  K-major, 32 B rows, 32B swizzle              128 rows x 16
+//   W image         K-major, 64 B rows, 64B swizzle, then its 32 B extra rows
+//   Z' image        K-major rows = channels, 128 B rows, 128B swizzle
+//   [F | 1]         MN-major, three 16-channel blocks, 32B swizzle (TMA)
 #include "fs_tc.h"
 #include "fs_tc_ptx.cuh"
 
@@ -46,18 +55,21 @@ using namespace tc;
 
 constexpr int kThreads = 384;
 constexpr int kTile = 128;        // points per tile
+constexpr int kGC = 128;          // slots per logits block
 constexpr int kD = 32;            // head width of the tensor-core path
 constexpr int kSoftmaxWarp0 = 4;  // warps 4..11: two softmax warpgroups
 constexpr int kStages = 3;        // x-tile pipeline depth (stats / deslice)
-constexpr int kSliceStages = 3;   // slice pipeline depth
-constexpr uint32_t kXBytes = kTile * 64;    // 128 points x 32 bf16
-constexpr uint32_t kXeBytes = kTile * 32;   // 128 points x 16 bf16
-constexpr uint32_t kFBlock = kTile * 32;    // 128 points x 16 channels
-constexpr int kSliceRange = 512;            // slots per slice CTA at most
+constexpr int kSliceStages = 5;   // slice pipeline depth
+constexpr int kSBuf = 3;          // S buffers (logits run up to two blocks ahead)
+constexpr uint32_t kXBytes = kTile * 64;   // 128 points x 32 bf16
+constexpr uint32_t kExBytes = kTile * 32;  // 128 rows x 16 bf16
+constexpr uint32_t kFBlock = kTile * 32;   // 128 points x 16 channels
+constexpr uint32_t kLseBytes = kTile * 4;  // 128 fp32
+constexpr uint64_t kWaitNs = 2000000000ull;
 
-// ---- operand images written by the prep kernel -------------------------------------------
+// ---- operand images written by the prep kernels -------------------------------------------
 // W image for head h: G rows (slots) x 64 B of W*log2e/tau (64B swizzle), then
-// G rows x 32 B of [beta'_hi, beta'_lo, 1, 1, 0...] (32B swizzle).
+// G rows x 32 B of [b'_hi, b'_lo, 0...] (32B swizzle).
 __device__ __forceinline__ uint32_t off_sw64(int row, int k) {  // k in [0, 32)
   const int chunk = k >> 3;
   return (uint32_t)((row >> 3) * 512 + (row & 7) * 64 + ((chunk ^ ((row & 7) >> 1)) << 4) + (k & 7) * 2);
@@ -80,7 +92,7 @@ __global__ void k_prep_w(const float* __restrict__ W, const float* __restrict__ 
   const int h = (int)(i / G), g = (int)(i % G);
   const float t = tau[h];
   if (!(t > 0.f && t < INFINITY)) {
-    atomicCAS(status, 0u, 5u);
+    atomicCAS(status, 0u, (uint32_t)FS_ERR_BAD_TAU);
     return;
   }
   const float scale = kLog2e / t;
@@ -92,14 +104,7 @@ __global__ void k_prep_w(const float* __restrict__ W, const float* __restrict__ 
   const float b2 = bias[(int64_t)h * G + g] * scale;
   const __nv_bfloat16 hi = __float2bfloat16_rn(b2);
   const __nv_bfloat16 lo = __float2bfloat16_rn(b2 - __bfloat162float(hi));
-  const __nv_bfloat16 one = __float2bfloat16_rn(1.f), zero = __float2bfloat16_rn(0.f);
-  for (int k = 0; k < 16; k++) {
-    __nv_bfloat16 v = zero;
-    if (k == 0) v = hi;
-    else if (k == 1) v = lo;
-    else if (k == 2 || k == 3) v = one;
-    ep[off_sw32(g, k) / 2] = v;
-  }
+  for (int k = 0; k < 16; k++) ep[off_sw32(g, k) / 2] = k == 0 ? hi : (k == 1 ? lo : __float2bfloat16_rn(0.f));
 }
 
 __global__ void k_prep_z(const float* __restrict__ zp, uint8_t* __restrict__ img, int64_t BH, int G) {
@@ -113,7 +118,7 @@ __global__ void k_prep_z(const float* __restrict__ zp, uint8_t* __restrict__ img
   out[off_z(c, g) / 2] = __float2bfloat16_rn(zp[i]);
 }
 
-// ---- shared pieces of the three streaming kernels ----------------------------------------------
+// ---- shared pieces -------------------------------------------------------------------------
 struct Work {
   int64_t bh;      // batch * H + head
   int64_t tile0;   // first point tile of this CTA
@@ -131,34 +136,38 @@ __device__ __forceinline__ Work work_of(int64_t N, int splits) {
   return w;
 }
 
-// Row r of the per-tile A extra block: [1, 1, -l_hi, -l_lo, 0 x 12] (32B swizzle).
-__device__ __forceinline__ void write_a_extra(uint8_t* xe, int r, float l2) {
-  const __nv_bfloat16 hi = __float2bfloat16_rn(l2);
-  const __nv_bfloat16 lo = __float2bfloat16_rn(l2 - __bfloat162float(hi));
-  const uint32_t one = 0x3F80u;
-  const uint32_t w0 = one | (one << 16);
-  const uint32_t nhi = (uint32_t)__bfloat16_as_ushort(__hneg(hi));
-  const uint32_t nlo = (uint32_t)__bfloat16_as_ushort(__hneg(lo));
-  const uint32_t w1 = nhi | (nlo << 16);
-  const uint32_t base = smem_u32(xe) + (uint32_t)((r >> 3) * 256 + (r & 7) * 32);
-  const uint32_t sw = (uint32_t)((r & 7) >> 2);
-  st_shared_v4(base + ((0u ^ sw) << 4), w0, w1, 0u, 0u);
-  st_shared_v4(base + ((1u ^ sw) << 4), 0u, 0u, 0u, 0u);
+// The constant point-side extra block: every row [1, 1, 0 x 14] (32B swizzle).
+__device__ __forceinline__ void write_const_extra(uint8_t* ex) {
+  for (int r = threadIdx.x; r < kTile; r += blockDim.x) {
+    const uint32_t base = smem_u32(ex) + (uint32_t)((r >> 3) * 256 + (r & 7) * 32);
+    const uint32_t sw = (uint32_t)((r & 7) >> 2);
+    st_shared_v4(base + ((0u ^ sw) << 4), 0x3F803F80u, 0u, 0u, 0u);
+    st_shared_v4(base + ((1u ^ sw) << 4), 0u, 0u, 0u, 0u);
+  }
 }
 
-// Issues the K = 48 logits MMA chain for chunk `c` into TMEM column `d_col`.
-template <int GC>
-__device__ __forceinline__ void issue_logits(uint32_t tmem_d, uint32_t x_s, uint32_t xe_s, uint32_t w_img,
-                                             uint32_t we_img, int c) {
-  constexpr uint32_t idesc = idesc_bf16(128, GC, false, false);
-  const uint32_t wc = w_img + (uint32_t)c * GC * 64;
-  const uint32_t wec = we_img + (uint32_t)c * GC * 32;
-  mma_ss(tmem_d, sdesc(x_s, 16, 512, kSw64), sdesc(wc, 16, 512, kSw64), idesc, 0);
-  mma_ss(tmem_d, sdesc(x_s + 32, 16, 512, kSw64), sdesc(wc + 32, 16, 512, kSw64), idesc, 1);
-  mma_ss(tmem_d, sdesc(xe_s, 16, 256, kSw32), sdesc(wec, 16, 256, kSw32), idesc, 1);
+// Base-2 logits of 128 points x 128 slots (chunk c of the W image) into TMEM.
+//   point_major: A = points (x tile), B = slots (W);  else A = slots, B = points.
+__device__ __forceinline__ void issue_logits(uint32_t tmem_d, uint32_t x_s, uint32_t ex_s, uint32_t w_img,
+                                             uint32_t we_img, int c, bool point_major) {
+  constexpr uint32_t idesc = idesc_bf16(128, kGC, false, false);
+  const uint32_t wc = w_img + (uint32_t)c * kGC * 64;
+  const uint32_t wec = we_img + (uint32_t)c * kGC * 32;
+  const uint64_t x0 = sdesc(x_s, 16, 512, kSw64), x1 = sdesc(x_s + 32, 16, 512, kSw64);
+  const uint64_t w0 = sdesc(wc, 16, 512, kSw64), w1 = sdesc(wc + 32, 16, 512, kSw64);
+  const uint64_t xe = sdesc(ex_s, 16, 256, kSw32), we = sdesc(wec, 16, 256, kSw32);
+  if (point_major) {
+    mma_ss(tmem_d, x0, w0, idesc, 0);
+    mma_ss(tmem_d, x1, w1, idesc, 1);
+    mma_ss(tmem_d, xe, we, idesc, 1);
+  } else {
+    mma_ss(tmem_d, w0, x0, idesc, 0);
+    mma_ss(tmem_d, w1, x1, idesc, 1);
+    mma_ss(tmem_d, we, xe, idesc, 1);
+  }
 }
 
-// Producer-side loads of one W image (and optionally a Z' image) into smem.
+// Producer-side bulk loads of an image into smem (pieces of at most 32 KB).
 __device__ __forceinline__ void load_images(uint8_t* dst, const uint8_t* src, uint32_t bytes, uint64_t* bar) {
   constexpr uint32_t kPiece = 32768;
   for (uint32_t off = 0; off < bytes; off += kPiece) {
@@ -167,69 +176,80 @@ __device__ __forceinline__ void load_images(uint8_t* dst, const uint8_t* src, ui
   }
 }
 
+// 2^(v + d) for 64 logits (d = -lse2, packed pairs) -> 32 bf16x2 words.
+__device__ __forceinline__ void weights64(const uint32_t (&v0)[32], const uint32_t (&v1)[32], const uint64_t (&d)[32],
+                                          uint32_t (&p0)[16], uint32_t (&p1)[16]) {
+#pragma unroll
+  for (int k = 0; k < 16; k++) {
+    const uint64_t a = add2(pack2(v0[2 * k], v0[2 * k + 1]), d[k]);
+    const uint64_t b = add2(pack2(v1[2 * k], v1[2 * k + 1]), d[16 + k]);
+    p0[k] = pack_bf16(ex2(lo_f(a)), ex2(hi_f(a)));
+    p1[k] = pack_bf16(ex2(lo_f(b)), ex2(hi_f(b)));
+  }
+}
+
 // =========================================================================================
 // Deslice: out_n = sum_g w_ng z'_g.
-// smem: [W img G*96][Z' img G*64][x stages][xe stages][barriers]
-// TMEM: three S buffers [0, 3*GC), O buffers [3*GC, 3*GC + 64).  The logits run
-// two chunks ahead of the softmax.  The two softmax warpgroups split every
-// chunk's columns: warpgroup wg reads S columns [64 wg, 64 wg + 64) and writes
-// their bf16 weights back, packed in pairs, into columns [64 wg, 64 wg + 32) of
-// the same buffer, which the P x Z' MMA reads as its A operand.
+// smem: [W img G*96][Z' img G*64][x stages][constant extra][barriers]
+// TMEM: S buffers [0, 384); P x Z' accumulators O_0 [384, 448), O_1 [448, 512),
+// each double-buffered by tile parity.  Softmax warpgroup wg reads S columns
+// [64 wg, 64 wg + 64) and writes their bf16 weights, packed in pairs, into
+// columns [64 wg, 64 wg + 32) of the same buffer; warp 2 + wg turns exactly
+// those into its products (K-steps [4 wg, 4 wg + 4) of the block).
 // =========================================================================================
-constexpr int kSBuf = 3;
-
-template <int GC>
 __global__ void __launch_bounds__(kThreads, 1)
     k_deslice(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ wimg,
               const uint8_t* __restrict__ zimg, const float* __restrict__ lse, __nv_bfloat16* __restrict__ out,
               int64_t N, int H, int G, int splits, uint32_t* status) {
-  static_assert(GC == 128, "chunk width");
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t wbytes = (uint32_t)G * 96, zbytes = (uint32_t)G * 64;
   uint8_t* s_w = smem;
   uint8_t* s_z = s_w + wbytes;
   uint8_t* s_x = s_z + zbytes;
-  uint8_t* s_xe = s_x + kStages * kXBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_xe + kStages * kXeBytes);
+  uint8_t* s_ex = s_x + kStages * kXBytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_ex + kExBytes);
   uint64_t* wz_full = bars;
   uint64_t* x_full = bars + 1;
   uint64_t* x_empty = x_full + kStages;
-  uint64_t* xe_ready = x_empty + kStages;
-  uint64_t* s_full = xe_ready + kStages;
+  uint64_t* s_full = x_empty + kStages;
   uint64_t* p_ready = s_full + kSBuf;
-  uint64_t* o_full = p_ready + kSBuf;
+  uint64_t* pv_done = p_ready + kSBuf;
+  uint64_t* o_full = pv_done + kSBuf;
   uint64_t* o_free = o_full + 2;
-  uint64_t* drain = o_free + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* drain = o_free + 2;  // one per issuing warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 3);
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const Work wk = work_of(N, splits);
   const int64_t b = wk.bh / H;
   const int h = (int)(wk.bh % H);
-  const int nch = G / GC;
-  constexpr uint32_t kO = kSBuf * GC;  // TMEM column base of the O buffers
+  const int nch = G / kGC;
+  constexpr uint32_t kO = kSBuf * kGC;  // TMEM column base of the O accumulators
+  const int64_t total = wk.ntiles * nch;
 
   if (threadIdx.x == 0) {
     mbar_init(wz_full, 1);
     for (int s = 0; s < kStages; s++) {
       mbar_init(&x_full[s], 1);
       mbar_init(&x_empty[s], 1);
-      mbar_init(&xe_ready[s], 4);
     }
     for (int i = 0; i < kSBuf; i++) {
       mbar_init(&s_full[i], 1);
       mbar_init(&p_ready[i], 8);
+      mbar_init(&pv_done[i], 2);
     }
     for (int i = 0; i < 2; i++) {
-      mbar_init(&o_full[i], 1);
+      mbar_init(&o_full[i], 2);
       mbar_init(&o_free[i], 8);
     }
-    mbar_init(drain, 1);
+    for (int i = 0; i < 3; i++) mbar_init(&drain[i], 1);
     ab->flag = 0;
     fence_mbar_init();
   }
+  write_const_extra(s_ex);
+  fence_proxy_async_smem();
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
   __syncthreads();
@@ -252,59 +272,59 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // Drain: the newest load of each stage has landed before the CTA exits.
       for (int64_t j = (i > kStages ? i - kStages : 0); j < i; j++)
-        mbar_wait(&x_full[j % kStages], (uint32_t)((j / kStages) & 1), ab, nullptr, 2000000000ull);
-      mbar_wait(wz_full, 0, ab, nullptr, 2000000000ull);
+        mbar_wait(&x_full[j % kStages], (uint32_t)((j / kStages) & 1), ab, nullptr, kWaitNs);
+      mbar_wait(wz_full, 0, ab, nullptr, kWaitNs);
     }
   } else if (warp == 1) {
-    // ------------------------------ MMA issuer ------------------------------
-    // One flattened sequence q = tile * nch + chunk; the logits of q+2 are issued
-    // before waiting for the softmax of q, across tile boundaries.  A buffer is
-    // rewritten only by an MMA issued after the P x Z' MMA that last read it, and
-    // tcgen05.mma executes in issue order.
+    // ------------------------------ logits issuer ------------------------------
+    // Block q uses S buffer q % 3; it is rewritten only after the products of
+    // block q - 3 (issued by the other warps) have completed.
     if (lane == 0 && wk.ntiles > 0) {
-      constexpr uint32_t idesc_pv = idesc_bf16(128, kD, false, false);
-      const uint32_t sw = smem_u32(s_w), swe = sw + (uint32_t)G * 64, sz = smem_u32(s_z);
-      const int64_t total = wk.ntiles * nch;
-      auto logits = [&](int64_t qq) -> bool {
-        const int64_t i = qq / nch;
-        const int c = (int)(qq % nch);
+      const uint32_t sw = smem_u32(s_w), swe = sw + (uint32_t)G * 64;
+      bool ok = mbar_wait(wz_full, 0, ab, status);
+      for (int64_t q = 0; ok && q < total; q++) {
+        const int64_t i = q / nch;
+        const int c = (int)(q % nch);
         const int s = (int)(i % kStages);
-        if (c == 0) {
-          const uint32_t par = (uint32_t)((i / kStages) & 1);
-          if (!mbar_wait(&x_full[s], par, ab, status) || !mbar_wait(&xe_ready[s], par, ab, status)) return false;
-          tc_fence_after();
-        }
-        const int bb = (int)(qq % kSBuf);
-        issue_logits<GC>(tmem + (uint32_t)bb * GC, smem_u32(s_x + s * kXBytes), smem_u32(s_xe + s * kXeBytes), sw,
-                         swe, c);
+        const int bb = (int)(q % kSBuf);
+        if (c == 0 && !(ok = mbar_wait(&x_full[s], (uint32_t)((i / kStages) & 1), ab, status))) break;
+        if (q >= kSBuf && !(ok = mbar_wait(&pv_done[bb], (uint32_t)(((q / kSBuf) - 1) & 1), ab, status))) break;
+        tc_fence_after();
+        issue_logits(tmem + (uint32_t)bb * kGC, smem_u32(s_x + s * kXBytes), smem_u32(s_ex), sw, swe, c, true);
         mma_commit(&s_full[bb]);
         if (c == nch - 1) mma_commit(&x_empty[s]);
-        return true;
-      };
-      bool ok = mbar_wait(wz_full, 0, ab, status) && logits(0) && (total < 2 || logits(1));
+      }
+      mma_commit(&drain[0]);
+      mbar_wait(&drain[0], 0, ab, nullptr, kWaitNs);
+    }
+  } else if (warp == 2 || warp == 3) {
+    // ------------------------------ P x Z' issuers ------------------------------
+    const int j = warp - 2;  // K-steps [4j, 4j + 4) of every block, accumulator O_j
+    if (lane == 0 && wk.ntiles > 0) {
+      constexpr uint32_t idesc_pv = idesc_bf16(128, kD, false, false);
+      const uint32_t sz = smem_u32(s_z);
+      bool ok = mbar_wait(wz_full, 0, ab, status);
       for (int64_t q = 0; ok && q < total; q++) {
         const int64_t i = q / nch;
         const int c = (int)(q % nch);
         const int ob = (int)(i & 1);
         const int bb = (int)(q % kSBuf);
-        if (q + 2 < total && !(ok = logits(q + 2))) break;
         if (c == 0 && i >= 2 && !(ok = mbar_wait(&o_free[ob], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
         if (!(ok = mbar_wait(&p_ready[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t tS = tmem + (uint32_t)bb * GC;
-        const uint32_t tO = tmem + kO + (uint32_t)ob * kD;
+        const uint32_t tP = tmem + (uint32_t)bb * kGC + (uint32_t)j * 64;
+        const uint32_t tO = tmem + kO + (uint32_t)(j * 2 + ob) * kD;
 #pragma unroll
-        for (int k = 0; k < GC / 16; k++) {
-          const int g0 = c * GC + k * 16;
+        for (int kk = 0; kk < 4; kk++) {
+          const int g0 = c * kGC + (4 * j + kk) * 16;
           const uint32_t zaddr = sz + (uint32_t)((g0 >> 6) * 4096 + (g0 & 63) * 2);
-          const uint32_t tP = tS + (uint32_t)((k >> 2) * 64 + (k & 3) * 8);
-          mma_ts(tO, tP, sdesc(zaddr, 16, 1024, kSw128), idesc_pv, (c > 0 || k > 0) ? 1u : 0u);
+          mma_ts(tO, tP + (uint32_t)kk * 8, sdesc(zaddr, 16, 1024, kSw128), idesc_pv, (c > 0 || kk > 0) ? 1u : 0u);
         }
+        mma_commit(&pv_done[bb]);
         if (c == nch - 1) mma_commit(&o_full[ob]);
       }
-      // Drain every MMA issued by this thread before TMEM is freed.
-      mma_commit(drain);
-      mbar_wait(drain, 0, ab, nullptr, 2000000000ull);
+      mma_commit(&drain[1 + j]);
+      mbar_wait(&drain[1 + j], 0, ab, nullptr, kWaitNs);
     }
   } else if (warp >= kSoftmaxWarp0) {
     // ------------------------------ softmax warpgroups ------------------------------
@@ -314,80 +334,65 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     int64_t q = 0;
     bool ok = true;
-    // lse of tile j, loaded two tiles ahead of its use.
-    auto load_l2 = [&](int64_t j) -> float {
+    // -lse2 of this thread's point in tile j, loaded two tiles ahead of its use.
+    auto load_nl2 = [&](int64_t j) -> float {
       const int64_t nn = (wk.tile0 + j) * kTile + r;
-      return (j < wk.ntiles && nn < N) ? lse[wk.bh * N + nn] * kLog2e : 0.f;
+      return (j < wk.ntiles && nn < N) ? -lse[wk.bh * N + nn] * kLog2e : 0.f;
     };
-    // The A extra block of tile j carries -lse of its points; warpgroup 0 writes
-    // it one tile ahead so the MMA warp can run the next tile's logits early.
-    auto put_extra = [&](int64_t j, float l2) -> bool {
-      const int s = (int)(j % kStages);
-      if (j >= kStages && !mbar_wait(&x_empty[s], (uint32_t)(((j / kStages) - 1) & 1), ab, status)) return false;
-      write_a_extra(s_xe + s * kXeBytes, r, l2);
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&xe_ready[s]);
-      return true;
-    };
-    // Output of tile t: this warpgroup's 16 channels of O -> bf16 -> global.
+    // Output of tile t: this warpgroup's 16 channels of O_0 + O_1 -> bf16 -> global.
     auto epilogue = [&](int64_t t) -> bool {
       const int ob = (int)(t & 1);
       if (!mbar_wait(&o_full[ob], (uint32_t)((t >> 1) & 1), ab, status)) return false;
       tc_fence_after();
-      uint32_t o[16];
-      tmem_ld16(tmem + lane_addr + kO + (uint32_t)ob * kD + (uint32_t)wg * 16, o);
-      tmem_wait_ld(o);
+      uint32_t o0[16], o1[16];
+      tmem_ld16(tmem + lane_addr + kO + (uint32_t)ob * kD + (uint32_t)wg * 16, o0);
+      tmem_ld16(tmem + lane_addr + kO + (uint32_t)(2 + ob) * kD + (uint32_t)wg * 16, o1);
+      tmem_wait_ld(o0);
+      tmem_wait_ld(o1);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&o_free[ob]);
       const int64_t n = (wk.tile0 + t) * kTile + r;
       if (n < N) {
+        float o[16];
+#pragma unroll
+        for (int k = 0; k < 16; k++) o[k] = __uint_as_float(o0[k]) + __uint_as_float(o1[k]);
         uint4* dst = reinterpret_cast<uint4*>(out + ((b * N + n) * H + h) * kD + wg * 16);
 #pragma unroll
-        for (int j = 0; j < 2; j++)
-          dst[j] = make_uint4(pack_bf16(__uint_as_float(o[8 * j]), __uint_as_float(o[8 * j + 1])),
-                              pack_bf16(__uint_as_float(o[8 * j + 2]), __uint_as_float(o[8 * j + 3])),
-                              pack_bf16(__uint_as_float(o[8 * j + 4]), __uint_as_float(o[8 * j + 5])),
-                              pack_bf16(__uint_as_float(o[8 * j + 6]), __uint_as_float(o[8 * j + 7])));
+        for (int k = 0; k < 2; k++)
+          dst[k] = make_uint4(pack_bf16(o[8 * k], o[8 * k + 1]), pack_bf16(o[8 * k + 2], o[8 * k + 3]),
+                              pack_bf16(o[8 * k + 4], o[8 * k + 5]), pack_bf16(o[8 * k + 6], o[8 * k + 7]));
       }
       return true;
     };
-    float l2_next = 0.f;
-    if (wg == 0 && wk.ntiles > 0) {
-      const float l2_0 = load_l2(0);
-      l2_next = load_l2(1);
-      ok = put_extra(0, l2_0);
-    }
+    float nl2 = load_nl2(0), nl2_next = load_nl2(1);
     for (int64_t i = 0; ok && i < wk.ntiles; i++) {
-      if (wg == 0 && i + 1 < wk.ntiles) {
-        const float l2 = l2_next;
-        l2_next = load_l2(i + 2);
-        if (!(ok = put_extra(i + 1, l2))) break;
-      }
+      const float nl2_cur = nl2;
+      nl2 = nl2_next;
+      nl2_next = load_nl2(i + 2);
+      uint64_t d[32];
+      const uint32_t nb = __float_as_uint(nl2_cur);
+#pragma unroll
+      for (int k = 0; k < 32; k++) d[k] = pack2(nb, nb);
       for (int c = 0; c < nch; c++, q++) {
         const int bb = (int)(q % kSBuf);
         if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t tS = tmem + lane_addr + (uint32_t)bb * GC + (uint32_t)wg * 64;
+        const uint32_t tS = tmem + lane_addr + (uint32_t)bb * kGC + (uint32_t)wg * 64;
         uint32_t v0[32], v1[32];
         tmem_ld32(tS, v0);
         tmem_ld32(tS + 32, v1);
         tmem_wait_ld2(v0, v1);
         uint32_t pk0[16], pk1[16];
-#pragma unroll
-        for (int j = 0; j < 16; j++) {
-          pk0[j] = pack_bf16(ex2(__uint_as_float(v0[2 * j])), ex2(__uint_as_float(v0[2 * j + 1])));
-          pk1[j] = pack_bf16(ex2(__uint_as_float(v1[2 * j])), ex2(__uint_as_float(v1[2 * j + 1])));
-        }
+        weights64(v0, v1, d, pk0, pk1);
         tmem_st16(tS, pk0);
         tmem_st16(tS + 16, pk1);
         tmem_wait_st();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&p_ready[bb]);
-        // The output of the previous tile is drained after this tile's first chunk,
-        // when its last P x Z' MMA has long finished.
+        // The output of the previous tile is drained after this tile's first block,
+        // when its last products have long finished.
         if (c == 0 && i > 0 && !(ok = epilogue(i - 1))) break;
       }
     }
@@ -400,23 +405,25 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // =========================================================================================
-// Statistics: lse_n = log sum_g exp(a_ng)  (natural log), written to lse[bh*N + n].
-// Same logits pipeline as the deslice with A extra = [1, 1, 0, 0].  Each
-// softmax warpgroup keeps a running (max, sum) over its half of every chunk;
+// Statistics: lse_n = log sum_g exp(a_ng) (natural log) to lse[bh*N + n], and
+// -lse2 = -lse*log2(e) to the padded copy nl2p[bh*Np + n] (Np = N rounded up to
+// a whole tile; padded points get -1e30 so that their weights vanish).
+// Two logits issuers (warp 1 + j issues the blocks c with c % 2 == j).  Each
+// softmax warpgroup keeps a running (max, sum) over its half of every block;
 // the halves are combined through shared memory at the end of a tile.
+// smem: [W img G*96][x stages][constant extra][ml exchange][barriers]
+// TMEM: two S buffers [0, 256).
 // =========================================================================================
-template <int GC>
 __global__ void __launch_bounds__(kThreads, 1)
     k_stats(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ wimg, float* __restrict__ lse,
-            int64_t N, int H, int G, int splits, uint32_t* status) {
-  static_assert(GC == 128, "chunk width");
+            float* __restrict__ nl2p, int64_t N, int64_t Np, int H, int G, int splits, uint32_t* status) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t wbytes = (uint32_t)G * 96;
   uint8_t* s_w = smem;
   uint8_t* s_x = s_w + wbytes;
-  uint8_t* s_xe = s_x + kStages * kXBytes;
-  float2* s_ml = reinterpret_cast<float2*>(s_xe + kStages * kXeBytes);  // [2][128] warpgroup-1 partials
+  uint8_t* s_ex = s_x + kStages * kXBytes;
+  float2* s_ml = reinterpret_cast<float2*>(s_ex + kExBytes);  // [2][128] warpgroup-1 partials
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_ml + 2 * kTile);
   uint64_t* w_full = bars;
   uint64_t* x_full = bars + 1;
@@ -425,21 +432,21 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* s_free = s_full + 2;
   uint64_t* ml_full = s_free + 2;   // warpgroup 1 partials written   (per tile parity)
   uint64_t* ml_empty = ml_full + 2; // warpgroup 0 has read them
-  uint64_t* drain = ml_empty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* drain = ml_empty + 2;   // one per issuing warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 2);
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const Work wk = work_of(N, splits);
   const int64_t b = wk.bh / H;
   const int h = (int)(wk.bh % H);
-  const int nch = G / GC;
+  const int nch = G / kGC;
 
   if (threadIdx.x == 0) {
     mbar_init(w_full, 1);
     for (int s = 0; s < kStages; s++) {
       mbar_init(&x_full[s], 1);
-      mbar_init(&x_empty[s], 1);
+      mbar_init(&x_empty[s], (uint32_t)(nch < 2 ? nch : 2));
     }
     for (int i = 0; i < 2; i++) {
       mbar_init(&s_full[i], 1);
@@ -447,13 +454,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&ml_full[i], 4);
       mbar_init(&ml_empty[i], 4);
     }
-    mbar_init(drain, 1);
+    mbar_init(&drain[0], 1);
+    mbar_init(&drain[1], 1);
     ab->flag = 0;
     fence_mbar_init();
   }
-  // The A extra block is constant here: [1, 1, 0, 0, ...] for every row and stage.
-  for (int idx = threadIdx.x; idx < kStages * kTile; idx += kThreads)
-    write_a_extra(s_xe + (idx / kTile) * kXeBytes, idx % kTile, 0.f);
+  write_const_extra(s_ex);
   fence_proxy_async_smem();
   if (warp == 1) tmem_alloc(tmem_slot, 256);
   tc_fence_before();
@@ -474,30 +480,30 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_3d(s_x + s * kXBytes, &xmap, h * kD, (int)((wk.tile0 + i) * kTile), (int)b, &x_full[s]);
       }
       for (int64_t j = (i > kStages ? i - kStages : 0); j < i; j++)
-        mbar_wait(&x_full[j % kStages], (uint32_t)((j / kStages) & 1), ab, nullptr, 2000000000ull);
-      mbar_wait(w_full, 0, ab, nullptr, 2000000000ull);
+        mbar_wait(&x_full[j % kStages], (uint32_t)((j / kStages) & 1), ab, nullptr, kWaitNs);
+      mbar_wait(w_full, 0, ab, nullptr, kWaitNs);
     }
-  } else if (warp == 1) {
-    if (lane == 0 && wk.ntiles > 0) {
+  } else if (warp == 1 || warp == 2) {
+    const int j = warp - 1;
+    if (lane == 0 && wk.ntiles > 0 && j < nch) {
       const uint32_t sw = smem_u32(s_w), swe = sw + (uint32_t)G * 64;
       bool ok = mbar_wait(w_full, 0, ab, status);
-      int64_t q = 0;
-      for (int64_t i = 0; ok && i < wk.ntiles; i++) {
+      const int c_last = ((nch - 1 - j) / 2) * 2 + j;
+      const int64_t total = wk.ntiles * nch;
+      for (int64_t q = 0; ok && q < total; q++) {
+        const int64_t i = q / nch;
+        const int c = (int)(q % nch);
+        if ((c & 1) != j) continue;
         const int s = (int)(i % kStages);
-        if (!(ok = mbar_wait(&x_full[s], (uint32_t)((i / kStages) & 1), ab, status))) break;
+        if (c == j && !(ok = mbar_wait(&x_full[s], (uint32_t)((i / kStages) & 1), ab, status))) break;
+        if (q >= 2 && !(ok = mbar_wait(&s_free[q & 1], (uint32_t)(((q >> 1) - 1) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t xs = smem_u32(s_x + s * kXBytes), xes = smem_u32(s_xe + s * kXeBytes);
-        for (int c = 0; c < nch; c++, q++) {
-          if (q >= 2 && !(ok = mbar_wait(&s_free[q & 1], (uint32_t)(((q >> 1) - 1) & 1), ab, status))) break;
-          tc_fence_after();
-          issue_logits<GC>(tmem + (uint32_t)(q & 1) * GC, xs, xes, sw, swe, c);
-          mma_commit(&s_full[q & 1]);
-        }
-        if (!ok) break;
-        mma_commit(&x_empty[s]);
+        issue_logits(tmem + (uint32_t)(q & 1) * kGC, smem_u32(s_x + s * kXBytes), smem_u32(s_ex), sw, swe, c, true);
+        mma_commit(&s_full[q & 1]);
+        if (c == c_last) mma_commit(&x_empty[s]);
       }
-      mma_commit(drain);
-      mbar_wait(drain, 0, ab, nullptr, 2000000000ull);
+      mma_commit(&drain[j]);
+      mbar_wait(&drain[j], 0, ab, nullptr, kWaitNs);
     }
   } else if (warp >= kSoftmaxWarp0) {
     const int wg = (warp - kSoftmaxWarp0) >> 2;
@@ -512,7 +518,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int c = 0; c < nch; c++, q++) {
         if (!(ok = mbar_wait(&s_full[q & 1], (uint32_t)((q >> 1) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t tS = tmem + lane_addr + (uint32_t)(q & 1) * GC + (uint32_t)wg * (GC / 2);
+        const uint32_t tS = tmem + lane_addr + (uint32_t)(q & 1) * kGC + (uint32_t)wg * (kGC / 2);
         uint32_t v0[32], v1[32];
         tmem_ld32(tS, v0);
         tmem_ld32(tS + 32, v1);
@@ -520,25 +526,29 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&s_free[q & 1]);
-        // Chunk maximum as a tree of three-input maxima (short dependency chains).
+        // Block maximum as a tree of three-input maxima (short dependency chains).
         float t[22];
 #pragma unroll
-        for (int j = 0; j < 10; j++) {
-          t[j] = max3(__uint_as_float(v0[3 * j]), __uint_as_float(v0[3 * j + 1]), __uint_as_float(v0[3 * j + 2]));
-          t[10 + j] = max3(__uint_as_float(v1[3 * j]), __uint_as_float(v1[3 * j + 1]), __uint_as_float(v1[3 * j + 2]));
+        for (int k = 0; k < 10; k++) {
+          t[k] = max3(__uint_as_float(v0[3 * k]), __uint_as_float(v0[3 * k + 1]), __uint_as_float(v0[3 * k + 2]));
+          t[10 + k] = max3(__uint_as_float(v1[3 * k]), __uint_as_float(v1[3 * k + 1]), __uint_as_float(v1[3 * k + 2]));
         }
         t[20] = max3(__uint_as_float(v0[30]), __uint_as_float(v0[31]), __uint_as_float(v1[30]));
         t[21] = fmaxf(__uint_as_float(v1[31]), m);
 #pragma unroll
-        for (int j = 0; j < 7; j++) t[j] = max3(t[3 * j], t[3 * j + 1], t[3 * j + 2]);
+        for (int k = 0; k < 7; k++) t[k] = max3(t[3 * k], t[3 * k + 1], t[3 * k + 2]);
         const float mn = max3(max3(t[0], t[1], t[2]), max3(t[3], t[4], t[5]), fmaxf(t[6], t[21]));
+        const uint32_t nmb = __float_as_uint(-mn);
+        const uint64_t nm2 = pack2(nmb, nmb);
         float acc[8];
 #pragma unroll
-        for (int j = 0; j < 8; j++) acc[j] = 0.f;
+        for (int k = 0; k < 8; k++) acc[k] = 0.f;
 #pragma unroll
-        for (int j = 0; j < 32; j++) {
-          acc[j & 7] += ex2(__uint_as_float(v0[j]) - mn);
-          acc[(j + 4) & 7] += ex2(__uint_as_float(v1[j]) - mn);
+        for (int k = 0; k < 16; k++) {
+          const uint64_t a = add2(pack2(v0[2 * k], v0[2 * k + 1]), nm2);
+          const uint64_t bq = add2(pack2(v1[2 * k], v1[2 * k + 1]), nm2);
+          acc[k & 7] += ex2(lo_f(a)) + ex2(hi_f(a));
+          acc[(k + 4) & 7] += ex2(lo_f(bq)) + ex2(hi_f(bq));
         }
         const float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
         l = l * ex2(m - mn) + sum;
@@ -558,7 +568,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(&ml_empty[pb]);
         const float M = fmaxf(m, o.x);
         const float L = l * ex2(m - M) + o.y * ex2(o.x - M);
-        if (n < N) lse[wk.bh * N + n] = (M + log2f(L)) * kLn2;
+        const float lse2 = M + log2f(L);
+        if (n < N) {
+          lse[wk.bh * N + n] = lse2 * kLn2;
+          nl2p[wk.bh * Np + n] = -lse2;
+        } else if (n < Np) {
+          nl2p[wk.bh * Np + n] = -1e30f;
+        }
       }
     }
   }
@@ -569,75 +585,74 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // =========================================================================================
-// Slice (slot-owned, split over points): the G/128 slot chunks of a head are cut
-// into `ranges` balanced ranges of at most 4 chunks; CTA (p, bh, r) owns range r
-// and point split p: U_g = sum_n w_ng f_n, S_g = sum_n w_ng with w from lse.
+// Slice (slot-owned, split over points), slot-major: CTA (p, bh, j) owns the
+// 128-slot block j of head h and point split p and computes for its slots
+//   U_g = sum_n w_ng f_n,  S_g = sum_n w_ng,  w_ng = 2^(a2_ng - lse2_n).
+// The logits are formed transposed (M = 128 slots, N = 128 points), so TMEM
+// lane = slot and column = point; -lse2 of the tile's points arrives by TMA
+// with the tile and is added per column.  The bf16 weights written back in
+// place serve directly as the TMEM A operand of U|S += E [F | 1] (K = points),
+// so the weight tile never passes through shared memory.
 // Writes part[p][bh][g][0..32] = (U_g, S_g).
-// smem: [W img of the range, up to 512*96][stages: x | xe | F_lo F_hi ones][E buffers 2 x 32 KB][bars]
-// TMEM: S buffers [0, 256), accumulators [256 + 48 j, ...) for M-tile j.
-// Warpgroup wg writes the E rows of slots [64 wg, 64 wg + 64) of every chunk.
+// smem: [W img block 128*96][stages: x | F_lo F_hi ones | -lse2][constant extra][barriers]
+// TMEM: S buffers [0, 384); U|S accumulators A_0 [384, 432), A_1 [432, 480).
+// Warp 1 issues the logits; warp 2 + wg issues the products of points
+// [64 wg, 64 wg + 64) of every tile (the columns softmax warpgroup wg wrote)
+// into its own accumulator A_wg (the two are summed in a fixed order).
 // =========================================================================================
-constexpr uint32_t kStageBytes = kXBytes + kXeBytes + 3 * kFBlock;  // 8 + 4 + 12 KB
-constexpr uint32_t kEBytes = 128 * kTile * 2;                       // 128 slots x 128 points bf16
+constexpr uint32_t kStageBytes = kXBytes + 3 * kFBlock + 1024;  // x, [F | 1], -lse2 (padded to 1 KB)
+constexpr uint32_t kWBlock = 128 * 96;                          // one 128-slot block of the W image
 
 __global__ void __launch_bounds__(kThreads, 1)
     k_slice(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap fmap,
-            const uint8_t* __restrict__ wimg, const float* __restrict__ lse, float* __restrict__ part, int64_t N,
-            int H, int G, int splits, int ranges, uint32_t* status) {
-  constexpr int GC = 128;
-  const int nchunks = G / GC;
-  const int rng = blockIdx.z;  // slot range
-  const int c_lo = rng * nchunks / ranges, c_hi = (rng + 1) * nchunks / ranges;
-  const int NCH = c_hi - c_lo;  // chunks of this CTA, 1..4
-  const int GS = NCH * GC;
-  const int g_base = c_lo * GC;
+            const __grid_constant__ CUtensorMap lmap, const uint8_t* __restrict__ wimg, float* __restrict__ part,
+            int64_t N, int H, int G, int splits, uint32_t* status) {
+  const int g_base = blockIdx.z * kGC;  // slot block
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  constexpr uint32_t wbytes = (uint32_t)kSliceRange * 96;
   uint8_t* s_w = smem;
-  uint8_t* s_st = s_w + wbytes;
-  uint8_t* s_e = s_st + kSliceStages * kStageBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_e + 2 * kEBytes);
+  uint8_t* s_st = s_w + kWBlock;
+  uint8_t* s_ex = s_st + kSliceStages * kStageBytes;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_ex + kExBytes);
   uint64_t* w_full = bars;
   uint64_t* x_full = bars + 1;
-  uint64_t* xe_ready = x_full + kSliceStages;
-  uint64_t* st_empty = xe_ready + kSliceStages;
+  uint64_t* st_empty = x_full + kSliceStages;
   uint64_t* s_full = st_empty + kSliceStages;
-  uint64_t* s_free = s_full + 2;
-  uint64_t* e_ready = s_free + 2;
-  uint64_t* e_free = e_ready + 2;
-  uint64_t* acc_full = e_free + 2;
-  uint64_t* drain = acc_full + 1;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* p_ready = s_full + kSBuf;
+  uint64_t* pv_done = p_ready + kSBuf;
+  uint64_t* acc_full = pv_done + kSBuf;
+  uint64_t* drain = acc_full + 1;  // one per issuing warp
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 3);
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const Work wk = work_of(N, splits);
   const int64_t b = wk.bh / H;
   const int h = (int)(wk.bh % H);
+  constexpr uint32_t kA = kSBuf * kGC;  // TMEM column base of the accumulators
+  constexpr uint32_t kFOff = kXBytes, kLOff = kXBytes + 3 * kFBlock;
 
   if (threadIdx.x == 0) {
     mbar_init(w_full, 1);
     for (int s = 0; s < kSliceStages; s++) {
       mbar_init(&x_full[s], 1);
-      mbar_init(&xe_ready[s], 4);
-      mbar_init(&st_empty[s], 1);
+      mbar_init(&st_empty[s], 3);  // the logits issuer and both product issuers
     }
-    for (int i = 0; i < 2; i++) {
+    for (int i = 0; i < kSBuf; i++) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_free[i], 8);
-      mbar_init(&e_ready[i], 8);
-      mbar_init(&e_free[i], 1);
+      mbar_init(&p_ready[i], 8);
+      mbar_init(&pv_done[i], 2);
     }
-    mbar_init(acc_full, 1);
-    mbar_init(drain, 1);
+    mbar_init(acc_full, 2);
+    for (int i = 0; i < 3; i++) mbar_init(&drain[i], 1);
     ab->flag = 0;
     fence_mbar_init();
   }
+  write_const_extra(s_ex);
   // Constant "ones" block of every stage: row n = [1, 0 x 15] (32B swizzle).
   for (int idx = threadIdx.x; idx < kSliceStages * kTile; idx += kThreads) {
     const int s = idx / kTile, r = idx % kTile;
-    const uint32_t base = smem_u32(s_st + s * kStageBytes + kXBytes + kXeBytes + 2 * kFBlock) +
+    const uint32_t base = smem_u32(s_st + s * kStageBytes + kFOff + 2 * kFBlock) +
                           (uint32_t)((r >> 3) * 256 + (r & 7) * 32);
     const uint32_t sw = (uint32_t)((r & 7) >> 2);
     st_shared_v4(base + ((0u ^ sw) << 4), 0x3F80u, 0u, 0u, 0u);
@@ -654,12 +669,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       prefetch_tmap(&xmap);
       prefetch_tmap(&fmap);
-      // W image rows g_base .. g_base+GS of head h: the W' part and the extra part are
-      // separate row arrays in the global image (G rows each).
-      mbar_expect_tx(w_full, (uint32_t)GS * 96);
+      prefetch_tmap(&lmap);
+      // The slot block's rows of the W image: 128 rows of W' (64 B) then 128 rows of
+      // the extra block (32 B); the global image holds G rows of each.
+      mbar_expect_tx(w_full, kWBlock);
       const uint8_t* src = wimg + (size_t)h * G * 96;
-      load_images(s_w, src + (size_t)g_base * 64, GS * 64, w_full);
-      load_images(s_w + GS * 64, src + (size_t)G * 64 + (size_t)g_base * 32, GS * 32, w_full);
+      load_images(s_w, src + (size_t)g_base * 64, kGC * 64, w_full);
+      load_images(s_w + kGC * 64, src + (size_t)G * 64 + (size_t)g_base * 32, kGC * 32, w_full);
       int64_t i = 0;
       for (; i < wk.ntiles; i++) {
         const int s = (int)(i % kSliceStages);
@@ -668,153 +684,120 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         uint8_t* st = s_st + s * kStageBytes;
         const int n0 = (int)((wk.tile0 + i) * kTile);
-        mbar_expect_tx(&x_full[s], kXBytes + 2 * kFBlock);
+        mbar_expect_tx(&x_full[s], kXBytes + 2 * kFBlock + kLseBytes);
         tma_load_3d(st, &xmap, h * kD, n0, (int)b, &x_full[s]);
-        tma_load_3d(st + kXBytes + kXeBytes, &fmap, h * kD, n0, (int)b, &x_full[s]);
-        tma_load_3d(st + kXBytes + kXeBytes + kFBlock, &fmap, h * kD + 16, n0, (int)b, &x_full[s]);
+        tma_load_3d(st + kFOff, &fmap, h * kD, n0, (int)b, &x_full[s]);
+        tma_load_3d(st + kFOff + kFBlock, &fmap, h * kD + 16, n0, (int)b, &x_full[s]);
+        tma_load_2d(st + kLOff, &lmap, n0, (int)wk.bh, &x_full[s]);
       }
       for (int64_t j = (i > kSliceStages ? i - kSliceStages : 0); j < i; j++)
-        mbar_wait(&x_full[j % kSliceStages], (uint32_t)((j / kSliceStages) & 1), ab, nullptr, 2000000000ull);
-      mbar_wait(w_full, 0, ab, nullptr, 2000000000ull);
+        mbar_wait(&x_full[j % kSliceStages], (uint32_t)((j / kSliceStages) & 1), ab, nullptr, kWaitNs);
+      mbar_wait(w_full, 0, ab, nullptr, kWaitNs);
     }
   } else if (warp == 1) {
+    // ------------------------------ logits issuer (transposed) ------------------------------
     if (lane == 0) {
-      constexpr uint32_t idesc_sl = idesc_bf16(128, 48, true, true);
-      const uint32_t sw = smem_u32(s_w), swe = sw + GS * 64;
-      const int64_t total = wk.ntiles * NCH;
-      auto logits = [&](int64_t qq) -> bool {
-        const int64_t i = qq / NCH;
-        const int c = (int)(qq % NCH);
+      const uint32_t sw = smem_u32(s_w), swe = sw + kGC * 64;
+      bool ok = mbar_wait(w_full, 0, ab, status);
+      for (int64_t i = 0; ok && i < wk.ntiles; i++) {
         const int s = (int)(i % kSliceStages);
-        if (c == 0) {
-          const uint32_t par = (uint32_t)((i / kSliceStages) & 1);
-          if (!mbar_wait(&x_full[s], par, ab, status) || !mbar_wait(&xe_ready[s], par, ab, status)) return false;
-        }
-        if (qq >= 2 && !mbar_wait(&s_free[qq & 1], (uint32_t)(((qq >> 1) - 1) & 1), ab, status)) return false;
+        const int bb = (int)(i % kSBuf);
+        if (!(ok = mbar_wait(&x_full[s], (uint32_t)((i / kSliceStages) & 1), ab, status))) break;
+        if (i >= kSBuf && !(ok = mbar_wait(&pv_done[bb], (uint32_t)(((i / kSBuf) - 1) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t st = smem_u32(s_st + s * kStageBytes);
-        issue_logits<GC>(tmem + (uint32_t)(qq & 1) * GC, st, st + kXBytes, sw, swe, c);
-        mma_commit(&s_full[qq & 1]);
-        return true;
-      };
-      bool ok = mbar_wait(w_full, 0, ab, status) && (total == 0 || logits(0));
-      for (int64_t q = 0; ok && q < total; q++) {
-        const int64_t i = q / NCH;
-        const int c = (int)(q % NCH);
+        issue_logits(tmem + (uint32_t)bb * kGC, smem_u32(s_st + s * kStageBytes), smem_u32(s_ex), sw, swe, 0, false);
+        mma_commit(&s_full[bb]);
+        mma_commit(&st_empty[s]);
+      }
+      mma_commit(&drain[0]);
+      mbar_wait(&drain[0], 0, ab, nullptr, kWaitNs);
+    }
+  } else if (warp == 2 || warp == 3) {
+    // ------------------------------ product issuers ------------------------------
+    const int j = warp - 2;  // points [64 j, 64 j + 64) of every tile, accumulator A_j
+    if (lane == 0) {
+      constexpr uint32_t idesc_sl = idesc_bf16(128, 48, false, true);
+      bool ok = true;
+      for (int64_t i = 0; ok && i < wk.ntiles; i++) {
         const int s = (int)(i % kSliceStages);
-        if (q + 1 < total && !(ok = logits(q + 1))) break;
-        if (!(ok = mbar_wait(&e_ready[q & 1], (uint32_t)((q >> 1) & 1), ab, status))) break;
+        const int bb = (int)(i % kSBuf);
+        if (!(ok = mbar_wait(&p_ready[bb], (uint32_t)((i / kSBuf) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t ebase = smem_u32(s_e + (q & 1) * kEBytes);
-        const uint32_t fs = smem_u32(s_st + s * kStageBytes) + kXBytes + kXeBytes;
-        const uint32_t tacc = tmem + 256 + (uint32_t)c * 48;
+        const uint32_t tE = tmem + (uint32_t)bb * kGC + (uint32_t)j * 64;
+        const uint32_t fs = smem_u32(s_st + s * kStageBytes) + kFOff + (uint32_t)j * 2048;
+        const uint32_t tacc = tmem + kA + (uint32_t)j * 48;
 #pragma unroll
-        for (int k = 0; k < kTile / 16; k++)
-          mma_ss(tacc, sdesc(ebase + (uint32_t)k * 2048, 16384, 1024, kSw128),
-                 sdesc(fs + (uint32_t)k * 512, kFBlock, 256, kSw32), idesc_sl, (i > 0 || k > 0) ? 1u : 0u);
-        mma_commit(&e_free[q & 1]);
-        if (c == NCH - 1) mma_commit(&st_empty[s]);
+        for (int kk = 0; kk < 4; kk++)
+          mma_ts(tacc, tE + (uint32_t)kk * 8, sdesc(fs + (uint32_t)kk * 512, kFBlock, 256, kSw32), idesc_sl,
+                 (i > 0 || kk > 0) ? 1u : 0u);
+        mma_commit(&pv_done[bb]);
+        mma_commit(&st_empty[s]);
       }
       if (ok) mma_commit(acc_full);
-      mma_commit(drain);
-      mbar_wait(drain, 0, ab, nullptr, 2000000000ull);
+      mma_commit(&drain[1 + j]);
+      mbar_wait(&drain[1 + j], 0, ab, nullptr, kWaitNs);
     }
   } else if (warp >= kSoftmaxWarp0) {
     const int wg = (warp - kSoftmaxWarp0) >> 2;
     const int wq = warp & 3;
-    const int r = wq * 32 + lane;
+    const int r = wq * 32 + lane;  // TMEM lane: slot g_base + r
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
-    int64_t q = 0;
     bool ok = true;
-    auto load_l2 = [&](int64_t j) -> float {
-      const int64_t nn = (wk.tile0 + j) * kTile + r;
-      return (j < wk.ntiles && nn < N) ? lse[wk.bh * N + nn] * kLog2e : 0.f;
-    };
-    auto put_extra = [&](int64_t j, float l2) -> bool {
-      const int s = (int)(j % kSliceStages);
-      if (j >= kSliceStages && !mbar_wait(&st_empty[s], (uint32_t)(((j / kSliceStages) - 1) & 1), ab, status))
-        return false;
-      write_a_extra(s_st + s * kStageBytes + kXBytes, r, l2);
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&xe_ready[s]);
-      return true;
-    };
-    float l2_next = 0.f;
-    if (wg == 0 && wk.ntiles > 0) {
-      const float l2_0 = load_l2(0);
-      l2_next = load_l2(1);
-      ok = put_extra(0, l2_0);
-    }
     for (int64_t i = 0; ok && i < wk.ntiles; i++) {
-      const int64_t n = (wk.tile0 + i) * kTile + r;
-      const bool valid = n < N;
-      if (wg == 0 && i + 1 < wk.ntiles) {
-        const float l2 = l2_next;
-        l2_next = load_l2(i + 2);
-        if (!(ok = put_extra(i + 1, l2))) break;
-      }
-      for (int c = 0; c < NCH; c++, q++) {
-        if (!(ok = mbar_wait(&s_full[q & 1], (uint32_t)((q >> 1) & 1), ab, status))) break;
-        tc_fence_after();
-        const uint32_t tS = tmem + lane_addr + (uint32_t)(q & 1) * GC + (uint32_t)wg * 64;
-        uint32_t v0[32], v1[32];
-        tmem_ld32(tS, v0);
-        tmem_ld32(tS + 32, v1);
-        tmem_wait_ld2(v0, v1);
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&s_free[q & 1]);
-        // w = 2^(a2 - lse2); padded points contribute nothing.
-        uint32_t pk[32];
+      const int s = (int)(i % kSliceStages);
+      const int bb = (int)(i % kSBuf);
+      // The -lse2 values come with the tile (TMA): wait for the stage, then for the logits.
+      if (!(ok = mbar_wait(&x_full[s], (uint32_t)((i / kSliceStages) & 1), ab, status))) break;
+      const float4* nl = reinterpret_cast<const float4*>(s_st + s * kStageBytes + kLOff) + wg * 16;
+      uint64_t d[32];
 #pragma unroll
-        for (int j = 0; j < 16; j++) {
-          pk[j] = valid ? pack_bf16(ex2(__uint_as_float(v0[2 * j])), ex2(__uint_as_float(v0[2 * j + 1]))) : 0u;
-          pk[16 + j] = valid ? pack_bf16(ex2(__uint_as_float(v1[2 * j])), ex2(__uint_as_float(v1[2 * j + 1]))) : 0u;
-        }
-        if (q >= 2 && !(ok = mbar_wait(&e_free[q & 1], (uint32_t)(((q >> 1) - 1) & 1), ab, status))) break;
-        // E[r][g], g in this warpgroup's 64 slots: MN-major m-block wg (16 KB apart), k-group r/8.
-        const uint32_t eb = smem_u32(s_e + (q & 1) * kEBytes) + (uint32_t)wg * 16384 +
-                            (uint32_t)((r >> 3) * 1024 + (r & 7) * 128);
-#pragma unroll
-        for (int j = 0; j < 8; j++)
-          st_shared_v4(eb + (((uint32_t)j ^ (uint32_t)(r & 7)) << 4), pk[4 * j], pk[4 * j + 1], pk[4 * j + 2],
-                       pk[4 * j + 3]);
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&e_ready[q & 1]);
+      for (int k = 0; k < 16; k++) {
+        const float4 t4 = nl[k];
+        d[2 * k] = pack2(__float_as_uint(t4.x), __float_as_uint(t4.y));
+        d[2 * k + 1] = pack2(__float_as_uint(t4.z), __float_as_uint(t4.w));
       }
+      if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((i / kSBuf) & 1), ab, status))) break;
+      tc_fence_after();
+      const uint32_t tS = tmem + lane_addr + (uint32_t)bb * kGC + (uint32_t)wg * 64;
+      uint32_t v0[32], v1[32];
+      tmem_ld32(tS, v0);
+      tmem_ld32(tS + 32, v1);
+      tmem_wait_ld2(v0, v1);
+      uint32_t pk0[16], pk1[16];
+      weights64(v0, v1, d, pk0, pk1);
+      tmem_st16(tS, pk0);
+      tmem_st16(tS + 16, pk1);
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_ready[bb]);
     }
-    // Epilogue: the accumulators of this CTA's slot range -> partials
+    // Epilogue: the accumulators of this CTA's slot block -> partials
     // (warpgroup 0 the numerators U, warpgroup 1 the weight sums S).
     const int64_t BH = gridDim.y;
+    float* o = part + (((int64_t)blockIdx.x * BH + wk.bh) * G + g_base + r) * (kD + 1);
     if (ok && wk.ntiles > 0 && mbar_wait(acc_full, 0, ab, status)) {
       tc_fence_after();
-      for (int j = 0; j < NCH; j++) {
-        const int g = g_base + j * GC + r;
-        float* o = part + (((int64_t)blockIdx.x * BH + wk.bh) * G + g) * (kD + 1);
-        if (wg == 0) {
-          uint32_t u[32];
-          tmem_ld32(tmem + lane_addr + 256 + j * 48, u);
-          tmem_wait_ld(u);
+      if (wg == 0) {
+        uint32_t u0[32], u1[32];
+        tmem_ld32(tmem + lane_addr + kA, u0);
+        tmem_ld32(tmem + lane_addr + kA + 48, u1);
+        tmem_wait_ld2(u0, u1);
 #pragma unroll
-          for (int k = 0; k < kD; k++) o[k] = __uint_as_float(u[k]);
-        } else {
-          uint32_t sv[16];
-          tmem_ld16(tmem + lane_addr + 256 + j * 48 + 32, sv);
-          tmem_wait_ld(sv);
-          o[kD] = __uint_as_float(sv[0]);
-        }
+        for (int k = 0; k < kD; k++) o[k] = __uint_as_float(u0[k]) + __uint_as_float(u1[k]);
+      } else {
+        uint32_t s0[16], s1[16];
+        tmem_ld16(tmem + lane_addr + kA + 32, s0);
+        tmem_ld16(tmem + lane_addr + kA + 48 + 32, s1);
+        tmem_wait_ld(s0);
+        tmem_wait_ld(s1);
+        o[kD] = __uint_as_float(s0[0]) + __uint_as_float(s1[0]);
       }
     } else if (ok && wk.ntiles == 0) {
-      for (int j = 0; j < NCH; j++) {
-        const int g = g_base + j * GC + r;
-        float* o = part + (((int64_t)blockIdx.x * BH + wk.bh) * G + g) * (kD + 1);
-        if (wg == 0)
-          for (int k = 0; k < kD; k++) o[k] = 0.f;
-        else
-          o[kD] = 0.f;
-      }
+      if (wg == 0)
+        for (int k = 0; k < kD; k++) o[k] = 0.f;
+      else
+        o[kD] = 0.f;
     }
   }
   tc_fence_before();
@@ -852,29 +835,50 @@ bool make_point_map(CUtensorMap* map, const void* ptr, const Shape& s, int box_c
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 2-D view of the padded [B*H, Np] fp32 -lse2 copy; box = (128 points, 1).
+bool make_lse_map(CUtensorMap* map, const float* ptr, int64_t BH, int64_t Np) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)Np, (cuuint64_t)BH};
+  cuuint64_t strides[1] = {(cuuint64_t)Np * 4};
+  cuuint32_t box[2] = {(cuuint32_t)kTile, 1};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(ptr), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 size_t w_image_bytes(const Shape& s) { return (size_t)s.H * s.G * 96; }
 size_t z_image_bytes(const Shape& s) { return (size_t)s.BH() * s.G * 64; }
+int64_t padded_n(const Shape& s) { return (s.N + kTile - 1) / kTile * kTile; }
+size_t nl2_bytes(const Shape& s) { return (size_t)s.BH() * padded_n(s) * sizeof(float); }
 
+// Point splits per work unit for one-CTA-per-SM kernels: the split count P that
+// minimises the makespan in units of one unit's work, ceil(units * P / SMs) / P
+// (whole waves of CTAs), smallest P on ties; at most one split per point tile.
 int point_splits(const Shape& s, int units) {
   const int64_t tiles = (s.N + kTile - 1) / kTile;
-  int64_t p = num_sms() / (units < 1 ? 1 : units);
-  if (p < 1) p = 1;
-  if (p > tiles) p = tiles;
-  if (p > 65535) p = 65535;
-  return (int)p;
+  const int64_t sms = num_sms();
+  if (units < 1) units = 1;
+  int64_t best = 1;
+  double best_t = 1e30;
+  for (int64_t p = 1; p <= 2 * sms && p <= tiles; p++) {
+    const double t = (double)((units * p + sms - 1) / sms) / (double)p;
+    if (t < best_t - 1e-12) {
+      best_t = t;
+      best = p;
+    }
+  }
+  return (int)best;
 }
 
-// Balanced ranges of at most kSliceRange/128 whole 128-slot chunks per head.
-int slice_ranges(const Shape& s) {
-  const int chunks = s.G / 128, per = kSliceRange / 128;
-  const int r = (chunks + per - 1) / per;
-  return r < 1 ? 1 : r;
-}
-int slice_splits(const Shape& s) { return point_splits(s, (int)(s.BH() * slice_ranges(s))); }
+// One slice CTA per (point split, batch-head, 128-slot block).
+int slice_blocks(const Shape& s) { return s.G / kGC < 1 ? 1 : s.G / kGC; }
+int slice_splits(const Shape& s) { return point_splits(s, (int)(s.BH() * slice_blocks(s))); }
 
-size_t smem_deslice(int G) { return 1024 + (size_t)G * 160 + kStages * (kXBytes + kXeBytes) + 256; }
-size_t smem_stats(int G) { return 1024 + (size_t)G * 96 + kStages * (kXBytes + kXeBytes) + 2 * kTile * 8 + 256; }
-size_t smem_slice() { return 1024 + (size_t)kSliceRange * 96 + kSliceStages * kStageBytes + 2 * kEBytes + 256; }
+size_t smem_deslice(int G) { return 1024 + (size_t)G * 160 + kStages * kXBytes + kExBytes + 512; }
+size_t smem_stats(int G) { return 1024 + (size_t)G * 96 + kStages * kXBytes + kExBytes + 2 * kTile * 8 + 512; }
+size_t smem_slice() { return 1024 + (size_t)kWBlock + kSliceStages * kStageBytes + kExBytes + 512; }
 
 template <typename K>
 cudaError_t set_smem(K kernel, size_t bytes) {
@@ -888,10 +892,24 @@ cudaError_t prep_w(const Shape& s, const float* W, const float* bias, const floa
   return cudaGetLastError();
 }
 
+// Statistics into lse [B,H,N] and the padded -lse2 copy at nl2p.
+cudaError_t run_stats(const Shape& s, const void* x, const uint8_t* wimg, float* lse, float* nl2p, uint32_t* status,
+                      cudaStream_t st) {
+  CUtensorMap xmap;
+  if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
+  const int P = point_splits(s, (int)s.BH());
+  const size_t sm = smem_stats(s.G);
+  cudaError_t e = set_smem(k_stats, sm);
+  if (e != cudaSuccess) return e;
+  k_stats<<<dim3((unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(xmap, wimg, lse, nl2p, s.N, padded_n(s), s.H,
+                                                                     s.G, P, status);
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 bool tc_forward_supported(const Shape& s) {
-  return s.dtype == FS_BF16 && s.d == kD && s.G % 128 == 0 && s.G <= 1024 && s.N >= 1 && encode_fn() != nullptr;
+  return s.dtype == FS_BF16 && s.d == kD && s.G % kGC == 0 && s.G <= 1024 && s.N >= 1 && encode_fn() != nullptr;
 }
 
 int tc_forward_launch_count(const Shape&) { return 4 /*prep_w, stats, slice, reduce*/ + 3 /*prep_w, prep_z, deslice*/; }
@@ -900,44 +918,40 @@ size_t tc_slice_partials_bytes(const Shape& s) {
   if (!tc_forward_supported(s)) return 0;
   return (size_t)slice_splits(s) * s.BH() * s.G * (kD + 1) * sizeof(float);
 }
-size_t tc_slice_prep_bytes(const Shape& s) { return tc_forward_supported(s) ? w_image_bytes(s) : 0; }
+size_t tc_slice_prep_bytes(const Shape& s) {
+  return tc_forward_supported(s) ? align_up(w_image_bytes(s), 256) + nl2_bytes(s) : 0;
+}
 size_t tc_deslice_prep_bytes(const Shape& s) {
-  return tc_forward_supported(s) ? align_up(w_image_bytes(s), 256) + z_image_bytes(s) : 0;
+  return tc_forward_supported(s) ? align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256) + nl2_bytes(s)
+                                 : 0;
 }
 
 cudaError_t tc_stats(const Shape& s, const void* x, const float* W, const float* bias, const float* tau, float* lse,
                      void* prep, uint32_t* status, cudaStream_t st) {
   uint8_t* wimg = static_cast<uint8_t*>(prep);
+  float* nl2p = reinterpret_cast<float*>(wimg + align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256));
   cudaError_t e = prep_w(s, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
-  CUtensorMap xmap;
-  if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
-  const int P = point_splits(s, (int)s.BH());
-  const size_t sm = smem_stats(s.G);
-  dim3 grid((unsigned)P, (unsigned)s.BH());
-  if (s.G % 128 == 0) {
-    if ((e = set_smem(k_stats<128>, sm)) != cudaSuccess) return e;
-    k_stats<128><<<grid, kThreads, sm, st>>>(xmap, wimg, lse, s.N, s.H, s.G, P, status);
-  } else {
-    return cudaErrorInvalidValue;
-  }
-  return cudaGetLastError();
+  return run_stats(s, x, wimg, lse, nl2p, status, st);
 }
 
 cudaError_t tc_slice_fwd(const Shape& s, const void* x, const void* f, const float* W, const float* bias,
                          const float* tau, float* tokens, float* wsum, float* lse, int finalize, float* part,
                          void* prep, uint32_t* status, cudaStream_t st) {
-  cudaError_t e = tc_stats(s, x, W, bias, tau, lse, prep, status, st);
-  if (e != cudaSuccess) return e;
   uint8_t* wimg = static_cast<uint8_t*>(prep);
-  CUtensorMap xmap, fmap;
+  float* nl2p = reinterpret_cast<float*>(wimg + align_up(w_image_bytes(s), 256));
+  cudaError_t e = prep_w(s, W, bias, tau, wimg, status, st);
+  if (e != cudaSuccess) return e;
+  if ((e = run_stats(s, x, wimg, lse, nl2p, status, st)) != cudaSuccess) return e;
+  CUtensorMap xmap, fmap, lmap;
   if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
   if (!make_point_map(&fmap, f, s, 16, CU_TENSOR_MAP_SWIZZLE_32B)) return cudaErrorInvalidValue;
-  const int R = slice_ranges(s), P = slice_splits(s);
+  if (!make_lse_map(&lmap, nl2p, s.BH(), padded_n(s))) return cudaErrorInvalidValue;
+  const int R = slice_blocks(s), P = slice_splits(s);
   dim3 grid((unsigned)P, (unsigned)s.BH(), (unsigned)R);
   const size_t sm = smem_slice();
   if ((e = set_smem(k_slice, sm)) != cudaSuccess) return e;
-  k_slice<<<grid, kThreads, sm, st>>>(xmap, fmap, wimg, lse, part, s.N, s.H, s.G, P, R, status);
+  k_slice<<<grid, kThreads, sm, st>>>(xmap, fmap, lmap, wimg, part, s.N, s.H, s.G, P, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   return simt_reduce_tokens(s, P, part, tokens, wsum, finalize, st);
 }
@@ -957,9 +971,9 @@ cudaError_t tc_deslice_fwd(const Shape& s, const void* x, const float* W, const 
   const int P = point_splits(s, (int)s.BH());
   const size_t sm = smem_deslice(s.G);
   dim3 grid((unsigned)P, (unsigned)s.BH());
-  if ((e = set_smem(k_deslice<128>, sm)) != cudaSuccess) return e;
-  k_deslice<128><<<grid, kThreads, sm, st>>>(xmap, wimg, zimg, lse, static_cast<__nv_bfloat16*>(out), s.N, s.H,
-                                             s.G, P, status);
+  if ((e = set_smem(k_deslice, sm)) != cudaSuccess) return e;
+  k_deslice<<<grid, kThreads, sm, st>>>(xmap, wimg, zimg, lse, static_cast<__nv_bfloat16*>(out), s.N, s.H, s.G, P,
+                                        status);
   return cudaGetLastError();
 }
 
