@@ -9,14 +9,17 @@
 //
 // Logits.  A 128-point x 128-slot block of base-2 logits a2 = a * log2(e) is one
 // tcgen05.mma chain with K = 48:
-//   point side [ x (32 bf16) | 1, 1, 0 ... ]            (the last block constant)
-//   slot side  [ W*log2e/tau (32) | b'_hi, b'_lo, 0 ... ]  (b' = bias*log2e/tau in
+//   point side [ x (32 bf16) | 1, 1, -lse2_hi, -lse2_lo, 0 ... ]  (stats: 1, 1, 0 ...)
+//   slot side  [ W*log2e/tau (32) | b'_hi, b'_lo, 1, 1, 0 ... ]  (b' = bias*log2e/tau in
 //                                                           two bf16 halves)
 // The point-major passes (stats, deslice) put points on the MMA's M (TMEM lane
 // = point); the slice swaps the operands, so its TMEM lane is a slot and its
-// column a point.  The normaliser lse2 is subtracted in registers (packed
-// f32x2 adds) and never written into an MMA operand: no thread writes a
-// tensor-core operand per tile (that costs a generic -> async proxy fence).
+// column a point.  In the slice and the deslice the point side's extra block is
+// [1, 1, -lse2_hi, -lse2_lo, 0 ...], so the accumulator holds a2 - lse2, the
+// log2 of the slice weight itself.  The stats pass writes these 16-byte rows per
+// point to memory and the later passes load them by TMA with each tile: no
+// thread writes a tensor-core operand per tile (that would cost a generic ->
+// async proxy fence per tile).
 //
 // Products.  The bf16 weights are written back into the S buffer they came
 // from and feed the second MMA as its TMEM A operand: P x Z' in the deslice
@@ -38,6 +41,8 @@
 // Shared-memory operand layouts (all bases 1024-byte aligned):
 //   x tile          K-major, 64 B rows, 64B swizzle (TMA)        128 points x 32
 //   constant extra  K-major, 32 B rows, 32B swizzle              128 rows x 16
+//   point extra     K-major, no swizzle: core matrices of 8 rows x 16 B, the
+//                   k = 0..7 half from memory (TMA), the k = 8..15 half zero
 //   W image         K-major, 64 B rows, 64B swizzle, then its 32 B extra rows
 //   Z' image        K-major rows = channels, 128 B rows, 128B swizzle
 //   [F | 1]         MN-major, three 16-channel blocks, 32B swizzle (TMA)
@@ -64,12 +69,12 @@ constexpr int kSBuf = 3;          // S buffers (logits run up to two blocks ahea
 constexpr uint32_t kXBytes = kTile * 64;   // 128 points x 32 bf16
 constexpr uint32_t kExBytes = kTile * 32;  // 128 rows x 16 bf16
 constexpr uint32_t kFBlock = kTile * 32;   // 128 points x 16 channels
-constexpr uint32_t kLseBytes = kTile * 4;  // 128 fp32
+constexpr uint32_t kPxBytes = kTile * 16;  // 128 point-extra rows of 8 bf16 (k = 0..7)
 constexpr uint64_t kWaitNs = 2000000000ull;
 
 // ---- operand images written by the prep kernels -------------------------------------------
 // W image for head h: G rows (slots) x 64 B of W*log2e/tau (64B swizzle), then
-// G rows x 32 B of [b'_hi, b'_lo, 0...] (32B swizzle).
+// G rows x 32 B of [b'_hi, b'_lo, 1, 1, 0...] (32B swizzle).
 __device__ __forceinline__ uint32_t off_sw64(int row, int k) {  // k in [0, 32)
   const int chunk = k >> 3;
   return (uint32_t)((row >> 3) * 512 + (row & 7) * 64 + ((chunk ^ ((row & 7) >> 1)) << 4) + (k & 7) * 2);
@@ -104,7 +109,10 @@ __global__ void k_prep_w(const float* __restrict__ W, const float* __restrict__ 
   const float b2 = bias[(int64_t)h * G + g] * scale;
   const __nv_bfloat16 hi = __float2bfloat16_rn(b2);
   const __nv_bfloat16 lo = __float2bfloat16_rn(b2 - __bfloat162float(hi));
-  for (int k = 0; k < 16; k++) ep[off_sw32(g, k) / 2] = k == 0 ? hi : (k == 1 ? lo : __float2bfloat16_rn(0.f));
+  // k = 2, 3 multiply the point side's -lse2 halves (zero in the statistics pass).
+  for (int k = 0; k < 16; k++)
+    ep[off_sw32(g, k) / 2] =
+        k == 0 ? hi : (k == 1 ? lo : __float2bfloat16_rn((k == 2 || k == 3) ? 1.f : 0.f));
 }
 
 __global__ void k_prep_z(const float* __restrict__ zp, uint8_t* __restrict__ img, int64_t BH, int G) {
@@ -146,16 +154,26 @@ __device__ __forceinline__ void write_const_extra(uint8_t* ex) {
   }
 }
 
+// Descriptors of the two kinds of point-side extra block: the constant one
+// (32B swizzle) and the per-tile one loaded by TMA (no swizzle; the k = 0..7
+// core matrices at px, the zero k = 8..15 half kPxBytes further on).
+__device__ __forceinline__ uint64_t const_extra_desc(uint32_t ex_s) { return sdesc(ex_s, 16, 256, kSw32); }
+__device__ __forceinline__ uint64_t point_extra_desc(uint32_t px_s) { return sdesc(px_s, kPxBytes, 128, 0); }
+__device__ __forceinline__ void zero_smem(uint8_t* p, uint32_t bytes) {
+  for (uint32_t o = threadIdx.x * 16; o < bytes; o += blockDim.x * 16) st_shared_v4(smem_u32(p) + o, 0u, 0u, 0u, 0u);
+}
+
 // Base-2 logits of 128 points x 128 slots (chunk c of the W image) into TMEM.
 //   point_major: A = points (x tile), B = slots (W);  else A = slots, B = points.
-__device__ __forceinline__ void issue_logits(uint32_t tmem_d, uint32_t x_s, uint32_t ex_s, uint32_t w_img,
+//   xe: descriptor of the point-side extra block.
+__device__ __forceinline__ void issue_logits(uint32_t tmem_d, uint32_t x_s, uint64_t xe, uint32_t w_img,
                                              uint32_t we_img, int c, bool point_major) {
   constexpr uint32_t idesc = idesc_bf16(128, kGC, false, false);
   const uint32_t wc = w_img + (uint32_t)c * kGC * 64;
   const uint32_t wec = we_img + (uint32_t)c * kGC * 32;
   const uint64_t x0 = sdesc(x_s, 16, 512, kSw64), x1 = sdesc(x_s + 32, 16, 512, kSw64);
   const uint64_t w0 = sdesc(wc, 16, 512, kSw64), w1 = sdesc(wc + 32, 16, 512, kSw64);
-  const uint64_t xe = sdesc(ex_s, 16, 256, kSw32), we = sdesc(wec, 16, 256, kSw32);
+  const uint64_t we = sdesc(wec, 16, 256, kSw32);
   if (point_major) {
     mma_ss(tmem_d, x0, w0, idesc, 0);
     mma_ss(tmem_d, x1, w1, idesc, 1);
@@ -176,39 +194,51 @@ __device__ __forceinline__ void load_images(uint8_t* dst, const uint8_t* src, ui
   }
 }
 
-// 2^(v + d) for 64 logits (d = -lse2, packed pairs) -> 32 bf16x2 words.
-__device__ __forceinline__ void weights64(const uint32_t (&v0)[32], const uint32_t (&v1)[32], const uint64_t (&d)[32],
-                                          uint32_t (&p0)[16], uint32_t (&p1)[16]) {
+// 2^t for 64 log2-weights -> 32 bf16x2 words.
+__device__ __forceinline__ void weights64(const uint32_t (&v0)[32], const uint32_t (&v1)[32], uint32_t (&p0)[16],
+                                          uint32_t (&p1)[16]) {
 #pragma unroll
   for (int k = 0; k < 16; k++) {
-    const uint64_t a = add2(pack2(v0[2 * k], v0[2 * k + 1]), d[k]);
-    const uint64_t b = add2(pack2(v1[2 * k], v1[2 * k + 1]), d[16 + k]);
-    p0[k] = pack_bf16(ex2(lo_f(a)), ex2(hi_f(a)));
-    p1[k] = pack_bf16(ex2(lo_f(b)), ex2(hi_f(b)));
+    p0[k] = pack_bf16(ex2(__uint_as_float(v0[2 * k])), ex2(__uint_as_float(v0[2 * k + 1])));
+    p1[k] = pack_bf16(ex2(__uint_as_float(v1[2 * k])), ex2(__uint_as_float(v1[2 * k + 1])));
   }
+}
+
+// Point-extra rows [1, 1, -lse2_hi, -lse2_lo, 0, 0, 0, 0] (bf16) from lse [B,H,N]
+// (natural log) into px [B*H, Np, 8]; padded points (n >= N) get -1e30 so that
+// their weights vanish.
+__global__ void k_prep_px(const float* __restrict__ lse, uint4* __restrict__ px, int64_t BH, int64_t N, int64_t Np) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= BH * Np) return;
+  const int64_t bh = i / Np, n = i % Np;
+  const float nl2 = n < N ? -lse[bh * N + n] * kLog2e : -1e30f;
+  const __nv_bfloat16 hi = __float2bfloat16_rn(nl2);
+  const __nv_bfloat16 lo = __float2bfloat16_rn(nl2 - __bfloat162float(hi));
+  px[i] = make_uint4(0x3F803F80u, (uint32_t)__bfloat16_as_ushort(hi) | ((uint32_t)__bfloat16_as_ushort(lo) << 16), 0u, 0u);
 }
 
 // =========================================================================================
 // Deslice: out_n = sum_g w_ng z'_g.
-// smem: [W img G*96][Z' img G*64][x stages][constant extra][barriers]
+// smem: [W img G*96][Z' img G*64][stages: x | point extra (TMA half, zero half)][barriers]
 // TMEM: S buffers [0, 384); P x Z' accumulators O_0 [384, 448), O_1 [448, 512),
 // each double-buffered by tile parity.  Softmax warpgroup wg reads S columns
 // [64 wg, 64 wg + 64) and writes their bf16 weights, packed in pairs, into
 // columns [64 wg, 64 wg + 32) of the same buffer; warp 2 + wg turns exactly
 // those into its products (K-steps [4 wg, 4 wg + 4) of the block).
 // =========================================================================================
+constexpr uint32_t kDStage = kXBytes + 2 * kPxBytes;  // x tile, point extra (both halves)
+
 __global__ void __launch_bounds__(kThreads, 1)
-    k_deslice(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ wimg,
-              const uint8_t* __restrict__ zimg, const float* __restrict__ lse, __nv_bfloat16* __restrict__ out,
-              int64_t N, int H, int G, int splits, uint32_t* status) {
+    k_deslice(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap pmap,
+              const uint8_t* __restrict__ wimg, const uint8_t* __restrict__ zimg, __nv_bfloat16* __restrict__ out,
+              int64_t N, int64_t Np, int H, int G, int splits, uint32_t* status) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t wbytes = (uint32_t)G * 96, zbytes = (uint32_t)G * 64;
   uint8_t* s_w = smem;
   uint8_t* s_z = s_w + wbytes;
-  uint8_t* s_x = s_z + zbytes;
-  uint8_t* s_ex = s_x + kStages * kXBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_ex + kExBytes);
+  uint8_t* s_x = s_z + zbytes;  // stage s at s_x + s * kDStage
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_x + kStages * kDStage);
   uint64_t* wz_full = bars;
   uint64_t* x_full = bars + 1;
   uint64_t* x_empty = x_full + kStages;
@@ -248,7 +278,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     ab->flag = 0;
     fence_mbar_init();
   }
-  write_const_extra(s_ex);
+  for (int s = 0; s < kStages; s++) zero_smem(s_x + s * kDStage + kXBytes + kPxBytes, kPxBytes);
   fence_proxy_async_smem();
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
@@ -260,6 +290,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------ producer ------------------------------
     if (lane == 0 && wk.ntiles > 0) {
       prefetch_tmap(&xmap);
+      prefetch_tmap(&pmap);
       mbar_expect_tx(wz_full, wbytes + zbytes);
       load_images(s_w, wimg + (size_t)h * wbytes, wbytes, wz_full);
       load_images(s_z, zimg + (size_t)wk.bh * zbytes, zbytes, wz_full);
@@ -267,8 +298,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (; i < wk.ntiles; i++) {
         const int s = (int)(i % kStages);
         if (i >= kStages && !mbar_wait(&x_empty[s], (uint32_t)(((i / kStages) - 1) & 1), ab, status)) break;
-        mbar_expect_tx(&x_full[s], kXBytes);
-        tma_load_3d(s_x + s * kXBytes, &xmap, h * kD, (int)((wk.tile0 + i) * kTile), (int)b, &x_full[s]);
+        const int n0 = (int)((wk.tile0 + i) * kTile);
+        mbar_expect_tx(&x_full[s], kXBytes + kPxBytes);
+        tma_load_3d(s_x + s * kDStage, &xmap, h * kD, n0, (int)b, &x_full[s]);
+        tma_load_2d(s_x + s * kDStage + kXBytes, &pmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
       }
       // Drain: the newest load of each stage has landed before the CTA exits.
       for (int64_t j = (i > kStages ? i - kStages : 0); j < i; j++)
@@ -290,7 +323,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (c == 0 && !(ok = mbar_wait(&x_full[s], (uint32_t)((i / kStages) & 1), ab, status))) break;
         if (q >= kSBuf && !(ok = mbar_wait(&pv_done[bb], (uint32_t)(((q / kSBuf) - 1) & 1), ab, status))) break;
         tc_fence_after();
-        issue_logits(tmem + (uint32_t)bb * kGC, smem_u32(s_x + s * kXBytes), smem_u32(s_ex), sw, swe, c, true);
+        const uint32_t xs = smem_u32(s_x + s * kDStage);
+        issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kXBytes), sw, swe, c, true);
         mma_commit(&s_full[bb]);
         if (c == nch - 1) mma_commit(&x_empty[s]);
       }
@@ -334,11 +368,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     int64_t q = 0;
     bool ok = true;
-    // -lse2 of this thread's point in tile j, loaded two tiles ahead of its use.
-    auto load_nl2 = [&](int64_t j) -> float {
-      const int64_t nn = (wk.tile0 + j) * kTile + r;
-      return (j < wk.ntiles && nn < N) ? -lse[wk.bh * N + nn] * kLog2e : 0.f;
-    };
     // Output of tile t: this warpgroup's 16 channels of O_0 + O_1 -> bf16 -> global.
     auto epilogue = [&](int64_t t) -> bool {
       const int ob = (int)(t & 1);
@@ -365,15 +394,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       return true;
     };
-    float nl2 = load_nl2(0), nl2_next = load_nl2(1);
     for (int64_t i = 0; ok && i < wk.ntiles; i++) {
-      const float nl2_cur = nl2;
-      nl2 = nl2_next;
-      nl2_next = load_nl2(i + 2);
-      uint64_t d[32];
-      const uint32_t nb = __float_as_uint(nl2_cur);
-#pragma unroll
-      for (int k = 0; k < 32; k++) d[k] = pack2(nb, nb);
       for (int c = 0; c < nch; c++, q++) {
         const int bb = (int)(q % kSBuf);
         if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
@@ -384,7 +405,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld32(tS + 32, v1);
         tmem_wait_ld2(v0, v1);
         uint32_t pk0[16], pk1[16];
-        weights64(v0, v1, d, pk0, pk1);
+        weights64(v0, v1, pk0, pk1);
         tmem_st16(tS, pk0);
         tmem_st16(tS + 16, pk1);
         tmem_wait_st();
@@ -406,8 +427,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // =========================================================================================
 // Statistics: lse_n = log sum_g exp(a_ng) (natural log) to lse[bh*N + n], and
-// -lse2 = -lse*log2(e) to the padded copy nl2p[bh*Np + n] (Np = N rounded up to
-// a whole tile; padded points get -1e30 so that their weights vanish).
+// the point-extra row [1, 1, -lse2_hi, -lse2_lo, 0 x 4] (lse2 = lse*log2(e)) to
+// px[bh*Np + n] (Np = N rounded up to a whole tile; padded points get -1e30 so
+// that their weights vanish).
 // Two logits issuers (warp 1 + j issues the blocks c with c % 2 == j).  Each
 // softmax warpgroup keeps a running (max, sum) over its half of every block;
 // the halves are combined through shared memory at the end of a tile.
@@ -416,7 +438,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // =========================================================================================
 __global__ void __launch_bounds__(kThreads, 1)
     k_stats(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ wimg, float* __restrict__ lse,
-            float* __restrict__ nl2p, int64_t N, int64_t Np, int H, int G, int splits, uint32_t* status) {
+            uint4* __restrict__ px, int64_t N, int64_t Np, int H, int G, int splits, uint32_t* status) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const uint32_t wbytes = (uint32_t)G * 96;
@@ -498,7 +520,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (c == j && !(ok = mbar_wait(&x_full[s], (uint32_t)((i / kStages) & 1), ab, status))) break;
         if (q >= 2 && !(ok = mbar_wait(&s_free[q & 1], (uint32_t)(((q >> 1) - 1) & 1), ab, status))) break;
         tc_fence_after();
-        issue_logits(tmem + (uint32_t)(q & 1) * kGC, smem_u32(s_x + s * kXBytes), smem_u32(s_ex), sw, swe, c, true);
+        issue_logits(tmem + (uint32_t)(q & 1) * kGC, smem_u32(s_x + s * kXBytes), const_extra_desc(smem_u32(s_ex)), sw,
+                     swe, c, true);
         mma_commit(&s_full[q & 1]);
         if (c == c_last) mma_commit(&x_empty[s]);
       }
@@ -569,11 +592,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float M = fmaxf(m, o.x);
         const float L = l * ex2(m - M) + o.y * ex2(o.x - M);
         const float lse2 = M + log2f(L);
-        if (n < N) {
-          lse[wk.bh * N + n] = lse2 * kLn2;
-          nl2p[wk.bh * Np + n] = -lse2;
-        } else if (n < Np) {
-          nl2p[wk.bh * Np + n] = -1e30f;
+        if (n < Np) {
+          const float nl2 = n < N ? -lse2 : -1e30f;
+          const __nv_bfloat16 hi = __float2bfloat16_rn(nl2);
+          const __nv_bfloat16 lo = __float2bfloat16_rn(nl2 - __bfloat162float(hi));
+          px[wk.bh * Np + n] =
+              make_uint4(0x3F803F80u, (uint32_t)__bfloat16_as_ushort(hi) | ((uint32_t)__bfloat16_as_ushort(lo) << 16),
+                         0u, 0u);
+          if (n < N) lse[wk.bh * N + n] = lse2 * kLn2;
         }
       }
     }
@@ -589,31 +615,31 @@ __global__ void __launch_bounds__(kThreads, 1)
 // 128-slot block j of head h and point split p and computes for its slots
 //   U_g = sum_n w_ng f_n,  S_g = sum_n w_ng,  w_ng = 2^(a2_ng - lse2_n).
 // The logits are formed transposed (M = 128 slots, N = 128 points), so TMEM
-// lane = slot and column = point; -lse2 of the tile's points arrives by TMA
-// with the tile and is added per column.  The bf16 weights written back in
-// place serve directly as the TMEM A operand of U|S += E [F | 1] (K = points),
-// so the weight tile never passes through shared memory.
+// lane = slot and column = point; the point-extra rows of the tile arrive by
+// TMA with it, so the accumulator holds log2 of the weights.  The bf16 weights
+// written back in place serve directly as the TMEM A operand of
+// U|S += E [F | 1] (K = points), so the weight tile never passes through
+// shared memory.
 // Writes part[p][bh][g][0..32] = (U_g, S_g).
-// smem: [W img block 128*96][stages: x | F_lo F_hi ones | -lse2][constant extra][barriers]
+// smem: [W img block 128*96][stages: x | F_lo F_hi ones | point extra (2 halves)][barriers]
 // TMEM: S buffers [0, 384); U|S accumulators A_0 [384, 432), A_1 [432, 480).
 // Warp 1 issues the logits; warp 2 + wg issues the products of points
 // [64 wg, 64 wg + 64) of every tile (the columns softmax warpgroup wg wrote)
 // into its own accumulator A_wg (the two are summed in a fixed order).
 // =========================================================================================
-constexpr uint32_t kStageBytes = kXBytes + 3 * kFBlock + 1024;  // x, [F | 1], -lse2 (padded to 1 KB)
-constexpr uint32_t kWBlock = 128 * 96;                          // one 128-slot block of the W image
+constexpr uint32_t kStageBytes = kXBytes + 3 * kFBlock + 2 * kPxBytes;  // x, [F | 1], point extra
+constexpr uint32_t kWBlock = 128 * 96;                                  // one 128-slot block of the W image
 
 __global__ void __launch_bounds__(kThreads, 1)
     k_slice(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap fmap,
-            const __grid_constant__ CUtensorMap lmap, const uint8_t* __restrict__ wimg, float* __restrict__ part,
-            int64_t N, int H, int G, int splits, uint32_t* status) {
+            const __grid_constant__ CUtensorMap pmap, const uint8_t* __restrict__ wimg, float* __restrict__ part,
+            int64_t N, int64_t Np, int H, int G, int splits, uint32_t* status) {
   const int g_base = blockIdx.z * kGC;  // slot block
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* s_w = smem;
   uint8_t* s_st = s_w + kWBlock;
-  uint8_t* s_ex = s_st + kSliceStages * kStageBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_ex + kExBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_st + kSliceStages * kStageBytes);
   uint64_t* w_full = bars;
   uint64_t* x_full = bars + 1;
   uint64_t* st_empty = x_full + kSliceStages;
@@ -630,7 +656,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int64_t b = wk.bh / H;
   const int h = (int)(wk.bh % H);
   constexpr uint32_t kA = kSBuf * kGC;  // TMEM column base of the accumulators
-  constexpr uint32_t kFOff = kXBytes, kLOff = kXBytes + 3 * kFBlock;
+  constexpr uint32_t kFOff = kXBytes, kPOff = kXBytes + 3 * kFBlock;
 
   if (threadIdx.x == 0) {
     mbar_init(w_full, 1);
@@ -648,7 +674,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     ab->flag = 0;
     fence_mbar_init();
   }
-  write_const_extra(s_ex);
+  for (int s = 0; s < kSliceStages; s++) zero_smem(s_st + s * kStageBytes + kPOff + kPxBytes, kPxBytes);
   // Constant "ones" block of every stage: row n = [1, 0 x 15] (32B swizzle).
   for (int idx = threadIdx.x; idx < kSliceStages * kTile; idx += kThreads) {
     const int s = idx / kTile, r = idx % kTile;
@@ -669,7 +695,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0) {
       prefetch_tmap(&xmap);
       prefetch_tmap(&fmap);
-      prefetch_tmap(&lmap);
+      prefetch_tmap(&pmap);
       // The slot block's rows of the W image: 128 rows of W' (64 B) then 128 rows of
       // the extra block (32 B); the global image holds G rows of each.
       mbar_expect_tx(w_full, kWBlock);
@@ -684,11 +710,11 @@ __global__ void __launch_bounds__(kThreads, 1)
           break;
         uint8_t* st = s_st + s * kStageBytes;
         const int n0 = (int)((wk.tile0 + i) * kTile);
-        mbar_expect_tx(&x_full[s], kXBytes + 2 * kFBlock + kLseBytes);
+        mbar_expect_tx(&x_full[s], kXBytes + 2 * kFBlock + kPxBytes);
         tma_load_3d(st, &xmap, h * kD, n0, (int)b, &x_full[s]);
         tma_load_3d(st + kFOff, &fmap, h * kD, n0, (int)b, &x_full[s]);
         tma_load_3d(st + kFOff + kFBlock, &fmap, h * kD + 16, n0, (int)b, &x_full[s]);
-        tma_load_2d(st + kLOff, &lmap, n0, (int)wk.bh, &x_full[s]);
+        tma_load_2d(st + kPOff, &pmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
       }
       for (int64_t j = (i > kSliceStages ? i - kSliceStages : 0); j < i; j++)
         mbar_wait(&x_full[j % kSliceStages], (uint32_t)((j / kSliceStages) & 1), ab, nullptr, kWaitNs);
@@ -705,7 +731,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(ok = mbar_wait(&x_full[s], (uint32_t)((i / kSliceStages) & 1), ab, status))) break;
         if (i >= kSBuf && !(ok = mbar_wait(&pv_done[bb], (uint32_t)(((i / kSBuf) - 1) & 1), ab, status))) break;
         tc_fence_after();
-        issue_logits(tmem + (uint32_t)bb * kGC, smem_u32(s_st + s * kStageBytes), smem_u32(s_ex), sw, swe, 0, false);
+        const uint32_t xs = smem_u32(s_st + s * kStageBytes);
+        issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kPOff), sw, swe, 0, false);
         mma_commit(&s_full[bb]);
         mma_commit(&st_empty[s]);
       }
@@ -744,18 +771,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     bool ok = true;
     for (int64_t i = 0; ok && i < wk.ntiles; i++) {
-      const int s = (int)(i % kSliceStages);
       const int bb = (int)(i % kSBuf);
-      // The -lse2 values come with the tile (TMA): wait for the stage, then for the logits.
-      if (!(ok = mbar_wait(&x_full[s], (uint32_t)((i / kSliceStages) & 1), ab, status))) break;
-      const float4* nl = reinterpret_cast<const float4*>(s_st + s * kStageBytes + kLOff) + wg * 16;
-      uint64_t d[32];
-#pragma unroll
-      for (int k = 0; k < 16; k++) {
-        const float4 t4 = nl[k];
-        d[2 * k] = pack2(__float_as_uint(t4.x), __float_as_uint(t4.y));
-        d[2 * k + 1] = pack2(__float_as_uint(t4.z), __float_as_uint(t4.w));
-      }
       if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((i / kSBuf) & 1), ab, status))) break;
       tc_fence_after();
       const uint32_t tS = tmem + lane_addr + (uint32_t)bb * kGC + (uint32_t)wg * 64;
@@ -764,7 +780,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld32(tS + 32, v1);
       tmem_wait_ld2(v0, v1);
       uint32_t pk0[16], pk1[16];
-      weights64(v0, v1, d, pk0, pk1);
+      weights64(v0, v1, pk0, pk1);
       tmem_st16(tS, pk0);
       tmem_st16(tS + 16, pk1);
       tmem_wait_st();
@@ -835,15 +851,15 @@ bool make_point_map(CUtensorMap* map, const void* ptr, const Shape& s, int box_c
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// 2-D view of the padded [B*H, Np] fp32 -lse2 copy; box = (128 points, 1).
-bool make_lse_map(CUtensorMap* map, const float* ptr, int64_t BH, int64_t Np) {
+// 2-D view of the point-extra rows [B*H*Np, 8] bf16; box = (8, 128 points).
+bool make_px_map(CUtensorMap* map, const void* ptr, int64_t BH, int64_t Np) {
   auto fn = encode_fn();
   if (!fn) return false;
-  cuuint64_t dims[2] = {(cuuint64_t)Np, (cuuint64_t)BH};
-  cuuint64_t strides[1] = {(cuuint64_t)Np * 4};
-  cuuint32_t box[2] = {(cuuint32_t)kTile, 1};
+  cuuint64_t dims[2] = {8, (cuuint64_t)(BH * Np)};
+  cuuint64_t strides[1] = {16};
+  cuuint32_t box[2] = {8, (cuuint32_t)kTile};
   cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(ptr), dims, strides, box, estr,
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -851,7 +867,7 @@ bool make_lse_map(CUtensorMap* map, const float* ptr, int64_t BH, int64_t Np) {
 size_t w_image_bytes(const Shape& s) { return (size_t)s.H * s.G * 96; }
 size_t z_image_bytes(const Shape& s) { return (size_t)s.BH() * s.G * 64; }
 int64_t padded_n(const Shape& s) { return (s.N + kTile - 1) / kTile * kTile; }
-size_t nl2_bytes(const Shape& s) { return (size_t)s.BH() * padded_n(s) * sizeof(float); }
+size_t px_bytes(const Shape& s) { return (size_t)s.BH() * padded_n(s) * 16; }
 
 // Point splits per work unit for one-CTA-per-SM kernels: the split count P that
 // minimises the makespan in units of one unit's work, ceil(units * P / SMs) / P
@@ -876,9 +892,9 @@ int point_splits(const Shape& s, int units) {
 int slice_blocks(const Shape& s) { return s.G / kGC < 1 ? 1 : s.G / kGC; }
 int slice_splits(const Shape& s) { return point_splits(s, (int)(s.BH() * slice_blocks(s))); }
 
-size_t smem_deslice(int G) { return 1024 + (size_t)G * 160 + kStages * kXBytes + kExBytes + 512; }
+size_t smem_deslice(int G) { return 1024 + (size_t)G * 160 + kStages * kDStage + 512; }
 size_t smem_stats(int G) { return 1024 + (size_t)G * 96 + kStages * kXBytes + kExBytes + 2 * kTile * 8 + 512; }
-size_t smem_slice() { return 1024 + (size_t)kWBlock + kSliceStages * kStageBytes + kExBytes + 512; }
+size_t smem_slice() { return 1024 + (size_t)kWBlock + kSliceStages * kStageBytes + 512; }
 
 template <typename K>
 cudaError_t set_smem(K kernel, size_t bytes) {
@@ -892,8 +908,8 @@ cudaError_t prep_w(const Shape& s, const float* W, const float* bias, const floa
   return cudaGetLastError();
 }
 
-// Statistics into lse [B,H,N] and the padded -lse2 copy at nl2p.
-cudaError_t run_stats(const Shape& s, const void* x, const uint8_t* wimg, float* lse, float* nl2p, uint32_t* status,
+// Statistics into lse [B,H,N] and the point-extra rows at px.
+cudaError_t run_stats(const Shape& s, const void* x, const uint8_t* wimg, float* lse, void* px, uint32_t* status,
                       cudaStream_t st) {
   CUtensorMap xmap;
   if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
@@ -901,8 +917,8 @@ cudaError_t run_stats(const Shape& s, const void* x, const uint8_t* wimg, float*
   const size_t sm = smem_stats(s.G);
   cudaError_t e = set_smem(k_stats, sm);
   if (e != cudaSuccess) return e;
-  k_stats<<<dim3((unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(xmap, wimg, lse, nl2p, s.N, padded_n(s), s.H,
-                                                                     s.G, P, status);
+  k_stats<<<dim3((unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(xmap, wimg, lse, static_cast<uint4*>(px), s.N,
+                                                                     padded_n(s), s.H, s.G, P, status);
   return cudaGetLastError();
 }
 
@@ -912,46 +928,48 @@ bool tc_forward_supported(const Shape& s) {
   return s.dtype == FS_BF16 && s.d == kD && s.G % kGC == 0 && s.G <= 1024 && s.N >= 1 && encode_fn() != nullptr;
 }
 
-int tc_forward_launch_count(const Shape&) { return 4 /*prep_w, stats, slice, reduce*/ + 3 /*prep_w, prep_z, deslice*/; }
+int tc_forward_launch_count(const Shape&) {
+  return 4 /*prep_w, stats, slice, reduce*/ + 4 /*prep_w, prep_z, prep_px, deslice*/;
+}
 
 size_t tc_slice_partials_bytes(const Shape& s) {
   if (!tc_forward_supported(s)) return 0;
   return (size_t)slice_splits(s) * s.BH() * s.G * (kD + 1) * sizeof(float);
 }
 size_t tc_slice_prep_bytes(const Shape& s) {
-  return tc_forward_supported(s) ? align_up(w_image_bytes(s), 256) + nl2_bytes(s) : 0;
+  return tc_forward_supported(s) ? align_up(w_image_bytes(s), 256) + px_bytes(s) : 0;
 }
 size_t tc_deslice_prep_bytes(const Shape& s) {
-  return tc_forward_supported(s) ? align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256) + nl2_bytes(s)
+  return tc_forward_supported(s) ? align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256) + px_bytes(s)
                                  : 0;
 }
 
 cudaError_t tc_stats(const Shape& s, const void* x, const float* W, const float* bias, const float* tau, float* lse,
                      void* prep, uint32_t* status, cudaStream_t st) {
   uint8_t* wimg = static_cast<uint8_t*>(prep);
-  float* nl2p = reinterpret_cast<float*>(wimg + align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256));
+  uint8_t* px = wimg + align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256);
   cudaError_t e = prep_w(s, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
-  return run_stats(s, x, wimg, lse, nl2p, status, st);
+  return run_stats(s, x, wimg, lse, px, status, st);
 }
 
 cudaError_t tc_slice_fwd(const Shape& s, const void* x, const void* f, const float* W, const float* bias,
                          const float* tau, float* tokens, float* wsum, float* lse, int finalize, float* part,
                          void* prep, uint32_t* status, cudaStream_t st) {
   uint8_t* wimg = static_cast<uint8_t*>(prep);
-  float* nl2p = reinterpret_cast<float*>(wimg + align_up(w_image_bytes(s), 256));
+  uint8_t* px = wimg + align_up(w_image_bytes(s), 256);
   cudaError_t e = prep_w(s, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
-  if ((e = run_stats(s, x, wimg, lse, nl2p, status, st)) != cudaSuccess) return e;
-  CUtensorMap xmap, fmap, lmap;
+  if ((e = run_stats(s, x, wimg, lse, px, status, st)) != cudaSuccess) return e;
+  CUtensorMap xmap, fmap, pmap;
   if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
   if (!make_point_map(&fmap, f, s, 16, CU_TENSOR_MAP_SWIZZLE_32B)) return cudaErrorInvalidValue;
-  if (!make_lse_map(&lmap, nl2p, s.BH(), padded_n(s))) return cudaErrorInvalidValue;
+  if (!make_px_map(&pmap, px, s.BH(), padded_n(s))) return cudaErrorInvalidValue;
   const int R = slice_blocks(s), P = slice_splits(s);
   dim3 grid((unsigned)P, (unsigned)s.BH(), (unsigned)R);
   const size_t sm = smem_slice();
   if ((e = set_smem(k_slice, sm)) != cudaSuccess) return e;
-  k_slice<<<grid, kThreads, sm, st>>>(xmap, fmap, lmap, wimg, part, s.N, s.H, s.G, P, status);
+  k_slice<<<grid, kThreads, sm, st>>>(xmap, fmap, pmap, wimg, part, s.N, padded_n(s), s.H, s.G, P, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   return simt_reduce_tokens(s, P, part, tokens, wsum, finalize, st);
 }
@@ -961,19 +979,24 @@ cudaError_t tc_deslice_fwd(const Shape& s, const void* x, const float* W, const 
                            cudaStream_t st) {
   uint8_t* wimg = static_cast<uint8_t*>(prep);
   uint8_t* zimg = wimg + align_up(w_image_bytes(s), 256);
+  uint8_t* px = zimg + align_up(z_image_bytes(s), 256);
   cudaError_t e = prep_w(s, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
   const int64_t nz = s.BH() * s.G * kD;
   k_prep_z<<<(unsigned)((nz + 255) / 256), 256, 0, st>>>(zp, zimg, s.BH(), s.G);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  CUtensorMap xmap;
+  const int64_t Np = padded_n(s), npx = s.BH() * Np;
+  k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(px), s.BH(), s.N, Np);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  CUtensorMap xmap, pmap;
   if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
+  if (!make_px_map(&pmap, px, s.BH(), Np)) return cudaErrorInvalidValue;
   const int P = point_splits(s, (int)s.BH());
   const size_t sm = smem_deslice(s.G);
   dim3 grid((unsigned)P, (unsigned)s.BH());
   if ((e = set_smem(k_deslice, sm)) != cudaSuccess) return e;
-  k_deslice<<<grid, kThreads, sm, st>>>(xmap, wimg, zimg, lse, static_cast<__nv_bfloat16*>(out), s.N, s.H, s.G, P,
-                                        status);
+  k_deslice<<<grid, kThreads, sm, st>>>(xmap, pmap, wimg, zimg, static_cast<__nv_bfloat16*>(out), s.N, Np, s.H, s.G,
+                                        P, status);
   return cudaGetLastError();
 }
 
