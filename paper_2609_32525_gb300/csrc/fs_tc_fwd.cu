@@ -26,17 +26,17 @@
 // (M = points, K = slots, N = 32 channels), E x [F | 1] in the slice (M =
 // slots, K = points, N = 48: 32 channels and a ones column for the weight sums).
 //
-// Issue.  A tcgen05.mma from one thread takes ~130 cycles before the thread can
-// issue the next, whatever N; separate warps overlap.  Warp 1 issues the logits
-// (stats: warps 1 and 2), warps 2 and 3 each issue half of every block's K-steps
-// of the product into an accumulator of their own; the two are summed in a
-// fixed order, so the result is deterministic.
+// Issue.  Each MMA-issuing role is a whole converged warp in which one elected
+// lane issues (a lone lane in a divergent branch issues several times slower).
+// Warp 1 issues the logits (stats: warps 1 and 2); warps 2 and 3 issue the
+// products into accumulators of their own, which are summed in a fixed order,
+// so the result is deterministic.
 //
 // CTA (384 threads): warp 0 TMA producer, warps 1..3 MMA issuers, warps 4..11
-// two softmax warpgroups that split the columns of every block; a thread owns
-// one TMEM lane (tcgen05.ld/st 32x32b).  Every wait is bounded (2 s): a wait
-// that gives up writes FS_ERR_TIMEOUT to the status word, the CTA drains its
-// copies and MMAs, frees TMEM and exits.
+// two softmax warpgroups that take alternate blocks (so they run out of phase);
+// a thread owns one TMEM lane (tcgen05.ld/st 32x32b).  Every wait is bounded
+// (2 s): a wait that gives up writes FS_ERR_TIMEOUT to the status word, the CTA
+// drains its copies and MMAs, frees TMEM and exits.
 //
 // Shared-memory operand layouts (all bases 1024-byte aligned):
 //   x tile          K-major, 64 B rows, 64B swizzle (TMA)        128 points x 32
@@ -130,7 +130,21 @@ __global__ void k_prep_z(const float* __restrict__ zp, uint8_t* __restrict__ img
 struct Work {
   int64_t bh;      // batch * H + head
   int64_t tile0;   // first point tile of this CTA
-  int64_t ntiles;  // number of point tiles
+  int ntiles;      // number of point tiles (the host keeps all point indices below 2^31)
+};
+
+// Tile i and slot block c of block q = i * nb + c, kept up to date while q walks
+// with a fixed stride, so that no loop divides by the runtime block count (a
+// 64-bit division per block cost as much as a block's exponentials).
+struct BlockPos {
+  int i, c;
+  __device__ __forceinline__ BlockPos(int q0, int nb) : i(0), c(q0) {
+    while (c >= nb) { c -= nb; ++i; }
+  }
+  __device__ __forceinline__ void step(int by, int nb) {
+    c += by;
+    while (c >= nb) { c -= nb; ++i; }
+  }
 };
 
 // CTA (split p of unit bh) processes a contiguous range of point tiles.
@@ -140,7 +154,7 @@ __device__ __forceinline__ Work work_of(int64_t N, int splits) {
   const int64_t tiles = (N + kTile - 1) / kTile;
   const int p = blockIdx.x;
   w.tile0 = tiles * p / splits;
-  w.ntiles = tiles * (p + 1) / splits - w.tile0;
+  w.ntiles = (int)(tiles * (p + 1) / splits - w.tile0);
   return w;
 }
 
@@ -175,13 +189,13 @@ __device__ __forceinline__ void issue_logits(uint32_t tmem_d, uint32_t x_s, uint
   const uint64_t w0 = sdesc(wc, 16, 512, kSw64), w1 = sdesc(wc + 32, 16, 512, kSw64);
   const uint64_t we = sdesc(wec, 16, 256, kSw32);
   if (point_major) {
-    mma_ss(tmem_d, x0, w0, idesc, 0);
-    mma_ss(tmem_d, x1, w1, idesc, 1);
-    mma_ss(tmem_d, xe, we, idesc, 1);
+    mma_ss_w(tmem_d, x0, w0, idesc, 0);
+    mma_ss_w(tmem_d, x1, w1, idesc, 1);
+    mma_ss_w(tmem_d, xe, we, idesc, 1);
   } else {
-    mma_ss(tmem_d, w0, x0, idesc, 0);
-    mma_ss(tmem_d, w1, x1, idesc, 1);
-    mma_ss(tmem_d, we, xe, idesc, 1);
+    mma_ss_w(tmem_d, w0, x0, idesc, 0);
+    mma_ss_w(tmem_d, w1, x1, idesc, 1);
+    mma_ss_w(tmem_d, we, xe, idesc, 1);
   }
 }
 
@@ -221,10 +235,11 @@ __global__ void k_prep_px(const float* __restrict__ lse, uint4* __restrict__ px,
 // Deslice: out_n = sum_g w_ng z'_g.
 // smem: [W img G*96][Z' img G*64][stages: x | point extra (TMA half, zero half)][barriers]
 // TMEM: S buffers [0, 384); P x Z' accumulators O_0 [384, 448), O_1 [448, 512),
-// each double-buffered by tile parity.  Softmax warpgroup wg reads S columns
-// [64 wg, 64 wg + 64) and writes their bf16 weights, packed in pairs, into
-// columns [64 wg, 64 wg + 32) of the same buffer; warp 2 + wg turns exactly
-// those into its products (K-steps [4 wg, 4 wg + 4) of the block).
+// each double-buffered by tile parity.  Block q (tile q / nb, slot block q % nb)
+// uses S buffer q % 3 and softmax warpgroup q % 2, which writes the bf16 weights
+// of its 128 slots, packed in pairs, into columns [0, 64) of the same buffer;
+// warp 2 + j turns slots [64 j, 64 j + 64) of every block into products
+// (K-steps [4 j, 4 j + 4)) accumulated in O_j.
 // =========================================================================================
 constexpr uint32_t kDStage = kXBytes + 2 * kPxBytes;  // x tile, point extra (both halves)
 
@@ -257,7 +272,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int h = (int)(wk.bh % H);
   const int nch = G / kGC;
   constexpr uint32_t kO = kSBuf * kGC;  // TMEM column base of the O accumulators
-  const int64_t total = wk.ntiles * nch;
+  const int total = wk.ntiles * nch;
 
   if (threadIdx.x == 0) {
     mbar_init(wz_full, 1);
@@ -267,12 +282,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < kSBuf; i++) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&p_ready[i], 8);
+      mbar_init(&p_ready[i], 4);  // the four warps of the warpgroup that owns the block
       mbar_init(&pv_done[i], 2);
     }
     for (int i = 0; i < 2; i++) {
       mbar_init(&o_full[i], 2);
-      mbar_init(&o_free[i], 8);
+      mbar_init(&o_free[i], 4);
     }
     for (int i = 0; i < 3; i++) mbar_init(&drain[i], 1);
     ab->flag = 0;
@@ -294,9 +309,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_expect_tx(wz_full, wbytes + zbytes);
       load_images(s_w, wimg + (size_t)h * wbytes, wbytes, wz_full);
       load_images(s_z, zimg + (size_t)wk.bh * zbytes, zbytes, wz_full);
-      int64_t i = 0;
+      int i = 0;
       for (; i < wk.ntiles; i++) {
-        const int s = (int)(i % kStages);
+        const int s = i % kStages;
         if (i >= kStages && !mbar_wait(&x_empty[s], (uint32_t)(((i / kStages) - 1) & 1), ab, status)) break;
         const int n0 = (int)((wk.tile0 + i) * kTile);
         mbar_expect_tx(&x_full[s], kXBytes + kPxBytes);
@@ -304,7 +319,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_2d(s_x + s * kDStage + kXBytes, &pmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
       }
       // Drain: the newest load of each stage has landed before the CTA exits.
-      for (int64_t j = (i > kStages ? i - kStages : 0); j < i; j++)
+      for (int j = (i > kStages ? i - kStages : 0); j < i; j++)
         mbar_wait(&x_full[j % kStages], (uint32_t)((j / kStages) & 1), ab, nullptr, kWaitNs);
       mbar_wait(wz_full, 0, ab, nullptr, kWaitNs);
     }
@@ -312,53 +327,53 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------ logits issuer ------------------------------
     // Block q uses S buffer q % 3; it is rewritten only after the products of
     // block q - 3 (issued by the other warps) have completed.
-    if (lane == 0 && wk.ntiles > 0) {
+    if (wk.ntiles > 0) {
       const uint32_t sw = smem_u32(s_w), swe = sw + (uint32_t)G * 64;
-      bool ok = mbar_wait(wz_full, 0, ab, status);
-      for (int64_t q = 0; ok && q < total; q++) {
-        const int64_t i = q / nch;
-        const int c = (int)(q % nch);
-        const int s = (int)(i % kStages);
-        const int bb = (int)(q % kSBuf);
-        if (c == 0 && !(ok = mbar_wait(&x_full[s], (uint32_t)((i / kStages) & 1), ab, status))) break;
-        if (q >= kSBuf && !(ok = mbar_wait(&pv_done[bb], (uint32_t)(((q / kSBuf) - 1) & 1), ab, status))) break;
+      bool ok = mbar_wait_w(wz_full, 0, ab, status);
+      BlockPos pos(0, nch);
+      for (int q = 0; ok && q < total; q++, pos.step(1, nch)) {
+        const int i = pos.i, c = pos.c;
+        const int s = i % kStages;
+        const int bb = q % kSBuf;
+        if (c == 0 && !(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kStages) & 1), ab, status))) break;
+        if (q >= kSBuf && !(ok = mbar_wait_w(&pv_done[bb], (uint32_t)(((q / kSBuf) - 1) & 1), ab, status))) break;
         tc_fence_after();
         const uint32_t xs = smem_u32(s_x + s * kDStage);
         issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kXBytes), sw, swe, c, true);
-        mma_commit(&s_full[bb]);
-        if (c == nch - 1) mma_commit(&x_empty[s]);
+        mma_commit_w(&s_full[bb]);
+        if (c == nch - 1) mma_commit_w(&x_empty[s]);
       }
-      mma_commit(&drain[0]);
-      mbar_wait(&drain[0], 0, ab, nullptr, kWaitNs);
+      mma_commit_w(&drain[0]);
+      mbar_wait_w(&drain[0], 0, ab, nullptr, kWaitNs);
     }
   } else if (warp == 2 || warp == 3) {
     // ------------------------------ P x Z' issuers ------------------------------
     const int j = warp - 2;  // K-steps [4j, 4j + 4) of every block, accumulator O_j
-    if (lane == 0 && wk.ntiles > 0) {
+    if (wk.ntiles > 0) {
       constexpr uint32_t idesc_pv = idesc_bf16(128, kD, false, false);
       const uint32_t sz = smem_u32(s_z);
-      bool ok = mbar_wait(wz_full, 0, ab, status);
-      for (int64_t q = 0; ok && q < total; q++) {
-        const int64_t i = q / nch;
-        const int c = (int)(q % nch);
-        const int ob = (int)(i & 1);
-        const int bb = (int)(q % kSBuf);
-        if (c == 0 && i >= 2 && !(ok = mbar_wait(&o_free[ob], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
-        if (!(ok = mbar_wait(&p_ready[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
+      bool ok = mbar_wait_w(wz_full, 0, ab, status);
+      BlockPos pos(0, nch);
+      for (int q = 0; ok && q < total; q++, pos.step(1, nch)) {
+        const int i = pos.i, c = pos.c;
+        const int ob = i & 1;
+        const int bb = q % kSBuf;
+        if (c == 0 && i >= 2 && !(ok = mbar_wait_w(&o_free[ob], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
+        if (!(ok = mbar_wait_w(&p_ready[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t tP = tmem + (uint32_t)bb * kGC + (uint32_t)j * 64;
+        const uint32_t tP = tmem + (uint32_t)bb * kGC + (uint32_t)j * 32;  // weights of slots 64j.. (packed pairs)
         const uint32_t tO = tmem + kO + (uint32_t)(j * 2 + ob) * kD;
 #pragma unroll
         for (int kk = 0; kk < 4; kk++) {
           const int g0 = c * kGC + (4 * j + kk) * 16;
           const uint32_t zaddr = sz + (uint32_t)((g0 >> 6) * 4096 + (g0 & 63) * 2);
-          mma_ts(tO, tP + (uint32_t)kk * 8, sdesc(zaddr, 16, 1024, kSw128), idesc_pv, (c > 0 || kk > 0) ? 1u : 0u);
+          mma_ts_w(tO, tP + (uint32_t)kk * 8, sdesc(zaddr, 16, 1024, kSw128), idesc_pv, (c > 0 || kk > 0) ? 1u : 0u);
         }
-        mma_commit(&pv_done[bb]);
-        if (c == nch - 1) mma_commit(&o_full[ob]);
+        mma_commit_w(&pv_done[bb]);
+        if (c == nch - 1) mma_commit_w(&o_full[ob]);
       }
-      mma_commit(&drain[1 + j]);
-      mbar_wait(&drain[1 + j], 0, ab, nullptr, kWaitNs);
+      mma_commit_w(&drain[1 + j]);
+      mbar_wait_w(&drain[1 + j], 0, ab, nullptr, kWaitNs);
     }
   } else if (warp >= kSoftmaxWarp0) {
     // ------------------------------ softmax warpgroups ------------------------------
@@ -366,58 +381,65 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int wq = warp & 3;  // TMEM sub-partition of this warp
     const int r = wq * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
-    int64_t q = 0;
     bool ok = true;
-    // Output of tile t: this warpgroup's 16 channels of O_0 + O_1 -> bf16 -> global.
-    auto epilogue = [&](int64_t t) -> bool {
+    // Output of tile t: O_0 + O_1 (fixed order) -> bf16 -> global, 64 B per point.
+    auto epilogue = [&](int t) -> bool {
       const int ob = (int)(t & 1);
       if (!mbar_wait(&o_full[ob], (uint32_t)((t >> 1) & 1), ab, status)) return false;
       tc_fence_after();
-      uint32_t o0[16], o1[16];
-      tmem_ld16(tmem + lane_addr + kO + (uint32_t)ob * kD + (uint32_t)wg * 16, o0);
-      tmem_ld16(tmem + lane_addr + kO + (uint32_t)(2 + ob) * kD + (uint32_t)wg * 16, o1);
-      tmem_wait_ld(o0);
-      tmem_wait_ld(o1);
+      uint32_t o0[32], o1[32];
+      tmem_ld32(tmem + lane_addr + kO + (uint32_t)ob * kD, o0);
+      tmem_ld32(tmem + lane_addr + kO + (uint32_t)(2 + ob) * kD, o1);
+      tmem_wait_ld2(o0, o1);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&o_free[ob]);
       const int64_t n = (wk.tile0 + t) * kTile + r;
       if (n < N) {
-        float o[16];
+        uint4* dst = reinterpret_cast<uint4*>(out + ((b * N + n) * H + h) * kD);
 #pragma unroll
-        for (int k = 0; k < 16; k++) o[k] = __uint_as_float(o0[k]) + __uint_as_float(o1[k]);
-        uint4* dst = reinterpret_cast<uint4*>(out + ((b * N + n) * H + h) * kD + wg * 16);
+        for (int k = 0; k < 4; k++) {
+          uint32_t w[4];
 #pragma unroll
-        for (int k = 0; k < 2; k++)
-          dst[k] = make_uint4(pack_bf16(o[8 * k], o[8 * k + 1]), pack_bf16(o[8 * k + 2], o[8 * k + 3]),
-                              pack_bf16(o[8 * k + 4], o[8 * k + 5]), pack_bf16(o[8 * k + 6], o[8 * k + 7]));
+          for (int e = 0; e < 4; e++)
+            w[e] = pack_bf16(__uint_as_float(o0[8 * k + 2 * e]) + __uint_as_float(o1[8 * k + 2 * e]),
+                             __uint_as_float(o0[8 * k + 2 * e + 1]) + __uint_as_float(o1[8 * k + 2 * e + 1]));
+          dst[k] = make_uint4(w[0], w[1], w[2], w[3]);
+        }
       }
       return true;
     };
-    for (int64_t i = 0; ok && i < wk.ntiles; i++) {
-      for (int c = 0; c < nch; c++, q++) {
-        const int bb = (int)(q % kSBuf);
-        if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
-        tc_fence_after();
-        const uint32_t tS = tmem + lane_addr + (uint32_t)bb * kGC + (uint32_t)wg * 64;
+    // Warpgroup wg takes the whole blocks q with q % 2 == wg, so the two warpgroups
+    // run half a block out of phase: one exponentiates while the other waits.
+    BlockPos pos(wg, nch);
+    for (int q = wg; ok && q < total; q += 2, pos.step(2, nch)) {
+      const int i = pos.i, c = pos.c;
+      const int bb = q % kSBuf;
+      if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
+      tc_fence_after();
+      const uint32_t tS = tmem + lane_addr + (uint32_t)bb * kGC;
+#pragma unroll 1
+      for (int half = 0; half < 2; half++) {
+        // Columns [64 half, 64 half + 64) -> packed weights in columns [32 half, 32 half + 32),
+        // which this thread has already read.
         uint32_t v0[32], v1[32];
-        tmem_ld32(tS, v0);
-        tmem_ld32(tS + 32, v1);
+        tmem_ld32(tS + half * 64, v0);
+        tmem_ld32(tS + half * 64 + 32, v1);
         tmem_wait_ld2(v0, v1);
         uint32_t pk0[16], pk1[16];
         weights64(v0, v1, pk0, pk1);
-        tmem_st16(tS, pk0);
-        tmem_st16(tS + 16, pk1);
-        tmem_wait_st();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&p_ready[bb]);
-        // The output of the previous tile is drained after this tile's first block,
-        // when its last products have long finished.
-        if (c == 0 && i > 0 && !(ok = epilogue(i - 1))) break;
+        tmem_st16(tS + half * 32, pk0);
+        tmem_st16(tS + half * 32 + 16, pk1);
       }
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_ready[bb]);
+      // The output of the previous tile is drained by the warpgroup that took the
+      // first block of this tile, when the last products of that tile have long finished.
+      if (c == 0 && i > 0 && !(ok = epilogue(i - 1))) break;
     }
-    if (ok && wk.ntiles > 0) epilogue(wk.ntiles - 1);
+    if (ok && total > 0 && total % 2 == wg) epilogue(wk.ntiles - 1);
   }
   tc_fence_before();
   __syncthreads();
@@ -430,9 +452,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 // the point-extra row [1, 1, -lse2_hi, -lse2_lo, 0 x 4] (lse2 = lse*log2(e)) to
 // px[bh*Np + n] (Np = N rounded up to a whole tile; padded points get -1e30 so
 // that their weights vanish).
-// Two logits issuers (warp 1 + j issues the blocks c with c % 2 == j).  Each
-// softmax warpgroup keeps a running (max, sum) over its half of every block;
-// the halves are combined through shared memory at the end of a tile.
+// Two logits issuers and two softmax warpgroups: block q (tile q / nb, slot block
+// q % nb) goes through S buffer q % 2, issuer 1 + q % 2 and warpgroup q % 2.  Each
+// warpgroup keeps a running (max, sum) over the blocks it took; the two shares of
+// a tile are combined through shared memory by the one that took its last block.
 // smem: [W img G*96][x stages][constant extra][ml exchange][barriers]
 // TMEM: two S buffers [0, 256).
 // =========================================================================================
@@ -472,7 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; i++) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_free[i], 8);
+      mbar_init(&s_free[i], 4);
       mbar_init(&ml_full[i], 4);
       mbar_init(&ml_empty[i], 4);
     }
@@ -494,61 +517,72 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&xmap);
       mbar_expect_tx(w_full, wbytes);
       load_images(s_w, wimg + (size_t)h * wbytes, wbytes, w_full);
-      int64_t i = 0;
+      int i = 0;
       for (; i < wk.ntiles; i++) {
-        const int s = (int)(i % kStages);
+        const int s = i % kStages;
         if (i >= kStages && !mbar_wait(&x_empty[s], (uint32_t)(((i / kStages) - 1) & 1), ab, status)) break;
         mbar_expect_tx(&x_full[s], kXBytes);
         tma_load_3d(s_x + s * kXBytes, &xmap, h * kD, (int)((wk.tile0 + i) * kTile), (int)b, &x_full[s]);
       }
-      for (int64_t j = (i > kStages ? i - kStages : 0); j < i; j++)
+      for (int j = (i > kStages ? i - kStages : 0); j < i; j++)
         mbar_wait(&x_full[j % kStages], (uint32_t)((j / kStages) & 1), ab, nullptr, kWaitNs);
       mbar_wait(w_full, 0, ab, nullptr, kWaitNs);
     }
   } else if (warp == 1 || warp == 2) {
+    // With two or more blocks per tile, issuer j takes the blocks q with q % 2 == j
+    // (always S buffer j, so each buffer has one producer and one consumer and
+    // both issuers touch every tile); with one block per tile issuer 0 takes all.
     const int j = warp - 1;
-    if (lane == 0 && wk.ntiles > 0 && j < nch) {
+    const int nis = nch >= 2 ? 2 : 1;
+    if (wk.ntiles > 0 && j < nis) {
       const uint32_t sw = smem_u32(s_w), swe = sw + (uint32_t)G * 64;
-      bool ok = mbar_wait(w_full, 0, ab, status);
-      const int c_last = ((nch - 1 - j) / 2) * 2 + j;
-      const int64_t total = wk.ntiles * nch;
-      for (int64_t q = 0; ok && q < total; q++) {
-        const int64_t i = q / nch;
-        const int c = (int)(q % nch);
-        if ((c & 1) != j) continue;
-        const int s = (int)(i % kStages);
-        if (c == j && !(ok = mbar_wait(&x_full[s], (uint32_t)((i / kStages) & 1), ab, status))) break;
-        if (q >= 2 && !(ok = mbar_wait(&s_free[q & 1], (uint32_t)(((q >> 1) - 1) & 1), ab, status))) break;
+      bool ok = mbar_wait_w(w_full, 0, ab, status);
+      const int total = wk.ntiles * nch;
+      BlockPos pos(j, nch);
+      for (int q = j; ok && q < total; q += nis, pos.step(nis, nch)) {
+        const int i = pos.i, c = pos.c;
+        const int s = i % kStages;
+        const int bb = q & 1;
+        if (c < nis && !(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kStages) & 1), ab, status))) break;
+        if (q >= 2 && !(ok = mbar_wait_w(&s_free[bb], (uint32_t)(((q >> 1) - 1) & 1), ab, status))) break;
         tc_fence_after();
-        issue_logits(tmem + (uint32_t)(q & 1) * kGC, smem_u32(s_x + s * kXBytes), const_extra_desc(smem_u32(s_ex)), sw,
-                     swe, c, true);
-        mma_commit(&s_full[q & 1]);
-        if (c == c_last) mma_commit(&x_empty[s]);
+        issue_logits(tmem + (uint32_t)bb * kGC, smem_u32(s_x + s * kXBytes), const_extra_desc(smem_u32(s_ex)), sw, swe,
+                     c, true);
+        mma_commit_w(&s_full[bb]);
+        if (c >= nch - nis) mma_commit_w(&x_empty[s]);
       }
-      mma_commit(&drain[j]);
-      mbar_wait(&drain[j], 0, ab, nullptr, kWaitNs);
+      mma_commit_w(&drain[j]);
+      mbar_wait_w(&drain[j], 0, ab, nullptr, kWaitNs);
     }
   } else if (warp >= kSoftmaxWarp0) {
     const int wg = (warp - kSoftmaxWarp0) >> 2;
     const int wq = warp & 3;
     const int r = wq * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
-    int64_t q = 0;
+    const int total = wk.ntiles * nch;
     bool ok = true;
-    for (int64_t i = 0; ok && i < wk.ntiles; i++) {
-      const int64_t n = (wk.tile0 + i) * kTile + r;
-      float m = -INFINITY, l = 0.f;
-      for (int c = 0; c < nch; c++, q++) {
-        if (!(ok = mbar_wait(&s_full[q & 1], (uint32_t)((q >> 1) & 1), ab, status))) break;
-        tc_fence_after();
-        const uint32_t tS = tmem + lane_addr + (uint32_t)(q & 1) * kGC + (uint32_t)wg * (kGC / 2);
+    float m = -INFINITY, l = 0.f;
+    // Warpgroup wg takes the whole blocks q with q % 2 == wg (always S buffer wg), so
+    // the two run out of phase.  A tile's last block is taken by the warpgroup that
+    // finalises the tile; with two or more blocks per tile the other warpgroup hands
+    // over its (max, sum) over the blocks it took.
+    BlockPos pos(wg, nch);
+    for (int q = wg; ok && q < total; q += 2, pos.step(2, nch)) {
+      const int i = pos.i, c = pos.c;
+      if (!(ok = mbar_wait(&s_full[wg], (uint32_t)((q >> 1) & 1), ab, status))) break;
+      tc_fence_after();
+#pragma unroll 1
+      for (int half = 0; half < 2; half++) {
+        const uint32_t tS = tmem + lane_addr + (uint32_t)wg * kGC + (uint32_t)half * 64;
         uint32_t v0[32], v1[32];
         tmem_ld32(tS, v0);
         tmem_ld32(tS + 32, v1);
         tmem_wait_ld2(v0, v1);
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&s_free[q & 1]);
+        if (half == 1) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&s_free[wg]);
+        }
         // Block maximum as a tree of three-input maxima (short dependency chains).
         float t[22];
 #pragma unroll
@@ -563,34 +597,45 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float mn = max3(max3(t[0], t[1], t[2]), max3(t[3], t[4], t[5]), fmaxf(t[6], t[21]));
         const uint32_t nmb = __float_as_uint(-mn);
         const uint64_t nm2 = pack2(nmb, nmb);
-        float acc[8];
-#pragma unroll
-        for (int k = 0; k < 8; k++) acc[k] = 0.f;
+        // Paired (f32x2) subtraction and accumulation: half an FMA-pipe instruction
+        // per element for each.
+        uint64_t acc[4] = {0, 0, 0, 0};
 #pragma unroll
         for (int k = 0; k < 16; k++) {
           const uint64_t a = add2(pack2(v0[2 * k], v0[2 * k + 1]), nm2);
           const uint64_t bq = add2(pack2(v1[2 * k], v1[2 * k + 1]), nm2);
-          acc[k & 7] += ex2(lo_f(a)) + ex2(hi_f(a));
-          acc[(k + 4) & 7] += ex2(lo_f(bq)) + ex2(hi_f(bq));
+          acc[k & 3] = add2(acc[k & 3], pack2(__float_as_uint(ex2(lo_f(a))), __float_as_uint(ex2(hi_f(a)))));
+          acc[(k + 2) & 3] =
+              add2(acc[(k + 2) & 3], pack2(__float_as_uint(ex2(lo_f(bq))), __float_as_uint(ex2(hi_f(bq)))));
         }
-        const float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+        const uint64_t acc01 = add2(acc[0], acc[1]), acc23 = add2(acc[2], acc[3]);
+        const uint64_t acc4 = add2(acc01, acc23);
+        const float sum = lo_f(acc4) + hi_f(acc4);
         l = l * ex2(m - mn) + sum;
         m = mn;
       }
-      if (!ok) break;
-      const int pb = (int)(i & 1);
-      if (wg == 1) {
+      const int pb = i & 1;
+      if (c == nch - 2) {
+        // Hand over this warpgroup's share of tile i.
         if (i >= 2 && !(ok = mbar_wait(&ml_empty[pb], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
         s_ml[pb * kTile + r] = make_float2(m, l);
         __syncwarp();
         if (lane == 0) mbar_arrive(&ml_full[pb]);
-      } else {
-        if (!(ok = mbar_wait(&ml_full[pb], (uint32_t)((i >> 1) & 1), ab, status))) break;
-        const float2 o = s_ml[pb * kTile + r];
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&ml_empty[pb]);
-        const float M = fmaxf(m, o.x);
-        const float L = l * ex2(m - M) + o.y * ex2(o.x - M);
+        m = -INFINITY;
+        l = 0.f;
+      } else if (c == nch - 1) {
+        float M = m, L = l;
+        if (nch >= 2) {
+          if (!(ok = mbar_wait(&ml_full[pb], (uint32_t)((i >> 1) & 1), ab, status))) break;
+          const float2 o = s_ml[pb * kTile + r];
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&ml_empty[pb]);
+          M = fmaxf(m, o.x);
+          L = l * ex2(m - M) + o.y * ex2(o.x - M);
+        }
+        m = -INFINITY;
+        l = 0.f;
+        const int64_t n = (wk.tile0 + i) * kTile + r;
         const float lse2 = M + log2f(L);
         if (n < Np) {
           const float nl2 = n < N ? -lse2 : -1e30f;
@@ -623,9 +668,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 // Writes part[p][bh][g][0..32] = (U_g, S_g).
 // smem: [W img block 128*96][stages: x | F_lo F_hi ones | point extra (2 halves)][barriers]
 // TMEM: S buffers [0, 384); U|S accumulators A_0 [384, 432), A_1 [432, 480).
-// Warp 1 issues the logits; warp 2 + wg issues the products of points
-// [64 wg, 64 wg + 64) of every tile (the columns softmax warpgroup wg wrote)
-// into its own accumulator A_wg (the two are summed in a fixed order).
+// Warp 1 issues the logits of every tile; softmax warpgroup wg takes the whole
+// tiles i with i % 2 == wg, and warp 2 + wg issues their products into its own
+// accumulator A_wg (the two are summed in a fixed order).
 // =========================================================================================
 constexpr uint32_t kStageBytes = kXBytes + 3 * kFBlock + 2 * kPxBytes;  // x, [F | 1], point extra
 constexpr uint32_t kWBlock = 128 * 96;                                  // one 128-slot block of the W image
@@ -644,8 +689,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* x_full = bars + 1;
   uint64_t* st_empty = x_full + kSliceStages;
   uint64_t* s_full = st_empty + kSliceStages;
-  uint64_t* p_ready = s_full + kSBuf;
-  uint64_t* pv_done = p_ready + kSBuf;
+  uint64_t* p_ready = s_full + kSBuf;   // [issuer][S buffer]
+  uint64_t* pv_done = p_ready + 2 * kSBuf;
   uint64_t* acc_full = pv_done + kSBuf;
   uint64_t* drain = acc_full + 1;  // one per issuing warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 3);
@@ -662,12 +707,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(w_full, 1);
     for (int s = 0; s < kSliceStages; s++) {
       mbar_init(&x_full[s], 1);
-      mbar_init(&st_empty[s], 3);  // the logits issuer and both product issuers
+      mbar_init(&st_empty[s], 2);  // the logits issuer and the tile's product issuer
     }
     for (int i = 0; i < kSBuf; i++) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&p_ready[i], 8);
-      mbar_init(&pv_done[i], 2);
+      mbar_init(&p_ready[i], 4);  // the four warps of the warpgroup that took the tile
+      mbar_init(&p_ready[kSBuf + i], 4);
+      mbar_init(&pv_done[i], 1);
     }
     mbar_init(acc_full, 2);
     for (int i = 0; i < 3; i++) mbar_init(&drain[i], 1);
@@ -702,9 +748,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint8_t* src = wimg + (size_t)h * G * 96;
       load_images(s_w, src + (size_t)g_base * 64, kGC * 64, w_full);
       load_images(s_w + kGC * 64, src + (size_t)G * 64 + (size_t)g_base * 32, kGC * 32, w_full);
-      int64_t i = 0;
+      int i = 0;
       for (; i < wk.ntiles; i++) {
-        const int s = (int)(i % kSliceStages);
+        const int s = i % kSliceStages;
         if (i >= kSliceStages &&
             !mbar_wait(&st_empty[s], (uint32_t)(((i / kSliceStages) - 1) & 1), ab, status))
           break;
@@ -716,53 +762,54 @@ __global__ void __launch_bounds__(kThreads, 1)
         tma_load_3d(st + kFOff + kFBlock, &fmap, h * kD + 16, n0, (int)b, &x_full[s]);
         tma_load_2d(st + kPOff, &pmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
       }
-      for (int64_t j = (i > kSliceStages ? i - kSliceStages : 0); j < i; j++)
+      for (int j = (i > kSliceStages ? i - kSliceStages : 0); j < i; j++)
         mbar_wait(&x_full[j % kSliceStages], (uint32_t)((j / kSliceStages) & 1), ab, nullptr, kWaitNs);
       mbar_wait(w_full, 0, ab, nullptr, kWaitNs);
     }
   } else if (warp == 1) {
     // ------------------------------ logits issuer (transposed) ------------------------------
-    if (lane == 0) {
+    {
       const uint32_t sw = smem_u32(s_w), swe = sw + kGC * 64;
-      bool ok = mbar_wait(w_full, 0, ab, status);
-      for (int64_t i = 0; ok && i < wk.ntiles; i++) {
-        const int s = (int)(i % kSliceStages);
-        const int bb = (int)(i % kSBuf);
-        if (!(ok = mbar_wait(&x_full[s], (uint32_t)((i / kSliceStages) & 1), ab, status))) break;
-        if (i >= kSBuf && !(ok = mbar_wait(&pv_done[bb], (uint32_t)(((i / kSBuf) - 1) & 1), ab, status))) break;
+      bool ok = mbar_wait_w(w_full, 0, ab, status);
+      for (int i = 0; ok && i < wk.ntiles; i++) {
+        const int s = i % kSliceStages;
+        const int bb = i % kSBuf;
+        if (!(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kSliceStages) & 1), ab, status))) break;
+        if (i >= kSBuf && !(ok = mbar_wait_w(&pv_done[bb], (uint32_t)(((i / kSBuf) - 1) & 1), ab, status))) break;
         tc_fence_after();
         const uint32_t xs = smem_u32(s_st + s * kStageBytes);
         issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kPOff), sw, swe, 0, false);
-        mma_commit(&s_full[bb]);
-        mma_commit(&st_empty[s]);
+        mma_commit_w(&s_full[bb]);
+        mma_commit_w(&st_empty[s]);
       }
-      mma_commit(&drain[0]);
-      mbar_wait(&drain[0], 0, ab, nullptr, kWaitNs);
+      mma_commit_w(&drain[0]);
+      mbar_wait_w(&drain[0], 0, ab, nullptr, kWaitNs);
     }
   } else if (warp == 2 || warp == 3) {
     // ------------------------------ product issuers ------------------------------
-    const int j = warp - 2;  // points [64 j, 64 j + 64) of every tile, accumulator A_j
-    if (lane == 0) {
+    const int j = warp - 2;  // tiles i with i % 2 == j, accumulator A_j
+    {
       constexpr uint32_t idesc_sl = idesc_bf16(128, 48, false, true);
       bool ok = true;
-      for (int64_t i = 0; ok && i < wk.ntiles; i++) {
-        const int s = (int)(i % kSliceStages);
-        const int bb = (int)(i % kSBuf);
-        if (!(ok = mbar_wait(&p_ready[bb], (uint32_t)((i / kSBuf) & 1), ab, status))) break;
+      for (int i = j; ok && i < wk.ntiles; i += 2) {
+        const int s = i % kSliceStages;
+        const int bb = i % kSBuf;
+        // This issuer's tiles on buffer bb are 2 kSBuf apart.
+        if (!(ok = mbar_wait_w(&p_ready[j * kSBuf + bb], (uint32_t)((i / (2 * kSBuf)) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t tE = tmem + (uint32_t)bb * kGC + (uint32_t)j * 64;
-        const uint32_t fs = smem_u32(s_st + s * kStageBytes) + kFOff + (uint32_t)j * 2048;
+        const uint32_t tE = tmem + (uint32_t)bb * kGC;  // packed weights of the 128 points
+        const uint32_t fs = smem_u32(s_st + s * kStageBytes) + kFOff;
         const uint32_t tacc = tmem + kA + (uint32_t)j * 48;
 #pragma unroll
-        for (int kk = 0; kk < 4; kk++)
-          mma_ts(tacc, tE + (uint32_t)kk * 8, sdesc(fs + (uint32_t)kk * 512, kFBlock, 256, kSw32), idesc_sl,
-                 (i > 0 || kk > 0) ? 1u : 0u);
-        mma_commit(&pv_done[bb]);
-        mma_commit(&st_empty[s]);
+        for (int kk = 0; kk < 8; kk++)
+          mma_ts_w(tacc, tE + (uint32_t)kk * 8, sdesc(fs + (uint32_t)kk * 512, kFBlock, 256, kSw32), idesc_sl,
+                 (i >= 2 || kk > 0) ? 1u : 0u);
+        mma_commit_w(&pv_done[bb]);
+        mma_commit_w(&st_empty[s]);
       }
-      if (ok) mma_commit(acc_full);
-      mma_commit(&drain[1 + j]);
-      mbar_wait(&drain[1 + j], 0, ab, nullptr, kWaitNs);
+      if (ok) mma_commit_w(acc_full);
+      mma_commit_w(&drain[1 + j]);
+      mbar_wait_w(&drain[1 + j], 0, ab, nullptr, kWaitNs);
     }
   } else if (warp >= kSoftmaxWarp0) {
     const int wg = (warp - kSoftmaxWarp0) >> 2;
@@ -770,23 +817,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = wq * 32 + lane;  // TMEM lane: slot g_base + r
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     bool ok = true;
-    for (int64_t i = 0; ok && i < wk.ntiles; i++) {
-      const int bb = (int)(i % kSBuf);
+    // Warpgroup wg takes the whole tiles i with i % 2 == wg (out of phase with the other).
+    for (int i = wg; ok && i < wk.ntiles; i += 2) {
+      const int bb = i % kSBuf;
       if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((i / kSBuf) & 1), ab, status))) break;
       tc_fence_after();
-      const uint32_t tS = tmem + lane_addr + (uint32_t)bb * kGC + (uint32_t)wg * 64;
-      uint32_t v0[32], v1[32];
-      tmem_ld32(tS, v0);
-      tmem_ld32(tS + 32, v1);
-      tmem_wait_ld2(v0, v1);
-      uint32_t pk0[16], pk1[16];
-      weights64(v0, v1, pk0, pk1);
-      tmem_st16(tS, pk0);
-      tmem_st16(tS + 16, pk1);
+      const uint32_t tS = tmem + lane_addr + (uint32_t)bb * kGC;
+#pragma unroll 1
+      for (int half = 0; half < 2; half++) {
+        // Points [64 half, 64 half + 64) -> packed weights in columns [32 half, 32 half + 32),
+        // which this thread has already read.
+        uint32_t v0[32], v1[32];
+        tmem_ld32(tS + half * 64, v0);
+        tmem_ld32(tS + half * 64 + 32, v1);
+        tmem_wait_ld2(v0, v1);
+        uint32_t pk0[16], pk1[16];
+        weights64(v0, v1, pk0, pk1);
+        tmem_st16(tS + half * 32, pk0);
+        tmem_st16(tS + half * 32 + 16, pk1);
+      }
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&p_ready[bb]);
+      if (lane == 0) mbar_arrive(&p_ready[wg * kSBuf + bb]);
     }
     // Epilogue: the accumulators of this CTA's slot block -> partials
     // (warpgroup 0 the numerators U, warpgroup 1 the weight sums S).
@@ -794,20 +847,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     float* o = part + (((int64_t)blockIdx.x * BH + wk.bh) * G + g_base + r) * (kD + 1);
     if (ok && wk.ntiles > 0 && mbar_wait(acc_full, 0, ab, status)) {
       tc_fence_after();
+      const bool two = wk.ntiles >= 2;  // A_1 holds tiles only when there are two (else unwritten)
       if (wg == 0) {
         uint32_t u0[32], u1[32];
         tmem_ld32(tmem + lane_addr + kA, u0);
         tmem_ld32(tmem + lane_addr + kA + 48, u1);
         tmem_wait_ld2(u0, u1);
 #pragma unroll
-        for (int k = 0; k < kD; k++) o[k] = __uint_as_float(u0[k]) + __uint_as_float(u1[k]);
+        for (int k = 0; k < kD; k++) o[k] = two ? __uint_as_float(u0[k]) + __uint_as_float(u1[k]) : __uint_as_float(u0[k]);
       } else {
         uint32_t s0[16], s1[16];
         tmem_ld16(tmem + lane_addr + kA + 32, s0);
         tmem_ld16(tmem + lane_addr + kA + 48 + 32, s1);
         tmem_wait_ld(s0);
         tmem_wait_ld(s1);
-        o[kD] = __uint_as_float(s0[0]) + __uint_as_float(s1[0]);
+        o[kD] = two ? __uint_as_float(s0[0]) + __uint_as_float(s1[0]) : __uint_as_float(s0[0]);
       }
     } else if (ok && wk.ntiles == 0) {
       if (wg == 0)
@@ -925,7 +979,10 @@ cudaError_t run_stats(const Shape& s, const void* x, const uint8_t* wimg, float*
 }  // namespace
 
 bool tc_forward_supported(const Shape& s) {
-  return s.dtype == FS_BF16 && s.d == kD && s.G % kGC == 0 && s.G <= 1024 && s.N >= 1 && encode_fn() != nullptr;
+  // TMA coordinates and the kernels' block counters are 32-bit.
+  const int64_t np = (s.N + kTile - 1) / kTile * kTile;
+  return s.dtype == FS_BF16 && s.d == kD && s.G % kGC == 0 && s.G <= 1024 && s.N >= 1 &&
+         s.BH() * np < (int64_t(1) << 31) && encode_fn() != nullptr;
 }
 
 int tc_forward_launch_count(const Shape&) {

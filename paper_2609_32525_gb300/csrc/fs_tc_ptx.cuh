@@ -226,6 +226,41 @@ __device__ __forceinline__ void mma_commit(uint64_t* bar) {
                : "memory");
 }
 
+// ---- warp-converged issue ---------------------------------------------------------------
+// The MMA-issuing roles run as whole, converged warps and let elect.sync pick the
+// lane that issues each tcgen05 instruction.  Measured on GB300, a converged warp
+// issues a small tcgen05.mma in ~25 cycles, a lone lane inside a divergent branch
+// in ~50-130.  With the full mask elect.sync picks the same lane every time, so
+// that lane's commits cover every MMA the warp issued.
+__device__ __forceinline__ void mma_ss_w(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p, e;\n setp.ne.b32 p, %4, 0;\n elect.sync _|e, 0xffffffff;\n"
+      " @e tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_ts_w(uint32_t d_tmem, uint32_t a_tmem, uint64_t b_desc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p, e;\n setp.ne.b32 p, %4, 0;\n elect.sync _|e, 0xffffffff;\n"
+      " @e tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit_w(uint64_t* bar) {
+  asm volatile(
+      "{\n .reg .pred e;\n elect.sync _|e, 0xffffffff;\n"
+      " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];\n}\n" ::"r"(smem_u32(bar))
+      : "memory");
+}
+// Bounded wait by a whole warp; the outcome is made warp-uniform so that the warp
+// stays converged (a lane that gave up makes the whole warp give up).
+__device__ __forceinline__ bool mbar_wait_w(uint64_t* bar, uint32_t parity, Abort* ab, uint32_t* status,
+                                            uint64_t limit_ns = 2000000000ull) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, ab, status, limit_ns));
+}
+
 // Shared-memory matrix descriptor (tcgen05 format).
 //   swizzle: 0 none, 2 128B, 4 64B, 6 32B.  lbo/sbo in bytes.
 __device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo, uint32_t swizzle) {
