@@ -67,7 +67,8 @@ typedef enum fs_status {
   FS_ERR_UNSUPPORTED = 2, /* well-formed shape that no kernel implements (e.g. d = 48) */
   FS_ERR_CUDA = 3,        /* a CUDA runtime call or kernel launch failed */
   FS_ERR_TIMEOUT = 4,     /* device: a bounded wait gave up (status word only) */
-  FS_ERR_BAD_TAU = 5      /* device: some tau[h] <= 0 or not finite (status word only) */
+  FS_ERR_BAD_TAU = 5,     /* device: some tau[h] <= 0 or not finite (status word only) */
+  FS_ERR_SCRATCH_TOO_SMALL = 6 /* fs_slice_fwd_noalloc: the shape needs more than its fixed scratch */
 } fs_status;
 
 typedef enum fs_dtype { FS_F32 = 0, FS_BF16 = 1 } fs_dtype;
@@ -150,6 +151,36 @@ fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx,
                        const float* d_tokens, void* dx_mid, void* dfx, float* dW,
                        float* dbias, float* dtau, int accumulate, void* ws,
                        size_t ws_bytes, fs_stream_t stream);
+
+/* Fixed-scratch variant of fs_slice_fwd.  The paper has no counterpart.
+ *
+ * For callers that cannot give the library device memory at the call site: a
+ * program that lays out all of its device memory once at start-up and may not
+ * allocate afterwards, or a caller (a plain C host, a foreign-language binding)
+ * that holds no device allocator of its own.  Instead of a workspace argument,
+ * this entry point uses one scratch buffer of FS_NOALLOC_SCRATCH_BYTES that is
+ * part of the library's device code (a static device array), so neither the
+ * caller nor the library allocates anything for the call.
+ *   - Arguments, outputs and numerics are those of fs_slice_fwd (it runs the
+ *     same kernels).  A shape whose fs_workspace_bytes(s, FS_OP_SLICE_FWD)
+ *     exceeds FS_NOALLOC_SCRATCH_BYTES is rejected with
+ *     FS_ERR_SCRATCH_TOO_SMALL before anything is launched; invalid or
+ *     unsupported shapes give fs_slice_fwd's errors.
+ *   - The first call on a device (with that device current) looks up the
+ *     scratch's device address through the CUDA runtime; later calls on that
+ *     device reuse it.  Make that first call before any stream capture begins.
+ *   - Each call clears the status word at the start of the scratch; nothing
+ *     else in the scratch has to start at zero.
+ *   - There is ONE scratch per device.  Calls that can overlap in time (on
+ *     different streams, or from different host threads) race on it and
+ *     corrupt each other's results: serialise them.
+ *   - scratch: if not NULL, receives the scratch's device address, which
+ *     fs_device_status accepts to read the call's device status. */
+#define FS_NOALLOC_SCRATCH_BYTES ((size_t)16 << 20)
+fs_status fs_slice_fwd_noalloc(const fs_shape* s, const void* x_mid, const void* fx,
+                               const float* W_slice, const float* bias, const float* tau,
+                               float* tokens, float* wsum, float* lse, int finalize,
+                               const void** scratch, fs_stream_t stream);
 
 /* Synchronises `stream` and returns the device status word of `ws`
  * (FS_OK, FS_ERR_TIMEOUT or FS_ERR_BAD_TAU), or FS_ERR_CUDA. */

@@ -150,6 +150,8 @@ const char* fs_status_string(fs_status st) {
     case FS_ERR_CUDA: return "FS_ERR_CUDA: CUDA runtime or launch failure";
     case FS_ERR_TIMEOUT: return "FS_ERR_TIMEOUT: device wait gave up";
     case FS_ERR_BAD_TAU: return "FS_ERR_BAD_TAU: tau <= 0 or not finite";
+    case FS_ERR_SCRATCH_TOO_SMALL:
+      return "FS_ERR_SCRATCH_TOO_SMALL: the shape needs more than the fixed scratch of fs_slice_fwd_noalloc";
   }
   return "unknown fs_status";
 }

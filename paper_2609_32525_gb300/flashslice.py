@@ -25,13 +25,14 @@ if not os.path.exists(_LIB_PATH):
                       "(the library has no CPU fallback)")
 _lib = ctypes.CDLL(_LIB_PATH)
 
-FS_OK, FS_ERR_INVALID, FS_ERR_UNSUPPORTED, FS_ERR_CUDA, FS_ERR_TIMEOUT, FS_ERR_BAD_TAU = range(6)
+FS_OK, FS_ERR_INVALID, FS_ERR_UNSUPPORTED, FS_ERR_CUDA, FS_ERR_TIMEOUT, FS_ERR_BAD_TAU, FS_ERR_SCRATCH_TOO_SMALL = range(7)
+FS_NOALLOC_SCRATCH_BYTES = 16 << 20
 FS_F32, FS_BF16 = 0, 1
 FS_OP_SLICE_FWD, FS_OP_DESLICE_FWD, FS_OP_DESLICE_BWD, FS_OP_SLICE_BWD = range(4)
 
 EXPORTED = ("fs_workspace_bytes", "fs_slice_fwd", "fs_slice_finalize", "fs_mix", "fs_deslice_fwd",
             "fs_deslice_bwd", "fs_mix_bwd", "fs_slice_bwd", "fs_device_status", "fs_status_string",
-            "fs_path_for_shape", "fs_forward_launch_count")
+            "fs_path_for_shape", "fs_forward_launch_count", "fs_slice_fwd_noalloc")
 
 
 class fs_shape(ctypes.Structure):
@@ -62,6 +63,7 @@ _sig = {
     "fs_status_string": (ctypes.c_char_p, [_I]),
     "fs_path_for_shape": (_I, [_S]),
     "fs_forward_launch_count": (_I, [_S]),
+    "fs_slice_fwd_noalloc": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _I, ctypes.POINTER(_P), _P]),
 }
 for _name, (_res, _args) in _sig.items():
     _f = getattr(_lib, _name)
@@ -167,6 +169,22 @@ def fs_slice_bwd(shape, x_mid, fx, W_slice, bias, tau, tokens, wsum, lse, d_toke
 
 def fs_device_status(ws, stream=None) -> int:
     return int(_lib.fs_device_status(_ptr(ws), _stream(stream)))
+
+
+def fs_slice_fwd_noalloc(shape, x_mid, fx, W_slice, bias, tau, tokens, wsum, lse, finalize, stream=None) -> int:
+    """fs_slice_fwd on the library's fixed device scratch (no workspace argument, nothing
+    allocated).  Returns the scratch's device address, for device_status_at."""
+    addr = _P()
+    st = _lib.fs_slice_fwd_noalloc(ctypes.byref(shape), _ptr(x_mid), _ptr(fx), _ptr(W_slice), _ptr(bias),
+                                   _ptr(tau), _ptr(tokens), _ptr(wsum), _ptr(lse), int(bool(finalize)),
+                                   ctypes.byref(addr), _stream(stream))
+    _check("fs_slice_fwd_noalloc", st)
+    return int(addr.value)
+
+
+def device_status_at(addr: int, stream=None) -> int:
+    """fs_device_status of a scratch given by its device address."""
+    return int(_lib.fs_device_status(_P(addr), _stream(stream)))
 
 
 # ---- convenience: one coupling, buffers allocated through torch ----------------------------
