@@ -172,6 +172,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--ref-points", type=int, default=16384)
+    ap.add_argument("--points", type=int, default=None,
+                    help="profiling runs only: the workload's recipe at a smaller N (the line says so)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -199,7 +201,7 @@ def main():
     from paper_2609_32525_gb300 import flashslice as fs
     from paper_2609_32525_gb300.workloads import make_named
 
-    wl = make_named(args.workload)
+    wl = make_named(args.workload, n_override=args.points)
     tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
 
     def put(a, dt):
@@ -312,6 +314,19 @@ def main():
                 "call_ms": {"fs_slice_fwd": slice_ms, "fs_mix": mix_ms, "fs_deslice_fwd": desl_ms},
                 "per_call_work": "4*C*G flops per point for each of slice and deslice (C=256)"}
 
+    # The kernels are bound by the exponentials (one per point, head and slot in each
+    # of the three sweeps: statistics, slice, deslice), so the MUFU rate is reported
+    # beside the tensor roofline: 32 ex2 per clock per SM (measured on GB300).
+    n_exp = float(wl.B * wl.N * wl.H * wl.G)
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    mufu_peak = 32.0 * sms * float(clocks.get("sm_mhz") or 2070.0) * 1e6 / 1e9
+    exps = {"fs_slice_fwd": 2 * n_exp, "fs_deslice_fwd": n_exp}
+    call_ms = {"fs_slice_fwd": slice_ms, "fs_deslice_fwd": desl_ms}
+    roofline["mufu"] = {"unit": "Gexp/s", "peak": mufu_peak, "exps_per_call": exps,
+                        "achieved": {k: exps[k] / (call_ms[k] * 1e-3) / 1e9 for k in exps},
+                        "frac": {k: exps[k] / (call_ms[k] * 1e-3) / 1e9 / mufu_peak for k in exps},
+                        "step_frac": 3 * n_exp / (ms_per_step * 1e-3) / 1e9 / mufu_peak}
+
     launches = fs.forward_launch_count(s) * args.steps
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
@@ -320,7 +335,9 @@ def main():
             "config": {"workload": wl.name, "B": wl.B, "N": wl.N, "H": wl.H, "d": wl.d, "G": wl.G,
                        "step": "fs_slice_fwd + fs_mix + fs_deslice_fwd", "parallelism": f"replicas x{world}",
                        "l2": "inputs 2 x %d MiB > 129 MB L2, no flush" % (hx.numel() * hx.element_size() >> 20),
-                       "path": ["simt", "tcgen05"][fs.path_for_shape(s)]},
+                       "path": ["simt", "tcgen05"][fs.path_for_shape(s)],
+                       **({"points_override": "N reduced for profiling; not the benchmark workload"}
+                          if args.points else {})},
             "clocks": clocks, "gpu_launches": launches, "roofline": roofline,
             "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "ms_per_step": e2e_ms}}

@@ -148,11 +148,10 @@ struct BlockPos {
 };
 
 // CTA (split p of unit bh) processes a contiguous range of point tiles.
-__device__ __forceinline__ Work work_of(int64_t N, int splits) {
+__device__ __forceinline__ Work work_of(int64_t N, int splits, int p, int64_t bh) {
   Work w;
-  w.bh = blockIdx.y;
+  w.bh = bh;
   const int64_t tiles = (N + kTile - 1) / kTile;
-  const int p = blockIdx.x;
   w.tile0 = tiles * p / splits;
   w.ntiles = (int)(tiles * (p + 1) / splits - w.tile0);
   return w;
@@ -267,7 +266,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const Work wk = work_of(N, splits);
+  const Work wk = work_of(N, splits, blockIdx.x, blockIdx.y);
   const int64_t b = wk.bh / H;
   const int h = (int)(wk.bh % H);
   const int nch = G / kGC;
@@ -482,7 +481,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const Work wk = work_of(N, splits);
+  const Work wk = work_of(N, splits, blockIdx.x, blockIdx.y);
   const int64_t b = wk.bh / H;
   const int h = (int)(wk.bh % H);
   const int nch = G / kGC;
@@ -679,7 +678,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     k_slice(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap fmap,
             const __grid_constant__ CUtensorMap pmap, const uint8_t* __restrict__ wimg, float* __restrict__ part,
             int64_t N, int64_t Np, int H, int G, int splits, uint32_t* status) {
-  const int g_base = blockIdx.z * kGC;  // slot block
+  // Grid (slot block, point split, bh): the CTAs of all slot blocks of one point
+  // range are adjacent in launch order, run together and share each x / F tile
+  // through L2 instead of re-reading it from DRAM once per slot block.
+  const int g_base = blockIdx.x * kGC;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* s_w = smem;
@@ -697,7 +699,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const Work wk = work_of(N, splits);
+  const Work wk = work_of(N, splits, blockIdx.y, blockIdx.z);
   const int64_t b = wk.bh / H;
   const int h = (int)(wk.bh % H);
   constexpr uint32_t kA = kSBuf * kGC;  // TMEM column base of the accumulators
@@ -843,8 +845,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     // Epilogue: the accumulators of this CTA's slot block -> partials
     // (warpgroup 0 the numerators U, warpgroup 1 the weight sums S).
-    const int64_t BH = gridDim.y;
-    float* o = part + (((int64_t)blockIdx.x * BH + wk.bh) * G + g_base + r) * (kD + 1);
+    const int64_t BH = gridDim.z;
+    float* o = part + (((int64_t)blockIdx.y * BH + wk.bh) * G + g_base + r) * (kD + 1);
     if (ok && wk.ntiles > 0 && mbar_wait(acc_full, 0, ab, status)) {
       tc_fence_after();
       const bool two = wk.ntiles >= 2;  // A_1 holds tiles only when there are two (else unwritten)
@@ -1023,7 +1025,7 @@ cudaError_t tc_slice_fwd(const Shape& s, const void* x, const void* f, const flo
   if (!make_point_map(&fmap, f, s, 16, CU_TENSOR_MAP_SWIZZLE_32B)) return cudaErrorInvalidValue;
   if (!make_px_map(&pmap, px, s.BH(), padded_n(s))) return cudaErrorInvalidValue;
   const int R = slice_blocks(s), P = slice_splits(s);
-  dim3 grid((unsigned)P, (unsigned)s.BH(), (unsigned)R);
+  dim3 grid((unsigned)R, (unsigned)P, (unsigned)s.BH());
   const size_t sm = smem_slice();
   if ((e = set_smem(k_slice, sm)) != cudaSuccess) return e;
   k_slice<<<grid, kThreads, sm, st>>>(xmap, fmap, pmap, wimg, part, s.N, padded_n(s), s.H, s.G, P, status);
