@@ -46,6 +46,33 @@ def _peaks():
     return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
 
 
+# DRAM traffic per C-ABI call at the full large_g_bf16 workload (N = 1,048,576).
+# Source: ncu dram__bytes_read.sum + dram__bytes_write.sum of each call's kernels,
+# captured at N = 262,144. The point-proportional kernels (stats, slice, px rows,
+# deslice) are scaled x4; the W/Z' images and the split-partial reduction are not.
+# Valid only for the kernel sources it was measured on, identified by their SHA-1.
+# When the sources change the figure is reported as null.
+_TRAFFIC = {"sources_sha1": "14986c1bd32fe0accef1bfc52d8f31446faac26d", "workload": "large_g_bf16", "N": 1048576,
+            "fs_slice_fwd": 2.4199e9, "fs_deslice_fwd": 1.0659e9}
+
+
+def _sources_sha1():
+    import glob
+    import hashlib
+
+    h = hashlib.sha1()
+    for f in sorted(glob.glob(os.path.join(ROOT, "paper_2609_32525_gb300", "csrc", "*"))):
+        if f.endswith((".cu", ".cuh", ".h")):
+            h.update(open(f, "rb").read())
+    return h.hexdigest()
+
+
+def _traffic(wl, call):
+    if wl.name != _TRAFFIC["workload"] or wl.N != _TRAFFIC["N"] or _sources_sha1() != _TRAFFIC["sources_sha1"]:
+        return None
+    return _TRAFFIC[call]
+
+
 def _algorithmic(wl):
     """Algorithmic work of one forward (per point, all heads; C = H*d):
     flops 8*C*G (logits twice, slice accumulate, deslice apply), bytes 4*C*e
@@ -307,7 +334,8 @@ def main():
     achieved_tf = alg["flops_per_call"] / (dom_ms * 1e-3) / 1e12
     roof_t = max(alg["flops"] / (peaks["bf16_tflops"] * 1e12), alg["bytes"] / (peaks["hbm_gbs"] * 1e9))
     roofline = {"bound": "tensor", "achieved": achieved_tf, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
-                "frac": achieved_tf / peaks["bf16_tflops"], "traffic": None, "kernel": dom_name,
+                "frac": achieved_tf / peaks["bf16_tflops"], "traffic": _traffic(wl, dom_name), "kernel": dom_name,
+                "traffic_unit": "bytes per call (ncu DRAM read + write)",
                 "peak_source": peaks["source"] + " bf16 burst",
                 "frac_sustained": achieved_tf / peaks["bf16_tflops_sustained"],
                 "step_frac": roof_t / (ms_per_step * 1e-3),
