@@ -64,7 +64,7 @@ constexpr int kGC = 128;          // slots per logits block
 constexpr int kD = 32;            // head width of the tensor-core path
 constexpr int kSoftmaxWarp0 = 4;  // warps 4..11: two softmax warpgroups
 constexpr int kStages = 3;        // x-tile pipeline depth (stats / deslice)
-constexpr int kSliceStages = 5;   // slice pipeline depth
+constexpr int kSliceStages = 8;   // slice pipeline depth (it streams x, F and px for every 128 slots)
 constexpr int kSBuf = 3;          // S buffers (logits run up to two blocks ahead)
 constexpr uint32_t kXBytes = kTile * 64;   // 128 points x 32 bf16
 constexpr uint32_t kExBytes = kTile * 32;  // 128 rows x 16 bf16
@@ -207,13 +207,28 @@ __device__ __forceinline__ void load_images(uint8_t* dst, const uint8_t* src, ui
   }
 }
 
-// 2^t for 64 log2-weights -> 32 bf16x2 words.
-__device__ __forceinline__ void weights64(const uint32_t (&v0)[32], const uint32_t (&v1)[32], uint32_t (&p0)[16],
-                                          uint32_t (&p1)[16]) {
+// 2^t for 32 log2-weights -> 16 bf16x2 words.
+__device__ __forceinline__ void weights32(const uint32_t (&v)[32], uint32_t (&p)[16]) {
 #pragma unroll
-  for (int k = 0; k < 16; k++) {
-    p0[k] = pack_bf16(ex2(__uint_as_float(v0[2 * k])), ex2(__uint_as_float(v0[2 * k + 1])));
-    p1[k] = pack_bf16(ex2(__uint_as_float(v1[2 * k])), ex2(__uint_as_float(v1[2 * k + 1])));
+  for (int k = 0; k < 16; k++) p[k] = pack_bf16(ex2(__uint_as_float(v[2 * k])), ex2(__uint_as_float(v[2 * k + 1])));
+}
+
+// The 128 log2-weights of one TMEM lane of an S buffer -> bf16 weights written back
+// in place, packed in pairs, into the first 64 columns, in two halves: columns
+// [64 h, 64 h + 64) -> packed weights in columns [32 h, 32 h + 32), which this
+// thread has already read.
+__device__ __forceinline__ void weights_in_halves(uint32_t tS) {
+#pragma unroll 1
+  for (int half = 0; half < 2; half++) {
+    uint32_t v0[32], v1[32];
+    tmem_ld32(tS + half * 64, v0);
+    tmem_ld32(tS + half * 64 + 32, v1);
+    tmem_wait_ld2(v0, v1);
+    uint32_t pk0[16], pk1[16];
+    weights32(v0, pk0);
+    weights32(v1, pk1);
+    tmem_st16(tS + half * 32, pk0);
+    tmem_st16(tS + half * 32 + 16, pk1);
   }
 }
 
@@ -416,20 +431,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int bb = q % kSBuf;
       if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
       tc_fence_after();
-      const uint32_t tS = tmem + lane_addr + (uint32_t)bb * kGC;
-#pragma unroll 1
-      for (int half = 0; half < 2; half++) {
-        // Columns [64 half, 64 half + 64) -> packed weights in columns [32 half, 32 half + 32),
-        // which this thread has already read.
-        uint32_t v0[32], v1[32];
-        tmem_ld32(tS + half * 64, v0);
-        tmem_ld32(tS + half * 64 + 32, v1);
-        tmem_wait_ld2(v0, v1);
-        uint32_t pk0[16], pk1[16];
-        weights64(v0, v1, pk0, pk1);
-        tmem_st16(tS + half * 32, pk0);
-        tmem_st16(tS + half * 32 + 16, pk1);
-      }
+      weights_in_halves(tmem + lane_addr + (uint32_t)bb * kGC);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
@@ -570,49 +572,55 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int i = pos.i, c = pos.c;
       if (!(ok = mbar_wait(&s_full[wg], (uint32_t)((q >> 1) & 1), ab, status))) break;
       tc_fence_after();
-#pragma unroll 1
-      for (int half = 0; half < 2; half++) {
-        const uint32_t tS = tmem + lane_addr + (uint32_t)wg * kGC + (uint32_t)half * 64;
-        uint32_t v0[32], v1[32];
-        tmem_ld32(tS, v0);
-        tmem_ld32(tS + 32, v1);
-        tmem_wait_ld2(v0, v1);
-        if (half == 1) {
-          tc_fence_before();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&s_free[wg]);
-        }
-        // Block maximum as a tree of three-input maxima (short dependency chains).
-        float t[22];
+      // The whole row of the block (128 logits) into registers, then S goes back to
+      // the issuer at once; the maximum, the 128 exponentials (independent, issued
+      // back to back) and a pairwise sum follow.
+      const uint32_t tS = tmem + lane_addr + (uint32_t)wg * kGC;
+      uint32_t v[4][32];
+      tmem_ld32(tS, v[0]);
+      tmem_ld32(tS + 32, v[1]);
+      tmem_ld32(tS + 64, v[2]);
+      tmem_ld32(tS + 96, v[3]);
+      tmem_wait_ld2(v[0], v[1]);
+      tmem_wait_ld2(v[2], v[3]);  // ties the other half's registers after the (already complete) wait
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&s_free[wg]);
+      float t[43];
 #pragma unroll
-        for (int k = 0; k < 10; k++) {
-          t[k] = max3(__uint_as_float(v0[3 * k]), __uint_as_float(v0[3 * k + 1]), __uint_as_float(v0[3 * k + 2]));
-          t[10 + k] = max3(__uint_as_float(v1[3 * k]), __uint_as_float(v1[3 * k + 1]), __uint_as_float(v1[3 * k + 2]));
-        }
-        t[20] = max3(__uint_as_float(v0[30]), __uint_as_float(v0[31]), __uint_as_float(v1[30]));
-        t[21] = fmaxf(__uint_as_float(v1[31]), m);
+      for (int k = 0; k < 42; k++)
+        t[k] = max3(__uint_as_float(v[(3 * k) >> 5][(3 * k) & 31]), __uint_as_float(v[(3 * k + 1) >> 5][(3 * k + 1) & 31]),
+                    __uint_as_float(v[(3 * k + 2) >> 5][(3 * k + 2) & 31]));
+      t[42] = max3(__uint_as_float(v[3][30]), __uint_as_float(v[3][31]), m);
 #pragma unroll
-        for (int k = 0; k < 7; k++) t[k] = max3(t[3 * k], t[3 * k + 1], t[3 * k + 2]);
-        const float mn = max3(max3(t[0], t[1], t[2]), max3(t[3], t[4], t[5]), fmaxf(t[6], t[21]));
-        const uint32_t nmb = __float_as_uint(-mn);
-        const uint64_t nm2 = pack2(nmb, nmb);
-        // Paired (f32x2) subtraction and accumulation: half an FMA-pipe instruction
-        // per element for each.
-        uint64_t acc[4] = {0, 0, 0, 0};
+      for (int k = 0; k < 14; k++) t[k] = max3(t[3 * k], t[3 * k + 1], t[3 * k + 2]);
+      t[14] = t[42];
+#pragma unroll
+      for (int k = 0; k < 5; k++) t[k] = max3(t[3 * k], t[3 * k + 1], t[3 * k + 2]);
+      const float mn = max3(max3(t[0], t[1], t[2]), t[3], t[4]);
+      const uint32_t nmb = __float_as_uint(-mn);
+      const uint64_t nm2 = pack2(nmb, nmb);
+      // Paired (f32x2) subtraction, then every exponential, then a pairwise f32x2 sum.
+#pragma unroll
+      for (int j = 0; j < 4; j++)
 #pragma unroll
         for (int k = 0; k < 16; k++) {
-          const uint64_t a = add2(pack2(v0[2 * k], v0[2 * k + 1]), nm2);
-          const uint64_t bq = add2(pack2(v1[2 * k], v1[2 * k + 1]), nm2);
-          acc[k & 3] = add2(acc[k & 3], pack2(__float_as_uint(ex2(lo_f(a))), __float_as_uint(ex2(hi_f(a)))));
-          acc[(k + 2) & 3] =
-              add2(acc[(k + 2) & 3], pack2(__float_as_uint(ex2(lo_f(bq))), __float_as_uint(ex2(hi_f(bq)))));
+          const uint64_t a = add2(pack2(v[j][2 * k], v[j][2 * k + 1]), nm2);
+          v[j][2 * k] = __float_as_uint(ex2(lo_f(a)));
+          v[j][2 * k + 1] = __float_as_uint(ex2(hi_f(a)));
         }
-        const uint64_t acc01 = add2(acc[0], acc[1]), acc23 = add2(acc[2], acc[3]);
-        const uint64_t acc4 = add2(acc01, acc23);
-        const float sum = lo_f(acc4) + hi_f(acc4);
-        l = l * ex2(m - mn) + sum;
-        m = mn;
-      }
+      uint64_t acc[16];
+#pragma unroll
+      for (int k = 0; k < 16; k++)
+        acc[k] = add2(add2(pack2(v[0][2 * k], v[0][2 * k + 1]), pack2(v[1][2 * k], v[1][2 * k + 1])),
+                      add2(pack2(v[2][2 * k], v[2][2 * k + 1]), pack2(v[3][2 * k], v[3][2 * k + 1])));
+#pragma unroll
+      for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+        for (int k = 0; k < w; k++) acc[k] = add2(acc[k], acc[k + w]);
+      const float sum = lo_f(acc[0]) + hi_f(acc[0]);
+      l = l * ex2(m - mn) + sum;
+      m = mn;
       const int pb = i & 1;
       if (c == nch - 2) {
         // Hand over this warpgroup's share of tile i.
@@ -824,20 +832,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int bb = i % kSBuf;
       if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((i / kSBuf) & 1), ab, status))) break;
       tc_fence_after();
-      const uint32_t tS = tmem + lane_addr + (uint32_t)bb * kGC;
-#pragma unroll 1
-      for (int half = 0; half < 2; half++) {
-        // Points [64 half, 64 half + 64) -> packed weights in columns [32 half, 32 half + 32),
-        // which this thread has already read.
-        uint32_t v0[32], v1[32];
-        tmem_ld32(tS + half * 64, v0);
-        tmem_ld32(tS + half * 64 + 32, v1);
-        tmem_wait_ld2(v0, v1);
-        uint32_t pk0[16], pk1[16];
-        weights64(v0, v1, pk0, pk1);
-        tmem_st16(tS + half * 32, pk0);
-        tmem_st16(tS + half * 32 + 16, pk1);
-      }
+      weights_in_halves(tmem + lane_addr + (uint32_t)bb * kGC);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();

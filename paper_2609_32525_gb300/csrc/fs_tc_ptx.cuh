@@ -46,29 +46,41 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// try_wait that lets the hardware suspend the thread until the phase completes or
+// about `hint_ns` nanoseconds have passed, so that a waiting warp takes no issue
+// slots from the warps that share its scheduler.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n"
+      " mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2, %3;\n"
+      " selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+
 // Shared state every role polls so that one timed-out wait ends the whole CTA.
 struct Abort {
   volatile int flag;
 };
 
-// Bounded wait: spins on try_wait; after `limit_ns` of wall time (checked every
-// 256 polls) it records FS timeout in *status, raises the CTA abort flag and
-// returns false.  Also returns false at once if the abort flag is already up.
+// Bounded wait: a first plain try_wait, then suspending try_waits of at most 20 us
+// each; after `limit_ns` of wall time it records FS timeout in *status, raises the
+// CTA abort flag and returns false.  Also returns false as soon as the abort flag
+// is up.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, Abort* ab, uint32_t* status,
                                           uint64_t limit_ns = 2000000000ull) {
   if (mbar_try_wait(bar, parity)) return true;
-  uint64_t t0 = 0;
-  for (uint32_t i = 1;; i++) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 0) {
-      if (ab->flag) return false;
-      const uint64_t t = globaltimer();
-      if (t0 == 0) t0 = t;
-      else if (t - t0 > limit_ns) {
-        ab->flag = 1;
-        if (status) atomicCAS(status, 0u, 4u /* FS_ERR_TIMEOUT */);
-        return false;
-      }
+  const uint64_t t0 = globaltimer();
+  for (;;) {
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if (ab->flag) return false;
+    if (globaltimer() - t0 > limit_ns) {
+      ab->flag = 1;
+      if (status) atomicCAS(status, 0u, 4u /* FS_ERR_TIMEOUT */);
+      return false;
     }
   }
 }
