@@ -209,20 +209,29 @@ __global__ void __launch_bounds__(kThreads) k_slice_partial(
 }
 
 // Fixed-order sum of the P partials, then (optionally) the normalisation.
+// One thread per (slot, column) of the partials [P, BHG, D+1]: consecutive threads
+// read consecutive words of every split.  The sum over splits runs in split order.
 __global__ void k_reduce_tokens(const float* __restrict__ part, int P, int64_t BHG, int D,
                                 float* __restrict__ tokens, float* __restrict__ wsum, int finalize,
                                 float eps) {
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= BHG) return;
-  float S = 0.f;
-  for (int p = 0; p < P; p++) S += part[((int64_t)p * BHG + i) * (D + 1) + D];
-  const float den = S + eps;
-  for (int c = 0; c < D; c++) {
-    float U = 0.f;
-    for (int p = 0; p < P; p++) U += part[((int64_t)p * BHG + i) * (D + 1) + c];
-    tokens[i * D + c] = finalize ? U / den : U;
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t stride = BHG * (D + 1);
+  if (idx >= stride) return;
+  const int64_t i = idx / (D + 1);
+  const int c = (int)(idx % (D + 1));
+  float v = 0.f;
+  for (int p = 0; p < P; p++) v += part[(int64_t)p * stride + idx];
+  if (c == D) {
+    wsum[i] = v;
+    return;
   }
-  wsum[i] = S;
+  if (!finalize) {
+    tokens[i * D + c] = v;
+    return;
+  }
+  float S = 0.f;
+  for (int p = 0; p < P; p++) S += part[(int64_t)p * stride + i * (D + 1) + D];
+  tokens[i * D + c] = v / (S + eps);
 }
 
 __global__ void k_finalize(float* __restrict__ tokens, const float* __restrict__ wsum, int64_t BHG,
@@ -686,8 +695,8 @@ cudaError_t simt_slice_partials(const Shape& s, int P, const void* x, const void
 cudaError_t simt_reduce_tokens(const Shape& s, int P, const float* part, float* tokens, float* wsum,
                                int finalize, cudaStream_t st) {
   const int64_t BHG = s.BH() * s.G;
-  k_reduce_tokens<<<(unsigned)((BHG + 255) / 256), 256, 0, st>>>(part, P, BHG, s.d, tokens, wsum, finalize,
-                                                                 s.eps);
+  const int64_t n = BHG * (s.d + 1);
+  k_reduce_tokens<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(part, P, BHG, s.d, tokens, wsum, finalize, s.eps);
   return cudaGetLastError();
 }
 
