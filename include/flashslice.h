@@ -73,6 +73,21 @@ typedef enum fs_status {
 
 typedef enum fs_dtype { FS_F32 = 0, FS_BF16 = 1 } fs_dtype;
 
+/* Arithmetic of the point-by-slot products for FS_BF16 shapes on the tensor
+ * cores (the paper's "dot levels", App. G.2; fp32 accumulation throughout):
+ *   FS_DOT_BF16   both operands of every product in bf16: W log2(e)/tau and the
+ *                 slice weights rounded to bf16 (the paper's "bf16" level).
+ *                 Outputs within ~1e-2 relative of exact.
+ *   FS_DOT_BF16X2 W log2(e)/tau and the slice weights each carried as two bf16
+ *                 halves (hi + lo, ~2^-16 relative) in the statistics and slice
+ *                 passes, and in the deslice where its images fit in shared
+ *                 memory (G <= 768): tokens, weight sums and lse to ~1e-4,
+ *                 which the temperature gradient needs (a near-cancelling sum).
+ *                 Slower: two more K-steps per logits block, twice the slice
+ *                 products.
+ * Ignored for FS_F32 shapes and on the SIMT path (fp32 FMA). */
+typedef enum fs_dot { FS_DOT_BF16 = 0, FS_DOT_BF16X2 = 1 } fs_dot;
+
 typedef struct fs_shape {
   int64_t B;     /* batch size, >= 1 */
   int64_t N;     /* points per sample, >= 1 */
@@ -81,6 +96,7 @@ typedef struct fs_shape {
   int32_t G;     /* slices per head, 1..4096 */
   int32_t dtype; /* fs_dtype of the [B,N,H,d] point tensors */
   float eps;     /* added to the weight sums before normalising, >= 0 (paper: 1e-5) */
+  int32_t dot;   /* fs_dot: product arithmetic of the tensor-core path */
 } fs_shape;
 
 typedef enum fs_op {
@@ -128,7 +144,10 @@ fs_status fs_deslice_fwd(const fs_shape* s, const void* x_mid, const float* W_sl
  *   d_tokens_mixed [B,H,G,d] = sum_n w_ng dout_n  (always overwritten)
  *   dx_mid [B,N,H,d], dW [H,d,G], dbias [H,G], dtau [H]: the contribution of
  *   the deslice weights; written if accumulate == 0, added if accumulate != 0.
- *   lse must be the statistics of the forward pass (not NULL). */
+ *   lse must be the statistics of the forward pass (not NULL).  The backward
+ *   forms its weights from fp32 logits; on shapes whose forward runs on the
+ *   tensor cores (fs_path_for_shape == 1), whose lse comes from logits with
+ *   bf16-rounded W log2(e)/tau, it recomputes lse in fp32 into ws instead. */
 fs_status fs_deslice_bwd(const fs_shape* s, const void* x_mid, const float* W_slice,
                          const float* bias, const float* tau, const float* tokens_mixed,
                          const float* lse, const void* dout, float* d_tokens_mixed,
@@ -142,7 +161,8 @@ fs_status fs_mix_bwd(const fs_shape* s, const float* M, const float* tokens,
                      fs_stream_t stream);
 
 /* Backward of the slice given d_tokens (the gradient w.r.t. the normalised
- * tokens); tokens and wsum are the forward's normalised tokens and S.
+ * tokens); tokens and wsum are the forward's normalised tokens and S; lse as
+ * in fs_deslice_bwd (recomputed in fp32 on the tensor-core path).
  *   dfx [B,N,H,d] (overwritten); dx_mid, dW, dbias, dtau: written if
  *   accumulate == 0, added if accumulate != 0. */
 fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx,

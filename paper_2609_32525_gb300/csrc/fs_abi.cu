@@ -35,6 +35,7 @@ bool valid_shape(const fs_shape* s) {
   if (s->B < 1 || s->N < 1 || s->H < 1 || s->d < 1 || s->G < 1) return false;
   if (s->dtype != FS_F32 && s->dtype != FS_BF16) return false;
   if (!(s->eps >= 0.f) || !std::isfinite(s->eps)) return false;
+  if (s->dot != FS_DOT_BF16 && s->dot != FS_DOT_BF16X2) return false;
   const double elems = (double)s->B * (double)s->N * (double)s->H * (double)s->d;
   if (elems >= 1099511627776.0) return false;  // 2^40
   return true;
@@ -44,13 +45,13 @@ bool supported_shape(const fs_shape* s) {
   return (s->d == 16 || s->d == 32 || s->d == 64) && s->G <= 4096 && (int64_t)s->B * s->H <= 65535;
 }
 
-Shape to_shape(const fs_shape* s) { return Shape{s->B, s->N, s->H, s->d, s->G, s->dtype, s->eps}; }
+Shape to_shape(const fs_shape* s) { return Shape{s->B, s->N, s->H, s->d, s->G, s->dtype, s->eps, s->dot}; }
 
 bool aligned(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Byte sizes of the regions each op places in `ws` (each 256-byte aligned).
 struct Regions {
-  size_t status, partials, stats, delta, dus, dtau_g, tc, total;
+  size_t status, partials, stats, delta, dus, dtau_p, tc, total;
 };
 
 Regions regions(const Shape& s, int op) {
@@ -82,13 +83,15 @@ Regions regions(const Shape& s, int op) {
     case FS_OP_DESLICE_BWD:
       r.delta = take(pts * sizeof(float));
       r.partials = take((size_t)P * BHG * (2 * s.d + 2) * sizeof(float));
-      r.dtau_g = take((size_t)s.H * s.G * sizeof(float));
+      r.dtau_p = take((size_t)s.BH() * simt_point_blocks(s) * sizeof(float));
+      r.stats = take(tc_forward_supported(s) ? pts * sizeof(float) : 0);
       break;
     case FS_OP_SLICE_BWD:
       r.delta = take(pts * sizeof(float));
       r.dus = take(BHG * (s.d + 1) * sizeof(float));
       r.partials = take((size_t)P * BHG * (s.d + 2) * sizeof(float));
-      r.dtau_g = take((size_t)s.H * s.G * sizeof(float));
+      r.dtau_p = take((size_t)s.BH() * simt_point_blocks(s) * sizeof(float));
+      r.stats = take(tc_forward_supported(s) ? pts * sizeof(float) : 0);
       break;
     default:
       return Regions{};
@@ -112,6 +115,20 @@ fs_status cuda_status(cudaError_t e) { return e == cudaSuccess ? FS_OK : FS_ERR_
 
 // Every ws-using call starts by clearing its status word.
 cudaError_t reset_status(void* ws, cudaStream_t st) { return cudaMemsetAsync(ws, 0, sizeof(uint32_t), st); }
+
+// The backward forms its weights from fp32 logits.  On shapes whose forward ran on
+// the tensor cores, the forward's lse comes from logits with bf16-rounded
+// W log2(e)/tau, so the backward recomputes it in fp32 (into ws) to normalise its
+// own weights exactly; elsewhere the caller's lse is used as it is.
+cudaError_t backward_stats(const Shape& sh, const void* x_mid, const float* W_slice, const float* bias,
+                           const float* tau, const float* lse, void* ws, const Regions& r, uint32_t* status,
+                           cudaStream_t st, const float** lse_use) {
+  *lse_use = lse;
+  if (!tc_forward_supported(sh)) return cudaSuccess;
+  float* buf = at<float>(ws, r.stats);
+  *lse_use = buf;
+  return simt_stats(sh, x_mid, W_slice, bias, tau, buf, status, st);
+}
 
 #define FS_CHECK_SHAPE(s)                               \
   do {                                                  \
@@ -247,9 +264,11 @@ fs_status fs_deslice_bwd(const fs_shape* s, const void* x_mid, const float* W_sl
   const Regions r = regions(sh, FS_OP_DESLICE_BWD);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   FS_CUDA(reset_status(ws, st));
-  return cuda_status(simt_deslice_bwd(sh, slot_splits(sh), x_mid, W_slice, bias, tau, tokens_mixed, lse, dout,
+  const float* lse_use = nullptr;
+  FS_CUDA(backward_stats(sh, x_mid, W_slice, bias, tau, lse, ws, r, at<uint32_t>(ws, r.status), st, &lse_use));
+  return cuda_status(simt_deslice_bwd(sh, slot_splits(sh), x_mid, W_slice, bias, tau, tokens_mixed, lse_use, dout,
                                       d_tokens_mixed, dx_mid, dW, dbias, dtau, accumulate, at<float>(ws, r.delta),
-                                      at<float>(ws, r.partials), at<float>(ws, r.dtau_g),
+                                      at<float>(ws, r.partials), at<float>(ws, r.dtau_p),
                                       at<uint32_t>(ws, r.status), st));
 }
 
@@ -275,9 +294,11 @@ fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx, con
   const Regions r = regions(sh, FS_OP_SLICE_BWD);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   FS_CUDA(reset_status(ws, st));
-  return cuda_status(simt_slice_bwd(sh, slot_splits(sh), x_mid, fx, W_slice, bias, tau, tokens, wsum, lse,
+  const float* lse_use = nullptr;
+  FS_CUDA(backward_stats(sh, x_mid, W_slice, bias, tau, lse, ws, r, at<uint32_t>(ws, r.status), st, &lse_use));
+  return cuda_status(simt_slice_bwd(sh, slot_splits(sh), x_mid, fx, W_slice, bias, tau, tokens, wsum, lse_use,
                                     d_tokens, dx_mid, dfx, dW, dbias, dtau, accumulate, at<float>(ws, r.delta),
-                                    at<float>(ws, r.dus), at<float>(ws, r.partials), at<float>(ws, r.dtau_g),
+                                    at<float>(ws, r.dus), at<float>(ws, r.partials), at<float>(ws, r.dtau_p),
                                     at<uint32_t>(ws, r.status), st));
 }
 

@@ -20,6 +20,7 @@ struct Shape {
   int H, d, G;
   int dtype;
   float eps;
+  int dot;  // fs_dot
   int64_t BH() const { return B * (int64_t)H; }
   int64_t points() const { return B * N; }
 };
@@ -31,6 +32,9 @@ int num_sms();
 int slot_splits(const Shape& s);
 
 // ---- SIMT kernels (fs_simt.cu) -------------------------------------------------
+// Point blocks per (b, h) of the SIMT point-owned kernels; the backward's dt_part
+// buffer holds one float per (b, h, point block).
+int64_t simt_point_blocks(const Shape& s);
 cudaError_t simt_stats(const Shape& s, const void* x, const float* W, const float* bias,
                        const float* tau, float* lse, uint32_t* status, cudaStream_t st);
 cudaError_t simt_slice_partials(const Shape& s, int P, const void* x, const void* f,
@@ -49,12 +53,12 @@ cudaError_t simt_deslice_bwd(const Shape& s, int P, const void* x, const float* 
                              const float* bias, const float* tau, const float* zp,
                              const float* lse, const void* dout, float* dzp, void* dx,
                              float* dW, float* db, float* dtau, int accumulate, float* delta,
-                             float* part, float* dtau_g, uint32_t* status, cudaStream_t st);
+                             float* part, float* dt_part, uint32_t* status, cudaStream_t st);
 cudaError_t simt_slice_bwd(const Shape& s, int P, const void* x, const void* f, const float* W,
                            const float* bias, const float* tau, const float* z,
                            const float* wsum, const float* lse, const float* dz, void* dx,
                            void* dfx, float* dW, float* db, float* dtau, int accumulate,
-                           float* delta, float* dUS, float* part, float* dtau_g,
+                           float* delta, float* dUS, float* part, float* dt_part,
                            uint32_t* status, cudaStream_t st);
 
 }  // namespace fs

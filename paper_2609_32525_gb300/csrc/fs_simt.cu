@@ -348,9 +348,10 @@ __global__ void __launch_bounds__(kThreads) k_bwd_point(
     const T* __restrict__ x, const T* __restrict__ v /* dout (MODE 0) or fx (MODE 1) */,
     const float* __restrict__ W, const float* __restrict__ bias, const float* __restrict__ tau,
     const float* __restrict__ tok /* z' (MODE 0) or (dU,dS) (MODE 1) */, const float* __restrict__ lse,
-    T* __restrict__ dx, T* __restrict__ dfx, float* __restrict__ delta, int accumulate, int64_t N, int H,
-    int G, uint32_t* status) {
+    T* __restrict__ dx, T* __restrict__ dfx, float* __restrict__ delta, float* __restrict__ dt_part,
+    int accumulate, int64_t N, int H, int G, uint32_t* status) {
   constexpr int GC = 16;
+  __shared__ float s_dt[kThreads];
   constexpr int TS = (MODE == 0) ? D : D + 1;  // token row stride
   __shared__ float sW[GC][D + 1];
   __shared__ float sT[GC][TS];
@@ -374,6 +375,10 @@ __global__ void __launch_bounds__(kThreads) k_bwd_point(
   }
   const float* tb = tok + bh * G * TS;
   float dl = 0.f;
+  // The point's term of the temperature gradient, sum_g da_g (a_g - lse) in base-2
+  // units: with the logits centred on lse (exact, since sum_g da_g = 0) the row
+  // sum carries no large cancelling parts (App. G.2).
+  float dtn = 0.f;
   for (int sweep = 0; sweep < 2; sweep++) {
     for (int g0 = 0; g0 < G; g0 += GC) {
       __syncthreads();
@@ -402,6 +407,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_point(
           const float da = w * (dw - dl);
 #pragma unroll
           for (int k = 0; k < D; k++) acc[k] = fmaf(da, sW[g][k], acc[k]);
+          if (valid) dtn = fmaf(da, a - l2, dtn);
         }
       }
     }
@@ -411,6 +417,14 @@ __global__ void __launch_bounds__(kThreads) k_bwd_point(
       for (int k = 0; k < D; k++) acc[k] = 0.f;
     }
   }
+  // Block sum of the temperature terms (fixed tree order) -> dt_part[bh][block].
+  s_dt[threadIdx.x] = dtn;
+  __syncthreads();
+  for (int w = kThreads / 2; w > 0; w >>= 1) {
+    if (threadIdx.x < w) s_dt[threadIdx.x] += s_dt[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) dt_part[bh * gridDim.x + blockIdx.x] = s_dt[0] * kLn2;
   if (!valid) return;
   delta[bh * N + n] = dl;
   // acc = sum_g da_g W[:,g] * log2e/tau ; dx = sum_g da_g W[:,g] / tau = acc * ln2.
@@ -451,7 +465,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_slot(
   if (!tau_ok(tau[h], status)) return;
   const float scale = kLog2e / tau[h];
   float wc[D], tg[D], dzp[D], dWa[D];
-  float bb = 0.f, dSg = 0.f, dba = 0.f, dta = 0.f;
+  float bb = 0.f, dSg = 0.f, dba = 0.f;
 #pragma unroll
   for (int k = 0; k < D; k++) {
     wc[k] = (g < G) ? W[((int64_t)h * D + k) * G + g] * scale : 0.f;
@@ -503,8 +517,6 @@ __global__ void __launch_bounds__(kThreads) k_bwd_slot(
 #pragma unroll
       for (int k = 0; k < D; k++) dWa[k] = fmaf(da, sx[j][k], dWa[k]);
       dba += da;
-      // a is the base-2 logit; the natural logit is a * ln2 (zero for padded points: w = 0).
-      dta = fmaf(da, a * kLn2, dta);
     }
   }
   if (g < G) {
@@ -518,7 +530,7 @@ __global__ void __launch_bounds__(kThreads) k_bwd_slot(
 #pragma unroll
     for (int k = 0; k < D; k++) o[off + k] = dWa[k];
     o[off + D] = dba;
-    o[off + D + 1] = dta;
+    o[off + D + 1] = 0.f;  // (the temperature gradient is formed per point, see k_bwd_point)
   }
 }
 
@@ -539,12 +551,11 @@ __global__ void k_slice_bwd_prep(const float* __restrict__ z, const float* __res
 }
 
 // Fixed-order reduction of slot-owned backward partials over (b, p).
-// Writes (or adds) dW[h][k][g], db[h][g]; dtau_g[h][g] = per-slot dtau terms;
-// optionally d_tokens_mixed[b][h][g][c] (sum over p only).
+// Writes (or adds) dW[h][k][g], db[h][g] (the temperature gradient is reduced
+// separately, from per-point row sums); optionally d_tokens_mixed[b][h][g][c] (sum over p only).
 __global__ void k_reduce_bwd(const float* __restrict__ part, int P, int64_t B, int H, int G, int D,
                              int PS, int has_dzp, const float* __restrict__ tau, float* __restrict__ dzp,
-                             float* __restrict__ dW, float* __restrict__ db, float* __restrict__ dtau_g,
-                             int accumulate) {
+                             float* __restrict__ dW, float* __restrict__ db, int accumulate) {
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= (int64_t)H * G) return;
   const int h = (int)(idx / G), g = (int)(idx % G);
@@ -560,35 +571,35 @@ __global__ void k_reduce_bwd(const float* __restrict__ part, int P, int64_t B, i
       }
     }
   }
-  for (int k = 0; k <= D + 1; k++) {
+  for (int k = 0; k <= D; k++) {
     float s = 0.f;
     for (int64_t b = 0; b < B; b++)
       for (int p = 0; p < P; p++) s += part[(((int64_t)p * BH + b * H + h) * G + g) * PS + off + k];
     if (k < D) {
       const int64_t o = ((int64_t)h * D + k) * G + g;
       dW[o] = (accumulate ? dW[o] : 0.f) + s * inv;
-    } else if (k == D) {
-      db[idx] = (accumulate ? db[idx] : 0.f) + s * inv;
     } else {
-      dtau_g[idx] = -s * inv;
+      db[idx] = (accumulate ? db[idx] : 0.f) + s * inv;
     }
   }
 }
 
-// dtau[h] (+)= sum_g dtau_g[h][g], fixed-order tree within one block per head.
-__global__ void k_reduce_dtau(const float* __restrict__ dtau_g, int G, float* __restrict__ dtau,
-                              int accumulate) {
+// dtau[h] (+)= -(1/tau_h) * sum over batches and point blocks of the block sums of
+// sum_g da (a - lse) (fixed order: strided per thread, then a tree).
+__global__ void k_reduce_dtau(const float* __restrict__ dt_part, int64_t B, int H, int64_t nblk,
+                              const float* __restrict__ tau, float* __restrict__ dtau, int accumulate) {
   __shared__ float s[256];
   const int h = blockIdx.x;
   float v = 0.f;
-  for (int g = threadIdx.x; g < G; g += 256) v += dtau_g[(int64_t)h * G + g];
+  for (int64_t b = 0; b < B; b++)
+    for (int64_t i = threadIdx.x; i < nblk; i += 256) v += dt_part[(b * H + h) * nblk + i];
   s[threadIdx.x] = v;
   __syncthreads();
   for (int w = 128; w > 0; w >>= 1) {
     if (threadIdx.x < w) s[threadIdx.x] += s[threadIdx.x + w];
     __syncthreads();
   }
-  if (threadIdx.x == 0) dtau[h] = (accumulate ? dtau[h] : 0.f) + s[0];
+  if (threadIdx.x == 0) dtau[h] = (accumulate ? dtau[h] : 0.f) - s[0] / tau[h];
 }
 
 inline dim3 point_grid(const Shape& s) {
@@ -627,10 +638,10 @@ cudaError_t launch_deslice(const Shape& s, const void* x, const float* W, const 
 template <int D, typename T, int MODE>
 cudaError_t launch_bwd(const Shape& s, int P, const void* x, const void* v, const float* W, const float* bias,
                        const float* tau, const float* tok, const float* lse, void* dx, void* dfx, float* delta,
-                       float* part, int accumulate, uint32_t* status, cudaStream_t st) {
+                       float* dt_part, float* part, int accumulate, uint32_t* status, cudaStream_t st) {
   k_bwd_point<D, T, MODE><<<point_grid(s), kThreads, 0, st>>>((const T*)x, (const T*)v, W, bias, tau, tok, lse,
-                                                               (T*)dx, (T*)dfx, delta, accumulate, s.N, s.H,
-                                                               s.G, status);
+                                                               (T*)dx, (T*)dfx, delta, dt_part, accumulate, s.N,
+                                                               s.H, s.G, status);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   k_bwd_slot<D, T, MODE><<<slot_grid(s, P), kThreads, 0, st>>>((const T*)x, (const T*)v, W, bias, tau, tok,
@@ -654,32 +665,35 @@ cudaError_t launch_bwd(const Shape& s, int P, const void* x, const void* v, cons
 template <int D, typename T>
 cudaError_t launch_bwd_deslice(const Shape& s, int P, const void* x, const void* v, const float* W,
                                const float* bias, const float* tau, const float* tok, const float* lse,
-                               void* dx, float* delta, float* part, int accumulate, uint32_t* status,
-                               cudaStream_t st) {
-  return launch_bwd<D, T, 0>(s, P, x, v, W, bias, tau, tok, lse, dx, nullptr, delta, part, accumulate, status,
-                             st);
+                               void* dx, float* delta, float* dt_part, float* part, int accumulate,
+                               uint32_t* status, cudaStream_t st) {
+  return launch_bwd<D, T, 0>(s, P, x, v, W, bias, tau, tok, lse, dx, nullptr, delta, dt_part, part, accumulate,
+                             status, st);
 }
 template <int D, typename T>
 cudaError_t launch_bwd_slice(const Shape& s, int P, const void* x, const void* v, const float* W,
                              const float* bias, const float* tau, const float* tok, const float* lse, void* dx,
-                             void* dfx, float* delta, float* part, int accumulate, uint32_t* status,
-                             cudaStream_t st) {
-  return launch_bwd<D, T, 1>(s, P, x, v, W, bias, tau, tok, lse, dx, dfx, delta, part, accumulate, status, st);
+                             void* dfx, float* delta, float* dt_part, float* part, int accumulate,
+                             uint32_t* status, cudaStream_t st) {
+  return launch_bwd<D, T, 1>(s, P, x, v, W, bias, tau, tok, lse, dx, dfx, delta, dt_part, part, accumulate,
+                             status, st);
 }
 
 cudaError_t reduce_params(const Shape& s, int P, const float* part, int PS, int has_dzp, const float* tau,
-                          float* dzp, float* dW, float* db, float* dtau, float* dtau_g, int accumulate,
+                          float* dzp, float* dW, float* db, float* dtau, const float* dt_part, int accumulate,
                           cudaStream_t st) {
   const int64_t HG = (int64_t)s.H * s.G;
   k_reduce_bwd<<<(unsigned)((HG + 127) / 128), 128, 0, st>>>(part, P, s.B, s.H, s.G, s.d, PS, has_dzp, tau,
-                                                              dzp, dW, db, dtau_g, accumulate);
+                                                              dzp, dW, db, accumulate);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_reduce_dtau<<<s.H, 256, 0, st>>>(dtau_g, s.G, dtau, accumulate);
+  k_reduce_dtau<<<s.H, 256, 0, st>>>(dt_part, s.B, s.H, simt_point_blocks(s), tau, dtau, accumulate);
   return cudaGetLastError();
 }
 
 }  // namespace
+
+int64_t simt_point_blocks(const Shape& s) { return (s.N + kThreads - 1) / kThreads; }
 
 cudaError_t simt_stats(const Shape& s, const void* x, const float* W, const float* bias, const float* tau,
                        float* lse, uint32_t* status, cudaStream_t st) {
@@ -731,30 +745,30 @@ cudaError_t simt_deslice(const Shape& s, const void* x, const float* W, const fl
 cudaError_t simt_deslice_bwd(const Shape& s, int P, const void* x, const float* W, const float* bias,
                              const float* tau, const float* zp, const float* lse, const void* dout, float* dzp,
                              void* dx, float* dW, float* db, float* dtau, int accumulate, float* delta,
-                             float* part, float* dtau_g, uint32_t* status, cudaStream_t st) {
+                             float* part, float* dt_part, uint32_t* status, cudaStream_t st) {
   cudaError_t e = [&]() -> cudaError_t {
-    FS_DISPATCH(s, launch_bwd_deslice, s, P, x, dout, W, bias, tau, zp, lse, dx, delta, part, accumulate,
-                status, st);
+    FS_DISPATCH(s, launch_bwd_deslice, s, P, x, dout, W, bias, tau, zp, lse, dx, delta, dt_part, part,
+                accumulate, status, st);
   }();
   if (e != cudaSuccess) return e;
-  return reduce_params(s, P, part, 2 * s.d + 2, 1, tau, dzp, dW, db, dtau, dtau_g, accumulate, st);
+  return reduce_params(s, P, part, 2 * s.d + 2, 1, tau, dzp, dW, db, dtau, dt_part, accumulate, st);
 }
 
 cudaError_t simt_slice_bwd(const Shape& s, int P, const void* x, const void* f, const float* W,
                            const float* bias, const float* tau, const float* z, const float* wsum,
                            const float* lse, const float* dz, void* dx, void* dfx, float* dW, float* db,
-                           float* dtau, int accumulate, float* delta, float* dUS, float* part, float* dtau_g,
+                           float* dtau, int accumulate, float* delta, float* dUS, float* part, float* dt_part,
                            uint32_t* status, cudaStream_t st) {
   const int64_t BHG = s.BH() * s.G;
   k_slice_bwd_prep<<<(unsigned)((BHG + 255) / 256), 256, 0, st>>>(z, wsum, dz, dUS, BHG, s.d, s.eps);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   e = [&]() -> cudaError_t {
-    FS_DISPATCH(s, launch_bwd_slice, s, P, x, f, W, bias, tau, dUS, lse, dx, dfx, delta, part, accumulate,
-                status, st);
+    FS_DISPATCH(s, launch_bwd_slice, s, P, x, f, W, bias, tau, dUS, lse, dx, dfx, delta, dt_part, part,
+                accumulate, status, st);
   }();
   if (e != cudaSuccess) return e;
-  return reduce_params(s, P, part, s.d + 2, 0, tau, nullptr, dW, db, dtau, dtau_g, accumulate, st);
+  return reduce_params(s, P, part, s.d + 2, 0, tau, nullptr, dW, db, dtau, dt_part, accumulate, st);
 }
 
 }  // namespace fs

@@ -73,8 +73,13 @@ constexpr uint32_t kPxBytes = kTile * 16;  // 128 point-extra rows of 8 bf16 (k 
 constexpr uint64_t kWaitNs = 2000000000ull;
 
 // ---- operand images written by the prep kernels -------------------------------------------
-// W image for head h: G rows (slots) x 64 B of W*log2e/tau (64B swizzle), then
-// G rows x 32 B of [b'_hi, b'_lo, 1, 1, 0...] (32B swizzle).
+// W image for head h (kWRow = 160 bytes per slot): G rows (slots) x 64 B of
+// W' = W*log2e/tau rounded to bf16 (64B swizzle), then G rows x 32 B of
+// [b'_hi, b'_lo, 1, 1, 0...] (32B swizzle), then G rows x 64 B of the residual
+// W' - bf16(W') rounded to bf16 (64B swizzle).  The statistics and slice passes
+// use both halves of W' (their lse, tokens and weight sums then carry no
+// systematic per-slot rounding of the weights); the deslice uses the first half.
+constexpr uint32_t kWRow = 160;
 __device__ __forceinline__ uint32_t off_sw64(int row, int k) {  // k in [0, 32)
   const int chunk = k >> 3;
   return (uint32_t)((row >> 3) * 512 + (row & 7) * 64 + ((chunk ^ ((row & 7) >> 1)) << 4) + (k & 7) * 2);
@@ -101,10 +106,15 @@ __global__ void k_prep_w(const float* __restrict__ W, const float* __restrict__ 
     return;
   }
   const float scale = kLog2e / t;
-  uint8_t* base = img + (size_t)h * G * 96;
+  uint8_t* base = img + (size_t)h * G * kWRow;
   __nv_bfloat16* wp = reinterpret_cast<__nv_bfloat16*>(base);
-  for (int k = 0; k < kD; k++)
-    wp[off_sw64(g, k) / 2] = __float2bfloat16_rn(W[((int64_t)h * kD + k) * G + g] * scale);
+  __nv_bfloat16* wl = reinterpret_cast<__nv_bfloat16*>(base + (size_t)G * 96);
+  for (int k = 0; k < kD; k++) {
+    const float w2 = W[((int64_t)h * kD + k) * G + g] * scale;
+    const __nv_bfloat16 whi = __float2bfloat16_rn(w2);
+    wp[off_sw64(g, k) / 2] = whi;
+    wl[off_sw64(g, k) / 2] = __float2bfloat16_rn(w2 - __bfloat162float(whi));
+  }
   __nv_bfloat16* ep = reinterpret_cast<__nv_bfloat16*>(base + (size_t)G * 64);
   const float b2 = bias[(int64_t)h * G + g] * scale;
   const __nv_bfloat16 hi = __float2bfloat16_rn(b2);
@@ -179,8 +189,9 @@ __device__ __forceinline__ void zero_smem(uint8_t* p, uint32_t bytes) {
 // Base-2 logits of 128 points x 128 slots (chunk c of the W image) into TMEM.
 //   point_major: A = points (x tile), B = slots (W);  else A = slots, B = points.
 //   xe: descriptor of the point-side extra block.
+//   wl_img: the residual half of W' (0: bf16 W' only, K = 48; else K = 80).
 __device__ __forceinline__ void issue_logits(uint32_t tmem_d, uint32_t x_s, uint64_t xe, uint32_t w_img,
-                                             uint32_t we_img, int c, bool point_major) {
+                                             uint32_t we_img, uint32_t wl_img, int c, bool point_major) {
   constexpr uint32_t idesc = idesc_bf16(128, kGC, false, false);
   const uint32_t wc = w_img + (uint32_t)c * kGC * 64;
   const uint32_t wec = we_img + (uint32_t)c * kGC * 32;
@@ -190,12 +201,25 @@ __device__ __forceinline__ void issue_logits(uint32_t tmem_d, uint32_t x_s, uint
   if (point_major) {
     mma_ss_w(tmem_d, x0, w0, idesc, 0);
     mma_ss_w(tmem_d, x1, w1, idesc, 1);
-    mma_ss_w(tmem_d, xe, we, idesc, 1);
   } else {
     mma_ss_w(tmem_d, w0, x0, idesc, 0);
     mma_ss_w(tmem_d, w1, x1, idesc, 1);
-    mma_ss_w(tmem_d, we, xe, idesc, 1);
   }
+  if (wl_img) {
+    const uint32_t wlc = wl_img + (uint32_t)c * kGC * 64;
+    const uint64_t l0 = sdesc(wlc, 16, 512, kSw64), l1 = sdesc(wlc + 32, 16, 512, kSw64);
+    if (point_major) {
+      mma_ss_w(tmem_d, x0, l0, idesc, 1);
+      mma_ss_w(tmem_d, x1, l1, idesc, 1);
+    } else {
+      mma_ss_w(tmem_d, l0, x0, idesc, 1);
+      mma_ss_w(tmem_d, l1, x1, idesc, 1);
+    }
+  }
+  if (point_major)
+    mma_ss_w(tmem_d, xe, we, idesc, 1);
+  else
+    mma_ss_w(tmem_d, we, xe, idesc, 1);
 }
 
 // Producer-side bulk loads of an image into smem (pieces of at most 32 KB).
@@ -217,6 +241,51 @@ __device__ __forceinline__ void weights32(const uint32_t (&v)[32], uint32_t (&p)
 // in place, packed in pairs, into the first 64 columns, in two halves: columns
 // [64 h, 64 h + 64) -> packed weights in columns [32 h, 32 h + 32), which this
 // thread has already read.
+// 2^t for 32 log2-weights -> the bf16 pairs (hi) and the bf16 pairs of the
+// residuals w - hi (lo): w = hi + lo to ~2^-16 relative.
+__device__ __forceinline__ void weights32_hilo(const uint32_t (&v)[32], uint32_t (&hi)[16], uint32_t (&lo)[16]) {
+#pragma unroll
+  for (int k = 0; k < 16; k++) {
+    const float w0 = ex2(__uint_as_float(v[2 * k])), w1 = ex2(__uint_as_float(v[2 * k + 1]));
+    const uint32_t p = pack_bf16(w0, w1);
+    const float h0 = __uint_as_float(p << 16), h1 = __uint_as_float(p & 0xFFFF0000u);
+    hi[k] = p;
+    lo[k] = pack_bf16(w0 - h0, w1 - h1);
+  }
+}
+
+// Slice weights of one TMEM lane (a slot) of an S buffer, 128 points: the hi
+// halves packed in pairs into columns [0, 64), the lo halves into [64, 128).
+// Half h reads columns [64 h, 64 h + 64); the lo pairs of half 0 wait in
+// registers until half 1 has read the columns they go to.
+__device__ __forceinline__ void weights_hilo_in_place(uint32_t tS) {
+  uint32_t lo0[16], lo1[16];
+  {
+    uint32_t v0[32], v1[32];
+    tmem_ld32(tS, v0);
+    tmem_ld32(tS + 32, v1);
+    tmem_wait_ld2(v0, v1);
+    uint32_t hi0[16], hi1[16];
+    weights32_hilo(v0, hi0, lo0);
+    weights32_hilo(v1, hi1, lo1);
+    tmem_st16(tS, hi0);
+    tmem_st16(tS + 16, hi1);
+  }
+  uint32_t v0[32], v1[32];
+  tmem_ld32(tS + 64, v0);
+  tmem_ld32(tS + 96, v1);
+  tmem_wait_ld2(v0, v1);
+  tmem_st16(tS + 64, lo0);
+  tmem_st16(tS + 80, lo1);
+  uint32_t hi0[16], hi1[16];
+  weights32_hilo(v0, hi0, lo0);
+  weights32_hilo(v1, hi1, lo1);
+  tmem_st16(tS + 32, hi0);
+  tmem_st16(tS + 48, hi1);
+  tmem_st16(tS + 96, lo0);
+  tmem_st16(tS + 112, lo1);
+}
+
 __device__ __forceinline__ void weights_in_halves(uint32_t tS) {
 #pragma unroll 1
   for (int half = 0; half < 2; half++) {
@@ -260,10 +329,12 @@ constexpr uint32_t kDStage = kXBytes + 2 * kPxBytes;  // x tile, point extra (bo
 __global__ void __launch_bounds__(kThreads, 1)
     k_deslice(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap pmap,
               const uint8_t* __restrict__ wimg, const uint8_t* __restrict__ zimg, __nv_bfloat16* __restrict__ out,
-              int64_t N, int64_t Np, int H, int G, int splits, uint32_t* status) {
+              int64_t N, int64_t Np, int H, int G, int splits, int hilo, uint32_t* status) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const uint32_t wbytes = (uint32_t)G * 96, zbytes = (uint32_t)G * 64;
+  // hilo: the residual half of W' fits in shared memory too (K = 80 logits, as in
+  // the statistics pass); else bf16 W' only (K = 48).
+  const uint32_t wbytes = (uint32_t)G * (hilo ? kWRow : 96), zbytes = (uint32_t)G * 64;
   uint8_t* s_w = smem;
   uint8_t* s_z = s_w + wbytes;
   uint8_t* s_x = s_z + zbytes;  // stage s at s_x + s * kDStage
@@ -321,7 +392,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&xmap);
       prefetch_tmap(&pmap);
       mbar_expect_tx(wz_full, wbytes + zbytes);
-      load_images(s_w, wimg + (size_t)h * wbytes, wbytes, wz_full);
+      load_images(s_w, wimg + (size_t)h * G * kWRow, wbytes, wz_full);
       load_images(s_z, zimg + (size_t)wk.bh * zbytes, zbytes, wz_full);
       int i = 0;
       for (; i < wk.ntiles; i++) {
@@ -353,7 +424,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (q >= kSBuf && !(ok = mbar_wait_w(&pv_done[bb], (uint32_t)(((q / kSBuf) - 1) & 1), ab, status))) break;
         tc_fence_after();
         const uint32_t xs = smem_u32(s_x + s * kDStage);
-        issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kXBytes), sw, swe, c, true);
+        issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kXBytes), sw, swe,
+                     hilo ? sw + (uint32_t)G * 96 : 0u, c, true);
         mma_commit_w(&s_full[bb]);
         if (c == nch - 1) mma_commit_w(&x_empty[s]);
       }
@@ -460,12 +532,14 @@ __global__ void __launch_bounds__(kThreads, 1)
 // smem: [W img G*96][x stages][constant extra][ml exchange][barriers]
 // TMEM: two S buffers [0, 256).
 // =========================================================================================
+template <bool split>
 __global__ void __launch_bounds__(kThreads, 1)
     k_stats(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ wimg, float* __restrict__ lse,
             uint4* __restrict__ px, int64_t N, int64_t Np, int H, int G, int splits, uint32_t* status) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const uint32_t wbytes = (uint32_t)G * 96;
+  // split (FS_DOT_BF16X2): the residual half of W' too (K = 80 logits).
+  const uint32_t wbytes = (uint32_t)G * (split ? kWRow : 96);
   uint8_t* s_w = smem;
   uint8_t* s_x = s_w + wbytes;
   uint8_t* s_ex = s_x + kStages * kXBytes;
@@ -517,7 +591,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0 && wk.ntiles > 0) {
       prefetch_tmap(&xmap);
       mbar_expect_tx(w_full, wbytes);
-      load_images(s_w, wimg + (size_t)h * wbytes, wbytes, w_full);
+      load_images(s_w, wimg + (size_t)h * G * kWRow, wbytes, w_full);
       int i = 0;
       for (; i < wk.ntiles; i++) {
         const int s = i % kStages;
@@ -548,7 +622,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (q >= 2 && !(ok = mbar_wait_w(&s_free[bb], (uint32_t)(((q >> 1) - 1) & 1), ab, status))) break;
         tc_fence_after();
         issue_logits(tmem + (uint32_t)bb * kGC, smem_u32(s_x + s * kXBytes), const_extra_desc(smem_u32(s_ex)), sw, swe,
-                     c, true);
+                     split ? sw + (uint32_t)G * 96 : 0u, c, true);
         mma_commit_w(&s_full[bb]);
         if (c >= nch - nis) mma_commit_w(&x_empty[s]);
       }
@@ -680,12 +754,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 // accumulator A_wg (the two are summed in a fixed order).
 // =========================================================================================
 constexpr uint32_t kStageBytes = kXBytes + 3 * kFBlock + 2 * kPxBytes;  // x, [F | 1], point extra
-constexpr uint32_t kWBlock = 128 * 96;                                  // one 128-slot block of the W image
+constexpr uint32_t kWBlock = 128 * kWRow;                               // one 128-slot block of the W image
 
+template <bool split>
 __global__ void __launch_bounds__(kThreads, 1)
     k_slice(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap fmap,
             const __grid_constant__ CUtensorMap pmap, const uint8_t* __restrict__ wimg, float* __restrict__ part,
             int64_t N, int64_t Np, int H, int G, int splits, uint32_t* status) {
+  // split (FS_DOT_BF16X2): logits with both halves of W' (K = 80), and the
+  // weights as hi + lo bf16 halves in the products (twice the product MMAs).
   // Grid (slot block, point split, bh): the CTAs of all slot blocks of one point
   // range are adjacent in launch order, run together and share each x / F tile
   // through L2 instead of re-reading it from DRAM once per slot block.
@@ -754,10 +831,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&pmap);
       // The slot block's rows of the W image: 128 rows of W' (64 B) then 128 rows of
       // the extra block (32 B); the global image holds G rows of each.
-      mbar_expect_tx(w_full, kWBlock);
-      const uint8_t* src = wimg + (size_t)h * G * 96;
+      mbar_expect_tx(w_full, split ? kWBlock : kGC * 96);
+      const uint8_t* src = wimg + (size_t)h * G * kWRow;
       load_images(s_w, src + (size_t)g_base * 64, kGC * 64, w_full);
       load_images(s_w + kGC * 64, src + (size_t)G * 64 + (size_t)g_base * 32, kGC * 32, w_full);
+      if (split) load_images(s_w + kGC * 96, src + (size_t)G * 96 + (size_t)g_base * 64, kGC * 64, w_full);
       int i = 0;
       for (; i < wk.ntiles; i++) {
         const int s = i % kSliceStages;
@@ -788,7 +866,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (i >= kSBuf && !(ok = mbar_wait_w(&pv_done[bb], (uint32_t)(((i / kSBuf) - 1) & 1), ab, status))) break;
         tc_fence_after();
         const uint32_t xs = smem_u32(s_st + s * kStageBytes);
-        issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kPOff), sw, swe, 0, false);
+        issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kPOff), sw, swe, split ? sw + kGC * 96 : 0u,
+                     0, false);
         mma_commit_w(&s_full[bb]);
         mma_commit_w(&st_empty[s]);
       }
@@ -811,9 +890,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t fs = smem_u32(s_st + s * kStageBytes) + kFOff;
         const uint32_t tacc = tmem + kA + (uint32_t)j * 48;
 #pragma unroll
-        for (int kk = 0; kk < 8; kk++)
-          mma_ts_w(tacc, tE + (uint32_t)kk * 8, sdesc(fs + (uint32_t)kk * 512, kFBlock, 256, kSw32), idesc_sl,
-                 (i >= 2 || kk > 0) ? 1u : 0u);
+        for (int kk = 0; kk < 8; kk++) {
+          const uint64_t fdesc = sdesc(fs + (uint32_t)kk * 512, kFBlock, 256, kSw32);
+          mma_ts_w(tacc, tE + (uint32_t)kk * 8, fdesc, idesc_sl, (i >= 2 || kk > 0) ? 1u : 0u);
+          // The residual halves of the weights: U and S to ~2^-16.
+          if (split) mma_ts_w(tacc, tE + 64 + (uint32_t)kk * 8, fdesc, idesc_sl, 1u);
+        }
         mma_commit_w(&pv_done[bb]);
         mma_commit_w(&st_empty[s]);
       }
@@ -832,7 +914,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int bb = i % kSBuf;
       if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((i / kSBuf) & 1), ab, status))) break;
       tc_fence_after();
-      weights_in_halves(tmem + lane_addr + (uint32_t)bb * kGC);
+      if (split)
+        weights_hilo_in_place(tmem + lane_addr + (uint32_t)bb * kGC);
+      else
+        weights_in_halves(tmem + lane_addr + (uint32_t)bb * kGC);
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
@@ -915,7 +1000,7 @@ bool make_px_map(CUtensorMap* map, const void* ptr, int64_t BH, int64_t Np) {
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-size_t w_image_bytes(const Shape& s) { return (size_t)s.H * s.G * 96; }
+size_t w_image_bytes(const Shape& s) { return (size_t)s.H * s.G * kWRow; }
 size_t z_image_bytes(const Shape& s) { return (size_t)s.BH() * s.G * 64; }
 int64_t padded_n(const Shape& s) { return (s.N + kTile - 1) / kTile * kTile; }
 size_t px_bytes(const Shape& s) { return (size_t)s.BH() * padded_n(s) * 16; }
@@ -943,8 +1028,13 @@ int point_splits(const Shape& s, int units) {
 int slice_blocks(const Shape& s) { return s.G / kGC < 1 ? 1 : s.G / kGC; }
 int slice_splits(const Shape& s) { return point_splits(s, (int)(s.BH() * slice_blocks(s))); }
 
-size_t smem_deslice(int G) { return 1024 + (size_t)G * 160 + kStages * kDStage + 512; }
-size_t smem_stats(int G) { return 1024 + (size_t)G * 96 + kStages * kXBytes + kExBytes + 2 * kTile * 8 + 512; }
+size_t smem_deslice(int G, bool hilo) {
+  return 1024 + (size_t)G * ((hilo ? kWRow : 96) + 64) + kStages * kDStage + 512;
+}
+constexpr size_t kMaxSmem = 232448;  // opt-in shared memory per block on sm_103
+size_t smem_stats(int G, bool split) {
+  return 1024 + (size_t)G * (split ? kWRow : 96) + kStages * kXBytes + kExBytes + 2 * kTile * 8 + 512;
+}
 size_t smem_slice() { return 1024 + (size_t)kWBlock + kSliceStages * kStageBytes + 512; }
 
 template <typename K>
@@ -965,11 +1055,13 @@ cudaError_t run_stats(const Shape& s, const void* x, const uint8_t* wimg, float*
   CUtensorMap xmap;
   if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
   const int P = point_splits(s, (int)s.BH());
-  const size_t sm = smem_stats(s.G);
-  cudaError_t e = set_smem(k_stats, sm);
+  const bool split = s.dot == FS_DOT_BF16X2;
+  const size_t sm = smem_stats(s.G, split);
+  const auto kernel = split ? k_stats<true> : k_stats<false>;
+  cudaError_t e = set_smem(kernel, sm);
   if (e != cudaSuccess) return e;
-  k_stats<<<dim3((unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(xmap, wimg, lse, static_cast<uint4*>(px), s.N,
-                                                                     padded_n(s), s.H, s.G, P, status);
+  kernel<<<dim3((unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(xmap, wimg, lse, static_cast<uint4*>(px), s.N,
+                                                                    padded_n(s), s.H, s.G, P, status);
   return cudaGetLastError();
 }
 
@@ -1022,8 +1114,9 @@ cudaError_t tc_slice_fwd(const Shape& s, const void* x, const void* f, const flo
   const int R = slice_blocks(s), P = slice_splits(s);
   dim3 grid((unsigned)R, (unsigned)P, (unsigned)s.BH());
   const size_t sm = smem_slice();
-  if ((e = set_smem(k_slice, sm)) != cudaSuccess) return e;
-  k_slice<<<grid, kThreads, sm, st>>>(xmap, fmap, pmap, wimg, part, s.N, padded_n(s), s.H, s.G, P, status);
+  const auto kernel = s.dot == FS_DOT_BF16X2 ? k_slice<true> : k_slice<false>;
+  if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
+  kernel<<<grid, kThreads, sm, st>>>(xmap, fmap, pmap, wimg, part, s.N, padded_n(s), s.H, s.G, P, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   return simt_reduce_tokens(s, P, part, tokens, wsum, finalize, st);
 }
@@ -1046,11 +1139,12 @@ cudaError_t tc_deslice_fwd(const Shape& s, const void* x, const float* W, const 
   if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
   if (!make_px_map(&pmap, px, s.BH(), Np)) return cudaErrorInvalidValue;
   const int P = point_splits(s, (int)s.BH());
-  const size_t sm = smem_deslice(s.G);
+  const bool hilo = s.dot == FS_DOT_BF16X2 && smem_deslice(s.G, true) <= kMaxSmem;  // up to G = 768
+  const size_t sm = smem_deslice(s.G, hilo);
   dim3 grid((unsigned)P, (unsigned)s.BH());
   if ((e = set_smem(k_deslice, sm)) != cudaSuccess) return e;
   k_deslice<<<grid, kThreads, sm, st>>>(xmap, pmap, wimg, zimg, static_cast<__nv_bfloat16*>(out), s.N, Np, s.H, s.G,
-                                        P, status);
+                                        P, hilo ? 1 : 0, status);
   return cudaGetLastError();
 }
 

@@ -28,6 +28,7 @@ _lib = ctypes.CDLL(_LIB_PATH)
 FS_OK, FS_ERR_INVALID, FS_ERR_UNSUPPORTED, FS_ERR_CUDA, FS_ERR_TIMEOUT, FS_ERR_BAD_TAU, FS_ERR_SCRATCH_TOO_SMALL = range(7)
 FS_NOALLOC_SCRATCH_BYTES = 16 << 20
 FS_F32, FS_BF16 = 0, 1
+FS_DOT_BF16, FS_DOT_BF16X2 = 0, 1
 FS_OP_SLICE_FWD, FS_OP_DESLICE_FWD, FS_OP_DESLICE_BWD, FS_OP_SLICE_BWD = range(4)
 
 EXPORTED = ("fs_workspace_bytes", "fs_slice_fwd", "fs_slice_finalize", "fs_mix", "fs_deslice_fwd",
@@ -37,7 +38,7 @@ EXPORTED = ("fs_workspace_bytes", "fs_slice_fwd", "fs_slice_finalize", "fs_mix",
 
 class fs_shape(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int64), ("N", ctypes.c_int64), ("H", ctypes.c_int32), ("d", ctypes.c_int32),
-                ("G", ctypes.c_int32), ("dtype", ctypes.c_int32), ("eps", ctypes.c_float)]
+                ("G", ctypes.c_int32), ("dtype", ctypes.c_int32), ("eps", ctypes.c_float), ("dot", ctypes.c_int32)]
 
 
 class FlashSliceError(RuntimeError):
@@ -71,15 +72,17 @@ for _name, (_res, _args) in _sig.items():
     _f.argtypes = _args
 
 
-def make_shape(B, N, H, d, G, dtype=FS_F32, eps=1e-5) -> fs_shape:
+def make_shape(B, N, H, d, G, dtype=FS_F32, eps=1e-5, dot=None) -> fs_shape:
+    """dot: FS_DOT_BF16 (default) or FS_DOT_BF16X2 (see the header)."""
     if isinstance(dtype, torch.dtype):
         dtype = FS_BF16 if dtype == torch.bfloat16 else FS_F32
-    return fs_shape(int(B), int(N), int(H), int(d), int(G), int(dtype), float(eps))
+    return fs_shape(int(B), int(N), int(H), int(d), int(G), int(dtype), float(eps),
+                    int(FS_DOT_BF16 if dot is None else dot))
 
 
-def shape_of(x_mid: torch.Tensor, G: int, eps: float = 1e-5) -> fs_shape:
+def shape_of(x_mid: torch.Tensor, G: int, eps: float = 1e-5, dot=None) -> fs_shape:
     B, N, H, d = x_mid.shape
-    return make_shape(B, N, H, d, G, x_mid.dtype, eps)
+    return make_shape(B, N, H, d, G, x_mid.dtype, eps, dot)
 
 
 def _ptr(t):
@@ -194,8 +197,13 @@ class Coupling:
     """Allocates the outputs and scratch of one slice -> mix -> deslice coupling
     (forward, and backward when asked) once, then runs it through the C ABI."""
 
-    def __init__(self, B, N, H, d, G, dtype=torch.bfloat16, eps=1e-5, backward=False, device="cuda"):
-        self.shape = make_shape(B, N, H, d, G, dtype, eps)
+    def __init__(self, B, N, H, d, G, dtype=torch.bfloat16, eps=1e-5, backward=False, device="cuda", dot=None):
+        # A coupling that will be differentiated defaults to the split products
+        # (FS_DOT_BF16X2): the temperature gradient is a near-cancelling sum that
+        # bf16 tokens cannot resolve.
+        if dot is None:
+            dot = FS_DOT_BF16X2 if backward else FS_DOT_BF16
+        self.shape = make_shape(B, N, H, d, G, dtype, eps, dot)
         self.dtype = dtype
         f32 = dict(dtype=torch.float32, device=device)
         self.tokens = torch.empty(B, H, G, d, **f32)

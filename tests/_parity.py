@@ -73,3 +73,22 @@ def oracle_forward(wl, heads=None, points=None):
 
 def oracle_backward(wl, heads=None):
     return orc.backward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, wl.dout, eps=wl.eps, heads=heads)
+
+
+def lse_bound(wl, b, h, points, split=False):
+    """Per-point bound on |lse_gpu - lse_exact| for head h of batch b at `points`,
+    from the arithmetic of each path.
+    * fp32 path: fp32 accumulation of the logits: 1e-4 absolute.
+    * bf16 path (tensor cores): W' = W log2(e)/tau is rounded to bf16 (relative
+      error <= 2^-8), or with split products (FS_DOT_BF16X2) rides as two bf16
+      halves, hi + lo (residual <= 2^-16); x is bf16 already, exact; the bias
+      rides as two halves (<= 2^-16). lse is a smooth maximum of the logits, so
+      its error is at most the largest logit error of the point."""
+    pts = np.asarray(points)
+    if wl.dtype == "f32":
+        return np.full(len(pts), 1e-4)
+    Wp = np.abs(wl.W_slice[h].astype(np.float64)) * np.log2(np.e) / wl.tau[h]
+    bp = np.abs(wl.bias[h].astype(np.float64)).max() * np.log2(np.e) / wl.tau[h]
+    s = np.abs(wl.x_mid[b, pts, h, :].astype(np.float64)) @ Wp
+    rel = 2.0 ** -16 if split else 2.0 ** -8
+    return np.log(2.0) * (rel * s.max(axis=1) + 2.0 ** -16 * bp) + 1e-4

@@ -1,0 +1,87 @@
+"""Parity at the full sizes of the five named workloads, against the fp64 oracle.
+
+The GPU runs each workload whole (every batch, point, head and slot).  The
+oracle's cost is bounded by checking a subset that it can compute exactly.
+* Small workloads: every head and point.
+* Large workloads: one head h over all points, for the reductions over points
+  (tokens, weight sums, and for training dW, dbias, dtau, dM, d_tokens_mixed).
+* Outputs and point gradients: a point sample of that head. The sample holds
+  the first and last 64 points (the ragged tail of the last tile) and a
+  seeded random draw.
+Heads do not interact, so one head is checked as it stands in the full run.
+
+Tolerances: fp32 workloads, normwise max relative error <= 1e-4 per tensor;
+bf16 workloads, relative L2 <= 1e-2 per tensor; lse within its per-point
+arithmetic bound (_parity.lse_bound).
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import flashslice_oracle as orc
+from paper_2609_32525_gb300.workloads import NAMED, make_named
+
+from _parity import error, host, lse_bound, tol, upload
+
+pytestmark = pytest.mark.gpu
+
+HEAD = 3
+FULL_ORACLE_ELEMS = 1 << 26  # B*N*H*G up to which every head is checked
+
+
+def _points(N, seed, k=4096):
+    rng = np.random.default_rng(seed)
+    pts = np.concatenate([np.arange(min(64, N)), np.arange(max(0, N - 64), N),
+                          rng.integers(0, N, size=min(k, N))])
+    return np.unique(pts)
+
+
+def _check(name, got, ref, dtype):
+    e = error(got, ref, dtype)
+    assert e <= tol(dtype), f"{name}: error {e:.3e} > {tol(dtype):.0e}"
+
+
+def _gpu_run(lib, wl, dev):
+    tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    c = lib.Coupling(wl.B, wl.N, wl.H, wl.d, wl.G, tdt, wl.eps, backward=wl.dout is not None)
+    c.forward(dev["x_mid"], dev["fx"], dev["W_slice"], dev["bias"], dev["tau"], dev["M"])
+    g = None
+    if wl.dout is not None:
+        g = c.backward(dev["x_mid"], dev["fx"], dev["W_slice"], dev["bias"], dev["tau"], dev["M"], dev["dout"])
+    torch.cuda.synchronize()
+    assert c.device_status() == lib.FS_OK
+    return c, g
+
+
+@pytest.mark.parametrize("name", NAMED)
+def test_full_size_parity(lib, name):
+    wl = make_named(name)
+    dev = upload(wl)
+    c, g = _gpu_run(lib, wl, dev)
+    small = wl.B * wl.N * wl.H * wl.G <= FULL_ORACLE_ELEMS
+    heads = list(range(wl.H)) if small else [HEAD]
+    pts = np.arange(wl.N) if small else _points(wl.N, 1000 + NAMED.index(name))
+
+    ref = orc.forward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, eps=wl.eps, heads=heads, points=pts)
+    hs = np.array(heads)
+    _check("tokens", host(c.tokens)[:, hs], ref["tokens"][:, hs], wl.dtype)
+    _check("wsum", host(c.wsum)[:, hs], ref["wsum"][:, hs], wl.dtype)
+    _check("tokens_mixed", host(c.tokens_mixed)[:, hs], ref["tokens_mixed"][:, hs], wl.dtype)
+    out = host(c.out)
+    _check("out", out[:, pts][:, :, hs], ref["out"][:, pts][:, :, hs], wl.dtype)
+    lse = host(c.lse)  # [B, H, N]
+    for b in range(wl.B):
+        for h in heads:
+            dev_lse = np.abs(lse[b, h, pts] - ref["lse"][b, pts, h])
+            bound = lse_bound(wl, b, h, pts, split=c.shape.dot == lib.FS_DOT_BF16X2)
+            assert (dev_lse <= bound).all(), f"lse b={b} h={h}: worst ratio {(dev_lse / bound).max():.3f}"
+
+    if wl.dout is None:
+        return
+    rb = orc.backward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, wl.dout, eps=wl.eps, heads=heads)
+    _check("d_tokens_mixed", host(c.d_tokens_mixed)[:, hs], rb["d_tokens_mixed"][:, hs], wl.dtype)
+    for k in ("dW", "dbias", "dM"):
+        _check(k, host(g[k])[hs], rb[k][hs], wl.dtype)
+    _check("dtau", host(g["dtau"])[hs], rb["dtau"][hs], wl.dtype)
+    for k in ("dx_mid", "dfx"):
+        _check(k, host(g[k])[:, pts][:, :, hs], rb[k][:, pts][:, :, hs], wl.dtype)
