@@ -226,6 +226,7 @@ def main():
     if not os.path.exists(_build.LIB):
         _build.build()
     from paper_2609_32525_gb300 import flashslice as fs
+    from paper_2609_32525_gb300 import sharding
     from paper_2609_32525_gb300.workloads import make_named
 
     wl = make_named(args.workload, n_override=args.points)
@@ -285,12 +286,9 @@ def main():
     slice_ms = float(np.mean([e[0].elapsed_time(e[1]) for e in evs]))
     mix_ms = float(np.mean([e[1].elapsed_time(e[2]) for e in evs]))
     desl_ms = float(np.mean([e[2].elapsed_time(e[3]) for e in evs]))
-    if world > 1:
-        tt = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        total_ms = float(tt.item())
+    total_ms = sharding.job_time_ms(total_ms, dev)
     ms_per_step = total_ms / args.steps
-    value = world * wl.points / (ms_per_step * 1e-3) / 1e6
+    value = sharding.job_rate(wl.points, world, ms_per_step)
     assert c.device_status() == fs.FS_OK
 
     # End to end through the same C-ABI calls with host buffers: pinned host
@@ -320,11 +318,8 @@ def main():
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = e0.elapsed_time(e1) / args.e2e_steps
-    if world > 1:
-        tt = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        e2e_ms = float(tt.item())
-    e2e_val = world * wl.points / (e2e_ms * 1e-3) / 1e6
+    e2e_ms = sharding.job_time_ms(e2e_ms, dev)
+    e2e_val = sharding.job_rate(wl.points, world, e2e_ms)
     h2d = 2 * hx.numel() * hx.element_size()
     d2h = hout.numel() * hout.element_size()
 

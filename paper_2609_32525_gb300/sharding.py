@@ -1,0 +1,45 @@
+"""Multi-rank host logic: point sharding of one coupling (App. G.4) and the
+job-level timing of runs on several GPUs.  torch.distributed only; no compute.
+
+Point-sharded forward of one coupling over R ranks, rank r holding points
+point_range(N, r, R) of every batch:
+  1. fs_slice_fwd(..., finalize=0) on the local points: unnormalised U and S;
+  2. allreduce_partials(U, S): the sums over all points (the one exchange step,
+     B*H*G*(d+1) floats: 33 KB at H = 8, G = 32, d = 32);
+  3. fs_slice_finalize, fs_mix, then fs_deslice_fwd on the local points.
+The backward exchanges d_tokens_mixed the same way before fs_mix_bwd and
+fs_slice_bwd, and sums the parameter gradients at the end.
+"""
+from __future__ import annotations
+
+import torch
+import torch.distributed as dist
+
+
+def point_range(N: int, rank: int, world: int) -> tuple[int, int]:
+    """Contiguous, balanced point range [n0, n1) of `rank` among `world` ranks."""
+    if world < 1 or not 0 <= rank < world:
+        raise ValueError("rank must lie in [0, world)")
+    return N * rank // world, N * (rank + 1) // world
+
+
+def allreduce_partials(U: torch.Tensor, S: torch.Tensor, group=None) -> None:
+    """Sum the unnormalised numerators U [B,H,G,d] and weight sums S [B,H,G] of
+    all ranks in place (before fs_slice_finalize)."""
+    dist.all_reduce(U, op=dist.ReduceOp.SUM, group=group)
+    dist.all_reduce(S, op=dist.ReduceOp.SUM, group=group)
+
+
+def job_time_ms(local_ms: float, device=None) -> float:
+    """Job time of a timed region: the maximum over ranks of their local times
+    (every rank must call it; a single process returns its own time)."""
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(local_ms)
+    t = torch.tensor([float(local_ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(points_per_rank: int, world: int, ms: float) -> float:
+    """Whole-job throughput in Mpoints/s: every rank's points over the job time."""
+    return world * points_per_rank / (ms * 1e-3) / 1e6

@@ -1,0 +1,89 @@
+"""Multi-rank host logic on CPU: two gloo ranks (world_size 2, spawned processes).
+
+* Point sharding (App. G.4): each rank slices its own point range without
+  normalising (the oracle stands in for fs_slice_fwd on the rank's GPU). The
+  unnormalised numerators and weight sums are summed across ranks with
+  sharding.allreduce_partials, then finalised. The result must equal the
+  unsharded oracle, and so must each rank's deslice of its own points with
+  the reduced tokens.
+* Job timing: the job time is the maximum of the ranks' times, and the
+  job rate counts every rank's points.
+"""
+import os
+import socket
+
+import numpy as np
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+from paper_2609_32525_gb300 import sharding
+
+WORLD = 2
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _worker(rank, port, results):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=WORLD)
+    try:
+        from oracle import flashslice_oracle as orc
+        from paper_2609_32525_gb300.workloads import make_case
+
+        wl = make_case(2, 1001, 3, 8, 7, dtype="f32", seed=41, backward=False)
+        n0, n1 = sharding.point_range(wl.N, rank, WORLD)
+        local = orc.slice_fwd(wl.x_mid[:, n0:n1], wl.fx[:, n0:n1], wl.W_slice, wl.bias, wl.tau, eps=wl.eps,
+                              finalize=False)
+        U = torch.from_numpy(local["tokens"].copy())
+        S = torch.from_numpy(local["wsum"].copy())
+        sharding.allreduce_partials(U, S)
+        tokens = orc.slice_finalize(U.numpy(), S.numpy(), wl.eps)
+        zp = orc.mix(wl.M, tokens)
+        out_local = orc.deslice_fwd(wl.x_mid[:, n0:n1], wl.W_slice, wl.bias, wl.tau, zp)
+
+        ref = orc.forward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, eps=wl.eps)
+        ok_tokens = np.allclose(tokens, ref["tokens"], rtol=1e-12, atol=1e-14)
+        ok_wsum = np.allclose(S.numpy(), ref["wsum"], rtol=1e-12, atol=1e-14)
+        ok_out = np.allclose(out_local, ref["out"][:, n0:n1], rtol=1e-12, atol=1e-14)
+        t = sharding.job_time_ms(1.0 + rank)
+        results[rank] = (ok_tokens, ok_wsum, ok_out, t, (n0, n1))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_point_range_partitions_the_points():
+    for N in (1, 7, 1000, 1001):
+        for world in (1, 2, 3, 8):
+            ranges = [sharding.point_range(N, r, world) for r in range(world)]
+            assert ranges[0][0] == 0 and ranges[-1][1] == N
+            assert all(a[1] == b[0] for a, b in zip(ranges, ranges[1:]))
+            sizes = [b - a for a, b in ranges]
+            assert max(sizes) - min(sizes) <= 1
+    with pytest.raises(ValueError):
+        sharding.point_range(10, 2, 2)
+
+
+def test_single_process_job_time_and_rate():
+    assert sharding.job_time_ms(3.5) == 3.5
+    assert sharding.job_rate(1_000_000, 4, 10.0) == pytest.approx(400.0)
+
+
+def test_two_gloo_ranks_shard_points_and_time_the_job():
+    port = _free_port()
+    with mp.Manager() as mgr:
+        results = mgr.dict()
+        mp.spawn(_worker, args=(port, results), nprocs=WORLD, join=True)
+        res = dict(results)
+    assert sorted(res) == list(range(WORLD))
+    for rank, (ok_tokens, ok_wsum, ok_out, t, rng) in res.items():
+        assert ok_tokens and ok_wsum, f"rank {rank}: reduced tokens differ from the unsharded oracle"
+        assert ok_out, f"rank {rank}: local deslice differs"
+        assert t == float(WORLD)  # max over ranks of 1 + rank
+    assert res[0][4][1] == res[1][4][0]
