@@ -145,9 +145,10 @@ fs_status fs_deslice_fwd(const fs_shape* s, const void* x_mid, const float* W_sl
  *   dx_mid [B,N,H,d], dW [H,d,G], dbias [H,G], dtau [H]: the contribution of
  *   the deslice weights; written if accumulate == 0, added if accumulate != 0.
  *   lse must be the statistics of the forward pass (not NULL).  The backward
- *   forms its weights from fp32 logits; on shapes whose forward runs on the
- *   tensor cores (fs_path_for_shape == 1), whose lse comes from logits with
- *   bf16-rounded W log2(e)/tau, it recomputes lse in fp32 into ws instead. */
+ *   forms its weights from fp32 logits and needs lse to ~1e-5: on tensor-core
+ *   shapes (fs_path_for_shape == 1) with dot = FS_DOT_BF16, whose lse comes
+ *   from logits with bf16-rounded W log2(e)/tau, it recomputes lse with split
+ *   products into ws; otherwise it uses the caller's lse. */
 fs_status fs_deslice_bwd(const fs_shape* s, const void* x_mid, const float* W_slice,
                          const float* bias, const float* tau, const float* tokens_mixed,
                          const float* lse, const void* dout, float* d_tokens_mixed,
@@ -162,7 +163,7 @@ fs_status fs_mix_bwd(const fs_shape* s, const float* M, const float* tokens,
 
 /* Backward of the slice given d_tokens (the gradient w.r.t. the normalised
  * tokens); tokens and wsum are the forward's normalised tokens and S; lse as
- * in fs_deslice_bwd (recomputed in fp32 on the tensor-core path).
+ * in fs_deslice_bwd (recomputed with split products for FS_DOT_BF16).
  *   dfx [B,N,H,d] (overwritten); dx_mid, dW, dbias, dtau: written if
  *   accumulate == 0, added if accumulate != 0. */
 fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx,

@@ -85,6 +85,7 @@ Regions regions(const Shape& s, int op) {
       r.partials = take((size_t)P * BHG * (2 * s.d + 2) * sizeof(float));
       r.dtau_p = take((size_t)s.BH() * simt_point_blocks(s) * sizeof(float));
       r.stats = take(tc_forward_supported(s) ? pts * sizeof(float) : 0);
+      r.tc = take(tc_deslice_prep_bytes(s));
       break;
     case FS_OP_SLICE_BWD:
       r.delta = take(pts * sizeof(float));
@@ -92,6 +93,7 @@ Regions regions(const Shape& s, int op) {
       r.partials = take((size_t)P * BHG * (s.d + 2) * sizeof(float));
       r.dtau_p = take((size_t)s.BH() * simt_point_blocks(s) * sizeof(float));
       r.stats = take(tc_forward_supported(s) ? pts * sizeof(float) : 0);
+      r.tc = take(tc_deslice_prep_bytes(s));
       break;
     default:
       return Regions{};
@@ -116,18 +118,21 @@ fs_status cuda_status(cudaError_t e) { return e == cudaSuccess ? FS_OK : FS_ERR_
 // Every ws-using call starts by clearing its status word.
 cudaError_t reset_status(void* ws, cudaStream_t st) { return cudaMemsetAsync(ws, 0, sizeof(uint32_t), st); }
 
-// The backward forms its weights from fp32 logits.  On shapes whose forward ran on
-// the tensor cores, the forward's lse comes from logits with bf16-rounded
-// W log2(e)/tau, so the backward recomputes it in fp32 (into ws) to normalise its
-// own weights exactly; elsewhere the caller's lse is used as it is.
+// The backward forms its weights from fp32 logits, so it needs lse to ~1e-5.  On
+// tensor-core shapes with bf16 products the forward's lse comes from logits with
+// bf16-rounded W log2(e)/tau: the backward recomputes it with split products (the
+// statistics pass, into ws).  With split products (and on the SIMT path) the
+// caller's lse is already that accurate and is used as it is.
 cudaError_t backward_stats(const Shape& sh, const void* x_mid, const float* W_slice, const float* bias,
                            const float* tau, const float* lse, void* ws, const Regions& r, uint32_t* status,
                            cudaStream_t st, const float** lse_use) {
   *lse_use = lse;
-  if (!tc_forward_supported(sh)) return cudaSuccess;
+  if (!tc_forward_supported(sh) || sh.dot == FS_DOT_BF16X2) return cudaSuccess;
+  Shape split = sh;
+  split.dot = FS_DOT_BF16X2;
   float* buf = at<float>(ws, r.stats);
   *lse_use = buf;
-  return simt_stats(sh, x_mid, W_slice, bias, tau, buf, status, st);
+  return tc_stats(split, x_mid, W_slice, bias, tau, buf, at<void>(ws, r.tc), status, st);
 }
 
 #define FS_CHECK_SHAPE(s)                               \

@@ -122,3 +122,23 @@ def test_tc_full_chain_and_determinism(lib):
     assert rel_l2(host(outs[0][0]), ref["out"]) < 1e-2
     assert torch.equal(outs[0][0].view(torch.int16), outs[1][0].view(torch.int16))
     assert torch.equal(outs[0][1].view(torch.int32), outs[1][1].view(torch.int32))
+
+
+@pytest.mark.parametrize("dot", ["bf16", "bf16x2"])
+def test_tc_forward_then_backward(lib, dot):
+    """The backward after a tensor-core forward, at both product arithmetics: with
+    bf16 products the backward recomputes lse with split products; with split
+    products it takes the forward's.  Every gradient against the oracle."""
+    wl = make_case(2, 3000, 2, 32, 256, dtype="bf16", seed=88, backward=True)
+    dev = upload(wl)
+    c = lib.Coupling(wl.B, wl.N, wl.H, wl.d, wl.G, torch.bfloat16, wl.eps, backward=True,
+                     dot=lib.FS_DOT_BF16X2 if dot == "bf16x2" else lib.FS_DOT_BF16)
+    assert lib.path_for_shape(c.shape) == 1
+    c.forward(dev["x_mid"], dev["fx"], dev["W_slice"], dev["bias"], dev["tau"], dev["M"])
+    g = c.backward(dev["x_mid"], dev["fx"], dev["W_slice"], dev["bias"], dev["tau"], dev["M"], dev["dout"])
+    torch.cuda.synchronize()
+    assert c.device_status() == lib.FS_OK
+    ref = orc.backward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, wl.dout, eps=wl.eps)
+    for k in ("dx_mid", "dfx", "dW", "dbias", "dtau", "dM"):
+        e = rel_l2(host(g[k]), ref[k])
+        assert e < 1e-2, f"{k} rel L2 {e:.3e}"
