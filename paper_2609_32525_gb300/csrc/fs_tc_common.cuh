@@ -1,0 +1,356 @@
+// Pieces shared by the tensor-core kernels of the forward (fs_tc_fwd.cu) and the
+// backward (fs_tc_bwd.cu): tile constants, the operand images and their prep
+// kernels, block bookkeeping, the logits MMA chain, the slice-weight helpers and
+// the host-side tensor maps, splits and launch helpers.  Internal linkage: every
+// translation unit that includes it gets its own copy.
+#pragma once
+
+#include "fs_tc.h"
+#include "fs_tc_ptx.cuh"
+
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+#include <mutex>
+
+namespace fs {
+namespace {
+
+using namespace tc;
+
+constexpr int kThreads = 384;
+constexpr int kTile = 128;        // points per tile
+constexpr int kGC = 128;          // slots per logits block
+constexpr int kD = 32;            // head width of the tensor-core path
+constexpr int kSoftmaxWarp0 = 4;  // warps 4..11: two softmax warpgroups
+constexpr int kStages = 3;        // x-tile pipeline depth (stats / deslice)
+constexpr int kSliceStages = 8;   // slice pipeline depth (it streams x, F and px for every 128 slots)
+constexpr int kSBuf = 3;          // S buffers (logits run up to two blocks ahead)
+constexpr uint32_t kXBytes = kTile * 64;   // 128 points x 32 bf16
+constexpr uint32_t kExBytes = kTile * 32;  // 128 rows x 16 bf16
+constexpr uint32_t kFBlock = kTile * 32;   // 128 points x 16 channels
+constexpr uint32_t kPxBytes = kTile * 16;  // 128 point-extra rows of 8 bf16 (k = 0..7)
+constexpr uint64_t kWaitNs = 2000000000ull;
+
+// ---- operand images written by the prep kernels -------------------------------------------
+// W image for head h (kWRow = 160 bytes per slot): G rows (slots) x 64 B of
+// W' = W*log2e/tau rounded to bf16 (64B swizzle), then G rows x 32 B of
+// [b'_hi, b'_lo, 1, 1, 0...] (32B swizzle), then G rows x 64 B of the residual
+// W' - bf16(W') rounded to bf16 (64B swizzle).  The statistics and slice passes
+// use both halves of W' (their lse, tokens and weight sums then carry no
+// systematic per-slot rounding of the weights); the deslice uses the first half.
+constexpr uint32_t kWRow = 160;
+__device__ __forceinline__ uint32_t off_sw64(int row, int k) {  // k in [0, 32)
+  const int chunk = k >> 3;
+  return (uint32_t)((row >> 3) * 512 + (row & 7) * 64 + ((chunk ^ ((row & 7) >> 1)) << 4) + (k & 7) * 2);
+}
+__device__ __forceinline__ uint32_t off_sw32(int row, int k) {  // k in [0, 16)
+  const int chunk = k >> 3;
+  return (uint32_t)((row >> 3) * 256 + (row & 7) * 32 + ((chunk ^ ((row & 7) >> 2)) << 4) + (k & 7) * 2);
+}
+// Z' image for (b,h): blocks of 64 slots, each 32 rows (channels) x 128 B (128B swizzle).
+__device__ __forceinline__ uint32_t off_z(int c, int g) {
+  const int kb = g >> 6, w = g & 63;
+  return (uint32_t)(kb * 4096 + (c >> 3) * 1024 + (c & 7) * 128 + (((w >> 3) ^ (c & 7)) << 4) + (w & 7) * 2);
+}
+
+__global__ void k_prep_w(const float* __restrict__ W, const float* __restrict__ bias, const float* __restrict__ tau,
+                         uint8_t* __restrict__ img, int H, int G, uint32_t* status) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t total = (int64_t)H * G;
+  if (i >= total) return;
+  const int h = (int)(i / G), g = (int)(i % G);
+  const float t = tau[h];
+  if (!(t > 0.f && t < INFINITY)) {
+    atomicCAS(status, 0u, (uint32_t)FS_ERR_BAD_TAU);
+    return;
+  }
+  const float scale = kLog2e / t;
+  uint8_t* base = img + (size_t)h * G * kWRow;
+  __nv_bfloat16* wp = reinterpret_cast<__nv_bfloat16*>(base);
+  __nv_bfloat16* wl = reinterpret_cast<__nv_bfloat16*>(base + (size_t)G * 96);
+  for (int k = 0; k < kD; k++) {
+    const float w2 = W[((int64_t)h * kD + k) * G + g] * scale;
+    const __nv_bfloat16 whi = __float2bfloat16_rn(w2);
+    wp[off_sw64(g, k) / 2] = whi;
+    wl[off_sw64(g, k) / 2] = __float2bfloat16_rn(w2 - __bfloat162float(whi));
+  }
+  __nv_bfloat16* ep = reinterpret_cast<__nv_bfloat16*>(base + (size_t)G * 64);
+  const float b2 = bias[(int64_t)h * G + g] * scale;
+  const __nv_bfloat16 hi = __float2bfloat16_rn(b2);
+  const __nv_bfloat16 lo = __float2bfloat16_rn(b2 - __bfloat162float(hi));
+  // k = 2, 3 multiply the point side's -lse2 halves (zero in the statistics pass).
+  for (int k = 0; k < 16; k++)
+    ep[off_sw32(g, k) / 2] =
+        k == 0 ? hi : (k == 1 ? lo : __float2bfloat16_rn((k == 2 || k == 3) ? 1.f : 0.f));
+}
+
+__global__ void k_prep_z(const float* __restrict__ zp, uint8_t* __restrict__ img, int64_t BH, int G) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t total = BH * G * kD;
+  if (i >= total) return;
+  const int c = (int)(i % kD);
+  const int g = (int)((i / kD) % G);
+  const int64_t bh = i / ((int64_t)kD * G);
+  __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * G * 64);
+  out[off_z(c, g) / 2] = __float2bfloat16_rn(zp[i]);
+}
+
+// ---- shared pieces -------------------------------------------------------------------------
+struct Work {
+  int64_t bh;      // batch * H + head
+  int64_t tile0;   // first point tile of this CTA
+  int ntiles;      // number of point tiles (the host keeps all point indices below 2^31)
+};
+
+// Tile i and slot block c of block q = i * nb + c, kept up to date while q walks
+// with a fixed stride, so that no loop divides by the runtime block count (a
+// 64-bit division per block cost as much as a block's exponentials).
+struct BlockPos {
+  int i, c;
+  __device__ __forceinline__ BlockPos(int q0, int nb) : i(0), c(q0) {
+    while (c >= nb) { c -= nb; ++i; }
+  }
+  __device__ __forceinline__ void step(int by, int nb) {
+    c += by;
+    while (c >= nb) { c -= nb; ++i; }
+  }
+};
+
+// CTA (split p of unit bh) processes a contiguous range of point tiles.
+__device__ __forceinline__ Work work_of(int64_t N, int splits, int p, int64_t bh) {
+  Work w;
+  w.bh = bh;
+  const int64_t tiles = (N + kTile - 1) / kTile;
+  w.tile0 = tiles * p / splits;
+  w.ntiles = (int)(tiles * (p + 1) / splits - w.tile0);
+  return w;
+}
+
+// The constant point-side extra block: every row [1, 1, 0 x 14] (32B swizzle).
+__device__ __forceinline__ void write_const_extra(uint8_t* ex) {
+  for (int r = threadIdx.x; r < kTile; r += blockDim.x) {
+    const uint32_t base = smem_u32(ex) + (uint32_t)((r >> 3) * 256 + (r & 7) * 32);
+    const uint32_t sw = (uint32_t)((r & 7) >> 2);
+    st_shared_v4(base + ((0u ^ sw) << 4), 0x3F803F80u, 0u, 0u, 0u);
+    st_shared_v4(base + ((1u ^ sw) << 4), 0u, 0u, 0u, 0u);
+  }
+}
+
+// Descriptors of the two kinds of point-side extra block: the constant one
+// (32B swizzle) and the per-tile one loaded by TMA (no swizzle; the k = 0..7
+// core matrices at px, the zero k = 8..15 half kPxBytes further on).
+__device__ __forceinline__ uint64_t const_extra_desc(uint32_t ex_s) { return sdesc(ex_s, 16, 256, kSw32); }
+__device__ __forceinline__ uint64_t point_extra_desc(uint32_t px_s) { return sdesc(px_s, kPxBytes, 128, 0); }
+__device__ __forceinline__ void zero_smem(uint8_t* p, uint32_t bytes) {
+  for (uint32_t o = threadIdx.x * 16; o < bytes; o += blockDim.x * 16) st_shared_v4(smem_u32(p) + o, 0u, 0u, 0u, 0u);
+}
+
+// Base-2 logits of 128 points x 128 slots (chunk c of the W image) into TMEM.
+//   point_major: A = points (x tile), B = slots (W);  else A = slots, B = points.
+//   xe: descriptor of the point-side extra block.
+//   wl_img: the residual half of W' (0: bf16 W' only, K = 48; else K = 80).
+__device__ __forceinline__ void issue_logits(uint32_t tmem_d, uint32_t x_s, uint64_t xe, uint32_t w_img,
+                                             uint32_t we_img, uint32_t wl_img, int c, bool point_major) {
+  constexpr uint32_t idesc = idesc_bf16(128, kGC, false, false);
+  const uint32_t wc = w_img + (uint32_t)c * kGC * 64;
+  const uint32_t wec = we_img + (uint32_t)c * kGC * 32;
+  const uint64_t x0 = sdesc(x_s, 16, 512, kSw64), x1 = sdesc(x_s + 32, 16, 512, kSw64);
+  const uint64_t w0 = sdesc(wc, 16, 512, kSw64), w1 = sdesc(wc + 32, 16, 512, kSw64);
+  const uint64_t we = sdesc(wec, 16, 256, kSw32);
+  if (point_major) {
+    mma_ss_w(tmem_d, x0, w0, idesc, 0);
+    mma_ss_w(tmem_d, x1, w1, idesc, 1);
+  } else {
+    mma_ss_w(tmem_d, w0, x0, idesc, 0);
+    mma_ss_w(tmem_d, w1, x1, idesc, 1);
+  }
+  if (wl_img) {
+    const uint32_t wlc = wl_img + (uint32_t)c * kGC * 64;
+    const uint64_t l0 = sdesc(wlc, 16, 512, kSw64), l1 = sdesc(wlc + 32, 16, 512, kSw64);
+    if (point_major) {
+      mma_ss_w(tmem_d, x0, l0, idesc, 1);
+      mma_ss_w(tmem_d, x1, l1, idesc, 1);
+    } else {
+      mma_ss_w(tmem_d, l0, x0, idesc, 1);
+      mma_ss_w(tmem_d, l1, x1, idesc, 1);
+    }
+  }
+  if (point_major)
+    mma_ss_w(tmem_d, xe, we, idesc, 1);
+  else
+    mma_ss_w(tmem_d, we, xe, idesc, 1);
+}
+
+// Producer-side bulk loads of an image into smem (pieces of at most 32 KB).
+__device__ __forceinline__ void load_images(uint8_t* dst, const uint8_t* src, uint32_t bytes, uint64_t* bar) {
+  constexpr uint32_t kPiece = 32768;
+  for (uint32_t off = 0; off < bytes; off += kPiece) {
+    const uint32_t n = (bytes - off) < kPiece ? (bytes - off) : kPiece;
+    bulk_load(dst + off, src + off, n, bar);
+  }
+}
+
+// 2^t for 32 log2-weights -> 16 bf16x2 words.
+__device__ __forceinline__ void weights32(const uint32_t (&v)[32], uint32_t (&p)[16]) {
+#pragma unroll
+  for (int k = 0; k < 16; k++) p[k] = pack_bf16(ex2(__uint_as_float(v[2 * k])), ex2(__uint_as_float(v[2 * k + 1])));
+}
+
+// The 128 log2-weights of one TMEM lane of an S buffer -> bf16 weights written back
+// in place, packed in pairs, into the first 64 columns, in two halves: columns
+// [64 h, 64 h + 64) -> packed weights in columns [32 h, 32 h + 32), which this
+// thread has already read.
+// 2^t for 32 log2-weights -> the bf16 pairs (hi) and the bf16 pairs of the
+// residuals w - hi (lo): w = hi + lo to ~2^-16 relative.
+__device__ __forceinline__ void weights32_hilo(const uint32_t (&v)[32], uint32_t (&hi)[16], uint32_t (&lo)[16]) {
+#pragma unroll
+  for (int k = 0; k < 16; k++) {
+    const float w0 = ex2(__uint_as_float(v[2 * k])), w1 = ex2(__uint_as_float(v[2 * k + 1]));
+    const uint32_t p = pack_bf16(w0, w1);
+    const float h0 = __uint_as_float(p << 16), h1 = __uint_as_float(p & 0xFFFF0000u);
+    hi[k] = p;
+    lo[k] = pack_bf16(w0 - h0, w1 - h1);
+  }
+}
+
+// Slice weights of one TMEM lane (a slot) of an S buffer, 128 points: the hi
+// halves packed in pairs into columns [0, 64), the lo halves into [64, 128).
+// Half h reads columns [64 h, 64 h + 64); the lo pairs of half 0 wait in
+// registers until half 1 has read the columns they go to.
+__device__ __forceinline__ void weights_hilo_in_place(uint32_t tS) {
+  uint32_t lo0[16], lo1[16];
+  {
+    uint32_t v0[32], v1[32];
+    tmem_ld32(tS, v0);
+    tmem_ld32(tS + 32, v1);
+    tmem_wait_ld2(v0, v1);
+    uint32_t hi0[16], hi1[16];
+    weights32_hilo(v0, hi0, lo0);
+    weights32_hilo(v1, hi1, lo1);
+    tmem_st16(tS, hi0);
+    tmem_st16(tS + 16, hi1);
+  }
+  uint32_t v0[32], v1[32];
+  tmem_ld32(tS + 64, v0);
+  tmem_ld32(tS + 96, v1);
+  tmem_wait_ld2(v0, v1);
+  tmem_st16(tS + 64, lo0);
+  tmem_st16(tS + 80, lo1);
+  uint32_t hi0[16], hi1[16];
+  weights32_hilo(v0, hi0, lo0);
+  weights32_hilo(v1, hi1, lo1);
+  tmem_st16(tS + 32, hi0);
+  tmem_st16(tS + 48, hi1);
+  tmem_st16(tS + 96, lo0);
+  tmem_st16(tS + 112, lo1);
+}
+
+__device__ __forceinline__ void weights_in_halves(uint32_t tS) {
+#pragma unroll 1
+  for (int half = 0; half < 2; half++) {
+    uint32_t v0[32], v1[32];
+    tmem_ld32(tS + half * 64, v0);
+    tmem_ld32(tS + half * 64 + 32, v1);
+    tmem_wait_ld2(v0, v1);
+    uint32_t pk0[16], pk1[16];
+    weights32(v0, pk0);
+    weights32(v1, pk1);
+    tmem_st16(tS + half * 32, pk0);
+    tmem_st16(tS + half * 32 + 16, pk1);
+  }
+}
+
+// Point-extra rows [1, 1, -lse2_hi, -lse2_lo, 0, 0, 0, 0] (bf16) from lse [B,H,N]
+// (natural log) into px [B*H, Np, 8]; padded points (n >= N) get -1e30 so that
+// their weights vanish.
+__global__ void k_prep_px(const float* __restrict__ lse, uint4* __restrict__ px, int64_t BH, int64_t N, int64_t Np) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= BH * Np) return;
+  const int64_t bh = i / Np, n = i % Np;
+  const float nl2 = n < N ? -lse[bh * N + n] * kLog2e : -1e30f;
+  const __nv_bfloat16 hi = __float2bfloat16_rn(nl2);
+  const __nv_bfloat16 lo = __float2bfloat16_rn(nl2 - __bfloat162float(hi));
+  px[i] = make_uint4(0x3F803F80u, (uint32_t)__bfloat16_as_ushort(hi) | ((uint32_t)__bfloat16_as_ushort(lo) << 16), 0u, 0u);
+}
+
+// ---- host side -------------------------------------------------------------------------------
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 3-D view of a [B, N, C] bf16 tensor; box = (box_c channels, 128 points, 1).
+bool make_point_map(CUtensorMap* map, const void* ptr, const Shape& s, int box_c, CUtensorMapSwizzle sw) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  const uint64_t C = (uint64_t)s.H * s.d;
+  cuuint64_t dims[3] = {C, (cuuint64_t)s.N, (cuuint64_t)s.B};
+  cuuint64_t strides[2] = {C * 2, (cuuint64_t)s.N * C * 2};
+  cuuint32_t box[3] = {(cuuint32_t)box_c, (cuuint32_t)kTile, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// 2-D view of the point-extra rows [B*H*Np, 8] bf16; box = (8, 128 points).
+bool make_px_map(CUtensorMap* map, const void* ptr, int64_t BH, int64_t Np) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {8, (cuuint64_t)(BH * Np)};
+  cuuint64_t strides[1] = {16};
+  cuuint32_t box[2] = {8, (cuuint32_t)kTile};
+  cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+size_t w_image_bytes(const Shape& s) { return (size_t)s.H * s.G * kWRow; }
+size_t z_image_bytes(const Shape& s) { return (size_t)s.BH() * s.G * 64; }
+int64_t padded_n(const Shape& s) { return (s.N + kTile - 1) / kTile * kTile; }
+size_t px_bytes(const Shape& s) { return (size_t)s.BH() * padded_n(s) * 16; }
+
+// Point splits per work unit for one-CTA-per-SM kernels: the split count P that
+// minimises the makespan in units of one unit's work, ceil(units * P / SMs) / P
+// (whole waves of CTAs), smallest P on ties; at most one split per point tile.
+int point_splits(const Shape& s, int units) {
+  const int64_t tiles = (s.N + kTile - 1) / kTile;
+  const int64_t sms = num_sms();
+  if (units < 1) units = 1;
+  int64_t best = 1;
+  double best_t = 1e30;
+  for (int64_t p = 1; p <= 2 * sms && p <= tiles; p++) {
+    const double t = (double)((units * p + sms - 1) / sms) / (double)p;
+    if (t < best_t - 1e-12) {
+      best_t = t;
+      best = p;
+    }
+  }
+  return (int)best;
+}
+
+constexpr size_t kMaxSmem = 232448;  // opt-in shared memory per block on sm_103
+template <typename K>
+cudaError_t set_smem(K kernel, size_t bytes) {
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+}
+
+cudaError_t prep_w(const Shape& s, const float* W, const float* bias, const float* tau, uint8_t* img,
+                   uint32_t* status, cudaStream_t st) {
+  const int64_t n = (int64_t)s.H * s.G;
+  k_prep_w<<<(unsigned)((n + 127) / 128), 128, 0, st>>>(W, bias, tau, img, s.H, s.G, status);
+  return cudaGetLastError();
+}
+
+}  // namespace
+}  // namespace fs
