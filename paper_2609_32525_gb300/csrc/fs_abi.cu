@@ -3,6 +3,7 @@
 #include "fs_internal.h"
 #include "fs_tc.h"
 
+#include <algorithm>
 #include <cmath>
 #include <cstring>
 
@@ -81,6 +82,11 @@ Regions regions(const Shape& s, int op) {
       r.tc = take(tc_deslice_prep_bytes(s));
       break;
     case FS_OP_DESLICE_BWD:
+      if (tc_backward_supported(s)) {
+        r.stats = take(pts * sizeof(float));
+        r.tc = take(std::max(tc_backward_bytes(s, 1), tc_deslice_prep_bytes(s)));
+        break;
+      }
       r.delta = take(pts * sizeof(float));
       r.partials = take((size_t)P * BHG * (2 * s.d + 2) * sizeof(float));
       r.dtau_p = take((size_t)s.BH() * simt_point_blocks(s) * sizeof(float));
@@ -88,8 +94,13 @@ Regions regions(const Shape& s, int op) {
       r.tc = take(tc_deslice_prep_bytes(s));
       break;
     case FS_OP_SLICE_BWD:
-      r.delta = take(pts * sizeof(float));
       r.dus = take(BHG * (s.d + 1) * sizeof(float));
+      if (tc_backward_supported(s)) {
+        r.stats = take(pts * sizeof(float));
+        r.tc = take(std::max(tc_backward_bytes(s, 2), tc_deslice_prep_bytes(s)));
+        break;
+      }
+      r.delta = take(pts * sizeof(float));
       r.partials = take((size_t)P * BHG * (s.d + 2) * sizeof(float));
       r.dtau_p = take((size_t)s.BH() * simt_point_blocks(s) * sizeof(float));
       r.stats = take(tc_forward_supported(s) ? pts * sizeof(float) : 0);
@@ -183,6 +194,11 @@ int fs_path_for_shape(const fs_shape* s) {
   return tc_forward_supported(to_shape(s)) ? 1 : 0;
 }
 
+int fs_backward_path_for_shape(const fs_shape* s) {
+  if (!valid_shape(s) || !supported_shape(s)) return -1;
+  return tc_backward_supported(to_shape(s)) ? 1 : 0;
+}
+
 int fs_forward_launch_count(const fs_shape* s) {
   if (!valid_shape(s) || !supported_shape(s)) return -1;
   const Shape sh = to_shape(s);
@@ -271,6 +287,10 @@ fs_status fs_deslice_bwd(const fs_shape* s, const void* x_mid, const float* W_sl
   FS_CUDA(reset_status(ws, st));
   const float* lse_use = nullptr;
   FS_CUDA(backward_stats(sh, x_mid, W_slice, bias, tau, lse, ws, r, at<uint32_t>(ws, r.status), st, &lse_use));
+  if (tc_backward_supported(sh))
+    return cuda_status(tc_deslice_bwd(sh, x_mid, W_slice, bias, tau, tokens_mixed, lse_use, dout, d_tokens_mixed,
+                                      dx_mid, dW, dbias, dtau, accumulate, at<void>(ws, r.tc),
+                                      at<uint32_t>(ws, r.status), st));
   return cuda_status(simt_deslice_bwd(sh, slot_splits(sh), x_mid, W_slice, bias, tau, tokens_mixed, lse_use, dout,
                                       d_tokens_mixed, dx_mid, dW, dbias, dtau, accumulate, at<float>(ws, r.delta),
                                       at<float>(ws, r.partials), at<float>(ws, r.dtau_p),
@@ -301,6 +321,10 @@ fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx, con
   FS_CUDA(reset_status(ws, st));
   const float* lse_use = nullptr;
   FS_CUDA(backward_stats(sh, x_mid, W_slice, bias, tau, lse, ws, r, at<uint32_t>(ws, r.status), st, &lse_use));
+  if (tc_backward_supported(sh))
+    return cuda_status(tc_slice_bwd(sh, x_mid, fx, W_slice, bias, tau, tokens, wsum, lse_use, d_tokens, dx_mid, dfx,
+                                    dW, dbias, dtau, accumulate, at<float>(ws, r.dus), at<void>(ws, r.tc),
+                                    at<uint32_t>(ws, r.status), st));
   return cuda_status(simt_slice_bwd(sh, slot_splits(sh), x_mid, fx, W_slice, bias, tau, tokens, wsum, lse_use,
                                     d_tokens, dx_mid, dfx, dW, dbias, dtau, accumulate, at<float>(ws, r.delta),
                                     at<float>(ws, r.dus), at<float>(ws, r.partials), at<float>(ws, r.dtau_p),

@@ -679,19 +679,26 @@ cudaError_t launch_bwd_slice(const Shape& s, int P, const void* x, const void* v
                              status, st);
 }
 
-cudaError_t reduce_params(const Shape& s, int P, const float* part, int PS, int has_dzp, const float* tau,
-                          float* dzp, float* dW, float* db, float* dtau, const float* dt_part, int accumulate,
-                          cudaStream_t st) {
+}  // namespace
+
+cudaError_t simt_reduce_bwd(const Shape& s, int P, const float* part, int PS, int has_dzp, const float* tau,
+                            float* dzp, float* dW, float* db, float* dtau, const float* dt_part, int64_t nblk,
+                            int accumulate, cudaStream_t st) {
   const int64_t HG = (int64_t)s.H * s.G;
   k_reduce_bwd<<<(unsigned)((HG + 127) / 128), 128, 0, st>>>(part, P, s.B, s.H, s.G, s.d, PS, has_dzp, tau,
                                                               dzp, dW, db, accumulate);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_reduce_dtau<<<s.H, 256, 0, st>>>(dt_part, s.B, s.H, simt_point_blocks(s), tau, dtau, accumulate);
+  k_reduce_dtau<<<s.H, 256, 0, st>>>(dt_part, s.B, s.H, nblk, tau, dtau, accumulate);
   return cudaGetLastError();
 }
 
-}  // namespace
+cudaError_t simt_slice_bwd_prep(const Shape& s, const float* z, const float* wsum, const float* dz, float* dUS,
+                                cudaStream_t st) {
+  const int64_t BHG = s.BH() * s.G;
+  k_slice_bwd_prep<<<(unsigned)((BHG + 255) / 256), 256, 0, st>>>(z, wsum, dz, dUS, BHG, s.d, s.eps);
+  return cudaGetLastError();
+}
 
 int64_t simt_point_blocks(const Shape& s) { return (s.N + kThreads - 1) / kThreads; }
 
@@ -751,7 +758,8 @@ cudaError_t simt_deslice_bwd(const Shape& s, int P, const void* x, const float* 
                 accumulate, status, st);
   }();
   if (e != cudaSuccess) return e;
-  return reduce_params(s, P, part, 2 * s.d + 2, 1, tau, dzp, dW, db, dtau, dt_part, accumulate, st);
+  return simt_reduce_bwd(s, P, part, 2 * s.d + 2, 1, tau, dzp, dW, db, dtau, dt_part, simt_point_blocks(s),
+                         accumulate, st);
 }
 
 cudaError_t simt_slice_bwd(const Shape& s, int P, const void* x, const void* f, const float* W,
@@ -759,16 +767,15 @@ cudaError_t simt_slice_bwd(const Shape& s, int P, const void* x, const void* f, 
                            const float* lse, const float* dz, void* dx, void* dfx, float* dW, float* db,
                            float* dtau, int accumulate, float* delta, float* dUS, float* part, float* dt_part,
                            uint32_t* status, cudaStream_t st) {
-  const int64_t BHG = s.BH() * s.G;
-  k_slice_bwd_prep<<<(unsigned)((BHG + 255) / 256), 256, 0, st>>>(z, wsum, dz, dUS, BHG, s.d, s.eps);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = simt_slice_bwd_prep(s, z, wsum, dz, dUS, st);
   if (e != cudaSuccess) return e;
   e = [&]() -> cudaError_t {
     FS_DISPATCH(s, launch_bwd_slice, s, P, x, f, W, bias, tau, dUS, lse, dx, dfx, delta, dt_part, part,
                 accumulate, status, st);
   }();
   if (e != cudaSuccess) return e;
-  return reduce_params(s, P, part, s.d + 2, 0, tau, nullptr, dW, db, dtau, dt_part, accumulate, st);
+  return simt_reduce_bwd(s, P, part, s.d + 2, 0, tau, nullptr, dW, db, dtau, dt_part, simt_point_blocks(s),
+                         accumulate, st);
 }
 
 }  // namespace fs

@@ -1,0 +1,837 @@
+// Tensor-core backward (tcgen05 / TMEM / TMA) for bf16 inputs on sm_103a.
+//
+// The gradients of the slice and of the deslice (Sec. 3.3) share one form.  With
+// w_ng = softmax_g(a_ng), a per-point vector v_n and per-slot t_g, c_g:
+//   dw_ng = v_n . t_g + c_g,   delta_n = sum_g w_ng dw_ng,   da_ng = w_ng (dw_ng - delta_n)
+//   deslice: v = dO, t = z', c = 0;   slice: v = fx, t = dU = dz/(S+eps), c = dS = -dz.z/(S+eps)
+// and then
+//   dx_n = (1/tau) sum_g da_ng W[:,g],   dW[:,g] = (1/tau) sum_n da_ng x_n,
+//   dbias_g = (1/tau) sum_n da_ng,       dtau = -(1/tau) sum_n sum_g da_ng (a_ng - lse_n),
+//   deslice also d z'_g = sum_n w_ng dO_n;  slice also dfx_n = sum_g w_ng dU_g.
+// Three passes, w recomputed in each and never written to memory:
+//   rows  (point-owned; the deslice kernel in a backward mode): delta_n (and dfx_n);
+//   slot  (slot-owned, split over points): dW, dbias, dtau (and d z') partials;
+//   point (point-owned): dx.
+// dw - delta is one more MMA chain of the logits' shape: the slot side carries
+// [t_g | c_g halves, 1, 1] (the T image, laid out as the W image) and the point
+// side [v_n | 1, 1, -delta_n halves] (delta's point-extra rows).
+#include "fs_tc_common.cuh"
+
+namespace fs {
+namespace {
+
+using namespace tc;
+
+constexpr int kBStages = 6;                            // slot pass pipeline depth (point tiles)
+constexpr int kDxStages = 3;                           // point pass pipeline depth
+constexpr uint32_t kBStage = 2 * kXBytes + 2 * kPxBytes;  // x | v | lse rows | delta rows (TMA halves)
+constexpr uint32_t kPxZero = 2 * kPxBytes;             // one zero block for the k = 8..15 halves
+constexpr uint32_t kWBlockB = kGC * kWRow;             // one 128-slot block of a W or T image
+
+// ---- prep kernels ------------------------------------------------------------------------------
+
+// T image of (b,h), in the W image's layout (kWRow bytes per slot): t_g rounded to
+// bf16, the extra rows [c_hi, c_lo, 1, 1, 0...], the residual t_g - bf16(t_g).
+// t: [BH][G][tstride] fp32, c_g = t[..][32] when has_c.  Also writes c_g to c_out [BH][G].
+__global__ void k_prep_t(const float* __restrict__ t, int tstride, int has_c, uint8_t* __restrict__ img,
+                         float* __restrict__ c_out, int64_t BH, int G) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= BH * G) return;
+  const int64_t bh = i / G;
+  const int g = (int)(i % G);
+  const float* src = t + i * tstride;
+  uint8_t* base = img + (size_t)bh * G * kWRow;
+  __nv_bfloat16* hp = reinterpret_cast<__nv_bfloat16*>(base);
+  __nv_bfloat16* lp = reinterpret_cast<__nv_bfloat16*>(base + (size_t)G * 96);
+  for (int k = 0; k < kD; k++) {
+    const float v = src[k];
+    const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+    hp[off_sw64(g, k) / 2] = hi;
+    lp[off_sw64(g, k) / 2] = __float2bfloat16_rn(v - __bfloat162float(hi));
+  }
+  const float c = has_c ? src[kD] : 0.f;
+  if (c_out) c_out[i] = c;
+  const __nv_bfloat16 chi = __float2bfloat16_rn(c);
+  const __nv_bfloat16 clo = __float2bfloat16_rn(c - __bfloat162float(chi));
+  __nv_bfloat16* ep = reinterpret_cast<__nv_bfloat16*>(base + (size_t)G * 64);
+  for (int k = 0; k < 16; k++)
+    ep[off_sw32(g, k) / 2] = k == 0 ? chi : (k == 1 ? clo : __float2bfloat16_rn((k == 2 || k == 3) ? 1.f : 0.f));
+}
+
+// Z-layout image (blocks of 64 slots, 32 channel rows x 128 B, 128B swizzle) of
+// t [BH][G][tstride] per (b,h): the bf16 half, then the residual half (G*128 bytes per (b,h)).
+__global__ void k_prep_z2(const float* __restrict__ t, int tstride, uint8_t* __restrict__ img, int64_t BH, int G) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= BH * G * kD) return;
+  const int c = (int)(i % kD);
+  const int g = (int)((i / kD) % G);
+  const int64_t bh = i / ((int64_t)kD * G);
+  const float v = t[(bh * G + g) * tstride + c];
+  __nv_bfloat16* hp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * G * 128);
+  __nv_bfloat16* lp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * G * 128 + (size_t)G * 64);
+  const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+  hp[off_z(c, g) / 2] = hi;
+  lp[off_z(c, g) / 2] = __float2bfloat16_rn(v - __bfloat162float(hi));
+}
+
+// W'^T image of head h in the Z layout (channel rows, slots along K), W' =
+// W log2(e)/tau: the bf16 half, then the residual half (G*128 bytes per head).
+// It is the B operand of dx += da W'^T.
+__global__ void k_prep_wt(const float* __restrict__ W, const float* __restrict__ tau, uint8_t* __restrict__ img,
+                          int H, int G, uint32_t* status) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= (int64_t)H * kD * G) return;
+  const int g = (int)(i % G);
+  const int c = (int)((i / G) % kD);
+  const int h = (int)(i / ((int64_t)kD * G));
+  const float tv = tau[h];
+  if (!(tv > 0.f && tv < INFINITY)) {
+    atomicCAS(status, 0u, (uint32_t)FS_ERR_BAD_TAU);
+    return;
+  }
+  const float v = W[i] * (kLog2e / tv);
+  __nv_bfloat16* hp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)h * G * 128);
+  __nv_bfloat16* lp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)h * G * 128 + (size_t)G * 64);
+  const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+  hp[off_z(c, g) / 2] = hi;
+  lp[off_z(c, g) / 2] = __float2bfloat16_rn(v - __bfloat162float(hi));
+}
+
+// delta's point-extra rows [1, 1, -delta_hi, -delta_lo, 0, 0, 0, 0] into dpx [BH, Np, 8];
+// delta_n = delta[bh][n] (+ wds[0][bh][n] + wds[1][bh][n] when wds is given).
+__global__ void k_prep_dpx(const float* __restrict__ delta, const float* __restrict__ wds, uint4* __restrict__ dpx,
+                           int64_t BH, int64_t N, int64_t Np) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= BH * Np) return;
+  const int64_t bh = i / Np, n = i % Np;
+  float d = 0.f;
+  if (n < N) {
+    d = delta[bh * N + n];
+    if (wds) d += wds[bh * N + n] + wds[(BH + bh) * N + n];
+  }
+  const __nv_bfloat16 hi = __float2bfloat16_rn(-d);
+  const __nv_bfloat16 lo = __float2bfloat16_rn(-d - __bfloat162float(hi));
+  dpx[i] = make_uint4(0x3F803F80u, (uint32_t)__bfloat16_as_ushort(hi) | ((uint32_t)__bfloat16_as_ushort(lo) << 16),
+                      0u, 0u);
+}
+
+// ---- device pieces -----------------------------------------------------------------------------
+
+// M = 128 x N = 64 product with K = 48 (80 with the residual half, lo_a or lo_b):
+// a0/b0 are the K-major 64B-swizzled 32-channel blocks, ae/be the extra blocks.
+template <bool kLoA>
+__device__ __forceinline__ void issue_dot64(uint32_t d, uint32_t a, uint32_t b, uint64_t ae, uint64_t be,
+                                            uint32_t lo) {
+  constexpr uint32_t idesc = idesc_bf16(128, 64, false, false);
+  mma_ss_w(d, sdesc(a, 16, 512, kSw64), sdesc(b, 16, 512, kSw64), idesc, 0);
+  mma_ss_w(d, sdesc(a + 32, 16, 512, kSw64), sdesc(b + 32, 16, 512, kSw64), idesc, 1);
+  if (lo) {
+    if (kLoA) {
+      mma_ss_w(d, sdesc(lo, 16, 512, kSw64), sdesc(b, 16, 512, kSw64), idesc, 1);
+      mma_ss_w(d, sdesc(lo + 32, 16, 512, kSw64), sdesc(b + 32, 16, 512, kSw64), idesc, 1);
+    } else {
+      mma_ss_w(d, sdesc(a, 16, 512, kSw64), sdesc(lo, 16, 512, kSw64), idesc, 1);
+      mma_ss_w(d, sdesc(a + 32, 16, 512, kSw64), sdesc(lo + 32, 16, 512, kSw64), idesc, 1);
+    }
+  }
+  mma_ss_w(d, ae, be, idesc, 1);
+}
+
+// Point-extra descriptor (no swizzle, 16-byte rows) whose k = 8..15 half is the shared zero block.
+__device__ __forceinline__ uint64_t px_desc(uint32_t px_s, uint32_t zero_s) { return sdesc(px_s, zero_s - px_s, 128, 0); }
+
+// One 64-column unit of a TMEM lane: L (log2 weights) at tL, dw - delta at tD.
+// da = 2^L (dw - delta) goes back in place into the L columns as bf16 pairs: columns
+// [32 h, 32 h + 16) the hi halves of entries [32 h, 32 h + 32), [32 h + 16, 32 h + 32)
+// their lo halves (kSplit).  kW: the weights too, into the dw columns, same layout.
+// kSums: dt += sum da L, db += sum da.
+template <bool kSplit, bool kW, bool kSums>
+__device__ __forceinline__ void da_unit(uint32_t tL, uint32_t tD, float& dt, float& db) {
+#pragma unroll 1
+  for (int h2 = 0; h2 < 2; h2++) {
+    uint32_t l[32], dw[32];
+    tmem_ld32(tL + 32 * h2, l);
+    tmem_ld32(tD + 32 * h2, dw);
+    tmem_wait_ld2(l, dw);
+    uint32_t dh[16], dl[16], wh[16], wl[16];
+    float t = 0.f, sb = 0.f;
+#pragma unroll
+    for (int k = 0; k < 16; k++) {
+      const float L0 = __uint_as_float(l[2 * k]), L1 = __uint_as_float(l[2 * k + 1]);
+      const float w0 = ex2(L0), w1 = ex2(L1);
+      const float a0 = w0 * __uint_as_float(dw[2 * k]), a1 = w1 * __uint_as_float(dw[2 * k + 1]);
+      if (kSums) {
+        t = fmaf(a0, L0, t);
+        t = fmaf(a1, L1, t);
+        sb += a0;
+        sb += a1;
+      }
+      const uint32_t p = pack_bf16(a0, a1);
+      dh[k] = p;
+      if (kSplit) dl[k] = pack_bf16(a0 - __uint_as_float(p << 16), a1 - __uint_as_float(p & 0xFFFF0000u));
+      if (kW) {
+        const uint32_t q = pack_bf16(w0, w1);
+        wh[k] = q;
+        if (kSplit) wl[k] = pack_bf16(w0 - __uint_as_float(q << 16), w1 - __uint_as_float(q & 0xFFFF0000u));
+      }
+    }
+    tmem_st16(tL + 32 * h2, dh);
+    if (kSplit) tmem_st16(tL + 32 * h2 + 16, dl);
+    if (kW) {
+      tmem_st16(tD + 32 * h2, wh);
+      if (kSplit) tmem_st16(tD + 32 * h2 + 16, wl);
+    }
+    if (kSums) {
+      dt += t;
+      db += sb;
+    }
+  }
+}
+// TMEM column (within a unit) of the hi pairs of K-step kk (16 entries).
+__device__ __forceinline__ uint32_t da_col(int kk) { return (uint32_t)(32 * (kk >> 1) + 8 * (kk & 1)); }
+
+// =========================================================================================
+// Slot pass: CTA (slot block, point split p, bh) owns 128 slots.  Unit u is half
+// u & 1 (64 points) of point tile u >> 1.  Per unit, warp 1 forms, transposed
+// (M = 128 slots, N = 64 points, TMEM lane = slot),
+//   L = a2 - lse2 (W block vs [x | 1, 1, -lse2]) and dw - delta (T block vs [v | 1, 1, -delta]);
+// softmax warpgroup u % 2 turns them into da (and, MODE 1, w) in place and sums
+// da (a2 - lse2) and da per slot in registers; warp 2 + u % 2 issues
+//   dWx += da^T x   (K = points; x's 64B-swizzled tile read as an MN-major B operand)
+//   MODE 1: dZ += w^T dO (the token gradient), from dO's tile the same way.
+// Writes part[p][bh][g] = MODE 1: (dZ(32), dWx(32), sum da, 0); MODE 2: (dWx, sum da, 0)
+// and dt_part[bh][p * R + block] = ln2 * sum over the block's slots of sum da (a2 - lse2).
+// smem: [W block: hi 8K | extra 4K | lo 8K][T block: same][stages][zero 2K][red 1.5K][bars]
+// TMEM: unit u uses set u % 3: L [128 s, +64), dw [128 s + 64, +64); accumulators
+// dWx_j [384 + 32 j), dZ_j [448 + 32 j).
+// =========================================================================================
+template <int MODE, bool split>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_bwd_slot_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap vmap,
+                  const __grid_constant__ CUtensorMap pmap, const __grid_constant__ CUtensorMap dmap,
+                  const uint8_t* __restrict__ wimg, const uint8_t* __restrict__ timg, float* __restrict__ part,
+                  float* __restrict__ dt_part, int64_t N, int64_t Np, int H, int G, int splits,
+                  uint32_t* status) {
+  const int g_base = blockIdx.x * kGC;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* s_w = smem;               // W block
+  uint8_t* s_t = s_w + kWBlockB;     // T block
+  uint8_t* s_st = s_t + kWBlockB;    // stages
+  uint8_t* s_zero = s_st + kBStages * kBStage;
+  float* s_red = reinterpret_cast<float*>(s_zero + kPxZero);  // 3 x 128 floats
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_red + 3 * kGC);
+  uint64_t* w_full = bars;
+  uint64_t* x_full = bars + 1;
+  uint64_t* st_empty = x_full + kBStages;
+  uint64_t* s_full = st_empty + kBStages;
+  uint64_t* p_ready = s_full + kSBuf;  // [issuer][set]
+  uint64_t* pv_done = p_ready + 2 * kSBuf;
+  uint64_t* acc_full = pv_done + kSBuf;
+  uint64_t* drain = acc_full + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 3);
+  Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const Work wk = work_of(N, splits, blockIdx.y, blockIdx.z);
+  const int64_t b = wk.bh / H;
+  const int h = (int)(wk.bh % H);
+  const int units = 2 * wk.ntiles;
+  constexpr uint32_t kAccW = kSBuf * kGC, kAccZ = kAccW + 64;
+  constexpr uint32_t kVOff = kXBytes, kPOff = 2 * kXBytes, kDOff = 2 * kXBytes + kPxBytes;
+
+  if (threadIdx.x == 0) {
+    mbar_init(w_full, 1);
+    for (int s = 0; s < kBStages; s++) {
+      mbar_init(&x_full[s], 1);
+      mbar_init(&st_empty[s], 3);  // the logits issuer and both product issuers
+    }
+    for (int i = 0; i < kSBuf; i++) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&p_ready[i], 4);
+      mbar_init(&p_ready[kSBuf + i], 4);
+      mbar_init(&pv_done[i], 1);
+    }
+    mbar_init(acc_full, 2);
+    for (int i = 0; i < 3; i++) mbar_init(&drain[i], 1);
+    ab->flag = 0;
+    fence_mbar_init();
+  }
+  zero_smem(s_zero, kPxZero);
+  fence_proxy_async_smem();
+  if (warp == 1) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ------------------------------ producer ------------------------------
+    if (lane == 0) {
+      prefetch_tmap(&xmap);
+      prefetch_tmap(&vmap);
+      prefetch_tmap(&pmap);
+      prefetch_tmap(&dmap);
+      mbar_expect_tx(w_full, 2 * kWBlockB);
+      const uint8_t* ws = wimg + (size_t)h * G * kWRow;
+      const uint8_t* ts = timg + (size_t)wk.bh * G * kWRow;
+      for (int im = 0; im < 2; im++) {
+        const uint8_t* src = im ? ts : ws;
+        uint8_t* dst = im ? s_t : s_w;
+        load_images(dst, src + (size_t)g_base * 64, kGC * 64, w_full);
+        load_images(dst + kGC * 64, src + (size_t)G * 64 + (size_t)g_base * 32, kGC * 32, w_full);
+        load_images(dst + kGC * 96, src + (size_t)G * 96 + (size_t)g_base * 64, kGC * 64, w_full);
+      }
+      int i = 0;
+      for (; i < wk.ntiles; i++) {
+        const int s = i % kBStages;
+        if (i >= kBStages && !mbar_wait(&st_empty[s], (uint32_t)(((i / kBStages) - 1) & 1), ab, status)) break;
+        uint8_t* st = s_st + s * kBStage;
+        const int n0 = (int)((wk.tile0 + i) * kTile);
+        mbar_expect_tx(&x_full[s], kBStage);
+        tma_load_3d(st, &xmap, h * kD, n0, (int)b, &x_full[s]);
+        tma_load_3d(st + kVOff, &vmap, h * kD, n0, (int)b, &x_full[s]);
+        tma_load_2d(st + kPOff, &pmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
+        tma_load_2d(st + kDOff, &dmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
+      }
+      for (int j = (i > kBStages ? i - kBStages : 0); j < i; j++)
+        mbar_wait(&x_full[j % kBStages], (uint32_t)((j / kBStages) & 1), ab, nullptr, kWaitNs);
+      mbar_wait(w_full, 0, ab, nullptr, kWaitNs);
+    }
+  } else if (warp == 1) {
+    // ------------------------------ logits and dw issuer ------------------------------
+    const uint32_t sw = smem_u32(s_w), stt = smem_u32(s_t), sz = smem_u32(s_zero);
+    bool ok = mbar_wait_w(w_full, 0, ab, status);
+    for (int u = 0; ok && u < units; u++) {
+      const int i = u >> 1, half = u & 1;
+      const int s = i % kBStages;
+      const int bb = u % kSBuf;
+      if (half == 0 && !(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kBStages) & 1), ab, status))) break;
+      if (u >= kSBuf && !(ok = mbar_wait_w(&pv_done[bb], (uint32_t)(((u / kSBuf) - 1) & 1), ab, status))) break;
+      tc_fence_after();
+      const uint32_t st = smem_u32(s_st + s * kBStage);
+      const uint32_t rows = (uint32_t)half * 64 * 64;     // the unit's 64 points in the 64-byte-row tiles
+      const uint32_t prow = (uint32_t)half * 64 * 16;     // ... and in the 16-byte extra rows
+      const uint32_t tL = tmem + (uint32_t)bb * kGC;
+      issue_dot64<true>(tL, sw, st + rows, sdesc(sw + kGC * 64, 16, 256, kSw32), px_desc(st + kPOff + prow, sz),
+                        split ? sw + kGC * 96 : 0u);
+      issue_dot64<true>(tL + 64, stt, st + kVOff + rows, sdesc(stt + kGC * 64, 16, 256, kSw32),
+                        px_desc(st + kDOff + prow, sz), split ? stt + kGC * 96 : 0u);
+      mma_commit_w(&s_full[bb]);
+      if (half == 1) mma_commit_w(&st_empty[s]);
+    }
+    mma_commit_w(&drain[0]);
+    mbar_wait_w(&drain[0], 0, ab, nullptr, kWaitNs);
+  } else if (warp == 2 || warp == 3) {
+    // ------------------------------ product issuers ------------------------------
+    const int j = warp - 2;  // units u with u % 2 == j (half j of every tile)
+    constexpr uint32_t idesc = idesc_bf16(128, kD, false, true);
+    bool ok = true;
+    for (int u = j; ok && u < units; u += 2) {
+      const int i = u >> 1;
+      const int s = i % kBStages;
+      const int bb = u % kSBuf;
+      // This issuer's units on set bb are 2 kSBuf apart.
+      if (!(ok = mbar_wait_w(&p_ready[j * kSBuf + bb], (uint32_t)((u / (2 * kSBuf)) & 1), ab, status))) break;
+      tc_fence_after();
+      const uint32_t st = smem_u32(s_st + s * kBStage) + (uint32_t)j * 64 * 64;
+      const uint32_t tL = tmem + (uint32_t)bb * kGC, tD = tL + 64;
+#pragma unroll
+      for (int kk = 0; kk < 4; kk++) {
+        // 16 points: two 8-row groups of the 64B-swizzled tile (MN-major: channels contiguous).
+        const uint64_t xd = sdesc(st + (uint32_t)kk * 1024, 4096, 512, kSw64);
+        const uint32_t acc = (u >= 2 || kk > 0) ? 1u : 0u;
+        mma_ts_w(tmem + kAccW + (uint32_t)j * 32, tL + da_col(kk), xd, idesc, acc);
+        if (split) mma_ts_w(tmem + kAccW + (uint32_t)j * 32, tL + da_col(kk) + 16, xd, idesc, 1u);
+        if (MODE == 1) {
+          const uint64_t vd = sdesc(st + kVOff + (uint32_t)kk * 1024, 4096, 512, kSw64);
+          mma_ts_w(tmem + kAccZ + (uint32_t)j * 32, tD + da_col(kk), vd, idesc, acc);
+          if (split) mma_ts_w(tmem + kAccZ + (uint32_t)j * 32, tD + da_col(kk) + 16, vd, idesc, 1u);
+        }
+      }
+      mma_commit_w(&pv_done[bb]);
+      mma_commit_w(&st_empty[s]);
+    }
+    if (ok) mma_commit_w(acc_full);
+    mma_commit_w(&drain[1 + j]);
+    mbar_wait_w(&drain[1 + j], 0, ab, nullptr, kWaitNs);
+  } else {
+    // ------------------------------ softmax warpgroups ------------------------------
+    const int wg = (warp - kSoftmaxWarp0) >> 2;
+    const int wq = warp & 3;
+    const int r = wq * 32 + lane;  // TMEM lane: slot g_base + r
+    const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
+    bool ok = true;
+    float dt = 0.f, db = 0.f;
+    for (int u = wg; ok && u < units; u += 2) {
+      const int bb = u % kSBuf;
+      if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((u / kSBuf) & 1), ab, status))) break;
+      tc_fence_after();
+      const uint32_t tL = tmem + lane_addr + (uint32_t)bb * kGC;
+      float t = 0.f, sb = 0.f;
+      da_unit<split, MODE == 1, true>(tL, tL + 64, t, sb);
+      dt += t;
+      db += sb;
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_ready[wg * kSBuf + bb]);
+    }
+    // Epilogue: warpgroup 1 hands its sums to warpgroup 0, which writes dWx and the
+    // sums; warpgroup 1 writes dZ (MODE 1).
+    const int64_t BH = gridDim.z;
+    const int PS = MODE == 1 ? 2 * kD + 2 : kD + 2;
+    float* o = part + (((int64_t)blockIdx.y * BH + wk.bh) * G + g_base + r) * PS;
+    if (wg == 1) {
+      s_red[r] = dt;
+      s_red[kGC + r] = db;
+    }
+    named_barrier(1, 256);
+    const bool have = ok && wk.ntiles > 0 && mbar_wait(acc_full, 0, ab, status);
+    if (have) tc_fence_after();
+    if (wg == 0) {
+      dt += s_red[r];
+      db += s_red[kGC + r];
+      const int off = MODE == 1 ? kD : 0;
+      if (have) {
+        uint32_t a0[32], a1[32];
+        tmem_ld32(tmem + lane_addr + kAccW, a0);
+        tmem_ld32(tmem + lane_addr + kAccW + 32, a1);
+        tmem_wait_ld2(a0, a1);
+#pragma unroll
+        for (int k = 0; k < kD; k++) o[off + k] = __uint_as_float(a0[k]) + __uint_as_float(a1[k]);
+      } else {
+        for (int k = 0; k < kD; k++) o[off + k] = 0.f;
+      }
+      o[off + kD] = db;
+      o[off + kD + 1] = 0.f;
+      s_red[2 * kGC + r] = dt;
+      named_barrier(2, 128);
+      if (r == 0) {
+        float sum = 0.f;
+        for (int k = 0; k < kGC; k++) sum += s_red[2 * kGC + k];
+        dt_part[wk.bh * ((int64_t)gridDim.x * gridDim.y) + (int64_t)blockIdx.y * gridDim.x + blockIdx.x] = sum * kLn2;
+      }
+    } else if (MODE == 1) {
+      if (have) {
+        uint32_t z0[32], z1[32];
+        tmem_ld32(tmem + lane_addr + kAccZ, z0);
+        tmem_ld32(tmem + lane_addr + kAccZ + 32, z1);
+        tmem_wait_ld2(z0, z1);
+#pragma unroll
+        for (int k = 0; k < kD; k++) o[k] = __uint_as_float(z0[k]) + __uint_as_float(z1[k]);
+      } else {
+        for (int k = 0; k < kD; k++) o[k] = 0.f;
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+// =========================================================================================
+// Point pass: dx_n = ln2 * sum_g da_ng W'_g (W' = W log2(e)/tau).  CTA (split, bh)
+// walks its point tiles; block q is (tile q / nb, 64-slot chunk q % nb).  Warp 1
+// forms L (x tile vs W rows) and dw - delta (v tile vs T rows), M = 128 points,
+// N = 64 slots, into set q % 3; softmax warpgroup q % 2 writes da in place (hi, lo
+// pairs); warp 2 + j issues K-steps [2 j, 2 j + 2) of the chunk into O_j:
+//   O_j += da W'^T (B: the W'^T image, channel rows, slots along K).
+// smem: [W img G x (96 | 160)][T img G x 96][W'^T img G x 64][stages][zero 2K][bars]
+// TMEM: sets [0, 384) of (L 64 | dw 64); O_(j, tile parity) at [384 + 32 (2 j + parity)).
+// =========================================================================================
+template <bool split>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_bwd_dx_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap vmap,
+                const __grid_constant__ CUtensorMap pmap, const __grid_constant__ CUtensorMap dmap,
+                const uint8_t* __restrict__ wimg, const uint8_t* __restrict__ timg,
+                const uint8_t* __restrict__ wtimg, __nv_bfloat16* __restrict__ dx, int64_t N, int64_t Np, int H,
+                int G, int splits, int hilo, int accumulate, uint32_t* status) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const uint32_t wbytes = (uint32_t)G * (hilo ? kWRow : 96);
+  uint8_t* s_w = smem;
+  uint8_t* s_t = s_w + wbytes;
+  uint8_t* s_wt = s_t + (uint32_t)G * 96;
+  uint8_t* s_st = s_wt + (uint32_t)G * 64;
+  uint8_t* s_zero = s_st + kDxStages * kBStage;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_zero + kPxZero);
+  uint64_t* wz_full = bars;
+  uint64_t* x_full = bars + 1;
+  uint64_t* x_empty = x_full + kDxStages;
+  uint64_t* s_full = x_empty + kDxStages;
+  uint64_t* p_ready = s_full + kSBuf;
+  uint64_t* pv_done = p_ready + kSBuf;
+  uint64_t* o_full = pv_done + kSBuf;
+  uint64_t* o_free = o_full + 2;
+  uint64_t* drain = o_free + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 3);
+  Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const Work wk = work_of(N, splits, blockIdx.x, blockIdx.y);
+  const int64_t b = wk.bh / H;
+  const int h = (int)(wk.bh % H);
+  const int nch = G / 64;
+  const int total = wk.ntiles * nch;
+  constexpr uint32_t kO = kSBuf * kGC;
+  constexpr uint32_t kVOff = kXBytes, kPOff = 2 * kXBytes, kDOff = 2 * kXBytes + kPxBytes;
+
+  if (threadIdx.x == 0) {
+    mbar_init(wz_full, 1);
+    for (int s = 0; s < kDxStages; s++) {
+      mbar_init(&x_full[s], 1);
+      mbar_init(&x_empty[s], 1);
+    }
+    for (int i = 0; i < kSBuf; i++) {
+      mbar_init(&s_full[i], 1);
+      mbar_init(&p_ready[i], 4);
+      mbar_init(&pv_done[i], 2);
+    }
+    for (int i = 0; i < 2; i++) {
+      mbar_init(&o_full[i], 2);
+      mbar_init(&o_free[i], 4);
+    }
+    for (int i = 0; i < 3; i++) mbar_init(&drain[i], 1);
+    ab->flag = 0;
+    fence_mbar_init();
+  }
+  zero_smem(s_zero, kPxZero);
+  fence_proxy_async_smem();
+  if (warp == 1) tmem_alloc(tmem_slot, 512);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0 && wk.ntiles > 0) {
+      prefetch_tmap(&xmap);
+      prefetch_tmap(&vmap);
+      prefetch_tmap(&pmap);
+      prefetch_tmap(&dmap);
+      mbar_expect_tx(wz_full, wbytes + (uint32_t)G * 96 + (uint32_t)G * 64);
+      load_images(s_w, wimg + (size_t)h * G * kWRow, wbytes, wz_full);
+      load_images(s_t, timg + (size_t)wk.bh * G * kWRow, (uint32_t)G * 96, wz_full);
+      load_images(s_wt, wtimg + (size_t)h * G * 128, (uint32_t)G * 64, wz_full);
+      int i = 0;
+      for (; i < wk.ntiles; i++) {
+        const int s = i % kDxStages;
+        if (i >= kDxStages && !mbar_wait(&x_empty[s], (uint32_t)(((i / kDxStages) - 1) & 1), ab, status)) break;
+        uint8_t* st = s_st + s * kBStage;
+        const int n0 = (int)((wk.tile0 + i) * kTile);
+        mbar_expect_tx(&x_full[s], kBStage);
+        tma_load_3d(st, &xmap, h * kD, n0, (int)b, &x_full[s]);
+        tma_load_3d(st + kVOff, &vmap, h * kD, n0, (int)b, &x_full[s]);
+        tma_load_2d(st + kPOff, &pmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
+        tma_load_2d(st + kDOff, &dmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
+      }
+      for (int j = (i > kDxStages ? i - kDxStages : 0); j < i; j++)
+        mbar_wait(&x_full[j % kDxStages], (uint32_t)((j / kDxStages) & 1), ab, nullptr, kWaitNs);
+      mbar_wait(wz_full, 0, ab, nullptr, kWaitNs);
+    }
+  } else if (warp == 1) {
+    if (wk.ntiles > 0) {
+      const uint32_t sw = smem_u32(s_w), stt = smem_u32(s_t), sz = smem_u32(s_zero);
+      bool ok = mbar_wait_w(wz_full, 0, ab, status);
+      BlockPos pos(0, nch);
+      for (int q = 0; ok && q < total; q++, pos.step(1, nch)) {
+        const int i = pos.i, c = pos.c;
+        const int s = i % kDxStages;
+        const int bb = q % kSBuf;
+        if (c == 0 && !(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kDxStages) & 1), ab, status))) break;
+        if (q >= kSBuf && !(ok = mbar_wait_w(&pv_done[bb], (uint32_t)(((q / kSBuf) - 1) & 1), ab, status))) break;
+        tc_fence_after();
+        const uint32_t st = smem_u32(s_st + s * kBStage);
+        const uint32_t tL = tmem + (uint32_t)bb * kGC;
+        const uint32_t rows = (uint32_t)c * 64 * 64, erows = (uint32_t)c * 64 * 32;
+        issue_dot64<false>(tL, st, sw + rows, px_desc(st + kPOff, sz),
+                           sdesc(sw + (uint32_t)G * 64 + erows, 16, 256, kSw32),
+                           hilo ? sw + (uint32_t)G * 96 + rows : 0u);
+        issue_dot64<false>(tL + 64, st + kVOff, stt + rows, px_desc(st + kDOff, sz),
+                           sdesc(stt + (uint32_t)G * 64 + erows, 16, 256, kSw32), 0u);
+        mma_commit_w(&s_full[bb]);
+        if (c == nch - 1) mma_commit_w(&x_empty[s]);
+      }
+      mma_commit_w(&drain[0]);
+      mbar_wait_w(&drain[0], 0, ab, nullptr, kWaitNs);
+    }
+  } else if (warp == 2 || warp == 3) {
+    const int j = warp - 2;
+    if (wk.ntiles > 0) {
+      constexpr uint32_t idesc = idesc_bf16(128, kD, false, false);
+      const uint32_t swt = smem_u32(s_wt);
+      bool ok = mbar_wait_w(wz_full, 0, ab, status);
+      BlockPos pos(0, nch);
+      for (int q = 0; ok && q < total; q++, pos.step(1, nch)) {
+        const int i = pos.i, c = pos.c;
+        const int ob = i & 1;
+        const int bb = q % kSBuf;
+        if (c == 0 && i >= 2 && !(ok = mbar_wait_w(&o_free[ob], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
+        if (!(ok = mbar_wait_w(&p_ready[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
+        tc_fence_after();
+        const uint32_t tL = tmem + (uint32_t)bb * kGC;
+        const uint32_t tO = tmem + kO + (uint32_t)(j * 2 + ob) * kD;
+#pragma unroll
+        for (int e = 0; e < 2; e++) {
+          const int kk = 2 * j + e;
+          const uint64_t bd = sdesc(swt + (uint32_t)c * 4096 + (uint32_t)kk * 32, 16, 1024, kSw128);
+          mma_ts_w(tO, tL + da_col(kk), bd, idesc, (c > 0 || e > 0) ? 1u : 0u);
+          if (split) mma_ts_w(tO, tL + da_col(kk) + 16, bd, idesc, 1u);
+        }
+        mma_commit_w(&pv_done[bb]);
+        if (c == nch - 1) mma_commit_w(&o_full[ob]);
+      }
+      mma_commit_w(&drain[1 + j]);
+      mbar_wait_w(&drain[1 + j], 0, ab, nullptr, kWaitNs);
+    }
+  } else {
+    const int wg = (warp - kSoftmaxWarp0) >> 2;
+    const int wq = warp & 3;
+    const int r = wq * 32 + lane;
+    const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
+    bool ok = true;
+    auto epilogue = [&](int t) -> bool {
+      const int ob = t & 1;
+      if (!mbar_wait(&o_full[ob], (uint32_t)((t >> 1) & 1), ab, status)) return false;
+      tc_fence_after();
+      uint32_t o0[32], o1[32];
+      tmem_ld32(tmem + lane_addr + kO + (uint32_t)ob * kD, o0);
+      tmem_ld32(tmem + lane_addr + kO + (uint32_t)(2 + ob) * kD, o1);
+      tmem_wait_ld2(o0, o1);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&o_free[ob]);
+      const int64_t n = (wk.tile0 + t) * kTile + r;
+      if (n < N) {
+        uint4* dst = reinterpret_cast<uint4*>(dx + ((b * N + n) * H + h) * kD);
+        float add[kD];
+#pragma unroll
+        for (int k = 0; k < kD; k++) add[k] = 0.f;
+        if (accumulate) {
+#pragma unroll
+          for (int k = 0; k < 4; k++) {
+            const uint4 q4 = dst[k];
+            const uint32_t w[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+            for (int e = 0; e < 4; e++) {
+              add[8 * k + 2 * e] = __uint_as_float(w[e] << 16);
+              add[8 * k + 2 * e + 1] = __uint_as_float(w[e] & 0xFFFF0000u);
+            }
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < 4; k++) {
+          uint32_t w[4];
+#pragma unroll
+          for (int e = 0; e < 4; e++) {
+            const int c0 = 8 * k + 2 * e;
+            w[e] = pack_bf16(fmaf(__uint_as_float(o0[c0]) + __uint_as_float(o1[c0]), kLn2, add[c0]),
+                             fmaf(__uint_as_float(o0[c0 + 1]) + __uint_as_float(o1[c0 + 1]), kLn2, add[c0 + 1]));
+          }
+          dst[k] = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+      }
+      return true;
+    };
+    BlockPos pos(wg, nch);
+    for (int q = wg; ok && q < total; q += 2, pos.step(2, nch)) {
+      const int i = pos.i, c = pos.c;
+      const int bb = q % kSBuf;
+      if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
+      tc_fence_after();
+      const uint32_t tL = tmem + lane_addr + (uint32_t)bb * kGC;
+      float unused0 = 0.f, unused1 = 0.f;
+      da_unit<split, false, false>(tL, tL + 64, unused0, unused1);
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&p_ready[bb]);
+      if (c == 0 && i > 0 && !(ok = epilogue(i - 1))) break;
+    }
+    if (ok && total > 0 && total % 2 == wg) epilogue(wk.ntiles - 1);
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem, 512);
+}
+
+// ---- host side ---------------------------------------------------------------------------------
+
+size_t smem_bwd_slot() {
+  return 1024 + 2 * (size_t)kWBlockB + kBStages * (size_t)kBStage + kPxZero + 3 * kGC * 4 + 512;
+}
+size_t smem_bwd_dx(int G, bool hilo) {
+  return 1024 + (size_t)G * ((hilo ? kWRow : 96) + 96 + 64) + kDxStages * (size_t)kBStage + kPxZero + 512;
+}
+
+int bwd_slot_blocks(const Shape& s) { return s.G / kGC; }
+int bwd_slot_splits(const Shape& s) { return point_splits(s, (int)(s.BH() * bwd_slot_blocks(s))); }
+
+// Workspace layout of one tensor-core backward call (offsets from the tc region).
+struct BwdLayout {
+  size_t wimg, wtimg, timg, zimg, px, dpx, delta, wds, ds, dtp, part, total;
+};
+BwdLayout bwd_layout(const Shape& s, int mode) {
+  BwdLayout L{};
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  const size_t BHG = (size_t)s.BH() * s.G;
+  const size_t pts = (size_t)s.BH() * s.N;
+  const int P = bwd_slot_splits(s), R = bwd_slot_blocks(s);
+  L.wimg = take(w_image_bytes(s));
+  L.wtimg = take((size_t)s.H * s.G * 128);
+  L.timg = take(BHG * kWRow);
+  L.zimg = take(BHG * 128);
+  L.px = take(px_bytes(s));
+  L.dpx = take(px_bytes(s));
+  L.delta = take(pts * sizeof(float));
+  L.wds = take(mode == 2 ? 2 * pts * sizeof(float) : 0);
+  L.ds = take(BHG * sizeof(float));
+  L.dtp = take((size_t)s.BH() * P * R * sizeof(float));
+  L.part = take((size_t)P * BHG * (mode == 1 ? 2 * kD + 2 : kD + 2) * sizeof(float));
+  L.total = off;
+  return L;
+}
+
+bool make_maps(const Shape& s, const void* x, const void* v, const void* px, const void* dpx, CUtensorMap* xmap,
+               CUtensorMap* vmap, CUtensorMap* pmap, CUtensorMap* dmap) {
+  const int64_t Np = padded_n(s);
+  return make_point_map(xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B) &&
+         make_point_map(vmap, v, s, kD, CU_TENSOR_MAP_SWIZZLE_64B) && make_px_map(pmap, px, s.BH(), Np) &&
+         make_px_map(dmap, dpx, s.BH(), Np);
+}
+
+// The common part of both backward calls, after the T and Z images are written:
+// the W images and lse rows, the rows pass, delta's rows, the slot and the point passes.
+cudaError_t run_backward(const Shape& s, int mode, const void* x, const void* v, const float* W, const float* bias,
+                         const float* tau, const float* lse, void* dfx, void* dx, int accumulate, uint8_t* ws,
+                         const BwdLayout& L, uint32_t* status, cudaStream_t st) {
+  const int64_t Np = padded_n(s);
+  cudaError_t e = prep_w(s, W, bias, tau, ws + L.wimg, status, st);
+  if (e != cudaSuccess) return e;
+  const int64_t nwt = (int64_t)s.H * kD * s.G;
+  k_prep_wt<<<(unsigned)((nwt + 255) / 256), 256, 0, st>>>(W, tau, ws + L.wtimg, s.H, s.G, status);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const int64_t npx = s.BH() * Np;
+  k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(ws + L.px), s.BH(), s.N,
+                                                             Np);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  float* delta = reinterpret_cast<float*>(ws + L.delta);
+  float* wds = mode == 2 ? reinterpret_cast<float*>(ws + L.wds) : nullptr;
+  if (wds && (e = cudaMemsetAsync(wds, 0, 2 * (size_t)s.BH() * s.N * sizeof(float), st)) != cudaSuccess) return e;
+  if ((e = tc_rows_bwd(s, mode, x, ws + L.wimg, ws + L.zimg, ws + L.px, v, dfx, delta, wds,
+                       reinterpret_cast<const float*>(ws + L.ds), status, st)) != cudaSuccess)
+    return e;
+  k_prep_dpx<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(delta, wds, reinterpret_cast<uint4*>(ws + L.dpx),
+                                                              s.BH(), s.N, Np);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+
+  CUtensorMap xmap, vmap, pmap, dmap;
+  if (!make_maps(s, x, v, ws + L.px, ws + L.dpx, &xmap, &vmap, &pmap, &dmap)) return cudaErrorInvalidValue;
+  const bool split = s.dot == FS_DOT_BF16X2;
+  {
+    const int R = bwd_slot_blocks(s), P = bwd_slot_splits(s);
+    const size_t sm = smem_bwd_slot();
+    const auto kernel = mode == 1 ? (split ? k_bwd_slot_tc<1, true> : k_bwd_slot_tc<1, false>)
+                                  : (split ? k_bwd_slot_tc<2, true> : k_bwd_slot_tc<2, false>);
+    if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
+    kernel<<<dim3((unsigned)R, (unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(
+        xmap, vmap, pmap, dmap, ws + L.wimg, ws + L.timg, reinterpret_cast<float*>(ws + L.part),
+        reinterpret_cast<float*>(ws + L.dtp), s.N, Np, s.H, s.G, P, status);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  {
+    const bool hilo = split && smem_bwd_dx(s.G, true) <= kMaxSmem;
+    const size_t sm = smem_bwd_dx(s.G, hilo);
+    const int P = point_splits(s, (int)s.BH());
+    const auto kernel = split ? k_bwd_dx_tc<true> : k_bwd_dx_tc<false>;
+    if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
+    kernel<<<dim3((unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(
+        xmap, vmap, pmap, dmap, ws + L.wimg, ws + L.timg, ws + L.wtimg, static_cast<__nv_bfloat16*>(dx), s.N, Np,
+        s.H, s.G, P, hilo ? 1 : 0, accumulate, status);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t prep_t_images(const Shape& s, const float* t, int tstride, int has_c, uint8_t* ws, const BwdLayout& L,
+                          cudaStream_t st) {
+  const int64_t BHG = s.BH() * s.G;
+  k_prep_t<<<(unsigned)((BHG + 127) / 128), 128, 0, st>>>(t, tstride, has_c, ws + L.timg,
+                                                            reinterpret_cast<float*>(ws + L.ds), s.BH(), s.G);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_prep_z2<<<(unsigned)((BHG * kD + 255) / 256), 256, 0, st>>>(t, tstride, ws + L.zimg, s.BH(), s.G);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+// A single point (N = 1) takes the fp32 SIMT backward: every token is then that
+// point's fx times S/(S + eps), so the slice's gradients are O(eps) and come from
+// cancelling terms of size |dz||fx|/(S + eps) that split bf16 products resolve only
+// to ~2^-17 of that size.
+bool tc_backward_supported(const Shape& s) {
+  return tc_forward_supported(s) && s.N >= 2 && smem_bwd_dx(s.G, false) <= kMaxSmem &&
+         tc_rows_smem(s, 2, false, false) <= kMaxSmem;
+}
+
+size_t tc_backward_bytes(const Shape& s, int mode) {
+  return tc_backward_supported(s) ? bwd_layout(s, mode).total : 0;
+}
+
+int tc_backward_slot_splits(const Shape& s) { return bwd_slot_splits(s); }
+
+// The backward forms every weight with split products whatever the forward's
+// arithmetic: its lse comes from split products (recomputed when the forward's
+// did not), and weights from bf16 logits would not sum to one against it; the
+// excess would bias the gradients that are sums of cancelling terms (dbias, dtau).
+Shape split_shape(const Shape& s) {
+  Shape r = s;
+  r.dot = FS_DOT_BF16X2;
+  return r;
+}
+
+cudaError_t tc_deslice_bwd(const Shape& s0, const void* x, const float* W, const float* bias, const float* tau,
+                           const float* zp, const float* lse, const void* dout, float* dzp, void* dx, float* dW,
+                           float* db, float* dtau, int accumulate, void* ws_tc, uint32_t* status, cudaStream_t st) {
+  const Shape s = split_shape(s0);
+  const BwdLayout L = bwd_layout(s, 1);
+  uint8_t* ws = static_cast<uint8_t*>(ws_tc);
+  cudaError_t e = prep_t_images(s, zp, kD, 0, ws, L, st);
+  if (e != cudaSuccess) return e;
+  if ((e = run_backward(s, 1, x, dout, W, bias, tau, lse, nullptr, dx, accumulate, ws, L, status, st)) !=
+      cudaSuccess)
+    return e;
+  const int P = bwd_slot_splits(s);
+  return simt_reduce_bwd(s, P, reinterpret_cast<const float*>(ws + L.part), 2 * kD + 2, 1, tau, dzp, dW, db, dtau,
+                         reinterpret_cast<const float*>(ws + L.dtp), (int64_t)P * bwd_slot_blocks(s), accumulate,
+                         st);
+}
+
+cudaError_t tc_slice_bwd(const Shape& s0, const void* x, const void* f, const float* W, const float* bias,
+                         const float* tau, const float* z, const float* wsum, const float* lse, const float* dz,
+                         void* dx, void* dfx, float* dW, float* db, float* dtau, int accumulate, float* dUS,
+                         void* ws_tc, uint32_t* status, cudaStream_t st) {
+  const Shape s = split_shape(s0);
+  const BwdLayout L = bwd_layout(s, 2);
+  uint8_t* ws = static_cast<uint8_t*>(ws_tc);
+  cudaError_t e = simt_slice_bwd_prep(s, z, wsum, dz, dUS, st);
+  if (e != cudaSuccess) return e;
+  if ((e = prep_t_images(s, dUS, kD + 1, 1, ws, L, st)) != cudaSuccess) return e;
+  if ((e = run_backward(s, 2, x, f, W, bias, tau, lse, dfx, dx, accumulate, ws, L, status, st)) != cudaSuccess)
+    return e;
+  const int P = bwd_slot_splits(s);
+  return simt_reduce_bwd(s, P, reinterpret_cast<const float*>(ws + L.part), kD + 2, 0, tau, nullptr, dW, db, dtau,
+                         reinterpret_cast<const float*>(ws + L.dtp), (int64_t)P * bwd_slot_blocks(s), accumulate,
+                         st);
+}
+
+}  // namespace fs

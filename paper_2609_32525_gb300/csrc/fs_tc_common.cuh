@@ -260,6 +260,89 @@ __device__ __forceinline__ void weights_in_halves(uint32_t tS) {
   }
 }
 
+// The weight helpers above, plus acc += sum over the block's 128 slots of w_g ds[g]
+// (ds: the block's slice of a per-slot array in shared memory; every lane reads
+// the same address, a broadcast).  The backward of the slice needs this sum for
+// its delta (the dS term).
+__device__ __forceinline__ void weights32_ds(const uint32_t (&v)[32], uint32_t (&p)[16], const float* ds,
+                                             float& acc) {
+  const float4* d4 = reinterpret_cast<const float4*>(ds);
+#pragma unroll
+  for (int k = 0; k < 8; k++) {
+    const float4 q = d4[k];
+    const float w0 = ex2(__uint_as_float(v[4 * k])), w1 = ex2(__uint_as_float(v[4 * k + 1]));
+    const float w2 = ex2(__uint_as_float(v[4 * k + 2])), w3 = ex2(__uint_as_float(v[4 * k + 3]));
+    acc = fmaf(w0, q.x, acc);
+    acc = fmaf(w1, q.y, acc);
+    acc = fmaf(w2, q.z, acc);
+    acc = fmaf(w3, q.w, acc);
+    p[2 * k] = pack_bf16(w0, w1);
+    p[2 * k + 1] = pack_bf16(w2, w3);
+  }
+}
+__device__ __forceinline__ void weights32_hilo_ds(const uint32_t (&v)[32], uint32_t (&hi)[16], uint32_t (&lo)[16],
+                                                  const float* ds, float& acc) {
+  const float4* d4 = reinterpret_cast<const float4*>(ds);
+#pragma unroll
+  for (int k = 0; k < 8; k++) {
+    const float4 q = d4[k];
+    float w[4];
+#pragma unroll
+    for (int e = 0; e < 4; e++) w[e] = ex2(__uint_as_float(v[4 * k + e]));
+    acc = fmaf(w[0], q.x, acc);
+    acc = fmaf(w[1], q.y, acc);
+    acc = fmaf(w[2], q.z, acc);
+    acc = fmaf(w[3], q.w, acc);
+#pragma unroll
+    for (int e = 0; e < 2; e++) {
+      const uint32_t pk = pack_bf16(w[2 * e], w[2 * e + 1]);
+      hi[2 * k + e] = pk;
+      lo[2 * k + e] = pack_bf16(w[2 * e] - __uint_as_float(pk << 16), w[2 * e + 1] - __uint_as_float(pk & 0xFFFF0000u));
+    }
+  }
+}
+__device__ __forceinline__ void weights_in_halves_ds(uint32_t tS, const float* ds, float& acc) {
+#pragma unroll 1
+  for (int half = 0; half < 2; half++) {
+    uint32_t v0[32], v1[32];
+    tmem_ld32(tS + half * 64, v0);
+    tmem_ld32(tS + half * 64 + 32, v1);
+    tmem_wait_ld2(v0, v1);
+    uint32_t pk0[16], pk1[16];
+    weights32_ds(v0, pk0, ds + half * 64, acc);
+    weights32_ds(v1, pk1, ds + half * 64 + 32, acc);
+    tmem_st16(tS + half * 32, pk0);
+    tmem_st16(tS + half * 32 + 16, pk1);
+  }
+}
+__device__ __forceinline__ void weights_hilo_in_place_ds(uint32_t tS, const float* ds, float& acc) {
+  uint32_t lo0[16], lo1[16];
+  {
+    uint32_t v0[32], v1[32];
+    tmem_ld32(tS, v0);
+    tmem_ld32(tS + 32, v1);
+    tmem_wait_ld2(v0, v1);
+    uint32_t hi0[16], hi1[16];
+    weights32_hilo_ds(v0, hi0, lo0, ds, acc);
+    weights32_hilo_ds(v1, hi1, lo1, ds + 32, acc);
+    tmem_st16(tS, hi0);
+    tmem_st16(tS + 16, hi1);
+  }
+  uint32_t v0[32], v1[32];
+  tmem_ld32(tS + 64, v0);
+  tmem_ld32(tS + 96, v1);
+  tmem_wait_ld2(v0, v1);
+  tmem_st16(tS + 64, lo0);
+  tmem_st16(tS + 80, lo1);
+  uint32_t hi0[16], hi1[16];
+  weights32_hilo_ds(v0, hi0, lo0, ds + 64, acc);
+  weights32_hilo_ds(v1, hi1, lo1, ds + 96, acc);
+  tmem_st16(tS + 32, hi0);
+  tmem_st16(tS + 48, hi1);
+  tmem_st16(tS + 96, lo0);
+  tmem_st16(tS + 112, lo1);
+}
+
 // Point-extra rows [1, 1, -lse2_hi, -lse2_lo, 0, 0, 0, 0] (bf16) from lse [B,H,N]
 // (natural log) into px [B*H, Np, 8]; padded points (n >= N) get -1e30 so that
 // their weights vanish.

@@ -62,21 +62,35 @@ using namespace tc;
 // of its 128 slots, packed in pairs, into columns [0, 64) of the same buffer;
 // warp 2 + j turns slots [64 j, 64 j + 64) of every block into products
 // (K-steps [4 j, 4 j + 4)) accumulated in O_j.
+//
+// The same pass serves the backward (Sec. 3.3): with R_n = sum_g w_ng t_g,
+//   MODE 1 (deslice backward, t = z', v = dO): delta_n = dO_n . R_n (fp32);
+//   MODE 2 (slice backward, t = dU, v = fx): dfx_n = R_n (bf16, into out) and
+//     delta_n = fx_n . R_n + sum_g w_ng dS_g.  The second sum is formed by the
+//     softmax warpgroups from the fp32 weights; each warpgroup stores its own
+//     partial per point (wds[wg][bh][n], cleared beforehand) and the consumer adds them.
+// PS (split products): the weights and t as bf16 hi + lo halves, P t = Phi thi +
+// Plo thi + Phi tlo; the image then holds t's residual half after its bf16 half.
 // =========================================================================================
 constexpr uint32_t kDStage = kXBytes + 2 * kPxBytes;  // x tile, point extra (both halves)
 
+template <int MODE, bool PS>
 __global__ void __launch_bounds__(kThreads, 1)
     k_deslice(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap pmap,
               const uint8_t* __restrict__ wimg, const uint8_t* __restrict__ zimg, __nv_bfloat16* __restrict__ out,
-              int64_t N, int64_t Np, int H, int G, int splits, int hilo, uint32_t* status) {
+              const __nv_bfloat16* __restrict__ v, float* __restrict__ delta, float* __restrict__ wds,
+              const float* __restrict__ dS, int64_t N, int64_t Np, int H, int G, int splits, int hilo,
+              uint32_t zstride, uint32_t* status) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   // hilo: the residual half of W' fits in shared memory too (K = 80 logits, as in
   // the statistics pass); else bf16 W' only (K = 48).
-  const uint32_t wbytes = (uint32_t)G * (hilo ? kWRow : 96), zbytes = (uint32_t)G * 64;
+  const uint32_t wbytes = (uint32_t)G * (hilo ? kWRow : 96), zbytes = (uint32_t)G * (PS ? 128 : 64);
   uint8_t* s_w = smem;
   uint8_t* s_z = s_w + wbytes;
-  uint8_t* s_x = s_z + zbytes;  // stage s at s_x + s * kDStage
+  float* s_ds = reinterpret_cast<float*>(s_z + zbytes);  // MODE 2: dS of the G slots
+  // (the stages stay 1024-byte aligned for their swizzled tiles)
+  uint8_t* s_x = s_z + zbytes + (MODE == 2 ? (((uint32_t)G * 4 + 1023u) & ~1023u) : 0u);  // stage s at s_x + s * kDStage
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_x + kStages * kDStage);
   uint64_t* wz_full = bars;
   uint64_t* x_full = bars + 1;
@@ -118,6 +132,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_mbar_init();
   }
   for (int s = 0; s < kStages; s++) zero_smem(s_x + s * kDStage + kXBytes + kPxBytes, kPxBytes);
+  if (MODE == 2)
+    for (int g = threadIdx.x; g < G; g += kThreads) s_ds[g] = dS[wk.bh * G + g];
   fence_proxy_async_smem();
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
@@ -132,7 +148,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&pmap);
       mbar_expect_tx(wz_full, wbytes + zbytes);
       load_images(s_w, wimg + (size_t)h * G * kWRow, wbytes, wz_full);
-      load_images(s_z, zimg + (size_t)wk.bh * zbytes, zbytes, wz_full);
+      load_images(s_z, zimg + (size_t)wk.bh * zstride, zbytes, wz_full);
       int i = 0;
       for (; i < wk.ntiles; i++) {
         const int s = i % kStages;
@@ -193,6 +209,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int g0 = c * kGC + (4 * j + kk) * 16;
           const uint32_t zaddr = sz + (uint32_t)((g0 >> 6) * 4096 + (g0 & 63) * 2);
           mma_ts_w(tO, tP + (uint32_t)kk * 8, sdesc(zaddr, 16, 1024, kSw128), idesc_pv, (c > 0 || kk > 0) ? 1u : 0u);
+          if (PS) {
+            mma_ts_w(tO, tP + 64 + (uint32_t)kk * 8, sdesc(zaddr, 16, 1024, kSw128), idesc_pv, 1u);
+            mma_ts_w(tO, tP + (uint32_t)kk * 8, sdesc(zaddr + (uint32_t)G * 64, 16, 1024, kSw128), idesc_pv, 1u);
+          }
         }
         mma_commit_w(&pv_done[bb]);
         if (c == nch - 1) mma_commit_w(&o_full[ob]);
@@ -221,18 +241,49 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (lane == 0) mbar_arrive(&o_free[ob]);
       const int64_t n = (wk.tile0 + t) * kTile + r;
       if (n < N) {
-        uint4* dst = reinterpret_cast<uint4*>(out + ((b * N + n) * H + h) * kD);
+        const int64_t row = ((b * N + n) * H + h) * kD;
+        if (MODE != 1) {
+          uint4* dst = reinterpret_cast<uint4*>(out + row);
 #pragma unroll
-        for (int k = 0; k < 4; k++) {
-          uint32_t w[4];
+          for (int k = 0; k < 4; k++) {
+            uint32_t w[4];
 #pragma unroll
-          for (int e = 0; e < 4; e++)
-            w[e] = pack_bf16(__uint_as_float(o0[8 * k + 2 * e]) + __uint_as_float(o1[8 * k + 2 * e]),
-                             __uint_as_float(o0[8 * k + 2 * e + 1]) + __uint_as_float(o1[8 * k + 2 * e + 1]));
-          dst[k] = make_uint4(w[0], w[1], w[2], w[3]);
+            for (int e = 0; e < 4; e++)
+              w[e] = pack_bf16(__uint_as_float(o0[8 * k + 2 * e]) + __uint_as_float(o1[8 * k + 2 * e]),
+                               __uint_as_float(o0[8 * k + 2 * e + 1]) + __uint_as_float(o1[8 * k + 2 * e + 1]));
+            dst[k] = make_uint4(w[0], w[1], w[2], w[3]);
+          }
+        }
+        if (MODE != 0) {
+          // delta_n = v_n . R_n from the fp32 accumulators.
+          const uint4* src = reinterpret_cast<const uint4*>(v + row);
+          float acc = 0.f;
+#pragma unroll
+          for (int k = 0; k < 4; k++) {
+            const uint4 q4 = src[k];
+            const uint32_t w[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+            for (int e = 0; e < 4; e++) {
+              const int c0 = 8 * k + 2 * e;
+              acc = fmaf(__uint_as_float(w[e] << 16), __uint_as_float(o0[c0]) + __uint_as_float(o1[c0]), acc);
+              acc = fmaf(__uint_as_float(w[e] & 0xFFFF0000u), __uint_as_float(o0[c0 + 1]) + __uint_as_float(o1[c0 + 1]),
+                         acc);
+            }
+          }
+          delta[wk.bh * N + n] = acc;
         }
       }
       return true;
+    };
+    // MODE 2: this warpgroup's sum_g w dS_g for point r of its current tile.
+    float wds_acc = 0.f;
+    int wds_tile = -1;
+    auto flush_wds = [&]() {
+      if (MODE == 2 && wds_tile >= 0) {
+        const int64_t n = (wk.tile0 + wds_tile) * kTile + r;
+        if (n < N) wds[((int64_t)wg * gridDim.y + wk.bh) * N + n] = wds_acc;
+      }
+      wds_acc = 0.f;
     };
     // Warpgroup wg takes the whole blocks q with q % 2 == wg, so the two warpgroups
     // run half a block out of phase: one exponentiates while the other waits.
@@ -242,7 +293,20 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int bb = q % kSBuf;
       if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
       tc_fence_after();
-      weights_in_halves(tmem + lane_addr + (uint32_t)bb * kGC);
+      if (MODE == 2) {
+        if (i != wds_tile) {
+          flush_wds();
+          wds_tile = i;
+        }
+        if (PS)
+          weights_hilo_in_place_ds(tmem + lane_addr + (uint32_t)bb * kGC, s_ds + c * kGC, wds_acc);
+        else
+          weights_in_halves_ds(tmem + lane_addr + (uint32_t)bb * kGC, s_ds + c * kGC, wds_acc);
+      } else if (PS) {
+        weights_hilo_in_place(tmem + lane_addr + (uint32_t)bb * kGC);
+      } else {
+        weights_in_halves(tmem + lane_addr + (uint32_t)bb * kGC);
+      }
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
@@ -252,6 +316,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (c == 0 && i > 0 && !(ok = epilogue(i - 1))) break;
     }
     if (ok && total > 0 && total % 2 == wg) epilogue(wk.ntiles - 1);
+    if (ok) flush_wds();
   }
   tc_fence_before();
   __syncthreads();
@@ -701,8 +766,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 int slice_blocks(const Shape& s) { return s.G / kGC < 1 ? 1 : s.G / kGC; }
 int slice_splits(const Shape& s) { return point_splits(s, (int)(s.BH() * slice_blocks(s))); }
 
-size_t smem_deslice(int G, bool hilo) {
-  return 1024 + (size_t)G * ((hilo ? kWRow : 96) + 64) + kStages * kDStage + 512;
+size_t smem_deslice(int G, bool hilo, int mode = 0, bool ps = false) {
+  return 1024 + (size_t)G * ((hilo ? kWRow : 96) + (ps ? 128 : 64)) + (mode == 2 ? align_up((size_t)G * 4, 1024) : 0) +
+         kStages * kDStage + 512;
 }
 size_t smem_stats(int G, bool split) {
   return 1024 + (size_t)G * (split ? kWRow : 96) + kStages * kXBytes + kExBytes + 2 * kTile * 8 + 512;
@@ -802,9 +868,36 @@ cudaError_t tc_deslice_fwd(const Shape& s, const void* x, const float* W, const 
   const bool hilo = s.dot == FS_DOT_BF16X2 && smem_deslice(s.G, true) <= kMaxSmem;  // up to G = 768
   const size_t sm = smem_deslice(s.G, hilo);
   dim3 grid((unsigned)P, (unsigned)s.BH());
-  if ((e = set_smem(k_deslice, sm)) != cudaSuccess) return e;
-  k_deslice<<<grid, kThreads, sm, st>>>(xmap, pmap, wimg, zimg, static_cast<__nv_bfloat16*>(out), s.N, Np, s.H, s.G,
-                                        P, hilo ? 1 : 0, status);
+  if ((e = set_smem(k_deslice<0, false>, sm)) != cudaSuccess) return e;
+  k_deslice<0, false><<<grid, kThreads, sm, st>>>(xmap, pmap, wimg, zimg, static_cast<__nv_bfloat16*>(out), nullptr,
+                                                  nullptr, nullptr, nullptr, s.N, Np, s.H, s.G, P, hilo ? 1 : 0,
+                                                  (uint32_t)s.G * 64, status);
+  return cudaGetLastError();
+}
+
+size_t tc_rows_smem(const Shape& s, int mode, bool ps, bool hilo) { return smem_deslice(s.G, hilo, mode, ps); }
+
+cudaError_t tc_rows_bwd(const Shape& s, int mode, const void* x, const uint8_t* wimg, const uint8_t* zimg,
+                        const void* px, const void* v, void* dfx, float* delta, float* wds, const float* dS,
+                        uint32_t* status, cudaStream_t st) {
+  const bool split = s.dot == FS_DOT_BF16X2;
+  const bool ps = split && smem_deslice(s.G, false, mode, true) <= kMaxSmem;
+  const bool hilo = split && smem_deslice(s.G, true, mode, ps) <= kMaxSmem;
+  const size_t sm = smem_deslice(s.G, hilo, mode, ps);
+  if (sm > kMaxSmem) return cudaErrorInvalidValue;
+  const int64_t Np = padded_n(s);
+  CUtensorMap xmap, pmap;
+  if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
+  if (!make_px_map(&pmap, px, s.BH(), Np)) return cudaErrorInvalidValue;
+  const int P = point_splits(s, (int)s.BH());
+  dim3 grid((unsigned)P, (unsigned)s.BH());
+  const auto kernel = mode == 1 ? (ps ? k_deslice<1, true> : k_deslice<1, false>)
+                                : (ps ? k_deslice<2, true> : k_deslice<2, false>);
+  cudaError_t e = set_smem(kernel, sm);
+  if (e != cudaSuccess) return e;
+  kernel<<<grid, kThreads, sm, st>>>(xmap, pmap, wimg, zimg, static_cast<__nv_bfloat16*>(dfx),
+                                     static_cast<const __nv_bfloat16*>(v), delta, wds, dS, s.N, Np, s.H, s.G, P,
+                                     hilo ? 1 : 0, (uint32_t)s.G * 128, status);
   return cudaGetLastError();
 }
 

@@ -33,7 +33,7 @@ FS_OP_SLICE_FWD, FS_OP_DESLICE_FWD, FS_OP_DESLICE_BWD, FS_OP_SLICE_BWD = range(4
 
 EXPORTED = ("fs_workspace_bytes", "fs_slice_fwd", "fs_slice_finalize", "fs_mix", "fs_deslice_fwd",
             "fs_deslice_bwd", "fs_mix_bwd", "fs_slice_bwd", "fs_device_status", "fs_status_string",
-            "fs_path_for_shape", "fs_forward_launch_count", "fs_slice_fwd_noalloc")
+            "fs_path_for_shape", "fs_backward_path_for_shape", "fs_forward_launch_count", "fs_slice_fwd_noalloc")
 
 
 class fs_shape(ctypes.Structure):
@@ -63,6 +63,7 @@ _sig = {
     "fs_device_status": (_I, [_P, _P]),
     "fs_status_string": (ctypes.c_char_p, [_I]),
     "fs_path_for_shape": (_I, [_S]),
+    "fs_backward_path_for_shape": (_I, [_S]),
     "fs_forward_launch_count": (_I, [_S]),
     "fs_slice_fwd_noalloc": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _I, ctypes.POINTER(_P), _P]),
 }
@@ -115,6 +116,10 @@ def workspace(shape: fs_shape, op: int, device="cuda") -> torch.Tensor:
 
 def path_for_shape(shape: fs_shape) -> int:
     return int(_lib.fs_path_for_shape(ctypes.byref(shape)))
+
+
+def backward_path_for_shape(shape: fs_shape) -> int:
+    return int(_lib.fs_backward_path_for_shape(ctypes.byref(shape)))
 
 
 def forward_launch_count(shape: fs_shape) -> int:
