@@ -272,20 +272,55 @@ __global__ void k_mix_bwd_dz(const float* __restrict__ M, const float* __restric
   dz[bh * G * D + idx] = s;
 }
 
-// dM[h][g][k] = sum_b sum_c dzp[b,h,g,c] z[b,h,k,c]
-__global__ void k_mix_bwd_dM(const float* __restrict__ z, const float* __restrict__ dzp,
-                             float* __restrict__ dM, int64_t B, int H, int G, int D) {
-  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= (int64_t)H * G * G) return;
-  const int h = (int)(idx / ((int64_t)G * G));
-  const int g = (int)((idx / G) % G), k = (int)(idx % G);
-  float s = 0.f;
+// dM[h][g][k] = sum_b sum_c dzp[b,h,g,c] z[b,h,k,c]: per head a G x G product with
+// K = B*D, tiled 64 x 64 per block (16 x 16 threads, 4 x 4 outputs each), the two
+// operand tiles staged in shared memory 16 channels at a time; the sum runs over
+// b, then c, in a fixed order.
+__global__ void __launch_bounds__(256) k_mix_bwd_dM(const float* __restrict__ z, const float* __restrict__ dzp,
+                                                    float* __restrict__ dM, int64_t B, int H, int G, int D) {
+  constexpr int T = 64, KC = 16;
+  __shared__ float sa[KC][T + 1];
+  __shared__ float sb[KC][T + 1];
+  const int h = blockIdx.z;
+  const int g0 = blockIdx.y * T, k0 = blockIdx.x * T;
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  float acc[4][4] = {};
   for (int64_t b = 0; b < B; b++) {
-    const float* a = dzp + ((b * H + h) * G + g) * D;
-    const float* t = z + ((b * H + h) * G + k) * D;
-    for (int c = 0; c < D; c++) s = fmaf(a[c], t[c], s);
+    const float* A = dzp + (b * H + h) * (int64_t)G * D;
+    const float* Z = z + (b * H + h) * (int64_t)G * D;
+    for (int c0 = 0; c0 < D; c0 += KC) {
+      __syncthreads();
+      for (int i = threadIdx.x; i < T * KC; i += 256) {
+        const int r = i / KC, c = i % KC;
+        sa[c][r] = (g0 + r < G && c0 + c < D) ? A[(int64_t)(g0 + r) * D + c0 + c] : 0.f;
+        sb[c][r] = (k0 + r < G && c0 + c < D) ? Z[(int64_t)(k0 + r) * D + c0 + c] : 0.f;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int c = 0; c < KC; c++) {
+        float av[4], bv[4];
+#pragma unroll
+        for (int i = 0; i < 4; i++) {
+          av[i] = sa[c][ty + 16 * i];
+          bv[i] = sb[c][tx + 16 * i];
+        }
+#pragma unroll
+        for (int i = 0; i < 4; i++)
+#pragma unroll
+          for (int j = 0; j < 4; j++) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+      }
+    }
   }
-  dM[idx] = s;
+#pragma unroll
+  for (int i = 0; i < 4; i++) {
+    const int g = g0 + ty + 16 * i;
+    if (g >= G) continue;
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+      const int k = k0 + tx + 16 * j;
+      if (k < G) dM[((int64_t)h * G + g) * G + k] = acc[i][j];
+    }
+  }
 }
 
 // ---- deslice: point-owned ----------------------------------------------------------
@@ -550,38 +585,40 @@ __global__ void k_slice_bwd_prep(const float* __restrict__ z, const float* __res
   dUS[i * (D + 1) + D] = -s / den;
 }
 
-// Fixed-order reduction of slot-owned backward partials over (b, p).
-// Writes (or adds) dW[h][k][g], db[h][g] (the temperature gradient is reduced
-// separately, from per-point row sums); optionally d_tokens_mixed[b][h][g][c] (sum over p only).
-__global__ void k_reduce_bwd(const float* __restrict__ part, int P, int64_t B, int H, int G, int D,
-                             int PS, int has_dzp, const float* __restrict__ tau, float* __restrict__ dzp,
-                             float* __restrict__ dW, float* __restrict__ db, int accumulate) {
+// Fixed-order reduction of slot-owned backward partials over (b, p), one thread
+// per output word (consecutive threads read consecutive words of a partial row):
+//   k_reduce_bwd_params: dW[h][k][g], db[h][g] (written, or added), sums over b then p;
+//   k_reduce_bwd_tokens: d_tokens_mixed[b][h][g][c], sums over p.
+// The temperature gradient is reduced separately, from its own partials.
+__global__ void k_reduce_bwd_params(const float* __restrict__ part, int P, int64_t B, int H, int G, int D,
+                                    int PS, int off, const float* __restrict__ tau, float* __restrict__ dW,
+                                    float* __restrict__ db, int accumulate) {
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= (int64_t)H * G) return;
-  const int h = (int)(idx / G), g = (int)(idx % G);
-  const float inv = 1.f / tau[h];
-  const int off = has_dzp ? D : 0;
+  if (idx >= (int64_t)H * G * (D + 1)) return;
+  const int k = (int)(idx % (D + 1));
+  const int64_t hg = idx / (D + 1);
+  const int h = (int)(hg / G), g = (int)(hg % G);
   const int64_t BH = B * H;
-  if (has_dzp) {
-    for (int64_t b = 0; b < B; b++) {
-      for (int c = 0; c < D; c++) {
-        float s = 0.f;
-        for (int p = 0; p < P; p++) s += part[(((int64_t)p * BH + b * H + h) * G + g) * PS + c];
-        dzp[((b * H + h) * G + g) * D + c] = s;
-      }
-    }
+  float s = 0.f;
+  for (int64_t b = 0; b < B; b++)
+    for (int p = 0; p < P; p++) s += part[(((int64_t)p * BH + b * H + h) * G + g) * PS + off + k];
+  s *= 1.f / tau[h];
+  if (k < D) {
+    const int64_t o = ((int64_t)h * D + k) * G + g;
+    dW[o] = (accumulate ? dW[o] : 0.f) + s;
+  } else {
+    db[hg] = (accumulate ? db[hg] : 0.f) + s;
   }
-  for (int k = 0; k <= D; k++) {
-    float s = 0.f;
-    for (int64_t b = 0; b < B; b++)
-      for (int p = 0; p < P; p++) s += part[(((int64_t)p * BH + b * H + h) * G + g) * PS + off + k];
-    if (k < D) {
-      const int64_t o = ((int64_t)h * D + k) * G + g;
-      dW[o] = (accumulate ? dW[o] : 0.f) + s * inv;
-    } else {
-      db[idx] = (accumulate ? db[idx] : 0.f) + s * inv;
-    }
-  }
+}
+__global__ void k_reduce_bwd_tokens(const float* __restrict__ part, int P, int64_t BHG, int D, int PS,
+                                    float* __restrict__ dzp) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= BHG * D) return;
+  const int c = (int)(idx % D);
+  const int64_t row = idx / D;
+  float s = 0.f;
+  for (int p = 0; p < P; p++) s += part[((int64_t)p * BHG + row) * PS + c];
+  dzp[idx] = s;
 }
 
 // dtau[h] (+)= -(1/tau_h) * sum over batches and point blocks of the block sums of
@@ -684,11 +721,16 @@ cudaError_t launch_bwd_slice(const Shape& s, int P, const void* x, const void* v
 cudaError_t simt_reduce_bwd(const Shape& s, int P, const float* part, int PS, int has_dzp, const float* tau,
                             float* dzp, float* dW, float* db, float* dtau, const float* dt_part, int64_t nblk,
                             int accumulate, cudaStream_t st) {
-  const int64_t HG = (int64_t)s.H * s.G;
-  k_reduce_bwd<<<(unsigned)((HG + 127) / 128), 128, 0, st>>>(part, P, s.B, s.H, s.G, s.d, PS, has_dzp, tau,
-                                                              dzp, dW, db, accumulate);
+  const int64_t nw = (int64_t)s.H * s.G * (s.d + 1);
+  k_reduce_bwd_params<<<(unsigned)((nw + 255) / 256), 256, 0, st>>>(part, P, s.B, s.H, s.G, s.d, PS,
+                                                                     has_dzp ? s.d : 0, tau, dW, db, accumulate);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
+  if (has_dzp) {
+    const int64_t BHG = s.BH() * s.G;
+    k_reduce_bwd_tokens<<<(unsigned)((BHG * s.d + 255) / 256), 256, 0, st>>>(part, P, BHG, s.d, PS, dzp);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
   k_reduce_dtau<<<s.H, 256, 0, st>>>(dt_part, s.B, s.H, nblk, tau, dtau, accumulate);
   return cudaGetLastError();
 }
@@ -739,8 +781,8 @@ cudaError_t simt_mix_bwd(const Shape& s, const float* M, const float* z, const f
   k_mix_bwd_dz<<<grid, 256, 0, st>>>(M, dzp, dz, s.H, s.G, s.d);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const int64_t HGG = (int64_t)s.H * s.G * s.G;
-  k_mix_bwd_dM<<<(unsigned)((HGG + 255) / 256), 256, 0, st>>>(z, dzp, dM, s.B, s.H, s.G, s.d);
+  const dim3 tiles((unsigned)((s.G + 63) / 64), (unsigned)((s.G + 63) / 64), (unsigned)s.H);
+  k_mix_bwd_dM<<<tiles, 256, 0, st>>>(z, dzp, dM, s.B, s.H, s.G, s.d);
   return cudaGetLastError();
 }
 
