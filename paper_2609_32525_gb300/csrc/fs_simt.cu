@@ -242,34 +242,51 @@ __global__ void k_finalize(float* __restrict__ tokens, const float* __restrict__
 }
 
 // ---- mix and its backward ------------------------------------------------------------
-// zp[bh][g][c] = sum_k M[h][g][k] z[bh][k][c]; grid (ceil(G*D/256), B*H).
-__global__ void k_mix(const float* __restrict__ M, const float* __restrict__ z, float* __restrict__ zp,
-                      int H, int G, int D) {
-  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= G * D) return;
-  const int g = idx / D, c = idx % D;
+// out[bh][g][c] = sum_k A_h(g, k) in[bh][k][c] per (b, h), with A_h = M[h] (the mix,
+// z' = M z) or A_h = M[h]^T (its backward, dz = M^T dz').  Blocks of 16 rows g x 32
+// channels (16 x 16 threads, 2 outputs each; many blocks, so that the short K
+// loop's latency overlaps) stage A and `in` 64 k at a time in shared memory; the
+// sum over k runs in a fixed order.
+template <bool kTrans>
+__global__ void __launch_bounds__(256) k_mix_tiled(const float* __restrict__ M, const float* __restrict__ in,
+                                                   float* __restrict__ out, int H, int G, int D) {
+  constexpr int TG = 16, TC = 32, KC = 64;
+  __shared__ float sa[KC][TG + 1];
+  __shared__ float sb[KC][TC + 1];
   const int64_t bh = blockIdx.y;
   const int h = (int)(bh % H);
-  const float* Mr = M + ((int64_t)h * G + g) * G;
-  const float* zb = z + bh * G * D;
-  float s = 0.f;
-  for (int k = 0; k < G; k++) s = fmaf(Mr[k], zb[(int64_t)k * D + c], s);
-  zp[bh * G * D + idx] = s;
-}
-
-// dz[bh][k][c] = sum_g M[h][g][k] dzp[bh][g][c]
-__global__ void k_mix_bwd_dz(const float* __restrict__ M, const float* __restrict__ dzp,
-                             float* __restrict__ dz, int H, int G, int D) {
-  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= G * D) return;
-  const int k = idx / D, c = idx % D;
-  const int64_t bh = blockIdx.y;
-  const int h = (int)(bh % H);
+  const int g0 = blockIdx.x * TG, c0 = blockIdx.z * TC;
+  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
   const float* Mh = M + (int64_t)h * G * G;
-  const float* db = dzp + bh * G * D;
-  float s = 0.f;
-  for (int g = 0; g < G; g++) s = fmaf(Mh[(int64_t)g * G + k], db[(int64_t)g * D + c], s);
-  dz[bh * G * D + idx] = s;
+  const float* X = in + bh * (int64_t)G * D;
+  float acc0 = 0.f, acc1 = 0.f;
+  for (int k0 = 0; k0 < G; k0 += KC) {
+    __syncthreads();
+    for (int i = threadIdx.x; i < TG * KC; i += 256) {
+      // consecutive threads read consecutive addresses of M: k for the mix, g for its transpose
+      const int g = kTrans ? i % TG : i / KC, k = kTrans ? i / TG : i % KC;
+      float v = 0.f;
+      if (g0 + g < G && k0 + k < G)
+        v = kTrans ? Mh[(int64_t)(k0 + k) * G + g0 + g] : Mh[(int64_t)(g0 + g) * G + k0 + k];
+      sa[k][g] = v;
+    }
+    for (int i = threadIdx.x; i < KC * TC; i += 256) {
+      const int k = i / TC, c = i % TC;
+      sb[k][c] = (k0 + k < G && c0 + c < D) ? X[(int64_t)(k0 + k) * D + c0 + c] : 0.f;
+    }
+    __syncthreads();
+#pragma unroll 16
+    for (int k = 0; k < KC; k++) {
+      const float a = sa[k][ty];
+      acc0 = fmaf(a, sb[k][tx], acc0);
+      acc1 = fmaf(a, sb[k][tx + 16], acc1);
+    }
+  }
+  const int g = g0 + ty;
+  if (g < G) {
+    if (c0 + tx < D) out[(bh * G + g) * (int64_t)D + c0 + tx] = acc0;
+    if (c0 + tx + 16 < D) out[(bh * G + g) * (int64_t)D + c0 + tx + 16] = acc1;
+  }
 }
 
 // dM[h][g][k] = sum_b sum_c dzp[b,h,g,c] z[b,h,k,c]: per head a G x G product with
@@ -770,15 +787,15 @@ cudaError_t simt_finalize(const Shape& s, float* tokens, const float* wsum, cuda
 }
 
 cudaError_t simt_mix(const Shape& s, const float* M, const float* z, float* zp, cudaStream_t st) {
-  dim3 grid((unsigned)((s.G * s.d + 255) / 256), (unsigned)s.BH());
-  k_mix<<<grid, 256, 0, st>>>(M, z, zp, s.H, s.G, s.d);
+  const dim3 grid((unsigned)((s.G + 15) / 16), (unsigned)s.BH(), (unsigned)((s.d + 31) / 32));
+  k_mix_tiled<false><<<grid, 256, 0, st>>>(M, z, zp, s.H, s.G, s.d);
   return cudaGetLastError();
 }
 
 cudaError_t simt_mix_bwd(const Shape& s, const float* M, const float* z, const float* dzp, float* dz, float* dM,
                          cudaStream_t st) {
-  dim3 grid((unsigned)((s.G * s.d + 255) / 256), (unsigned)s.BH());
-  k_mix_bwd_dz<<<grid, 256, 0, st>>>(M, dzp, dz, s.H, s.G, s.d);
+  const dim3 grid((unsigned)((s.G + 15) / 16), (unsigned)s.BH(), (unsigned)((s.d + 31) / 32));
+  k_mix_tiled<true><<<grid, 256, 0, st>>>(M, dzp, dz, s.H, s.G, s.d);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const dim3 tiles((unsigned)((s.G + 63) / 64), (unsigned)((s.G + 63) / 64), (unsigned)s.H);
