@@ -10,6 +10,11 @@ workload, default N = 1,048,576 points, H = 8, d = 32, G = 1024, bf16
 (inputs 512 MiB each, larger than the 129 MB L2, so no flush is needed between
 steps).  Metric: Mpoints/s of the whole job (B*N points per step per rank).
 
+--workload train_bf16 (B = 2, N = 524,288, G = 512, the workload with an upstream
+gradient) times a training step instead: the forward and then fs_deslice_bwd ->
+fs_mix_bwd -> fs_slice_bwd, every gradient of the coupling, and reports that
+step's Mpoints/s on its own line (metric "train step ...").
+
 Multi-GPU: the workload is replicated (each rank runs its own full copy; no
 collective on the data path), so scaling is weak.  Launched with torchrun for
 N > 1; rank 0 prints the line.
@@ -52,8 +57,8 @@ def _peaks():
 # deslice) are scaled x4; the W/Z' images and the split-partial reduction are not.
 # Valid only for the kernel sources it was measured on, identified by their SHA-1.
 # When the sources change the figure is reported as null.
-_TRAFFIC = {"sources_sha1": "dabd91c7777d2244eec5ea07f2723cfb1311caea", "workload": "large_g_bf16", "N": 1048576,
-            "fs_slice_fwd": 2.5625e9, "fs_deslice_fwd": 1.0580e9}
+_TRAFFIC = {"sources_sha1": "1a646add9ab2e2759603c65d05661901255e2551", "workload": "large_g_bf16", "N": 1048576,
+            "fs_slice_fwd": 2.3552e9, "fs_deslice_fwd": 1.0585e9}
 
 
 def _sources_sha1():
@@ -131,7 +136,7 @@ class ClockSampler:
                 "samples": len(sm), "reasons": sorted(reasons)}
 
 
-def cpu_oracle_rate(wl, target_s=12.0):
+def cpu_oracle_rate(wl, target_s=12.0, train=False):
     """The fp64 oracle as it stands, forward (slice over the sample, mix, deslice
     of the sample) on the first n points of the workload, all heads.  Returns
     (Mpoints/s, sample description, threads)."""
@@ -139,7 +144,10 @@ def cpu_oracle_rate(wl, target_s=12.0):
 
     def run(n):
         t0 = time.perf_counter()
-        orc.forward(wl.x_mid[:, :n], wl.fx[:, :n], wl.W_slice, wl.bias, wl.tau, wl.M, eps=wl.eps)
+        if train:
+            orc.backward(wl.x_mid[:, :n], wl.fx[:, :n], wl.W_slice, wl.bias, wl.tau, wl.M, wl.dout[:, :n], eps=wl.eps)
+        else:
+            orc.forward(wl.x_mid[:, :n], wl.fx[:, :n], wl.W_slice, wl.bias, wl.tau, wl.M, eps=wl.eps)
         return time.perf_counter() - t0
 
     n = min(wl.N, 4096)
@@ -155,8 +163,9 @@ def cpu_oracle_rate(wl, target_s=12.0):
     except Exception:
         pass
     pts = wl.B * n2
-    desc = (f"{wl.name}: first {n2} of {wl.N} points x B={wl.B}, all {wl.H} heads, fp64 forward "
-            f"(slice over the sample, mix, deslice of the sample), {t2:.1f} s")
+    what = ("fp64 forward and backward (every gradient; the slice's sums over the sample)" if train else
+            "fp64 forward (slice over the sample, mix, deslice of the sample)")
+    desc = f"{wl.name}: first {n2} of {wl.N} points x B={wl.B}, all {wl.H} heads, {what}, {t2:.1f} s"
     return pts / t2 / 1e6, desc, threads
 
 
@@ -187,6 +196,142 @@ def run_reference(args):
                              "sample": f"first {n} points of {wl.name} per step, all heads, fp64 forward"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+TRAIN_METRIC = "train step (slice+mix+deslice forward and backward) Mpoints/s"
+
+
+def run_train(args, wl, dev, world, rank):
+    """A training step of the coupling through the C ABI: the forward, then the
+    backward of the deslice, the mix and the slice (every gradient)."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2609_32525_gb300 import flashslice as fs
+    from paper_2609_32525_gb300 import sharding
+
+    def put(a, dt):
+        return torch.from_numpy(a).to(device=dev, dtype=dt).contiguous()
+
+    tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    x, fx, dO = put(wl.x_mid, tdt), put(wl.fx, tdt), put(wl.dout, tdt)
+    W, b, t, M = (put(getattr(wl, k), torch.float32) for k in ("W_slice", "bias", "tau", "M"))
+    c = fs.Coupling(wl.B, wl.N, wl.H, wl.d, wl.G, tdt, wl.eps, device=dev, backward=True)
+    s = c.shape
+    stream = torch.cuda.current_stream()
+    names = ("fs_slice_fwd", "fs_mix", "fs_deslice_fwd", "fs_deslice_bwd", "fs_mix_bwd", "fs_slice_bwd")
+
+    def step(ev=None, xs=x, fs_=fx, ds=dO):
+        calls = (
+            lambda: fs.fs_slice_fwd(s, xs, fs_, W, b, t, c.tokens, c.wsum, c.lse, True, c.ws_slice),
+            lambda: fs.fs_mix(s, M, c.tokens, c.tokens_mixed),
+            lambda: fs.fs_deslice_fwd(s, xs, W, b, t, c.tokens_mixed, c.lse, c.out, c.ws_deslice),
+            lambda: fs.fs_deslice_bwd(s, xs, W, b, t, c.tokens_mixed, c.lse, ds, c.d_tokens_mixed, c.dx_mid, c.dW,
+                                      c.dbias, c.dtau, False, c.ws_dbwd),
+            lambda: fs.fs_mix_bwd(s, M, c.tokens, c.d_tokens_mixed, c.d_tokens, c.dM),
+            lambda: fs.fs_slice_bwd(s, xs, fs_, W, b, t, c.tokens, c.wsum, c.lse, c.d_tokens, c.dx_mid, c.dfx, c.dW,
+                                    c.dbias, c.dtau, True, c.ws_sbwd),
+        )
+        for i, call in enumerate(calls):
+            if ev is not None:
+                ev[i].record(stream)
+            call()
+        if ev is not None:
+            ev[len(calls)].record(stream)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if c.device_status() != fs.FS_OK:
+        raise RuntimeError("device status after warm-up: " + fs.status_string(c.device_status()))
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        pass
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)] for _ in range(args.steps)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(uuid)
+    time.sleep(0.3)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for i in range(args.steps):
+        step(evs[i])
+    t1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    ms_per_step = sharding.job_time_ms(t0.elapsed_time(t1), dev) / args.steps
+    value = sharding.job_rate(wl.points, world, ms_per_step)
+    call_ms = {n: float(np.mean([e[i].elapsed_time(e[i + 1]) for e in evs])) for i, n in enumerate(names)}
+    assert c.device_status() == fs.FS_OK
+
+    # End to end: pinned host x, fx, dO in; out, dx_mid and dfx back, every step.
+    hx, hf, hd = (torch.from_numpy(a).to(tdt).pin_memory() for a in (wl.x_mid, wl.fx, wl.dout))
+    hout = [torch.empty(c.out.shape, dtype=tdt).pin_memory() for _ in range(3)]
+    x2, f2, d2 = torch.empty_like(x), torch.empty_like(fx), torch.empty_like(dO)
+
+    def e2e_step():
+        x2.copy_(hx, non_blocking=True)
+        f2.copy_(hf, non_blocking=True)
+        d2.copy_(hd, non_blocking=True)
+        step(None, x2, f2, d2)
+        for h_, dv in zip(hout, (c.out, c.dx_mid, c.dfx)):
+            h_.copy_(dv, non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = sharding.job_time_ms(e0.elapsed_time(e1) / args.e2e_steps, dev)
+
+    # Algorithmic work of a training step per point (C = H*d): forward 8*C*G flops,
+    # each backward call 8*C*G (logits, dw and the two products of its pass), so
+    # 24*C*G in all; bytes 11*C*e (forward 4, deslice backward 3, slice backward 4).
+    C, e = wl.H * wl.d, (2 if wl.dtype == "bf16" else 4)
+    P = wl.B * wl.N
+    flops, bytes_ = 24.0 * C * wl.G * P, 11.0 * C * e * P
+    per_call = {"fs_slice_fwd": 4.0 * C * wl.G * P, "fs_deslice_fwd": 4.0 * C * wl.G * P,
+                "fs_deslice_bwd": 8.0 * C * wl.G * P, "fs_slice_bwd": 8.0 * C * wl.G * P}
+    peaks = _peaks()
+    dom = max(per_call, key=lambda k: call_ms[k])
+    achieved = per_call[dom] / (call_ms[dom] * 1e-3) / 1e12
+    roof_t = max(flops / (peaks["bf16_tflops"] * 1e12), bytes_ / (peaks["hbm_gbs"] * 1e9))
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": achieved / peaks["bf16_tflops"], "traffic": None, "kernel": dom,
+                "peak_source": peaks["source"] + " bf16 burst", "step_frac": roof_t / (ms_per_step * 1e-3),
+                "call_ms": call_ms,
+                "per_call_work": "forward calls 4*C*G flops per point each, backward calls 8*C*G (C=256)"}
+    line = {"metric": TRAIN_METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
+            "data": "synthetic (seeded; " + wl.recipe + ")",
+            "config": {"workload": wl.name, "B": wl.B, "N": wl.N, "H": wl.H, "d": wl.d, "G": wl.G,
+                       "step": " + ".join(names), "parallelism": f"replicas x{world}",
+                       "dot": ["bf16", "bf16x2"][s.dot],
+                       "path": {"forward": ["simt", "tcgen05"][fs.path_for_shape(s)],
+                                "backward": ["simt", "tcgen05"][fs.backward_path_for_shape(s)]},
+                       **({"points_override": "N reduced for profiling; not the benchmark workload"}
+                          if args.points else {})},
+            "clocks": clocks, "roofline": roofline,
+            "e2e": {"value": sharding.job_rate(wl.points, world, e2e_ms), "unit": UNIT,
+                    "h2d_bytes_per_step": 3 * hx.numel() * hx.element_size(),
+                    "d2h_bytes_per_step": sum(h_.numel() * h_.element_size() for h_ in hout), "ms_per_step": e2e_ms}}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, desc, threads = cpu_oracle_rate(wl, train=True)
+        line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": desc}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
 
 
 def main():
@@ -230,6 +375,8 @@ def main():
     from paper_2609_32525_gb300.workloads import make_named
 
     wl = make_named(args.workload, n_override=args.points)
+    if wl.dout is not None:
+        return run_train(args, wl, dev, world, rank)
     tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
 
     def put(a, dt):
@@ -337,9 +484,9 @@ def main():
                 "call_ms": {"fs_slice_fwd": slice_ms, "fs_mix": mix_ms, "fs_deslice_fwd": desl_ms},
                 "per_call_work": "4*C*G flops per point for each of slice and deslice (C=256)"}
 
-    # The kernels are bound by the exponentials (one per point, head and slot in each
-    # of the three sweeps: statistics, slice, deslice), so the MUFU rate is reported
-    # beside the tensor roofline: 32 ex2 per clock per SM (measured on GB300).
+    # Each of the three sweeps (statistics, slice, deslice) makes one exponential per
+    # point, head and slot; at 32 ex2 per clock per SM (measured on GB300) that floor
+    # lies above the tensor roofline, so the MUFU rate is reported beside it.
     n_exp = float(wl.B * wl.N * wl.H * wl.G)
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     mufu_peak = 32.0 * sms * float(clocks.get("sm_mhz") or 2070.0) * 1e6 / 1e9
