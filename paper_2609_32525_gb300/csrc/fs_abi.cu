@@ -228,7 +228,7 @@ fs_status fs_slice_fwd(const fs_shape* s, const void* x_mid, const void* fx, con
   float* part = at<float>(ws, r.partials);
   FS_CUDA(simt_stats(sh, x_mid, W_slice, bias, tau, lse_buf, status, st));
   FS_CUDA(simt_slice_partials(sh, P, x_mid, fx, W_slice, bias, tau, lse_buf, part, status, st));
-  FS_CUDA(simt_reduce_tokens(sh, P, part, tokens, wsum, finalize, st));
+  FS_CUDA(simt_reduce_tokens(sh, P, part, sh.G, tokens, wsum, finalize, st));
   return FS_OK;
 }
 

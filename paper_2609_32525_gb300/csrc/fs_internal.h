@@ -40,7 +40,9 @@ cudaError_t simt_stats(const Shape& s, const void* x, const float* W, const floa
 cudaError_t simt_slice_partials(const Shape& s, int P, const void* x, const void* f,
                                 const float* W, const float* bias, const float* tau,
                                 const float* lse, float* part, uint32_t* status, cudaStream_t st);
-cudaError_t simt_reduce_tokens(const Shape& s, int P, const float* part, float* tokens,
+// Fixed-order sum of split partials [P, B*H, Gs, d+1] (Gs >= G slot rows per (b, h);
+// the first G are reduced) into tokens (normalised when finalize) and wsum.
+cudaError_t simt_reduce_tokens(const Shape& s, int P, const float* part, int Gs, float* tokens,
                                float* wsum, int finalize, cudaStream_t st);
 cudaError_t simt_finalize(const Shape& s, float* tokens, const float* wsum, cudaStream_t st);
 cudaError_t simt_mix(const Shape& s, const float* M, const float* z, float* zp, cudaStream_t st);

@@ -211,16 +211,20 @@ __global__ void __launch_bounds__(kThreads) k_slice_partial(
 // Fixed-order sum of the P partials, then (optionally) the normalisation.
 // One thread per (slot, column) of the partials [P, BHG, D+1]: consecutive threads
 // read consecutive words of every split.  The sum over splits runs in split order.
-__global__ void k_reduce_tokens(const float* __restrict__ part, int P, int64_t BHG, int D,
+// Partials hold Gs >= G slot rows per (b, h) (the tensor-core path pads G to whole
+// 128-slot blocks); only the first G are reduced.
+__global__ void k_reduce_tokens(const float* __restrict__ part, int P, int64_t BH, int G, int Gs, int D,
                                 float* __restrict__ tokens, float* __restrict__ wsum, int finalize,
                                 float eps) {
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t stride = BHG * (D + 1);
-  if (idx >= stride) return;
-  const int64_t i = idx / (D + 1);
+  if (idx >= BH * G * (D + 1)) return;
+  const int64_t i = idx / (D + 1);  // output row bh * G + g
   const int c = (int)(idx % (D + 1));
+  const int64_t row = (i / G) * Gs + i % G;  // its partial row
+  const int64_t stride = BH * Gs * (D + 1);
+  const int64_t at = row * (D + 1) + c;
   float v = 0.f;
-  for (int p = 0; p < P; p++) v += part[(int64_t)p * stride + idx];
+  for (int p = 0; p < P; p++) v += part[(int64_t)p * stride + at];
   if (c == D) {
     wsum[i] = v;
     return;
@@ -230,7 +234,7 @@ __global__ void k_reduce_tokens(const float* __restrict__ part, int P, int64_t B
     return;
   }
   float S = 0.f;
-  for (int p = 0; p < P; p++) S += part[(int64_t)p * stride + i * (D + 1) + D];
+  for (int p = 0; p < P; p++) S += part[(int64_t)p * stride + row * (D + 1) + D];
   tokens[i * D + c] = v / (S + eps);
 }
 
@@ -772,11 +776,11 @@ cudaError_t simt_slice_partials(const Shape& s, int P, const void* x, const void
   FS_DISPATCH(s, launch_slice_partials, s, P, x, f, W, bias, tau, lse, part, status, st);
 }
 
-cudaError_t simt_reduce_tokens(const Shape& s, int P, const float* part, float* tokens, float* wsum,
+cudaError_t simt_reduce_tokens(const Shape& s, int P, const float* part, int Gs, float* tokens, float* wsum,
                                int finalize, cudaStream_t st) {
-  const int64_t BHG = s.BH() * s.G;
-  const int64_t n = BHG * (s.d + 1);
-  k_reduce_tokens<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(part, P, BHG, s.d, tokens, wsum, finalize, s.eps);
+  const int64_t n = s.BH() * s.G * (s.d + 1);
+  k_reduce_tokens<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(part, P, s.BH(), s.G, Gs, s.d, tokens, wsum, finalize,
+                                                               s.eps);
   return cudaGetLastError();
 }
 

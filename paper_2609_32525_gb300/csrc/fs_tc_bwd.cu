@@ -714,7 +714,7 @@ cudaError_t run_backward(const Shape& s, int mode, const void* x, const void* v,
                          const float* tau, const float* lse, void* dfx, void* dx, int accumulate, uint8_t* ws,
                          const BwdLayout& L, uint32_t* status, cudaStream_t st) {
   const int64_t Np = padded_n(s);
-  cudaError_t e = prep_w(s, W, bias, tau, ws + L.wimg, status, st);
+  cudaError_t e = prep_w(s, s.G, W, bias, tau, ws + L.wimg, status, st);
   if (e != cudaSuccess) return e;
   const int64_t nwt = (int64_t)s.H * kD * s.G;
   k_prep_wt<<<(unsigned)((nwt + 255) / 256), 256, 0, st>>>(W, tau, ws + L.wtimg, s.H, s.G, status);
@@ -779,7 +779,7 @@ cudaError_t prep_t_images(const Shape& s, const float* t, int tstride, int has_c
 // cancelling terms of size |dz||fx|/(S + eps) that split bf16 products resolve only
 // to ~2^-17 of that size.
 bool tc_backward_supported(const Shape& s) {
-  return tc_forward_supported(s) && s.N >= 2 && smem_bwd_dx(s.G, false) <= kMaxSmem &&
+  return tc_forward_supported(s) && s.G % kGC == 0 && s.N >= 2 && smem_bwd_dx(s.G, false) <= kMaxSmem &&
          tc_rows_smem(s, 2, false, false) <= kMaxSmem;
 }
 

@@ -53,29 +53,32 @@ __device__ __forceinline__ uint32_t off_z(int c, int g) {
   return (uint32_t)(kb * 4096 + (c >> 3) * 1024 + (c & 7) * 128 + (((w >> 3) ^ (c & 7)) << 4) + (w & 7) * 2);
 }
 
+// Slots [G, Gp) pad the image to whole 128-slot blocks: W' = 0 and b' = -1e30, so
+// their logits are -1e30 and their weights exactly 0 in every pass.
 __global__ void k_prep_w(const float* __restrict__ W, const float* __restrict__ bias, const float* __restrict__ tau,
-                         uint8_t* __restrict__ img, int H, int G, uint32_t* status) {
+                         uint8_t* __restrict__ img, int H, int G, int Gp, uint32_t* status) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t total = (int64_t)H * G;
+  const int64_t total = (int64_t)H * Gp;
   if (i >= total) return;
-  const int h = (int)(i / G), g = (int)(i % G);
+  const int h = (int)(i / Gp), g = (int)(i % Gp);
   const float t = tau[h];
   if (!(t > 0.f && t < INFINITY)) {
     atomicCAS(status, 0u, (uint32_t)FS_ERR_BAD_TAU);
     return;
   }
   const float scale = kLog2e / t;
-  uint8_t* base = img + (size_t)h * G * kWRow;
+  const bool real = g < G;
+  uint8_t* base = img + (size_t)h * Gp * kWRow;
   __nv_bfloat16* wp = reinterpret_cast<__nv_bfloat16*>(base);
-  __nv_bfloat16* wl = reinterpret_cast<__nv_bfloat16*>(base + (size_t)G * 96);
+  __nv_bfloat16* wl = reinterpret_cast<__nv_bfloat16*>(base + (size_t)Gp * 96);
   for (int k = 0; k < kD; k++) {
-    const float w2 = W[((int64_t)h * kD + k) * G + g] * scale;
+    const float w2 = real ? W[((int64_t)h * kD + k) * G + g] * scale : 0.f;
     const __nv_bfloat16 whi = __float2bfloat16_rn(w2);
     wp[off_sw64(g, k) / 2] = whi;
     wl[off_sw64(g, k) / 2] = __float2bfloat16_rn(w2 - __bfloat162float(whi));
   }
-  __nv_bfloat16* ep = reinterpret_cast<__nv_bfloat16*>(base + (size_t)G * 64);
-  const float b2 = bias[(int64_t)h * G + g] * scale;
+  __nv_bfloat16* ep = reinterpret_cast<__nv_bfloat16*>(base + (size_t)Gp * 64);
+  const float b2 = real ? bias[(int64_t)h * G + g] * scale : -1e30f;
   const __nv_bfloat16 hi = __float2bfloat16_rn(b2);
   const __nv_bfloat16 lo = __float2bfloat16_rn(b2 - __bfloat162float(hi));
   // k = 2, 3 multiply the point side's -lse2 halves (zero in the statistics pass).
@@ -84,15 +87,16 @@ __global__ void k_prep_w(const float* __restrict__ W, const float* __restrict__ 
         k == 0 ? hi : (k == 1 ? lo : __float2bfloat16_rn((k == 2 || k == 3) ? 1.f : 0.f));
 }
 
-__global__ void k_prep_z(const float* __restrict__ zp, uint8_t* __restrict__ img, int64_t BH, int G) {
+// Padding slots [G, Gp) get zero rows (their weights are 0, and 0 * 0 stays 0).
+__global__ void k_prep_z(const float* __restrict__ zp, uint8_t* __restrict__ img, int64_t BH, int G, int Gp) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t total = BH * G * kD;
+  const int64_t total = BH * Gp * kD;
   if (i >= total) return;
   const int c = (int)(i % kD);
-  const int g = (int)((i / kD) % G);
-  const int64_t bh = i / ((int64_t)kD * G);
-  __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * G * 64);
-  out[off_z(c, g) / 2] = __float2bfloat16_rn(zp[i]);
+  const int g = (int)((i / kD) % Gp);
+  const int64_t bh = i / ((int64_t)kD * Gp);
+  __nv_bfloat16* out = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * Gp * 64);
+  out[off_z(c, g) / 2] = __float2bfloat16_rn(g < G ? zp[(bh * G + g) * kD + c] : 0.f);
 }
 
 // ---- shared pieces -------------------------------------------------------------------------
@@ -398,6 +402,14 @@ bool make_px_map(CUtensorMap* map, const void* ptr, int64_t BH, int64_t Np) {
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The tensor-core kernels see G rounded up to whole 128-slot blocks (padding slots
+// carry weight 0); outputs keep the caller's G.
+Shape tc_padded(const Shape& s) {
+  Shape r = s;
+  r.G = (s.G + kGC - 1) / kGC * kGC;
+  return r;
+}
+
 size_t w_image_bytes(const Shape& s) { return (size_t)s.H * s.G * kWRow; }
 size_t z_image_bytes(const Shape& s) { return (size_t)s.BH() * s.G * 64; }
 int64_t padded_n(const Shape& s) { return (s.N + kTile - 1) / kTile * kTile; }
@@ -428,10 +440,11 @@ cudaError_t set_smem(K kernel, size_t bytes) {
   return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
 }
 
-cudaError_t prep_w(const Shape& s, const float* W, const float* bias, const float* tau, uint8_t* img,
+// W image of the padded shape sp (sp.G = G rounded up) from W [H, d, G].
+cudaError_t prep_w(const Shape& sp, int G, const float* W, const float* bias, const float* tau, uint8_t* img,
                    uint32_t* status, cudaStream_t st) {
-  const int64_t n = (int64_t)s.H * s.G;
-  k_prep_w<<<(unsigned)((n + 127) / 128), 128, 0, st>>>(W, bias, tau, img, s.H, s.G, status);
+  const int64_t n = (int64_t)sp.H * sp.G;
+  k_prep_w<<<(unsigned)((n + 127) / 128), 128, 0, st>>>(W, bias, tau, img, sp.H, G, sp.G, status);
   return cudaGetLastError();
 }
 

@@ -796,7 +796,7 @@ cudaError_t run_stats(const Shape& s, const void* x, const uint8_t* wimg, float*
 bool tc_forward_supported(const Shape& s) {
   // TMA coordinates and the kernels' block counters are 32-bit.
   const int64_t np = (s.N + kTile - 1) / kTile * kTile;
-  return s.dtype == FS_BF16 && s.d == kD && s.G % kGC == 0 && s.G <= 1024 && s.N >= 1 &&
+  return s.dtype == FS_BF16 && s.d == kD && s.G <= 1024 && s.N >= 1 &&
          s.BH() * np < (int64_t(1) << 31) && encode_fn() != nullptr;
 }
 
@@ -804,33 +804,38 @@ int tc_forward_launch_count(const Shape&) {
   return 4 /*prep_w, stats, slice, reduce*/ + 4 /*prep_w, prep_z, prep_px, deslice*/;
 }
 
-size_t tc_slice_partials_bytes(const Shape& s) {
-  if (!tc_forward_supported(s)) return 0;
+size_t tc_slice_partials_bytes(const Shape& s0) {
+  if (!tc_forward_supported(s0)) return 0;
+  const Shape s = tc_padded(s0);
   return (size_t)slice_splits(s) * s.BH() * s.G * (kD + 1) * sizeof(float);
 }
-size_t tc_slice_prep_bytes(const Shape& s) {
-  return tc_forward_supported(s) ? align_up(w_image_bytes(s), 256) + px_bytes(s) : 0;
+size_t tc_slice_prep_bytes(const Shape& s0) {
+  const Shape s = tc_padded(s0);
+  return tc_forward_supported(s0) ? align_up(w_image_bytes(s), 256) + px_bytes(s) : 0;
 }
-size_t tc_deslice_prep_bytes(const Shape& s) {
-  return tc_forward_supported(s) ? align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256) + px_bytes(s)
-                                 : 0;
+size_t tc_deslice_prep_bytes(const Shape& s0) {
+  const Shape s = tc_padded(s0);
+  return tc_forward_supported(s0) ? align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256) + px_bytes(s)
+                                  : 0;
 }
 
-cudaError_t tc_stats(const Shape& s, const void* x, const float* W, const float* bias, const float* tau, float* lse,
+cudaError_t tc_stats(const Shape& s0, const void* x, const float* W, const float* bias, const float* tau, float* lse,
                      void* prep, uint32_t* status, cudaStream_t st) {
+  const Shape s = tc_padded(s0);
   uint8_t* wimg = static_cast<uint8_t*>(prep);
   uint8_t* px = wimg + align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256);
-  cudaError_t e = prep_w(s, W, bias, tau, wimg, status, st);
+  cudaError_t e = prep_w(s, s0.G, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
   return run_stats(s, x, wimg, lse, px, status, st);
 }
 
-cudaError_t tc_slice_fwd(const Shape& s, const void* x, const void* f, const float* W, const float* bias,
+cudaError_t tc_slice_fwd(const Shape& s0, const void* x, const void* f, const float* W, const float* bias,
                          const float* tau, float* tokens, float* wsum, float* lse, int finalize, float* part,
                          void* prep, uint32_t* status, cudaStream_t st) {
+  const Shape s = tc_padded(s0);
   uint8_t* wimg = static_cast<uint8_t*>(prep);
   uint8_t* px = wimg + align_up(w_image_bytes(s), 256);
-  cudaError_t e = prep_w(s, W, bias, tau, wimg, status, st);
+  cudaError_t e = prep_w(s, s0.G, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
   if ((e = run_stats(s, x, wimg, lse, px, status, st)) != cudaSuccess) return e;
   CUtensorMap xmap, fmap, pmap;
@@ -844,19 +849,20 @@ cudaError_t tc_slice_fwd(const Shape& s, const void* x, const void* f, const flo
   if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
   kernel<<<grid, kThreads, sm, st>>>(xmap, fmap, pmap, wimg, part, s.N, padded_n(s), s.H, s.G, P, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  return simt_reduce_tokens(s, P, part, tokens, wsum, finalize, st);
+  return simt_reduce_tokens(s0, P, part, s.G, tokens, wsum, finalize, st);
 }
 
-cudaError_t tc_deslice_fwd(const Shape& s, const void* x, const float* W, const float* bias, const float* tau,
+cudaError_t tc_deslice_fwd(const Shape& s0, const void* x, const float* W, const float* bias, const float* tau,
                            const float* zp, const float* lse, void* out, void* prep, uint32_t* status,
                            cudaStream_t st) {
+  const Shape s = tc_padded(s0);
   uint8_t* wimg = static_cast<uint8_t*>(prep);
   uint8_t* zimg = wimg + align_up(w_image_bytes(s), 256);
   uint8_t* px = zimg + align_up(z_image_bytes(s), 256);
-  cudaError_t e = prep_w(s, W, bias, tau, wimg, status, st);
+  cudaError_t e = prep_w(s, s0.G, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
   const int64_t nz = s.BH() * s.G * kD;
-  k_prep_z<<<(unsigned)((nz + 255) / 256), 256, 0, st>>>(zp, zimg, s.BH(), s.G);
+  k_prep_z<<<(unsigned)((nz + 255) / 256), 256, 0, st>>>(zp, zimg, s.BH(), s0.G, s.G);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int64_t Np = padded_n(s), npx = s.BH() * Np;
   k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(px), s.BH(), s.N, Np);
