@@ -121,6 +121,17 @@ fs_status fs_slice_fwd(const fs_shape* s, const void* x_mid, const void* fx,
                        float* tokens, float* wsum, float* lse, int finalize,
                        void* ws, size_t ws_bytes, fs_stream_t stream);
 
+/* Slice given its statistics: fs_slice_fwd with lse [B,H,N] an input (as
+ * fs_slice_fwd writes it, natural log) and no statistics pass.  For the
+ * FrozenSlice variant (Sec. 3, the variants table: the slice weights of layer 1
+ * reused by every layer), where a later layer slices its own fx with the
+ * layer-1 logits input, weights and statistics; and for any caller that
+ * already holds lse for these weights.  ws: FS_OP_SLICE_FWD's workspace. */
+fs_status fs_slice_fwd_lse(const fs_shape* s, const void* x_mid, const void* fx,
+                           const float* W_slice, const float* bias, const float* tau,
+                           const float* lse, float* tokens, float* wsum, int finalize,
+                           void* ws, size_t ws_bytes, fs_stream_t stream);
+
 /* tokens <- tokens / (wsum + eps), in place ("column normalisation after
  * partials have been combined", App. G.1). */
 fs_status fs_slice_finalize(const fs_shape* s, float* tokens, const float* wsum,
@@ -133,7 +144,9 @@ fs_status fs_mix(const fs_shape* s, const float* M, const float* tokens,
 
 /* Deslice with tied weights (Sec. 2; App. G.1): out[b,n,h,:] = sum_g w z'_g.
  *   lse: statistics from fs_slice_fwd; NULL makes the call compute them first
- *   (into ws).  out has the dtype of the shape. */
+ *   (into ws).  out has the dtype of the shape.  The Untied variant (Sec. 3, the
+ *   variants table: the deslice gets its own projection and temperature) passes
+ *   its own W_slice, bias, tau and lse = NULL. */
 fs_status fs_deslice_fwd(const fs_shape* s, const void* x_mid, const float* W_slice,
                          const float* bias, const float* tau, const float* tokens_mixed,
                          const float* lse, void* out, void* ws, size_t ws_bytes,
@@ -144,7 +157,8 @@ fs_status fs_deslice_fwd(const fs_shape* s, const void* x_mid, const float* W_sl
  *   d_tokens_mixed [B,H,G,d] = sum_n w_ng dout_n  (always overwritten)
  *   dx_mid [B,N,H,d], dW [H,d,G], dbias [H,G], dtau [H]: the contribution of
  *   the deslice weights; written if accumulate == 0, added if accumulate != 0.
- *   lse must be the statistics of the forward pass (not NULL).  The backward
+ *   lse: the statistics of these weights from the forward, or NULL (an untied
+ *   deslice, which kept none): the call then computes them into ws.  The backward
  *   forms its weights from fp32 logits and needs lse to ~1e-5: on tensor-core
  *   shapes (fs_path_for_shape == 1) with dot = FS_DOT_BF16, whose lse comes
  *   from logits with bf16-rounded W log2(e)/tau, it recomputes lse with split
@@ -163,7 +177,8 @@ fs_status fs_mix_bwd(const fs_shape* s, const float* M, const float* tokens,
 
 /* Backward of the slice given d_tokens (the gradient w.r.t. the normalised
  * tokens); tokens and wsum are the forward's normalised tokens and S; lse as
- * in fs_deslice_bwd (recomputed with split products for FS_DOT_BF16).
+ * in fs_deslice_bwd (NULL: computed; recomputed with split products for
+ * FS_DOT_BF16).
  *   dfx [B,N,H,d] (overwritten); dx_mid, dW, dbias, dtau: written if
  *   accumulate == 0, added if accumulate != 0. */
 fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx,

@@ -90,7 +90,7 @@ Regions regions(const Shape& s, int op) {
       r.delta = take(pts * sizeof(float));
       r.partials = take((size_t)P * BHG * (2 * s.d + 2) * sizeof(float));
       r.dtau_p = take((size_t)s.BH() * simt_point_blocks(s) * sizeof(float));
-      r.stats = take(tc_forward_supported(s) ? pts * sizeof(float) : 0);
+      r.stats = take(pts * sizeof(float));
       r.tc = take(tc_deslice_prep_bytes(s));
       break;
     case FS_OP_SLICE_BWD:
@@ -103,7 +103,7 @@ Regions regions(const Shape& s, int op) {
       r.delta = take(pts * sizeof(float));
       r.partials = take((size_t)P * BHG * (s.d + 2) * sizeof(float));
       r.dtau_p = take((size_t)s.BH() * simt_point_blocks(s) * sizeof(float));
-      r.stats = take(tc_forward_supported(s) ? pts * sizeof(float) : 0);
+      r.stats = take(pts * sizeof(float));
       r.tc = take(tc_deslice_prep_bytes(s));
       break;
     default:
@@ -133,16 +133,20 @@ cudaError_t reset_status(void* ws, cudaStream_t st) { return cudaMemsetAsync(ws,
 // tensor-core shapes with bf16 products the forward's lse comes from logits with
 // bf16-rounded W log2(e)/tau: the backward recomputes it with split products (the
 // statistics pass, into ws).  With split products (and on the SIMT path) the
-// caller's lse is already that accurate and is used as it is.
+// caller's lse is already that accurate and is used as it is.  A caller without
+// statistics for these weights (an untied deslice, Sec. 3) passes NULL and the
+// backward computes them.
 cudaError_t backward_stats(const Shape& sh, const void* x_mid, const float* W_slice, const float* bias,
                            const float* tau, const float* lse, void* ws, const Regions& r, uint32_t* status,
                            cudaStream_t st, const float** lse_use) {
   *lse_use = lse;
-  if (!tc_forward_supported(sh) || sh.dot == FS_DOT_BF16X2) return cudaSuccess;
-  Shape split = sh;
-  split.dot = FS_DOT_BF16X2;
+  const bool tc = tc_forward_supported(sh);
+  if (lse && (!tc || sh.dot == FS_DOT_BF16X2)) return cudaSuccess;
   float* buf = at<float>(ws, r.stats);
   *lse_use = buf;
+  if (!tc) return simt_stats(sh, x_mid, W_slice, bias, tau, buf, status, st);
+  Shape split = sh;
+  split.dot = FS_DOT_BF16X2;
   return tc_stats(split, x_mid, W_slice, bias, tau, buf, at<void>(ws, r.tc), status, st);
 }
 
@@ -232,6 +236,28 @@ fs_status fs_slice_fwd(const fs_shape* s, const void* x_mid, const void* fx, con
   return FS_OK;
 }
 
+fs_status fs_slice_fwd_lse(const fs_shape* s, const void* x_mid, const void* fx, const float* W_slice,
+                           const float* bias, const float* tau, const float* lse, float* tokens, float* wsum,
+                           int finalize, void* ws, size_t ws_bytes, fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(x_mid); FS_CHECK_PTR(fx); FS_CHECK_PTR(W_slice); FS_CHECK_PTR(bias); FS_CHECK_PTR(tau);
+  FS_CHECK_PTR(lse); FS_CHECK_PTR(tokens); FS_CHECK_PTR(wsum);
+  const Shape sh = to_shape(s);
+  if (fs_status e = check_ws(sh, FS_OP_SLICE_FWD, ws, ws_bytes)) return e;
+  const Regions r = regions(sh, FS_OP_SLICE_FWD);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  uint32_t* status = at<uint32_t>(ws, r.status);
+  FS_CUDA(reset_status(ws, st));
+  if (tc_forward_supported(sh))
+    return cuda_status(tc_slice_fwd_lse(sh, x_mid, fx, W_slice, bias, tau, lse, tokens, wsum, finalize,
+                                        at<float>(ws, r.partials), at<void>(ws, r.tc), status, st));
+  const int P = slot_splits(sh);
+  float* part = at<float>(ws, r.partials);
+  FS_CUDA(simt_slice_partials(sh, P, x_mid, fx, W_slice, bias, tau, lse, part, status, st));
+  FS_CUDA(simt_reduce_tokens(sh, P, part, sh.G, tokens, wsum, finalize, st));
+  return FS_OK;
+}
+
 fs_status fs_slice_finalize(const fs_shape* s, float* tokens, const float* wsum, fs_stream_t stream) {
   FS_CHECK_SHAPE(s);
   FS_CHECK_PTR(tokens); FS_CHECK_PTR(wsum);
@@ -278,7 +304,8 @@ fs_status fs_deslice_bwd(const fs_shape* s, const void* x_mid, const float* W_sl
                          void* ws, size_t ws_bytes, fs_stream_t stream) {
   FS_CHECK_SHAPE(s);
   FS_CHECK_PTR(x_mid); FS_CHECK_PTR(W_slice); FS_CHECK_PTR(bias); FS_CHECK_PTR(tau);
-  FS_CHECK_PTR(tokens_mixed); FS_CHECK_PTR(lse); FS_CHECK_PTR(dout); FS_CHECK_PTR(d_tokens_mixed);
+  FS_CHECK_PTR(tokens_mixed); FS_CHECK_PTR(dout); FS_CHECK_PTR(d_tokens_mixed);
+  if (lse && !aligned(lse)) return FS_ERR_INVALID;
   FS_CHECK_PTR(dx_mid); FS_CHECK_PTR(dW); FS_CHECK_PTR(dbias); FS_CHECK_PTR(dtau);
   const Shape sh = to_shape(s);
   if (fs_status e = check_ws(sh, FS_OP_DESLICE_BWD, ws, ws_bytes)) return e;
@@ -312,7 +339,8 @@ fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx, con
                        float* dtau, int accumulate, void* ws, size_t ws_bytes, fs_stream_t stream) {
   FS_CHECK_SHAPE(s);
   FS_CHECK_PTR(x_mid); FS_CHECK_PTR(fx); FS_CHECK_PTR(W_slice); FS_CHECK_PTR(bias); FS_CHECK_PTR(tau);
-  FS_CHECK_PTR(tokens); FS_CHECK_PTR(wsum); FS_CHECK_PTR(lse); FS_CHECK_PTR(d_tokens);
+  FS_CHECK_PTR(tokens); FS_CHECK_PTR(wsum); FS_CHECK_PTR(d_tokens);
+  if (lse && !aligned(lse)) return FS_ERR_INVALID;
   FS_CHECK_PTR(dx_mid); FS_CHECK_PTR(dfx); FS_CHECK_PTR(dW); FS_CHECK_PTR(dbias); FS_CHECK_PTR(dtau);
   const Shape sh = to_shape(s);
   if (fs_status e = check_ws(sh, FS_OP_SLICE_BWD, ws, ws_bytes)) return e;

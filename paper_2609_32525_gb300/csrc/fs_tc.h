@@ -20,6 +20,10 @@ cudaError_t tc_stats(const Shape& s, const void* x, const float* W, const float*
 cudaError_t tc_slice_fwd(const Shape& s, const void* x, const void* f, const float* W, const float* bias,
                          const float* tau, float* tokens, float* wsum, float* lse, int finalize, float* part,
                          void* prep, uint32_t* status, cudaStream_t st);
+// The slice given the statistics lse (the statistics pass is skipped).
+cudaError_t tc_slice_fwd_lse(const Shape& s, const void* x, const void* f, const float* W, const float* bias,
+                             const float* tau, const float* lse, float* tokens, float* wsum, int finalize,
+                             float* part, void* prep, uint32_t* status, cudaStream_t st);
 cudaError_t tc_deslice_fwd(const Shape& s, const void* x, const float* W, const float* bias, const float* tau,
                            const float* zp, const float* lse, void* out, void* prep, uint32_t* status,
                            cudaStream_t st);

@@ -793,6 +793,10 @@ cudaError_t run_stats(const Shape& s, const void* x, const uint8_t* wimg, float*
 
 }  // namespace
 
+// The slice on prepared operands (defined below, after the C-ABI-facing helpers).
+cudaError_t run_slice(const Shape& s, int G, const void* x, const void* f, const uint8_t* wimg, void* px,
+                      float* tokens, float* wsum, int finalize, float* part, uint32_t* status, cudaStream_t st);
+
 bool tc_forward_supported(const Shape& s) {
   // TMA coordinates and the kernels' block counters are 32-bit.
   const int64_t np = (s.N + kTile - 1) / kTile * kTile;
@@ -838,6 +842,13 @@ cudaError_t tc_slice_fwd(const Shape& s0, const void* x, const void* f, const fl
   cudaError_t e = prep_w(s, s0.G, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
   if ((e = run_stats(s, x, wimg, lse, px, status, st)) != cudaSuccess) return e;
+  return run_slice(s, s0.G, x, f, wimg, px, tokens, wsum, finalize, part, status, st);
+}
+
+// The slice on prepared operands: the W image and the point-extra rows at px.
+cudaError_t run_slice(const Shape& s, int G, const void* x, const void* f, const uint8_t* wimg, void* px,
+                      float* tokens, float* wsum, int finalize, float* part, uint32_t* status, cudaStream_t st) {
+  cudaError_t e;
   CUtensorMap xmap, fmap, pmap;
   if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
   if (!make_point_map(&fmap, f, s, 16, CU_TENSOR_MAP_SWIZZLE_32B)) return cudaErrorInvalidValue;
@@ -849,7 +860,23 @@ cudaError_t tc_slice_fwd(const Shape& s0, const void* x, const void* f, const fl
   if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
   kernel<<<grid, kThreads, sm, st>>>(xmap, fmap, pmap, wimg, part, s.N, padded_n(s), s.H, s.G, P, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  return simt_reduce_tokens(s0, P, part, s.G, tokens, wsum, finalize, st);
+  Shape so = s;
+  so.G = G;
+  return simt_reduce_tokens(so, P, part, s.G, tokens, wsum, finalize, st);
+}
+
+cudaError_t tc_slice_fwd_lse(const Shape& s0, const void* x, const void* f, const float* W, const float* bias,
+                             const float* tau, const float* lse, float* tokens, float* wsum, int finalize,
+                             float* part, void* prep, uint32_t* status, cudaStream_t st) {
+  const Shape s = tc_padded(s0);
+  uint8_t* wimg = static_cast<uint8_t*>(prep);
+  uint8_t* px = wimg + align_up(w_image_bytes(s), 256);
+  cudaError_t e = prep_w(s, s0.G, W, bias, tau, wimg, status, st);
+  if (e != cudaSuccess) return e;
+  const int64_t Np = padded_n(s), npx = s.BH() * Np;
+  k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(px), s.BH(), s.N, Np);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  return run_slice(s, s0.G, x, f, wimg, px, tokens, wsum, finalize, part, status, st);
 }
 
 cudaError_t tc_deslice_fwd(const Shape& s0, const void* x, const float* W, const float* bias, const float* tau,

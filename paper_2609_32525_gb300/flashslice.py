@@ -33,7 +33,8 @@ FS_OP_SLICE_FWD, FS_OP_DESLICE_FWD, FS_OP_DESLICE_BWD, FS_OP_SLICE_BWD = range(4
 
 EXPORTED = ("fs_workspace_bytes", "fs_slice_fwd", "fs_slice_finalize", "fs_mix", "fs_deslice_fwd",
             "fs_deslice_bwd", "fs_mix_bwd", "fs_slice_bwd", "fs_device_status", "fs_status_string",
-            "fs_path_for_shape", "fs_backward_path_for_shape", "fs_forward_launch_count", "fs_slice_fwd_noalloc")
+            "fs_path_for_shape", "fs_backward_path_for_shape", "fs_forward_launch_count", "fs_slice_fwd_noalloc",
+            "fs_slice_fwd_lse")
 
 
 class fs_shape(ctypes.Structure):
@@ -54,6 +55,7 @@ _Z = ctypes.c_size_t
 _sig = {
     "fs_workspace_bytes": (_Z, [_S, _I]),
     "fs_slice_fwd": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _Z, _P]),
+    "fs_slice_fwd_lse": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _Z, _P]),
     "fs_slice_finalize": (_I, [_S, _P, _P, _P]),
     "fs_mix": (_I, [_S, _P, _P, _P, _P]),
     "fs_deslice_fwd": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _Z, _P]),
@@ -135,6 +137,13 @@ def fs_slice_fwd(shape, x_mid, fx, W_slice, bias, tau, tokens, wsum, lse, finali
                            _ptr(tokens), _ptr(wsum), _ptr(lse), int(bool(finalize)), _ptr(ws), ws.numel(),
                            _stream(stream))
     _check("fs_slice_fwd", st)
+
+
+def fs_slice_fwd_lse(shape, x_mid, fx, W_slice, bias, tau, lse, tokens, wsum, finalize, ws, stream=None):
+    st = _lib.fs_slice_fwd_lse(ctypes.byref(shape), _ptr(x_mid), _ptr(fx), _ptr(W_slice), _ptr(bias), _ptr(tau),
+                               _ptr(lse), _ptr(tokens), _ptr(wsum), int(bool(finalize)), _ptr(ws), ws.numel(),
+                               _stream(stream))
+    _check("fs_slice_fwd_lse", st)
 
 
 def fs_slice_finalize(shape, tokens, wsum, stream=None):
