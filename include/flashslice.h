@@ -230,9 +230,9 @@ const char* fs_status_string(fs_status st);
 int fs_path_for_shape(const fs_shape* s);
 
 /* Kernel path of the backward (fs_deslice_bwd, fs_slice_bwd) for this shape:
- * 0 = SIMT fp32 kernels, 1 = tcgen05 tensor-core kernels (bf16, d = 32, G a
- * multiple of 128 up to 640, N >= 2; the weights with split products whatever
- * s->dot says).  For tests and benchmarks. */
+ * 0 = SIMT fp32 kernels, 1 = tcgen05 tensor-core kernels (bf16, d = 32,
+ * G <= 640, N >= 2; the weights with split products whatever s->dot says).
+ * For tests and benchmarks. */
 int fs_backward_path_for_shape(const fs_shape* s);
 
 /* Number of kernels the forward (slice + mix + deslice) launches for this shape. */

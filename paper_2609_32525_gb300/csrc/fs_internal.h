@@ -59,10 +59,11 @@ cudaError_t simt_deslice_bwd(const Shape& s, int P, const void* x, const float* 
 // dUS[bh][g] = (dz_g / (S_g + eps), -(dz_g . z_g) / (S_g + eps)) (d + 1 floats per slot).
 cudaError_t simt_slice_bwd_prep(const Shape& s, const float* z, const float* wsum, const float* dz, float* dUS,
                                 cudaStream_t st);
-// Fixed-order reduction of slot-owned backward partials part[P][B*H][G][PS]
-// (PS = 2d + 2 with the token gradient first when has_dzp, else d + 2) into
-// dW, dbias (and dzp), and of dt_part[B*H][nblk] into dtau.
-cudaError_t simt_reduce_bwd(const Shape& s, int P, const float* part, int PS, int has_dzp, const float* tau,
+// Fixed-order reduction of slot-owned backward partials part[P][B*H][Gs][PS]
+// (Gs >= G slot rows per (b, h), the first G reduced; PS = 2d + 2 with the token
+// gradient first when has_dzp, else d + 2) into dW, dbias (and dzp), and of
+// dt_part[B*H][nblk] into dtau.
+cudaError_t simt_reduce_bwd(const Shape& s, int P, const float* part, int Gs, int PS, int has_dzp, const float* tau,
                             float* dzp, float* dW, float* db, float* dtau, const float* dt_part, int64_t nblk,
                             int accumulate, cudaStream_t st);
 cudaError_t simt_slice_bwd(const Shape& s, int P, const void* x, const void* f, const float* W,

@@ -611,7 +611,7 @@ __global__ void k_slice_bwd_prep(const float* __restrict__ z, const float* __res
 //   k_reduce_bwd_params: dW[h][k][g], db[h][g] (written, or added), sums over b then p;
 //   k_reduce_bwd_tokens: d_tokens_mixed[b][h][g][c], sums over p.
 // The temperature gradient is reduced separately, from its own partials.
-__global__ void k_reduce_bwd_params(const float* __restrict__ part, int P, int64_t B, int H, int G, int D,
+__global__ void k_reduce_bwd_params(const float* __restrict__ part, int P, int64_t B, int H, int G, int Gs, int D,
                                     int PS, int off, const float* __restrict__ tau, float* __restrict__ dW,
                                     float* __restrict__ db, int accumulate) {
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -622,7 +622,7 @@ __global__ void k_reduce_bwd_params(const float* __restrict__ part, int P, int64
   const int64_t BH = B * H;
   float s = 0.f;
   for (int64_t b = 0; b < B; b++)
-    for (int p = 0; p < P; p++) s += part[(((int64_t)p * BH + b * H + h) * G + g) * PS + off + k];
+    for (int p = 0; p < P; p++) s += part[(((int64_t)p * BH + b * H + h) * Gs + g) * PS + off + k];
   s *= 1.f / tau[h];
   if (k < D) {
     const int64_t o = ((int64_t)h * D + k) * G + g;
@@ -631,14 +631,15 @@ __global__ void k_reduce_bwd_params(const float* __restrict__ part, int P, int64
     db[hg] = (accumulate ? db[hg] : 0.f) + s;
   }
 }
-__global__ void k_reduce_bwd_tokens(const float* __restrict__ part, int P, int64_t BHG, int D, int PS,
+__global__ void k_reduce_bwd_tokens(const float* __restrict__ part, int P, int64_t BH, int G, int Gs, int D, int PS,
                                     float* __restrict__ dzp) {
   const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= BHG * D) return;
+  if (idx >= BH * G * D) return;
   const int c = (int)(idx % D);
-  const int64_t row = idx / D;
+  const int64_t i = idx / D;                  // output row bh * G + g
+  const int64_t row = (i / G) * Gs + i % G;  // its partial row
   float s = 0.f;
-  for (int p = 0; p < P; p++) s += part[((int64_t)p * BHG + row) * PS + c];
+  for (int p = 0; p < P; p++) s += part[((int64_t)p * BH * Gs + row) * PS + c];
   dzp[idx] = s;
 }
 
@@ -739,17 +740,18 @@ cudaError_t launch_bwd_slice(const Shape& s, int P, const void* x, const void* v
 
 }  // namespace
 
-cudaError_t simt_reduce_bwd(const Shape& s, int P, const float* part, int PS, int has_dzp, const float* tau,
+cudaError_t simt_reduce_bwd(const Shape& s, int P, const float* part, int Gs, int PS, int has_dzp, const float* tau,
                             float* dzp, float* dW, float* db, float* dtau, const float* dt_part, int64_t nblk,
                             int accumulate, cudaStream_t st) {
   const int64_t nw = (int64_t)s.H * s.G * (s.d + 1);
-  k_reduce_bwd_params<<<(unsigned)((nw + 255) / 256), 256, 0, st>>>(part, P, s.B, s.H, s.G, s.d, PS,
+  k_reduce_bwd_params<<<(unsigned)((nw + 255) / 256), 256, 0, st>>>(part, P, s.B, s.H, s.G, Gs, s.d, PS,
                                                                      has_dzp ? s.d : 0, tau, dW, db, accumulate);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   if (has_dzp) {
     const int64_t BHG = s.BH() * s.G;
-    k_reduce_bwd_tokens<<<(unsigned)((BHG * s.d + 255) / 256), 256, 0, st>>>(part, P, BHG, s.d, PS, dzp);
+    k_reduce_bwd_tokens<<<(unsigned)((BHG * s.d + 255) / 256), 256, 0, st>>>(part, P, s.BH(), s.G, Gs, s.d, PS,
+                                                                              dzp);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   k_reduce_dtau<<<s.H, 256, 0, st>>>(dt_part, s.B, s.H, nblk, tau, dtau, accumulate);
@@ -821,7 +823,7 @@ cudaError_t simt_deslice_bwd(const Shape& s, int P, const void* x, const float* 
                 accumulate, status, st);
   }();
   if (e != cudaSuccess) return e;
-  return simt_reduce_bwd(s, P, part, 2 * s.d + 2, 1, tau, dzp, dW, db, dtau, dt_part, simt_point_blocks(s),
+  return simt_reduce_bwd(s, P, part, s.G, 2 * s.d + 2, 1, tau, dzp, dW, db, dtau, dt_part, simt_point_blocks(s),
                          accumulate, st);
 }
 
@@ -837,7 +839,7 @@ cudaError_t simt_slice_bwd(const Shape& s, int P, const void* x, const void* f, 
                 accumulate, status, st);
   }();
   if (e != cudaSuccess) return e;
-  return simt_reduce_bwd(s, P, part, s.d + 2, 0, tau, nullptr, dW, db, dtau, dt_part, simt_point_blocks(s),
+  return simt_reduce_bwd(s, P, part, s.G, s.d + 2, 0, tau, nullptr, dW, db, dtau, dt_part, simt_point_blocks(s),
                          accumulate, st);
 }
 

@@ -39,7 +39,8 @@ size_t tc_rows_smem(const Shape& s, int mode, bool ps, bool hilo);
 
 // ---- tensor-core backward (fs_tc_bwd.cu) ----
 // True when the tensor-core backward implements this shape (the forward's
-// shapes with N >= 2 whose operand images fit in shared memory: G <= 640).
+// shapes with N >= 2 whose operand images fit in shared memory: G <= 640, padded
+// like the forward's to whole 128-slot blocks).
 bool tc_backward_supported(const Shape& s);
 // Workspace of one tensor-core backward call (mode 1 deslice, 2 slice).
 size_t tc_backward_bytes(const Shape& s, int mode);

@@ -32,66 +32,70 @@ constexpr uint32_t kWBlockB = kGC * kWRow;             // one 128-slot block of 
 
 // T image of (b,h), in the W image's layout (kWRow bytes per slot): t_g rounded to
 // bf16, the extra rows [c_hi, c_lo, 1, 1, 0...], the residual t_g - bf16(t_g).
-// t: [BH][G][tstride] fp32, c_g = t[..][32] when has_c.  Also writes c_g to c_out [BH][G].
+// t: [BH][G][tstride] fp32, c_g = t[..][32] when has_c.  Also writes c_g to c_out
+// [BH][Gp].  Padding slots [G, Gp) get t = 0 and c = 0 (their weights are 0).
 __global__ void k_prep_t(const float* __restrict__ t, int tstride, int has_c, uint8_t* __restrict__ img,
-                         float* __restrict__ c_out, int64_t BH, int G) {
+                         float* __restrict__ c_out, int64_t BH, int G, int Gp) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= BH * G) return;
-  const int64_t bh = i / G;
-  const int g = (int)(i % G);
-  const float* src = t + i * tstride;
-  uint8_t* base = img + (size_t)bh * G * kWRow;
+  if (i >= BH * Gp) return;
+  const int64_t bh = i / Gp;
+  const int g = (int)(i % Gp);
+  const bool real = g < G;
+  const float* src = t + (bh * G + (real ? g : 0)) * tstride;
+  uint8_t* base = img + (size_t)bh * Gp * kWRow;
   __nv_bfloat16* hp = reinterpret_cast<__nv_bfloat16*>(base);
-  __nv_bfloat16* lp = reinterpret_cast<__nv_bfloat16*>(base + (size_t)G * 96);
+  __nv_bfloat16* lp = reinterpret_cast<__nv_bfloat16*>(base + (size_t)Gp * 96);
   for (int k = 0; k < kD; k++) {
-    const float v = src[k];
+    const float v = real ? src[k] : 0.f;
     const __nv_bfloat16 hi = __float2bfloat16_rn(v);
     hp[off_sw64(g, k) / 2] = hi;
     lp[off_sw64(g, k) / 2] = __float2bfloat16_rn(v - __bfloat162float(hi));
   }
-  const float c = has_c ? src[kD] : 0.f;
+  const float c = (has_c && real) ? src[kD] : 0.f;
   if (c_out) c_out[i] = c;
   const __nv_bfloat16 chi = __float2bfloat16_rn(c);
   const __nv_bfloat16 clo = __float2bfloat16_rn(c - __bfloat162float(chi));
-  __nv_bfloat16* ep = reinterpret_cast<__nv_bfloat16*>(base + (size_t)G * 64);
+  __nv_bfloat16* ep = reinterpret_cast<__nv_bfloat16*>(base + (size_t)Gp * 64);
   for (int k = 0; k < 16; k++)
     ep[off_sw32(g, k) / 2] = k == 0 ? chi : (k == 1 ? clo : __float2bfloat16_rn((k == 2 || k == 3) ? 1.f : 0.f));
 }
 
 // Z-layout image (blocks of 64 slots, 32 channel rows x 128 B, 128B swizzle) of
-// t [BH][G][tstride] per (b,h): the bf16 half, then the residual half (G*128 bytes per (b,h)).
-__global__ void k_prep_z2(const float* __restrict__ t, int tstride, uint8_t* __restrict__ img, int64_t BH, int G) {
+// t [BH][G][tstride] per (b,h): the bf16 half, then the residual half (Gp*128 bytes
+// per (b,h)); padding slots [G, Gp) are zero.
+__global__ void k_prep_z2(const float* __restrict__ t, int tstride, uint8_t* __restrict__ img, int64_t BH, int G,
+                          int Gp) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= BH * G * kD) return;
+  if (i >= BH * Gp * kD) return;
   const int c = (int)(i % kD);
-  const int g = (int)((i / kD) % G);
-  const int64_t bh = i / ((int64_t)kD * G);
-  const float v = t[(bh * G + g) * tstride + c];
-  __nv_bfloat16* hp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * G * 128);
-  __nv_bfloat16* lp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * G * 128 + (size_t)G * 64);
+  const int g = (int)((i / kD) % Gp);
+  const int64_t bh = i / ((int64_t)kD * Gp);
+  const float v = g < G ? t[(bh * G + g) * tstride + c] : 0.f;
+  __nv_bfloat16* hp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * Gp * 128);
+  __nv_bfloat16* lp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * Gp * 128 + (size_t)Gp * 64);
   const __nv_bfloat16 hi = __float2bfloat16_rn(v);
   hp[off_z(c, g) / 2] = hi;
   lp[off_z(c, g) / 2] = __float2bfloat16_rn(v - __bfloat162float(hi));
 }
 
 // W'^T image of head h in the Z layout (channel rows, slots along K), W' =
-// W log2(e)/tau: the bf16 half, then the residual half (G*128 bytes per head).
-// It is the B operand of dx += da W'^T.
+// W log2(e)/tau: the bf16 half, then the residual half (Gp*128 bytes per head;
+// padding slots zero).  It is the B operand of dx += da W'^T.
 __global__ void k_prep_wt(const float* __restrict__ W, const float* __restrict__ tau, uint8_t* __restrict__ img,
-                          int H, int G, uint32_t* status) {
+                          int H, int G, int Gp, uint32_t* status) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= (int64_t)H * kD * G) return;
-  const int g = (int)(i % G);
-  const int c = (int)((i / G) % kD);
-  const int h = (int)(i / ((int64_t)kD * G));
+  if (i >= (int64_t)H * kD * Gp) return;
+  const int g = (int)(i % Gp);
+  const int c = (int)((i / Gp) % kD);
+  const int h = (int)(i / ((int64_t)kD * Gp));
   const float tv = tau[h];
   if (!(tv > 0.f && tv < INFINITY)) {
     atomicCAS(status, 0u, (uint32_t)FS_ERR_BAD_TAU);
     return;
   }
-  const float v = W[i] * (kLog2e / tv);
-  __nv_bfloat16* hp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)h * G * 128);
-  __nv_bfloat16* lp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)h * G * 128 + (size_t)G * 64);
+  const float v = g < G ? W[((int64_t)h * kD + c) * G + g] * (kLog2e / tv) : 0.f;
+  __nv_bfloat16* hp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)h * Gp * 128);
+  __nv_bfloat16* lp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)h * Gp * 128 + (size_t)Gp * 64);
   const __nv_bfloat16 hi = __float2bfloat16_rn(v);
   hp[off_z(c, g) / 2] = hi;
   lp[off_z(c, g) / 2] = __float2bfloat16_rn(v - __bfloat162float(hi));
@@ -710,14 +714,15 @@ bool make_maps(const Shape& s, const void* x, const void* v, const void* px, con
 
 // The common part of both backward calls, after the T and Z images are written:
 // the W images and lse rows, the rows pass, delta's rows, the slot and the point passes.
-cudaError_t run_backward(const Shape& s, int mode, const void* x, const void* v, const float* W, const float* bias,
-                         const float* tau, const float* lse, void* dfx, void* dx, int accumulate, uint8_t* ws,
-                         const BwdLayout& L, uint32_t* status, cudaStream_t st) {
+// s: the padded shape (s.G a whole number of 128-slot blocks); G: the caller's.
+cudaError_t run_backward(const Shape& s, int G, int mode, const void* x, const void* v, const float* W,
+                         const float* bias, const float* tau, const float* lse, void* dfx, void* dx, int accumulate,
+                         uint8_t* ws, const BwdLayout& L, uint32_t* status, cudaStream_t st) {
   const int64_t Np = padded_n(s);
-  cudaError_t e = prep_w(s, s.G, W, bias, tau, ws + L.wimg, status, st);
+  cudaError_t e = prep_w(s, G, W, bias, tau, ws + L.wimg, status, st);
   if (e != cudaSuccess) return e;
   const int64_t nwt = (int64_t)s.H * kD * s.G;
-  k_prep_wt<<<(unsigned)((nwt + 255) / 256), 256, 0, st>>>(W, tau, ws + L.wtimg, s.H, s.G, status);
+  k_prep_wt<<<(unsigned)((nwt + 255) / 256), 256, 0, st>>>(W, tau, ws + L.wtimg, s.H, G, s.G, status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int64_t npx = s.BH() * Np;
   k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(ws + L.px), s.BH(), s.N,
@@ -761,14 +766,14 @@ cudaError_t run_backward(const Shape& s, int mode, const void* x, const void* v,
   return cudaSuccess;
 }
 
-cudaError_t prep_t_images(const Shape& s, const float* t, int tstride, int has_c, uint8_t* ws, const BwdLayout& L,
-                          cudaStream_t st) {
+cudaError_t prep_t_images(const Shape& s, int G, const float* t, int tstride, int has_c, uint8_t* ws,
+                          const BwdLayout& L, cudaStream_t st) {
   const int64_t BHG = s.BH() * s.G;
   k_prep_t<<<(unsigned)((BHG + 127) / 128), 128, 0, st>>>(t, tstride, has_c, ws + L.timg,
-                                                            reinterpret_cast<float*>(ws + L.ds), s.BH(), s.G);
+                                                            reinterpret_cast<float*>(ws + L.ds), s.BH(), G, s.G);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_prep_z2<<<(unsigned)((BHG * kD + 255) / 256), 256, 0, st>>>(t, tstride, ws + L.zimg, s.BH(), s.G);
+  k_prep_z2<<<(unsigned)((BHG * kD + 255) / 256), 256, 0, st>>>(t, tstride, ws + L.zimg, s.BH(), G, s.G);
   return cudaGetLastError();
 }
 
@@ -778,13 +783,14 @@ cudaError_t prep_t_images(const Shape& s, const float* t, int tstride, int has_c
 // point's fx times S/(S + eps), so the slice's gradients are O(eps) and come from
 // cancelling terms of size |dz||fx|/(S + eps) that split bf16 products resolve only
 // to ~2^-17 of that size.
-bool tc_backward_supported(const Shape& s) {
-  return tc_forward_supported(s) && s.G % kGC == 0 && s.N >= 2 && smem_bwd_dx(s.G, false) <= kMaxSmem &&
-         tc_rows_smem(s, 2, false, false) <= kMaxSmem;
+bool tc_backward_supported(const Shape& s0) {
+  if (!tc_forward_supported(s0) || s0.N < 2) return false;
+  const Shape s = tc_padded(s0);
+  return smem_bwd_dx(s.G, false) <= kMaxSmem && tc_rows_smem(s, 2, false, false) <= kMaxSmem;
 }
 
 size_t tc_backward_bytes(const Shape& s, int mode) {
-  return tc_backward_supported(s) ? bwd_layout(s, mode).total : 0;
+  return tc_backward_supported(s) ? bwd_layout(tc_padded(s), mode).total : 0;
 }
 
 int tc_backward_slot_splits(const Shape& s) { return bwd_slot_splits(s); }
@@ -802,36 +808,36 @@ Shape split_shape(const Shape& s) {
 cudaError_t tc_deslice_bwd(const Shape& s0, const void* x, const float* W, const float* bias, const float* tau,
                            const float* zp, const float* lse, const void* dout, float* dzp, void* dx, float* dW,
                            float* db, float* dtau, int accumulate, void* ws_tc, uint32_t* status, cudaStream_t st) {
-  const Shape s = split_shape(s0);
+  const Shape s = tc_padded(split_shape(s0));
   const BwdLayout L = bwd_layout(s, 1);
   uint8_t* ws = static_cast<uint8_t*>(ws_tc);
-  cudaError_t e = prep_t_images(s, zp, kD, 0, ws, L, st);
+  cudaError_t e = prep_t_images(s, s0.G, zp, kD, 0, ws, L, st);
   if (e != cudaSuccess) return e;
-  if ((e = run_backward(s, 1, x, dout, W, bias, tau, lse, nullptr, dx, accumulate, ws, L, status, st)) !=
+  if ((e = run_backward(s, s0.G, 1, x, dout, W, bias, tau, lse, nullptr, dx, accumulate, ws, L, status, st)) !=
       cudaSuccess)
     return e;
   const int P = bwd_slot_splits(s);
-  return simt_reduce_bwd(s, P, reinterpret_cast<const float*>(ws + L.part), 2 * kD + 2, 1, tau, dzp, dW, db, dtau,
-                         reinterpret_cast<const float*>(ws + L.dtp), (int64_t)P * bwd_slot_blocks(s), accumulate,
-                         st);
+  return simt_reduce_bwd(s0, P, reinterpret_cast<const float*>(ws + L.part), s.G, 2 * kD + 2, 1, tau, dzp, dW, db,
+                         dtau, reinterpret_cast<const float*>(ws + L.dtp), (int64_t)P * bwd_slot_blocks(s),
+                         accumulate, st);
 }
 
 cudaError_t tc_slice_bwd(const Shape& s0, const void* x, const void* f, const float* W, const float* bias,
                          const float* tau, const float* z, const float* wsum, const float* lse, const float* dz,
                          void* dx, void* dfx, float* dW, float* db, float* dtau, int accumulate, float* dUS,
                          void* ws_tc, uint32_t* status, cudaStream_t st) {
-  const Shape s = split_shape(s0);
+  const Shape s = tc_padded(split_shape(s0));
   const BwdLayout L = bwd_layout(s, 2);
   uint8_t* ws = static_cast<uint8_t*>(ws_tc);
-  cudaError_t e = simt_slice_bwd_prep(s, z, wsum, dz, dUS, st);
+  cudaError_t e = simt_slice_bwd_prep(s0, z, wsum, dz, dUS, st);
   if (e != cudaSuccess) return e;
-  if ((e = prep_t_images(s, dUS, kD + 1, 1, ws, L, st)) != cudaSuccess) return e;
-  if ((e = run_backward(s, 2, x, f, W, bias, tau, lse, dfx, dx, accumulate, ws, L, status, st)) != cudaSuccess)
+  if ((e = prep_t_images(s, s0.G, dUS, kD + 1, 1, ws, L, st)) != cudaSuccess) return e;
+  if ((e = run_backward(s, s0.G, 2, x, f, W, bias, tau, lse, dfx, dx, accumulate, ws, L, status, st)) != cudaSuccess)
     return e;
   const int P = bwd_slot_splits(s);
-  return simt_reduce_bwd(s, P, reinterpret_cast<const float*>(ws + L.part), kD + 2, 0, tau, nullptr, dW, db, dtau,
-                         reinterpret_cast<const float*>(ws + L.dtp), (int64_t)P * bwd_slot_blocks(s), accumulate,
-                         st);
+  return simt_reduce_bwd(s0, P, reinterpret_cast<const float*>(ws + L.part), s.G, kD + 2, 0, tau, nullptr, dW, db,
+                         dtau, reinterpret_cast<const float*>(ws + L.dtp), (int64_t)P * bwd_slot_blocks(s),
+                         accumulate, st);
 }
 
 }  // namespace fs

@@ -1,5 +1,6 @@
-"""GPU parity of the tcgen05 tensor-core backward (bf16, d = 32, G a multiple of
-128 up to 640) against the fp64 oracle, at both product arithmetics.
+"""GPU parity of the tcgen05 tensor-core backward (bf16, d = 32, G up to 640,
+padded inside the kernels to whole 128-slot blocks) against the fp64 oracle, at
+both product arithmetics.
 
 Each backward call runs in isolation, fed with the ORACLE's forward values
 (mixed tokens, tokens, weight sums and lse), so that only the backward kernels
@@ -32,6 +33,8 @@ SHAPES = [
     (1, 5000, 2, 512),
     (1, 3001, 1, 640),
     (2, 2049, 2, 256),
+    (1, 1000, 2, 100),  # G padded to 128 inside the kernels
+    (2, 777, 1, 48),
 ]
 TOL = 1e-2
 
