@@ -122,3 +122,33 @@ def backward(x_mid, fx, W, bias, tau, M, eps, dout, B, N, H, d, G):
                     db[h][g] += da / tau[h]
                     dt[h] += -da * a[g] / tau[h]
     return {"dx_mid": dx, "dfx": dfx, "dW": dW, "dbias": db, "dtau": dt, "dM": dM}
+
+
+def mix_channels(Wc, tokens, B, H, G, d):
+    """z'[b][h][g][c] = sum_k Wc[h][c][k] z[b][h][g][k], by loops (the NoTokenAttn
+    core: a per-token channel map, Sec. 2 after Eq. (1))."""
+    out = [[[[0.0] * d for _ in range(G)] for _ in range(H)] for _ in range(B)]
+    for b in range(B):
+        for h in range(H):
+            for g in range(G):
+                for c in range(d):
+                    acc = 0.0
+                    for k in range(d):
+                        acc += Wc[h][c][k] * tokens[b][h][g][k]
+                    out[b][h][g][c] = acc
+    return out
+
+
+def mix_channels_bwd(Wc, tokens, d_tokens_mixed, B, H, G, d):
+    """Chain rule of mix_channels element by element: (d_tokens, dWc)."""
+    dz = [[[[0.0] * d for _ in range(G)] for _ in range(H)] for _ in range(B)]
+    dWc = [[[0.0] * d for _ in range(d)] for _ in range(H)]
+    for b in range(B):
+        for h in range(H):
+            for g in range(G):
+                for c in range(d):
+                    up = d_tokens_mixed[b][h][g][c]
+                    for k in range(d):
+                        dz[b][h][g][k] += Wc[h][c][k] * up
+                        dWc[h][c][k] += up * tokens[b][h][g][k]
+    return dz, dWc

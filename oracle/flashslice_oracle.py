@@ -224,6 +224,22 @@ def mix_bwd(M, tokens, d_tokens_mixed):
     return {"d_tokens": dz, "dM": dM}
 
 
+def mix_channels(Wc, tokens):
+    """Core of the attention-free variant (Sec. 2 after Eq. (1), Sec. 3 variants
+    table, "NoTokenAttn"): A is the identity, so the tokens do not interact, and a
+    learned linear map acts on the channels of each token, one d x d map per head:
+    z'[b,h,g,c] = sum_k Wc[h,c,k] z[b,h,g,k]."""
+    return np.einsum("hck,bhgk->bhgc", _f64(Wc), _f64(tokens))
+
+
+def mix_channels_bwd(Wc, tokens, d_tokens_mixed):
+    """Backward of z' = Wc z per token: dz = Wc^T dz', dWc = sum over b and g of dz' z^T."""
+    dzp = _f64(d_tokens_mixed)
+    dz = np.einsum("hck,bhgc->bhgk", _f64(Wc), dzp)
+    dWc = np.einsum("bhgc,bhgk->hck", dzp, _f64(tokens))
+    return {"d_tokens": dz, "dWc": dWc}
+
+
 def slice_bwd(x_mid, fx, W_slice, bias, tau, tokens, wsum, d_tokens, eps=DEFAULT_EPS, heads=None):
     """Gradients of z = U/(S+eps), U = w^T f, S = w^T 1 w.r.t. fx and the logit inputs.
 
