@@ -142,6 +142,21 @@ fs_status fs_slice_finalize(const fs_shape* s, float* tokens, const float* wsum,
 fs_status fs_mix(const fs_shape* s, const float* M, const float* tokens,
                  float* tokens_mixed, fs_stream_t stream);
 
+/* The attention-free core (Sec. 2 after Eq. (1); "NoTokenAttn" in the Sec. 3
+ * variants table): A is the identity, so the tokens do not interact, and a
+ * learned linear map acts on the channels of each token, one per head:
+ * tokens_mixed[b,h,g,c] = sum_k Wc[h,c,k] tokens[b,h,g,k].  Wc [H,d,d] fp32.
+ * Out-of-place only.  It may replace fs_mix, or follow it (the two commute). */
+fs_status fs_mix_channels(const fs_shape* s, const float* Wc, const float* tokens,
+                          float* tokens_mixed, fs_stream_t stream);
+
+/* Backward of fs_mix_channels: d_tokens[b,h,g,k] = sum_c Wc[h,c,k]
+ * d_tokens_mixed[b,h,g,c] (overwritten); dWc [H,d,d] = sum over b and g of
+ * d_tokens_mixed tokens^T (overwritten). */
+fs_status fs_mix_channels_bwd(const fs_shape* s, const float* Wc, const float* tokens,
+                              const float* d_tokens_mixed, float* d_tokens, float* dWc,
+                              fs_stream_t stream);
+
 /* Deslice with tied weights (Sec. 2; App. G.1): out[b,n,h,:] = sum_g w z'_g.
  *   lse: statistics from fs_slice_fwd; NULL makes the call compute them first
  *   (into ws).  out has the dtype of the shape.  The Untied variant (Sec. 3, the

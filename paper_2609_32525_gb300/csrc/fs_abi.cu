@@ -272,6 +272,23 @@ fs_status fs_mix(const fs_shape* s, const float* M, const float* tokens, float* 
   return cuda_status(simt_mix(to_shape(s), M, tokens, tokens_mixed, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+fs_status fs_mix_channels(const fs_shape* s, const float* Wc, const float* tokens, float* tokens_mixed,
+                          fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(Wc); FS_CHECK_PTR(tokens); FS_CHECK_PTR(tokens_mixed);
+  if (tokens == tokens_mixed) return FS_ERR_INVALID;
+  return cuda_status(simt_mix_channels(to_shape(s), Wc, tokens, tokens_mixed, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+fs_status fs_mix_channels_bwd(const fs_shape* s, const float* Wc, const float* tokens, const float* d_tokens_mixed,
+                              float* d_tokens, float* dWc, fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(Wc); FS_CHECK_PTR(tokens); FS_CHECK_PTR(d_tokens_mixed); FS_CHECK_PTR(d_tokens); FS_CHECK_PTR(dWc);
+  if (d_tokens == d_tokens_mixed) return FS_ERR_INVALID;
+  return cuda_status(simt_mix_channels_bwd(to_shape(s), Wc, tokens, d_tokens_mixed, d_tokens, dWc,
+                                           reinterpret_cast<cudaStream_t>(stream)));
+}
+
 fs_status fs_deslice_fwd(const fs_shape* s, const void* x_mid, const float* W_slice, const float* bias,
                          const float* tau, const float* tokens_mixed, const float* lse, void* out, void* ws,
                          size_t ws_bytes, fs_stream_t stream) {

@@ -46,6 +46,11 @@ cudaError_t simt_reduce_tokens(const Shape& s, int P, const float* part, int Gs,
                                float* wsum, int finalize, cudaStream_t st);
 cudaError_t simt_finalize(const Shape& s, float* tokens, const float* wsum, cudaStream_t st);
 cudaError_t simt_mix(const Shape& s, const float* M, const float* z, float* zp, cudaStream_t st);
+// The attention-free core: zp[b,h,g,:] = Wc[h] z[b,h,g,:]; its backward dz = Wc^T dzp,
+// dWc = sum over b and g of dzp z^T.
+cudaError_t simt_mix_channels(const Shape& s, const float* Wc, const float* z, float* zp, cudaStream_t st);
+cudaError_t simt_mix_channels_bwd(const Shape& s, const float* Wc, const float* z, const float* dzp, float* dz,
+                                  float* dWc, cudaStream_t st);
 cudaError_t simt_mix_bwd(const Shape& s, const float* M, const float* z, const float* dzp,
                          float* dz, float* dM, cudaStream_t st);
 cudaError_t simt_deslice(const Shape& s, const void* x, const float* W, const float* bias,

@@ -293,6 +293,38 @@ __global__ void __launch_bounds__(256) k_mix_tiled(const float* __restrict__ M, 
   }
 }
 
+// Per-token channel map (the attention-free core): out[bh][g][c] = sum_k A(c, k)
+// in[bh][g][k], with A = Wc[h] (forward) or Wc[h]^T (its token backward); one
+// thread per output word, the sum over k in a fixed order.
+template <bool kTrans>
+__global__ void k_mix_channels(const float* __restrict__ Wc, const float* __restrict__ in, float* __restrict__ out,
+                               int64_t BHG, int H, int G, int D) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= BHG * D) return;
+  const int c = (int)(idx % D);
+  const int64_t t = idx / D;  // token bh * G + g
+  const int h = (int)((t / G) % H);
+  const float* A = Wc + (int64_t)h * D * D;
+  const float* z = in + t * D;
+  float acc = 0.f;
+  for (int k = 0; k < D; k++) acc = fmaf(kTrans ? A[(int64_t)k * D + c] : A[(int64_t)c * D + k], z[k], acc);
+  out[idx] = acc;
+}
+
+// dWc[h][c][k] = sum over b and g of dzp[b,h,g,c] z[b,h,g,k] (fixed order: b, then g).
+__global__ void k_mix_channels_dW(const float* __restrict__ z, const float* __restrict__ dzp, float* __restrict__ dWc,
+                                  int64_t B, int H, int G, int D) {
+  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= (int64_t)H * D * D) return;
+  const int k = (int)(idx % D), c = (int)((idx / D) % D), h = (int)(idx / ((int64_t)D * D));
+  float acc = 0.f;
+  for (int64_t b = 0; b < B; b++) {
+    const int64_t base = (b * H + h) * (int64_t)G * D;
+    for (int g = 0; g < G; g++) acc = fmaf(dzp[base + (int64_t)g * D + c], z[base + (int64_t)g * D + k], acc);
+  }
+  dWc[idx] = acc;
+}
+
 // dM[h][g][k] = sum_b sum_c dzp[b,h,g,c] z[b,h,k,c]: per head a G x G product with
 // K = B*D, tiled 64 x 64 per block (16 x 16 threads, 4 x 4 outputs each), the two
 // operand tiles staged in shared memory 16 channels at a time; the sum runs over
@@ -806,6 +838,23 @@ cudaError_t simt_mix_bwd(const Shape& s, const float* M, const float* z, const f
   if (e != cudaSuccess) return e;
   const dim3 tiles((unsigned)((s.G + 63) / 64), (unsigned)((s.G + 63) / 64), (unsigned)s.H);
   k_mix_bwd_dM<<<tiles, 256, 0, st>>>(z, dzp, dM, s.B, s.H, s.G, s.d);
+  return cudaGetLastError();
+}
+
+cudaError_t simt_mix_channels(const Shape& s, const float* Wc, const float* z, float* zp, cudaStream_t st) {
+  const int64_t BHG = s.BH() * s.G;
+  k_mix_channels<false><<<(unsigned)((BHG * s.d + 255) / 256), 256, 0, st>>>(Wc, z, zp, BHG, s.H, s.G, s.d);
+  return cudaGetLastError();
+}
+
+cudaError_t simt_mix_channels_bwd(const Shape& s, const float* Wc, const float* z, const float* dzp, float* dz,
+                                  float* dWc, cudaStream_t st) {
+  const int64_t BHG = s.BH() * s.G;
+  k_mix_channels<true><<<(unsigned)((BHG * s.d + 255) / 256), 256, 0, st>>>(Wc, dzp, dz, BHG, s.H, s.G, s.d);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  const int64_t n = (int64_t)s.H * s.d * s.d;
+  k_mix_channels_dW<<<(unsigned)((n + 127) / 128), 128, 0, st>>>(z, dzp, dWc, s.B, s.H, s.G, s.d);
   return cudaGetLastError();
 }
 

@@ -34,7 +34,7 @@ FS_OP_SLICE_FWD, FS_OP_DESLICE_FWD, FS_OP_DESLICE_BWD, FS_OP_SLICE_BWD = range(4
 EXPORTED = ("fs_workspace_bytes", "fs_slice_fwd", "fs_slice_finalize", "fs_mix", "fs_deslice_fwd",
             "fs_deslice_bwd", "fs_mix_bwd", "fs_slice_bwd", "fs_device_status", "fs_status_string",
             "fs_path_for_shape", "fs_backward_path_for_shape", "fs_forward_launch_count", "fs_slice_fwd_noalloc",
-            "fs_slice_fwd_lse")
+            "fs_slice_fwd_lse", "fs_mix_channels", "fs_mix_channels_bwd")
 
 
 class fs_shape(ctypes.Structure):
@@ -57,6 +57,8 @@ _sig = {
     "fs_slice_fwd": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _Z, _P]),
     "fs_slice_fwd_lse": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _Z, _P]),
     "fs_slice_finalize": (_I, [_S, _P, _P, _P]),
+    "fs_mix_channels": (_I, [_S, _P, _P, _P, _P]),
+    "fs_mix_channels_bwd": (_I, [_S, _P, _P, _P, _P, _P, _P]),
     "fs_mix": (_I, [_S, _P, _P, _P, _P]),
     "fs_deslice_fwd": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _Z, _P]),
     "fs_deslice_bwd": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _Z, _P]),
@@ -144,6 +146,17 @@ def fs_slice_fwd_lse(shape, x_mid, fx, W_slice, bias, tau, lse, tokens, wsum, fi
                                _ptr(lse), _ptr(tokens), _ptr(wsum), int(bool(finalize)), _ptr(ws), ws.numel(),
                                _stream(stream))
     _check("fs_slice_fwd_lse", st)
+
+
+def fs_mix_channels(shape, Wc, tokens, tokens_mixed, stream=None):
+    _check("fs_mix_channels", _lib.fs_mix_channels(ctypes.byref(shape), _ptr(Wc), _ptr(tokens), _ptr(tokens_mixed),
+                                                   _stream(stream)))
+
+
+def fs_mix_channels_bwd(shape, Wc, tokens, d_tokens_mixed, d_tokens, dWc, stream=None):
+    _check("fs_mix_channels_bwd", _lib.fs_mix_channels_bwd(ctypes.byref(shape), _ptr(Wc), _ptr(tokens),
+                                                           _ptr(d_tokens_mixed), _ptr(d_tokens), _ptr(dWc),
+                                                           _stream(stream)))
 
 
 def fs_slice_finalize(shape, tokens, wsum, stream=None):
