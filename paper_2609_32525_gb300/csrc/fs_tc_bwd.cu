@@ -151,6 +151,8 @@ __device__ __forceinline__ uint64_t px_desc(uint32_t px_s, uint32_t zero_s) { re
 // kSums: dt += sum da L, db += sum da.
 template <bool kSplit, bool kW, bool kSums>
 __device__ __forceinline__ void da_unit(uint32_t tL, uint32_t tD, float& dt, float& db) {
+  // Pairs of entries go through the packed f32x2 forms (one instruction for both).
+  const uint64_t neg1 = pack2(__float_as_uint(-1.f), __float_as_uint(-1.f));
 #pragma unroll 1
   for (int h2 = 0; h2 < 2; h2++) {
     uint32_t l[32], dw[32];
@@ -158,25 +160,30 @@ __device__ __forceinline__ void da_unit(uint32_t tL, uint32_t tD, float& dt, flo
     tmem_ld32(tD + 32 * h2, dw);
     tmem_wait_ld2(l, dw);
     uint32_t dh[16], dl[16], wh[16], wl[16];
-    float t = 0.f, sb = 0.f;
+    uint64_t t2 = 0, sb2 = 0;  // (+0, +0)
 #pragma unroll
     for (int k = 0; k < 16; k++) {
-      const float L0 = __uint_as_float(l[2 * k]), L1 = __uint_as_float(l[2 * k + 1]);
-      const float w0 = ex2(L0), w1 = ex2(L1);
-      const float a0 = w0 * __uint_as_float(dw[2 * k]), a1 = w1 * __uint_as_float(dw[2 * k + 1]);
+      const uint64_t L2 = pack2(l[2 * k], l[2 * k + 1]);
+      const uint64_t w2 = pack2(__float_as_uint(ex2(__uint_as_float(l[2 * k]))),
+                                __float_as_uint(ex2(__uint_as_float(l[2 * k + 1]))));
+      const uint64_t a2 = mul2(w2, pack2(dw[2 * k], dw[2 * k + 1]));
       if (kSums) {
-        t = fmaf(a0, L0, t);
-        t = fmaf(a1, L1, t);
-        sb += a0;
-        sb += a1;
+        t2 = fma2(a2, L2, t2);
+        sb2 = add2(sb2, a2);
       }
-      const uint32_t p = pack_bf16(a0, a1);
+      const uint32_t p = pack_bf16(lo_f(a2), hi_f(a2));
       dh[k] = p;
-      if (kSplit) dl[k] = pack_bf16(a0 - __uint_as_float(p << 16), a1 - __uint_as_float(p & 0xFFFF0000u));
+      if (kSplit) {
+        const uint64_t r2 = fma2(pack2(p << 16, p & 0xFFFF0000u), neg1, a2);  // a - bf16(a)
+        dl[k] = pack_bf16(lo_f(r2), hi_f(r2));
+      }
       if (kW) {
-        const uint32_t q = pack_bf16(w0, w1);
+        const uint32_t q = pack_bf16(lo_f(w2), hi_f(w2));
         wh[k] = q;
-        if (kSplit) wl[k] = pack_bf16(w0 - __uint_as_float(q << 16), w1 - __uint_as_float(q & 0xFFFF0000u));
+        if (kSplit) {
+          const uint64_t r2 = fma2(pack2(q << 16, q & 0xFFFF0000u), neg1, w2);
+          wl[k] = pack_bf16(lo_f(r2), hi_f(r2));
+        }
       }
     }
     tmem_st16(tL + 32 * h2, dh);
@@ -186,8 +193,8 @@ __device__ __forceinline__ void da_unit(uint32_t tL, uint32_t tD, float& dt, flo
       if (kSplit) tmem_st16(tD + 32 * h2 + 16, wl);
     }
     if (kSums) {
-      dt += t;
-      db += sb;
+      dt += lo_f(t2) + hi_f(t2);
+      db += lo_f(sb2) + hi_f(sb2);
     }
   }
 }
