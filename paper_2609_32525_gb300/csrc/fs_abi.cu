@@ -140,8 +140,11 @@ cudaError_t backward_stats(const Shape& sh, const void* x_mid, const float* W_sl
                            const float* tau, const float* lse, void* ws, const Regions& r, uint32_t* status,
                            cudaStream_t st, const float** lse_use) {
   *lse_use = lse;
-  const bool tc = tc_forward_supported(sh);
-  if (lse && (!tc || sh.dot == FS_DOT_BF16X2)) return cudaSuccess;
+  // fp32 shapes take the fp32 SIMT backward: it gets exact fp32 statistics (the
+  // forward's come from split bf16 products on the tensor cores).
+  const bool tc = tc_forward_supported(sh) && sh.dtype == FS_BF16;
+  const bool fp32_tc = tc_forward_supported(sh) && sh.dtype == FS_F32;
+  if (lse && !fp32_tc && (!tc || sh.dot == FS_DOT_BF16X2)) return cudaSuccess;
   float* buf = at<float>(ws, r.stats);
   *lse_use = buf;
   if (!tc) return simt_stats(sh, x_mid, W_slice, bias, tau, buf, status, st);

@@ -60,24 +60,6 @@ __global__ void k_prep_t(const float* __restrict__ t, int tstride, int has_c, ui
     ep[off_sw32(g, k) / 2] = k == 0 ? chi : (k == 1 ? clo : __float2bfloat16_rn((k == 2 || k == 3) ? 1.f : 0.f));
 }
 
-// Z-layout image (blocks of 64 slots, 32 channel rows x 128 B, 128B swizzle) of
-// t [BH][G][tstride] per (b,h): the bf16 half, then the residual half (Gp*128 bytes
-// per (b,h)); padding slots [G, Gp) are zero.
-__global__ void k_prep_z2(const float* __restrict__ t, int tstride, uint8_t* __restrict__ img, int64_t BH, int G,
-                          int Gp) {
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (i >= BH * Gp * kD) return;
-  const int c = (int)(i % kD);
-  const int g = (int)((i / kD) % Gp);
-  const int64_t bh = i / ((int64_t)kD * Gp);
-  const float v = g < G ? t[(bh * G + g) * tstride + c] : 0.f;
-  __nv_bfloat16* hp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * Gp * 128);
-  __nv_bfloat16* lp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * Gp * 128 + (size_t)Gp * 64);
-  const __nv_bfloat16 hi = __float2bfloat16_rn(v);
-  hp[off_z(c, g) / 2] = hi;
-  lp[off_z(c, g) / 2] = __float2bfloat16_rn(v - __bfloat162float(hi));
-}
-
 // W'^T image of head h in the Z layout (channel rows, slots along K), W' =
 // W log2(e)/tau: the bf16 half, then the residual half (Gp*128 bytes per head;
 // padding slots zero).  It is the B operand of dx += da W'^T.
@@ -791,7 +773,7 @@ cudaError_t prep_t_images(const Shape& s, int G, const float* t, int tstride, in
 // cancelling terms of size |dz||fx|/(S + eps) that split bf16 products resolve only
 // to ~2^-17 of that size.
 bool tc_backward_supported(const Shape& s0) {
-  if (!tc_forward_supported(s0) || s0.N < 2) return false;
+  if (s0.dtype != FS_BF16 || !tc_forward_supported(s0) || s0.N < 2) return false;
   const Shape s = tc_padded(s0);
   return smem_bwd_dx(s.G, false) <= kMaxSmem && tc_rows_smem(s, 2, false, false) <= kMaxSmem;
 }

@@ -99,6 +99,24 @@ __global__ void k_prep_z(const float* __restrict__ zp, uint8_t* __restrict__ img
   out[off_z(c, g) / 2] = __float2bfloat16_rn(g < G ? zp[(bh * G + g) * kD + c] : 0.f);
 }
 
+// Z-layout image (blocks of 64 slots, 32 channel rows x 128 B, 128B swizzle) of
+// t [BH][G][tstride] per (b,h): the bf16 half, then the residual half (Gp*128 bytes
+// per (b,h)); padding slots [G, Gp) are zero.
+__global__ void k_prep_z2(const float* __restrict__ t, int tstride, uint8_t* __restrict__ img, int64_t BH, int G,
+                          int Gp) {
+  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= BH * Gp * kD) return;
+  const int c = (int)(i % kD);
+  const int g = (int)((i / kD) % Gp);
+  const int64_t bh = i / ((int64_t)kD * Gp);
+  const float v = g < G ? t[(bh * G + g) * tstride + c] : 0.f;
+  __nv_bfloat16* hp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * Gp * 128);
+  __nv_bfloat16* lp = reinterpret_cast<__nv_bfloat16*>(img + (size_t)bh * Gp * 128 + (size_t)Gp * 64);
+  const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+  hp[off_z(c, g) / 2] = hi;
+  lp[off_z(c, g) / 2] = __float2bfloat16_rn(v - __bfloat162float(hi));
+}
+
 // ---- shared pieces -------------------------------------------------------------------------
 struct Work {
   int64_t bh;      // batch * H + head
@@ -153,8 +171,10 @@ __device__ __forceinline__ void zero_smem(uint8_t* p, uint32_t bytes) {
 //   point_major: A = points (x tile), B = slots (W);  else A = slots, B = points.
 //   xe: descriptor of the point-side extra block.
 //   wl_img: the residual half of W' (0: bf16 W' only, K = 48; else K = 80).
+//   xr_s: the residual half of x, fp32 inputs (0: none; else two more K-steps, x_r W'_hi).
 __device__ __forceinline__ void issue_logits(uint32_t tmem_d, uint32_t x_s, uint64_t xe, uint32_t w_img,
-                                             uint32_t we_img, uint32_t wl_img, int c, bool point_major) {
+                                             uint32_t we_img, uint32_t wl_img, int c, bool point_major,
+                                             uint32_t xr_s = 0) {
   constexpr uint32_t idesc = idesc_bf16(128, kGC, false, false);
   const uint32_t wc = w_img + (uint32_t)c * kGC * 64;
   const uint32_t wec = we_img + (uint32_t)c * kGC * 32;
@@ -179,10 +199,36 @@ __device__ __forceinline__ void issue_logits(uint32_t tmem_d, uint32_t x_s, uint
       mma_ss_w(tmem_d, l1, x1, idesc, 1);
     }
   }
+  if (xr_s) {
+    const uint64_t r0 = sdesc(xr_s, 16, 512, kSw64), r1 = sdesc(xr_s + 32, 16, 512, kSw64);
+    if (point_major) {
+      mma_ss_w(tmem_d, r0, w0, idesc, 1);
+      mma_ss_w(tmem_d, r1, w1, idesc, 1);
+    } else {
+      mma_ss_w(tmem_d, w0, r0, idesc, 1);
+      mma_ss_w(tmem_d, w1, r1, idesc, 1);
+    }
+  }
   if (point_major)
     mma_ss_w(tmem_d, xe, we, idesc, 1);
   else
     mma_ss_w(tmem_d, we, xe, idesc, 1);
+}
+
+// fp32 point tensors -> bf16 hi and residual lo tensors of the same layout (v = hi + lo
+// to ~2^-16 relative): the tensor-core path's operands for fp32 inputs.
+__global__ void k_split_bf16(const float* __restrict__ v, __nv_bfloat16* __restrict__ hi,
+                             __nv_bfloat16* __restrict__ lo, int64_t n) {
+  const int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 4;
+  if (i >= n) return;
+  const float4 a = *reinterpret_cast<const float4*>(v + i);
+  const float e[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+  for (int k = 0; k < 4; k++) {
+    const __nv_bfloat16 h = __float2bfloat16_rn(e[k]);
+    hi[i + k] = h;
+    lo[i + k] = __float2bfloat16_rn(e[k] - __bfloat162float(h));
+  }
 }
 
 // Producer-side bulk loads of an image into smem (pieces of at most 32 KB).
@@ -411,7 +457,8 @@ Shape tc_padded(const Shape& s) {
 }
 
 size_t w_image_bytes(const Shape& s) { return (size_t)s.H * s.G * kWRow; }
-size_t z_image_bytes(const Shape& s) { return (size_t)s.BH() * s.G * 64; }
+// Z' image of the forward's deslice; fp32 inputs carry z' as hi and residual halves.
+size_t z_image_bytes(const Shape& s) { return (size_t)s.BH() * s.G * (s.dtype == FS_F32 ? 128 : 64); }
 int64_t padded_n(const Shape& s) { return (s.N + kTile - 1) / kTile * kTile; }
 size_t px_bytes(const Shape& s) { return (size_t)s.BH() * padded_n(s) * 16; }
 

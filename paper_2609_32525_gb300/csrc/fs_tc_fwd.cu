@@ -74,9 +74,12 @@ using namespace tc;
 // =========================================================================================
 constexpr uint32_t kDStage = kXBytes + 2 * kPxBytes;  // x tile, point extra (both halves)
 
-template <int MODE, bool PS>
+// X3 (fp32 inputs, MODE 0 with PS): each stage also holds x's residual tile
+// (xrmap), the logits add x_r W'_hi, and out is fp32.
+template <int MODE, bool PS, bool X3 = false>
 __global__ void __launch_bounds__(kThreads, 1)
     k_deslice(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap pmap,
+              const __grid_constant__ CUtensorMap xrmap,
               const uint8_t* __restrict__ wimg, const uint8_t* __restrict__ zimg, __nv_bfloat16* __restrict__ out,
               const __nv_bfloat16* __restrict__ v, float* __restrict__ delta, float* __restrict__ wds,
               const float* __restrict__ dS, int64_t N, int64_t Np, int H, int G, int splits, int hilo,
@@ -90,8 +93,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* s_z = s_w + wbytes;
   float* s_ds = reinterpret_cast<float*>(s_z + zbytes);  // MODE 2: dS of the G slots
   // (the stages stay 1024-byte aligned for their swizzled tiles)
-  uint8_t* s_x = s_z + zbytes + (MODE == 2 ? (((uint32_t)G * 4 + 1023u) & ~1023u) : 0u);  // stage s at s_x + s * kDStage
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_x + kStages * kDStage);
+  uint8_t* s_x = s_z + zbytes + (MODE == 2 ? (((uint32_t)G * 4 + 1023u) & ~1023u) : 0u);  // stage s at s_x + s * kDSt
+  constexpr uint32_t kDSt = kDStage + (X3 ? kXBytes : 0u);  // stage: x | px (2 halves) [| x residual]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_x + kStages * kDSt);
   uint64_t* wz_full = bars;
   uint64_t* x_full = bars + 1;
   uint64_t* x_empty = x_full + kStages;
@@ -131,7 +135,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     ab->flag = 0;
     fence_mbar_init();
   }
-  for (int s = 0; s < kStages; s++) zero_smem(s_x + s * kDStage + kXBytes + kPxBytes, kPxBytes);
+  for (int s = 0; s < kStages; s++) zero_smem(s_x + s * kDSt + kXBytes + kPxBytes, kPxBytes);
   if (MODE == 2)
     for (int g = threadIdx.x; g < G; g += kThreads) s_ds[g] = dS[wk.bh * G + g];
   fence_proxy_async_smem();
@@ -146,6 +150,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (lane == 0 && wk.ntiles > 0) {
       prefetch_tmap(&xmap);
       prefetch_tmap(&pmap);
+      if (X3) prefetch_tmap(&xrmap);
       mbar_expect_tx(wz_full, wbytes + zbytes);
       load_images(s_w, wimg + (size_t)h * G * kWRow, wbytes, wz_full);
       load_images(s_z, zimg + (size_t)wk.bh * zstride, zbytes, wz_full);
@@ -154,9 +159,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int s = i % kStages;
         if (i >= kStages && !mbar_wait(&x_empty[s], (uint32_t)(((i / kStages) - 1) & 1), ab, status)) break;
         const int n0 = (int)((wk.tile0 + i) * kTile);
-        mbar_expect_tx(&x_full[s], kXBytes + kPxBytes);
-        tma_load_3d(s_x + s * kDStage, &xmap, h * kD, n0, (int)b, &x_full[s]);
-        tma_load_2d(s_x + s * kDStage + kXBytes, &pmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
+        mbar_expect_tx(&x_full[s], kXBytes + kPxBytes + (X3 ? kXBytes : 0u));
+        tma_load_3d(s_x + s * kDSt, &xmap, h * kD, n0, (int)b, &x_full[s]);
+        tma_load_2d(s_x + s * kDSt + kXBytes, &pmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
+        if (X3) tma_load_3d(s_x + s * kDSt + kDStage, &xrmap, h * kD, n0, (int)b, &x_full[s]);
       }
       // Drain: the newest load of each stage has landed before the CTA exits.
       for (int j = (i > kStages ? i - kStages : 0); j < i; j++)
@@ -178,9 +184,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (c == 0 && !(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kStages) & 1), ab, status))) break;
         if (q >= kSBuf && !(ok = mbar_wait_w(&pv_done[bb], (uint32_t)(((q / kSBuf) - 1) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t xs = smem_u32(s_x + s * kDStage);
+        const uint32_t xs = smem_u32(s_x + s * kDSt);
         issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kXBytes), sw, swe,
-                     hilo ? sw + (uint32_t)G * 96 : 0u, c, true);
+                     hilo ? sw + (uint32_t)G * 96 : 0u, c, true, X3 ? xs + kDStage : 0u);
         mma_commit_w(&s_full[bb]);
         if (c == nch - 1) mma_commit_w(&x_empty[s]);
       }
@@ -242,7 +248,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int64_t n = (wk.tile0 + t) * kTile + r;
       if (n < N) {
         const int64_t row = ((b * N + n) * H + h) * kD;
-        if (MODE != 1) {
+        if (X3) {
+          float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(out) + row);
+#pragma unroll
+          for (int k = 0; k < 8; k++)
+            dst[k] = make_float4(__uint_as_float(o0[4 * k]) + __uint_as_float(o1[4 * k]),
+                                 __uint_as_float(o0[4 * k + 1]) + __uint_as_float(o1[4 * k + 1]),
+                                 __uint_as_float(o0[4 * k + 2]) + __uint_as_float(o1[4 * k + 2]),
+                                 __uint_as_float(o0[4 * k + 3]) + __uint_as_float(o1[4 * k + 3]));
+        } else if (MODE != 1) {
           uint4* dst = reinterpret_cast<uint4*>(out + row);
 #pragma unroll
           for (int k = 0; k < 4; k++) {
@@ -336,17 +350,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 // smem: [W img G*96][x stages][constant extra][ml exchange][barriers]
 // TMEM: two S buffers [0, 256).
 // =========================================================================================
-template <bool split>
+// X3 (fp32 inputs): x arrives as bf16 hi and residual tiles (xmap, xrmap), one stage
+// holding both, and the logits add x_r W'_hi.
+template <bool split, bool X3>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_stats(const __grid_constant__ CUtensorMap xmap, const uint8_t* __restrict__ wimg, float* __restrict__ lse,
-            uint4* __restrict__ px, int64_t N, int64_t Np, int H, int G, int splits, uint32_t* status) {
+    k_stats(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap xrmap,
+            const uint8_t* __restrict__ wimg, float* __restrict__ lse, uint4* __restrict__ px, int64_t N,
+            int64_t Np, int H, int G, int splits, uint32_t* status) {
+  constexpr uint32_t kXSt = X3 ? 2 * kXBytes : kXBytes;  // x stage
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   // split (FS_DOT_BF16X2): the residual half of W' too (K = 80 logits).
   const uint32_t wbytes = (uint32_t)G * (split ? kWRow : 96);
   uint8_t* s_w = smem;
   uint8_t* s_x = s_w + wbytes;
-  uint8_t* s_ex = s_x + kStages * kXBytes;
+  uint8_t* s_ex = s_x + kStages * kXSt;
   float2* s_ml = reinterpret_cast<float2*>(s_ex + kExBytes);  // [2][128] warpgroup-1 partials
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_ml + 2 * kTile);
   uint64_t* w_full = bars;
@@ -394,14 +412,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 0) {
     if (lane == 0 && wk.ntiles > 0) {
       prefetch_tmap(&xmap);
+      if (X3) prefetch_tmap(&xrmap);
       mbar_expect_tx(w_full, wbytes);
       load_images(s_w, wimg + (size_t)h * G * kWRow, wbytes, w_full);
       int i = 0;
       for (; i < wk.ntiles; i++) {
         const int s = i % kStages;
         if (i >= kStages && !mbar_wait(&x_empty[s], (uint32_t)(((i / kStages) - 1) & 1), ab, status)) break;
-        mbar_expect_tx(&x_full[s], kXBytes);
-        tma_load_3d(s_x + s * kXBytes, &xmap, h * kD, (int)((wk.tile0 + i) * kTile), (int)b, &x_full[s]);
+        mbar_expect_tx(&x_full[s], kXSt);
+        tma_load_3d(s_x + s * kXSt, &xmap, h * kD, (int)((wk.tile0 + i) * kTile), (int)b, &x_full[s]);
+        if (X3) tma_load_3d(s_x + s * kXSt + kXBytes, &xrmap, h * kD, (int)((wk.tile0 + i) * kTile), (int)b, &x_full[s]);
       }
       for (int j = (i > kStages ? i - kStages : 0); j < i; j++)
         mbar_wait(&x_full[j % kStages], (uint32_t)((j / kStages) & 1), ab, nullptr, kWaitNs);
@@ -425,8 +445,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (c < nis && !(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kStages) & 1), ab, status))) break;
         if (q >= 2 && !(ok = mbar_wait_w(&s_free[bb], (uint32_t)(((q >> 1) - 1) & 1), ab, status))) break;
         tc_fence_after();
-        issue_logits(tmem + (uint32_t)bb * kGC, smem_u32(s_x + s * kXBytes), const_extra_desc(smem_u32(s_ex)), sw, swe,
-                     split ? sw + (uint32_t)G * 96 : 0u, c, true);
+        const uint32_t xs = smem_u32(s_x + s * kXSt);
+        issue_logits(tmem + (uint32_t)bb * kGC, xs, const_extra_desc(smem_u32(s_ex)), sw, swe,
+                     split ? sw + (uint32_t)G * 96 : 0u, c, true, X3 ? xs + kXBytes : 0u);
         mma_commit_w(&s_full[bb]);
         if (c >= nch - nis) mma_commit_w(&x_empty[s]);
       }
@@ -560,11 +581,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 constexpr uint32_t kStageBytes = kXBytes + 3 * kFBlock + 2 * kPxBytes;  // x, [F | 1], point extra
 constexpr uint32_t kWBlock = 128 * kWRow;                               // one 128-slot block of the W image
 
-template <bool split>
+// X3 (fp32 inputs): each stage also holds the residual tiles of x and fx (xrmap,
+// frmap); the logits add x_r W'_hi and the products add P_hi F_r (N = 32: U only).
+// Its stages are larger, so there are half as many.
+template <bool split, bool X3>
 __global__ void __launch_bounds__(kThreads, 1)
     k_slice(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap fmap,
-            const __grid_constant__ CUtensorMap pmap, const uint8_t* __restrict__ wimg, float* __restrict__ part,
+            const __grid_constant__ CUtensorMap pmap, const __grid_constant__ CUtensorMap xrmap,
+            const __grid_constant__ CUtensorMap frmap, const uint8_t* __restrict__ wimg, float* __restrict__ part,
             int64_t N, int64_t Np, int H, int G, int splits, uint32_t* status) {
+  constexpr int kNSt = X3 ? kSliceStages / 2 : kSliceStages;
+  constexpr uint32_t kStB = kStageBytes + (X3 ? kXBytes + 2 * kFBlock : 0u);
+  constexpr uint32_t kXROff = kStageBytes, kFROff = kStageBytes + kXBytes;
   // split (FS_DOT_BF16X2): logits with both halves of W' (K = 80), and the
   // weights as hi + lo bf16 halves in the products (twice the product MMAs).
   // Grid (slot block, point split, bh): the CTAs of all slot blocks of one point
@@ -575,11 +603,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* s_w = smem;
   uint8_t* s_st = s_w + kWBlock;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_st + kSliceStages * kStageBytes);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_st + kNSt * kStB);
   uint64_t* w_full = bars;
   uint64_t* x_full = bars + 1;
-  uint64_t* st_empty = x_full + kSliceStages;
-  uint64_t* s_full = st_empty + kSliceStages;
+  uint64_t* st_empty = x_full + kNSt;
+  uint64_t* s_full = st_empty + kNSt;
   uint64_t* p_ready = s_full + kSBuf;   // [issuer][S buffer]
   uint64_t* pv_done = p_ready + 2 * kSBuf;
   uint64_t* acc_full = pv_done + kSBuf;
@@ -596,7 +624,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(w_full, 1);
-    for (int s = 0; s < kSliceStages; s++) {
+    for (int s = 0; s < kNSt; s++) {
       mbar_init(&x_full[s], 1);
       mbar_init(&st_empty[s], 2);  // the logits issuer and the tile's product issuer
     }
@@ -611,11 +639,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     ab->flag = 0;
     fence_mbar_init();
   }
-  for (int s = 0; s < kSliceStages; s++) zero_smem(s_st + s * kStageBytes + kPOff + kPxBytes, kPxBytes);
+  for (int s = 0; s < kNSt; s++) zero_smem(s_st + s * kStB + kPOff + kPxBytes, kPxBytes);
   // Constant "ones" block of every stage: row n = [1, 0 x 15] (32B swizzle).
-  for (int idx = threadIdx.x; idx < kSliceStages * kTile; idx += kThreads) {
+  for (int idx = threadIdx.x; idx < kNSt * kTile; idx += kThreads) {
     const int s = idx / kTile, r = idx % kTile;
-    const uint32_t base = smem_u32(s_st + s * kStageBytes + kFOff + 2 * kFBlock) +
+    const uint32_t base = smem_u32(s_st + s * kStB + kFOff + 2 * kFBlock) +
                           (uint32_t)((r >> 3) * 256 + (r & 7) * 32);
     const uint32_t sw = (uint32_t)((r & 7) >> 2);
     st_shared_v4(base + ((0u ^ sw) << 4), 0x3F80u, 0u, 0u, 0u);
@@ -633,6 +661,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&xmap);
       prefetch_tmap(&fmap);
       prefetch_tmap(&pmap);
+      if (X3) {
+        prefetch_tmap(&xrmap);
+        prefetch_tmap(&frmap);
+      }
       // The slot block's rows of the W image: 128 rows of W' (64 B) then 128 rows of
       // the extra block (32 B); the global image holds G rows of each.
       mbar_expect_tx(w_full, split ? kWBlock : kGC * 96);
@@ -642,20 +674,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (split) load_images(s_w + kGC * 96, src + (size_t)G * 96 + (size_t)g_base * 64, kGC * 64, w_full);
       int i = 0;
       for (; i < wk.ntiles; i++) {
-        const int s = i % kSliceStages;
-        if (i >= kSliceStages &&
-            !mbar_wait(&st_empty[s], (uint32_t)(((i / kSliceStages) - 1) & 1), ab, status))
+        const int s = i % kNSt;
+        if (i >= kNSt &&
+            !mbar_wait(&st_empty[s], (uint32_t)(((i / kNSt) - 1) & 1), ab, status))
           break;
-        uint8_t* st = s_st + s * kStageBytes;
+        uint8_t* st = s_st + s * kStB;
         const int n0 = (int)((wk.tile0 + i) * kTile);
-        mbar_expect_tx(&x_full[s], kXBytes + 2 * kFBlock + kPxBytes);
+        mbar_expect_tx(&x_full[s], kXBytes + 2 * kFBlock + kPxBytes + (X3 ? kXBytes + 2 * kFBlock : 0u));
         tma_load_3d(st, &xmap, h * kD, n0, (int)b, &x_full[s]);
         tma_load_3d(st + kFOff, &fmap, h * kD, n0, (int)b, &x_full[s]);
         tma_load_3d(st + kFOff + kFBlock, &fmap, h * kD + 16, n0, (int)b, &x_full[s]);
         tma_load_2d(st + kPOff, &pmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
+        if (X3) {
+          tma_load_3d(st + kXROff, &xrmap, h * kD, n0, (int)b, &x_full[s]);
+          tma_load_3d(st + kFROff, &frmap, h * kD, n0, (int)b, &x_full[s]);
+          tma_load_3d(st + kFROff + kFBlock, &frmap, h * kD + 16, n0, (int)b, &x_full[s]);
+        }
       }
-      for (int j = (i > kSliceStages ? i - kSliceStages : 0); j < i; j++)
-        mbar_wait(&x_full[j % kSliceStages], (uint32_t)((j / kSliceStages) & 1), ab, nullptr, kWaitNs);
+      for (int j = (i > kNSt ? i - kNSt : 0); j < i; j++)
+        mbar_wait(&x_full[j % kNSt], (uint32_t)((j / kNSt) & 1), ab, nullptr, kWaitNs);
       mbar_wait(w_full, 0, ab, nullptr, kWaitNs);
     }
   } else if (warp == 1) {
@@ -664,14 +701,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t sw = smem_u32(s_w), swe = sw + kGC * 64;
       bool ok = mbar_wait_w(w_full, 0, ab, status);
       for (int i = 0; ok && i < wk.ntiles; i++) {
-        const int s = i % kSliceStages;
+        const int s = i % kNSt;
         const int bb = i % kSBuf;
-        if (!(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kSliceStages) & 1), ab, status))) break;
+        if (!(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kNSt) & 1), ab, status))) break;
         if (i >= kSBuf && !(ok = mbar_wait_w(&pv_done[bb], (uint32_t)(((i / kSBuf) - 1) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t xs = smem_u32(s_st + s * kStageBytes);
+        const uint32_t xs = smem_u32(s_st + s * kStB);
         issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kPOff), sw, swe, split ? sw + kGC * 96 : 0u,
-                     0, false);
+                     0, false, X3 ? xs + kXROff : 0u);
         mma_commit_w(&s_full[bb]);
         mma_commit_w(&st_empty[s]);
       }
@@ -685,13 +722,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idesc_sl = idesc_bf16(128, 48, false, true);
       bool ok = true;
       for (int i = j; ok && i < wk.ntiles; i += 2) {
-        const int s = i % kSliceStages;
+        const int s = i % kNSt;
         const int bb = i % kSBuf;
         // This issuer's tiles on buffer bb are 2 kSBuf apart.
         if (!(ok = mbar_wait_w(&p_ready[j * kSBuf + bb], (uint32_t)((i / (2 * kSBuf)) & 1), ab, status))) break;
         tc_fence_after();
         const uint32_t tE = tmem + (uint32_t)bb * kGC;  // packed weights of the 128 points
-        const uint32_t fs = smem_u32(s_st + s * kStageBytes) + kFOff;
+        const uint32_t fs = smem_u32(s_st + s * kStB) + kFOff;
         const uint32_t tacc = tmem + kA + (uint32_t)j * 48;
 #pragma unroll
         for (int kk = 0; kk < 8; kk++) {
@@ -699,6 +736,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           mma_ts_w(tacc, tE + (uint32_t)kk * 8, fdesc, idesc_sl, (i >= 2 || kk > 0) ? 1u : 0u);
           // The residual halves of the weights: U and S to ~2^-16.
           if (split) mma_ts_w(tacc, tE + 64 + (uint32_t)kk * 8, fdesc, idesc_sl, 1u);
+          if (X3)  // the weights against fx's residual half (U only)
+            mma_ts_w(tacc, tE + (uint32_t)kk * 8, sdesc(fs - kFOff + kFROff + (uint32_t)kk * 512, kFBlock, 256, kSw32),
+                     idesc_bf16(128, 32, false, true), 1u);
         }
         mma_commit_w(&pv_done[bb]);
         mma_commit_w(&st_empty[s]);
@@ -766,46 +806,74 @@ __global__ void __launch_bounds__(kThreads, 1)
 int slice_blocks(const Shape& s) { return s.G / kGC < 1 ? 1 : s.G / kGC; }
 int slice_splits(const Shape& s) { return point_splits(s, (int)(s.BH() * slice_blocks(s))); }
 
-size_t smem_deslice(int G, bool hilo, int mode = 0, bool ps = false) {
-  return 1024 + (size_t)G * ((hilo ? kWRow : 96) + (ps ? 128 : 64)) + (mode == 2 ? align_up((size_t)G * 4, 1024) : 0) +
-         kStages * kDStage + 512;
-}
-size_t smem_stats(int G, bool split) {
-  return 1024 + (size_t)G * (split ? kWRow : 96) + kStages * kXBytes + kExBytes + 2 * kTile * 8 + 512;
-}
-size_t smem_slice() { return 1024 + (size_t)kWBlock + kSliceStages * kStageBytes + 512; }
+// fp32 point tensors take the tensor-core path with every operand as two bf16 halves
+// (x, fx and W', the weights, z'): the X3 kernels.  Their inputs are first split
+// into bf16 hi and residual tensors in the workspace (k_split_bf16).
+bool x3_shape(const Shape& s) { return s.dtype == FS_F32; }
+size_t half_bytes(const Shape& s) { return align_up((size_t)s.B * s.N * s.H * s.d * 2, 256); }
 
-// Statistics into lse [B,H,N] and the point-extra rows at px.
-cudaError_t run_stats(const Shape& s, const void* x, const uint8_t* wimg, float* lse, void* px, uint32_t* status,
-                      cudaStream_t st) {
-  CUtensorMap xmap;
+size_t smem_deslice(int G, bool hilo, int mode = 0, bool ps = false, bool x3 = false) {
+  return 1024 + (size_t)G * ((hilo ? kWRow : 96) + (ps ? 128 : 64)) + (mode == 2 ? align_up((size_t)G * 4, 1024) : 0) +
+         kStages * (kDStage + (x3 ? kXBytes : 0)) + 512;
+}
+size_t smem_stats(int G, bool split, bool x3 = false) {
+  return 1024 + (size_t)G * (split ? kWRow : 96) + kStages * kXBytes * (x3 ? 2 : 1) + kExBytes + 2 * kTile * 8 + 512;
+}
+size_t smem_slice(bool x3 = false) {
+  return 1024 + (size_t)kWBlock +
+         (x3 ? (size_t)(kSliceStages / 2) * (kStageBytes + kXBytes + 2 * kFBlock) : (size_t)kSliceStages * kStageBytes) +
+         512;
+}
+
+// v (fp32 [B,N,H,d]) -> bf16 hi at dst, bf16 residual at dst + half_bytes(s).
+cudaError_t split_points(const Shape& s, const void* v, uint8_t* dst, cudaStream_t st) {
+  const int64_t n = s.B * s.N * s.H * s.d;
+  k_split_bf16<<<(unsigned)((n / 4 + 255) / 256), 256, 0, st>>>(
+      static_cast<const float*>(v), reinterpret_cast<__nv_bfloat16*>(dst),
+      reinterpret_cast<__nv_bfloat16*>(dst + half_bytes(s)), n);
+  return cudaGetLastError();
+}
+
+// Statistics into lse [B,H,N] and the point-extra rows at px.  xr: x's residual
+// half (X3), else null.
+cudaError_t run_stats(const Shape& s, const void* x, const void* xr, const uint8_t* wimg, float* lse, void* px,
+                      uint32_t* status, cudaStream_t st) {
+  CUtensorMap xmap, xrmap;
   if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
+  if (!make_point_map(&xrmap, xr ? xr : x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
   const int P = point_splits(s, (int)s.BH());
-  const bool split = s.dot == FS_DOT_BF16X2;
-  const size_t sm = smem_stats(s.G, split);
-  const auto kernel = split ? k_stats<true> : k_stats<false>;
+  const bool x3 = xr != nullptr;
+  const bool split = s.dot == FS_DOT_BF16X2 || x3;
+  const size_t sm = smem_stats(s.G, split, x3);
+  const auto kernel = x3 ? k_stats<true, true> : (split ? k_stats<true, false> : k_stats<false, false>);
   cudaError_t e = set_smem(kernel, sm);
   if (e != cudaSuccess) return e;
-  kernel<<<dim3((unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(xmap, wimg, lse, static_cast<uint4*>(px), s.N,
-                                                                    padded_n(s), s.H, s.G, P, status);
+  kernel<<<dim3((unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(xmap, xrmap, wimg, lse, static_cast<uint4*>(px),
+                                                                    s.N, padded_n(s), s.H, s.G, P, status);
   return cudaGetLastError();
 }
 
 }  // namespace
 
 // The slice on prepared operands (defined below, after the C-ABI-facing helpers).
-cudaError_t run_slice(const Shape& s, int G, const void* x, const void* f, const uint8_t* wimg, void* px,
-                      float* tokens, float* wsum, int finalize, float* part, uint32_t* status, cudaStream_t st);
+cudaError_t run_slice(const Shape& s, int G, const void* x, const void* f, const void* xr, const void* fr,
+                      const uint8_t* wimg, void* px, float* tokens, float* wsum, int finalize, float* part,
+                      uint32_t* status, cudaStream_t st);
 
 bool tc_forward_supported(const Shape& s) {
   // TMA coordinates and the kernels' block counters are 32-bit.
   const int64_t np = (s.N + kTile - 1) / kTile * kTile;
-  return s.dtype == FS_BF16 && s.d == kD && s.G <= 1024 && s.N >= 1 &&
+  // fp32 inputs need the residual half of W' in the deslice's shared memory (G <= 512),
+  // and take the tensor cores only when there is enough work to pay for splitting
+  // their inputs: B*N*H*G >= 2^24 (smaller problems keep the exact fp32 SIMT kernels).
+  const bool fp32_ok = s.dtype == FS_F32 && s.G <= 512 && (double)s.BH() * s.N * s.G >= 16777216.0;
+  return (s.dtype == FS_BF16 || fp32_ok) && s.d == kD && s.G <= 1024 && s.N >= 1 &&
          s.BH() * np < (int64_t(1) << 31) && encode_fn() != nullptr;
 }
 
-int tc_forward_launch_count(const Shape&) {
-  return 4 /*prep_w, stats, slice, reduce*/ + 4 /*prep_w, prep_z, prep_px, deslice*/;
+int tc_forward_launch_count(const Shape& s) {
+  return 4 /*prep_w, stats, slice, reduce*/ + 4 /*prep_w, prep_z, prep_px, deslice*/ +
+         (x3_shape(s) ? 3 /*splits of x, fx; of x*/ : 0);
 }
 
 size_t tc_slice_partials_bytes(const Shape& s0) {
@@ -813,13 +881,18 @@ size_t tc_slice_partials_bytes(const Shape& s0) {
   const Shape s = tc_padded(s0);
   return (size_t)slice_splits(s) * s.BH() * s.G * (kD + 1) * sizeof(float);
 }
+// Layouts of the prepared operands: slice [W img | px | (X3) x hi, x r, fx hi, fx r];
+// deslice and statistics [W img | Z' img | px | (X3) x hi, x r].
 size_t tc_slice_prep_bytes(const Shape& s0) {
   const Shape s = tc_padded(s0);
-  return tc_forward_supported(s0) ? align_up(w_image_bytes(s), 256) + px_bytes(s) : 0;
+  return tc_forward_supported(s0)
+             ? align_up(w_image_bytes(s), 256) + align_up(px_bytes(s), 256) + (x3_shape(s) ? 4 * half_bytes(s) : 0)
+             : 0;
 }
 size_t tc_deslice_prep_bytes(const Shape& s0) {
   const Shape s = tc_padded(s0);
-  return tc_forward_supported(s0) ? align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256) + px_bytes(s)
+  return tc_forward_supported(s0) ? align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256) +
+                                        align_up(px_bytes(s), 256) + (x3_shape(s) ? 2 * half_bytes(s) : 0)
                                   : 0;
 }
 
@@ -828,9 +901,12 @@ cudaError_t tc_stats(const Shape& s0, const void* x, const float* W, const float
   const Shape s = tc_padded(s0);
   uint8_t* wimg = static_cast<uint8_t*>(prep);
   uint8_t* px = wimg + align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256);
+  uint8_t* xh = px + align_up(px_bytes(s), 256);
   cudaError_t e = prep_w(s, s0.G, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
-  return run_stats(s, x, wimg, lse, px, status, st);
+  if (!x3_shape(s)) return run_stats(s, x, nullptr, wimg, lse, px, status, st);
+  if ((e = split_points(s, x, xh, st)) != cudaSuccess) return e;
+  return run_stats(s, xh, xh + half_bytes(s), wimg, lse, px, status, st);
 }
 
 cudaError_t tc_slice_fwd(const Shape& s0, const void* x, const void* f, const float* W, const float* bias,
@@ -839,26 +915,43 @@ cudaError_t tc_slice_fwd(const Shape& s0, const void* x, const void* f, const fl
   const Shape s = tc_padded(s0);
   uint8_t* wimg = static_cast<uint8_t*>(prep);
   uint8_t* px = wimg + align_up(w_image_bytes(s), 256);
+  uint8_t* xh = px + align_up(px_bytes(s), 256);
+  uint8_t* fh = xh + 2 * half_bytes(s);
   cudaError_t e = prep_w(s, s0.G, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
-  if ((e = run_stats(s, x, wimg, lse, px, status, st)) != cudaSuccess) return e;
-  return run_slice(s, s0.G, x, f, wimg, px, tokens, wsum, finalize, part, status, st);
+  const void *xr = nullptr, *fr = nullptr;
+  if (x3_shape(s)) {
+    if ((e = split_points(s, x, xh, st)) != cudaSuccess) return e;
+    if ((e = split_points(s, f, fh, st)) != cudaSuccess) return e;
+    x = xh;
+    xr = xh + half_bytes(s);
+    f = fh;
+    fr = fh + half_bytes(s);
+  }
+  if ((e = run_stats(s, x, xr, wimg, lse, px, status, st)) != cudaSuccess) return e;
+  return run_slice(s, s0.G, x, f, xr, fr, wimg, px, tokens, wsum, finalize, part, status, st);
 }
 
-// The slice on prepared operands: the W image and the point-extra rows at px.
-cudaError_t run_slice(const Shape& s, int G, const void* x, const void* f, const uint8_t* wimg, void* px,
-                      float* tokens, float* wsum, int finalize, float* part, uint32_t* status, cudaStream_t st) {
+// The slice on prepared operands: the W image and the point-extra rows at px; xr and
+// fr the residual halves of x and fx (X3), else null.
+cudaError_t run_slice(const Shape& s, int G, const void* x, const void* f, const void* xr, const void* fr,
+                      const uint8_t* wimg, void* px, float* tokens, float* wsum, int finalize, float* part,
+                      uint32_t* status, cudaStream_t st) {
   cudaError_t e;
-  CUtensorMap xmap, fmap, pmap;
+  const bool x3 = xr != nullptr;
+  CUtensorMap xmap, fmap, pmap, xrmap, frmap;
   if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
   if (!make_point_map(&fmap, f, s, 16, CU_TENSOR_MAP_SWIZZLE_32B)) return cudaErrorInvalidValue;
   if (!make_px_map(&pmap, px, s.BH(), padded_n(s))) return cudaErrorInvalidValue;
+  if (!make_point_map(&xrmap, x3 ? xr : x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
+  if (!make_point_map(&frmap, x3 ? fr : f, s, 16, CU_TENSOR_MAP_SWIZZLE_32B)) return cudaErrorInvalidValue;
   const int R = slice_blocks(s), P = slice_splits(s);
   dim3 grid((unsigned)R, (unsigned)P, (unsigned)s.BH());
-  const size_t sm = smem_slice();
-  const auto kernel = s.dot == FS_DOT_BF16X2 ? k_slice<true> : k_slice<false>;
+  const size_t sm = smem_slice(x3);
+  const auto kernel = x3 ? k_slice<true, true> : (s.dot == FS_DOT_BF16X2 ? k_slice<true, false> : k_slice<false, false>);
   if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
-  kernel<<<grid, kThreads, sm, st>>>(xmap, fmap, pmap, wimg, part, s.N, padded_n(s), s.H, s.G, P, status);
+  kernel<<<grid, kThreads, sm, st>>>(xmap, fmap, pmap, xrmap, frmap, wimg, part, s.N, padded_n(s), s.H, s.G, P,
+                                     status);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   Shape so = s;
   so.G = G;
@@ -871,40 +964,64 @@ cudaError_t tc_slice_fwd_lse(const Shape& s0, const void* x, const void* f, cons
   const Shape s = tc_padded(s0);
   uint8_t* wimg = static_cast<uint8_t*>(prep);
   uint8_t* px = wimg + align_up(w_image_bytes(s), 256);
+  uint8_t* xh = px + align_up(px_bytes(s), 256);
+  uint8_t* fh = xh + 2 * half_bytes(s);
   cudaError_t e = prep_w(s, s0.G, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
   const int64_t Np = padded_n(s), npx = s.BH() * Np;
   k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(px), s.BH(), s.N, Np);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  return run_slice(s, s0.G, x, f, wimg, px, tokens, wsum, finalize, part, status, st);
+  const void *xr = nullptr, *fr = nullptr;
+  if (x3_shape(s)) {
+    if ((e = split_points(s, x, xh, st)) != cudaSuccess) return e;
+    if ((e = split_points(s, f, fh, st)) != cudaSuccess) return e;
+    x = xh;
+    xr = xh + half_bytes(s);
+    f = fh;
+    fr = fh + half_bytes(s);
+  }
+  return run_slice(s, s0.G, x, f, xr, fr, wimg, px, tokens, wsum, finalize, part, status, st);
 }
 
 cudaError_t tc_deslice_fwd(const Shape& s0, const void* x, const float* W, const float* bias, const float* tau,
                            const float* zp, const float* lse, void* out, void* prep, uint32_t* status,
                            cudaStream_t st) {
   const Shape s = tc_padded(s0);
+  const bool x3 = x3_shape(s);
   uint8_t* wimg = static_cast<uint8_t*>(prep);
   uint8_t* zimg = wimg + align_up(w_image_bytes(s), 256);
   uint8_t* px = zimg + align_up(z_image_bytes(s), 256);
+  uint8_t* xh = px + align_up(px_bytes(s), 256);
   cudaError_t e = prep_w(s, s0.G, W, bias, tau, wimg, status, st);
   if (e != cudaSuccess) return e;
   const int64_t nz = s.BH() * s.G * kD;
-  k_prep_z<<<(unsigned)((nz + 255) / 256), 256, 0, st>>>(zp, zimg, s.BH(), s0.G, s.G);
+  // With split products the image holds z' hi then its residual (G*128 bytes per (b,h)).
+  const bool ps = x3;
+  if (ps)
+    k_prep_z2<<<(unsigned)((nz + 255) / 256), 256, 0, st>>>(zp, kD, zimg, s.BH(), s0.G, s.G);
+  else
+    k_prep_z<<<(unsigned)((nz + 255) / 256), 256, 0, st>>>(zp, zimg, s.BH(), s0.G, s.G);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   const int64_t Np = padded_n(s), npx = s.BH() * Np;
   k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(px), s.BH(), s.N, Np);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  CUtensorMap xmap, pmap;
-  if (!make_point_map(&xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
+  if (x3 && (e = split_points(s, x, xh, st)) != cudaSuccess) return e;
+  CUtensorMap xmap, pmap, xrmap;
+  if (!make_point_map(&xmap, x3 ? xh : x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B)) return cudaErrorInvalidValue;
+  if (!make_point_map(&xrmap, x3 ? xh + half_bytes(s) : x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B))
+    return cudaErrorInvalidValue;
   if (!make_px_map(&pmap, px, s.BH(), Np)) return cudaErrorInvalidValue;
   const int P = point_splits(s, (int)s.BH());
-  const bool hilo = s.dot == FS_DOT_BF16X2 && smem_deslice(s.G, true) <= kMaxSmem;  // up to G = 768
-  const size_t sm = smem_deslice(s.G, hilo);
+  const bool split = s.dot == FS_DOT_BF16X2 || x3;
+  const bool hilo = split && smem_deslice(s.G, true, 0, ps, x3) <= kMaxSmem;  // up to G = 768 (bf16)
+  const size_t sm = smem_deslice(s.G, hilo, 0, ps, x3);
+  if (sm > kMaxSmem) return cudaErrorInvalidValue;
   dim3 grid((unsigned)P, (unsigned)s.BH());
-  if ((e = set_smem(k_deslice<0, false>, sm)) != cudaSuccess) return e;
-  k_deslice<0, false><<<grid, kThreads, sm, st>>>(xmap, pmap, wimg, zimg, static_cast<__nv_bfloat16*>(out), nullptr,
-                                                  nullptr, nullptr, nullptr, s.N, Np, s.H, s.G, P, hilo ? 1 : 0,
-                                                  (uint32_t)s.G * 64, status);
+  const auto kernel = x3 ? k_deslice<0, true, true> : k_deslice<0, false>;
+  if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
+  kernel<<<grid, kThreads, sm, st>>>(xmap, pmap, xrmap, wimg, zimg, static_cast<__nv_bfloat16*>(out), nullptr,
+                                     nullptr, nullptr, nullptr, s.N, Np, s.H, s.G, P, hilo ? 1 : 0,
+                                     (uint32_t)s.G * (ps ? 128 : 64), status);
   return cudaGetLastError();
 }
 
@@ -928,7 +1045,7 @@ cudaError_t tc_rows_bwd(const Shape& s, int mode, const void* x, const uint8_t* 
                                 : (ps ? k_deslice<2, true> : k_deslice<2, false>);
   cudaError_t e = set_smem(kernel, sm);
   if (e != cudaSuccess) return e;
-  kernel<<<grid, kThreads, sm, st>>>(xmap, pmap, wimg, zimg, static_cast<__nv_bfloat16*>(dfx),
+  kernel<<<grid, kThreads, sm, st>>>(xmap, pmap, xmap, wimg, zimg, static_cast<__nv_bfloat16*>(dfx),
                                      static_cast<const __nv_bfloat16*>(v), delta, wds, dS, s.N, Np, s.H, s.G, P,
                                      hilo ? 1 : 0, (uint32_t)s.G * 128, status);
   return cudaGetLastError();
