@@ -44,10 +44,23 @@
  *    points are reduced in a fixed order, so repeated calls on the same
  *    device agree bit for bit.
  *  - Supported: d in {16, 32, 64}; G in [1, 4096]; B*H <= 65535; B*N*H*d < 2^40.
- *    Precision: FS_F32 computes every product in fp32 FMA; FS_BF16 computes
- *    the point-by-slot products on bf16 tensor cores with fp32 accumulation
- *    (bf16 operands, the paper's "bf16" dot level, Appendix G.2 Table of dot
- *    levels) where a tensor-core kernel exists for the shape, else in fp32.
+ *    Kernels (fs_path_for_shape, fs_backward_path_for_shape say which):
+ *      FS_BF16, d = 32, G <= 1024: tcgen05 tensor cores, fp32 accumulation, at
+ *        the dot level of fs_shape.dot (below); the backward on tensor cores for
+ *        G <= 640 (always with split products), else in fp32 FMA.
+ *      FS_F32, d = 32, G <= 512, B*N*H*G >= 2^24: the forward on tensor cores
+ *        with every operand split into two bf16 halves (normwise relative error
+ *        ~1e-5); the backward in fp32 FMA.
+ *      everything else: fp32 FMA (SIMT) kernels.
+ *
+ * Call sequence of one coupling (a training step):
+ *   fs_slice_fwd   (x_mid, fx)            -> tokens, wsum, lse
+ *   fs_mix         (M, tokens)            -> tokens_mixed   (or fs_mix_channels)
+ *   fs_deslice_fwd (x_mid, tokens_mixed, lse) -> out
+ *   fs_deslice_bwd (..., dout)            -> d_tokens_mixed, dx_mid, dW, dbias, dtau
+ *   fs_mix_bwd     (M, tokens, d_tokens_mixed) -> d_tokens, dM
+ *   fs_slice_bwd   (..., d_tokens, accumulate = 1) -> dfx; adds to dx_mid, dW, dbias, dtau
+ * Each call that takes `ws` gets scratch sized by fs_workspace_bytes for its op.
  */
 #ifndef FLASHSLICE_H
 #define FLASHSLICE_H
@@ -85,7 +98,8 @@ typedef enum fs_dtype { FS_F32 = 0, FS_BF16 = 1 } fs_dtype;
  *                 which the temperature gradient needs (a near-cancelling sum).
  *                 Slower: two more K-steps per logits block, twice the slice
  *                 products.
- * Ignored for FS_F32 shapes and on the SIMT path (fp32 FMA). */
+ * Ignored for FS_F32 shapes (split into bf16 halves on the tensor cores, or
+ * fp32 FMA) and on the SIMT path. */
 typedef enum fs_dot { FS_DOT_BF16 = 0, FS_DOT_BF16X2 = 1 } fs_dot;
 
 typedef struct fs_shape {
