@@ -1,6 +1,8 @@
 // SIMT fp32 kernels: every step of the coupling with fp32 FMA products and fp32
-// accumulation.  They serve fp32 inputs (the paper's default "ieee" dot level,
-// Appendix G.2) and every shape the tensor-core kernels do not cover.
+// accumulation (the paper's "ieee" dot level, Appendix G.2).  They serve every
+// shape the tensor-core kernels do not cover (d != 32, G above their limits, small
+// fp32 problems, the backward of fp32 inputs), and the small steps every path
+// shares: the fixed-order reductions, the mixes and their backward.
 //
 // Ownership follows the paper's G-blocked family (Appendix G.1): a statistics
 // pass per point; slot-owned split-N partial numerators and weight sums with a

@@ -1,4 +1,10 @@
-// Tensor-core forward path for bf16 inputs on sm_103a (tcgen05 + TMEM + TMA).
+// Tensor-core forward path on sm_103a (tcgen05 + TMEM + TMA), and the rows pass
+// of the backward (the deslice kernel in modes 1 and 2, see k_deslice).
+//
+// Inputs: bf16 point tensors as they are; fp32 point tensors split beforehand
+// into bf16 hi and residual tensors (k_split_bf16), with the residual products
+// added in the X3 instantiations.  G is padded to whole 128-slot blocks whose
+// padding slots carry weight 0.
 //
 // The three streaming passes of the paper's G-blocked family (Appendix G.1):
 //   k_stats   : per point and head, lse_n = log sum_g exp(a_ng)        (point-owned)
