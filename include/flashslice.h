@@ -117,7 +117,8 @@ typedef enum fs_op {
   FS_OP_SLICE_FWD = 0,
   FS_OP_DESLICE_FWD = 1,
   FS_OP_DESLICE_BWD = 2,
-  FS_OP_SLICE_BWD = 3
+  FS_OP_SLICE_BWD = 3,
+  FS_OP_STATS = 4
 } fs_op;
 
 /* Bytes of scratch `ws` that entry point `op` needs for this shape on the
@@ -134,6 +135,16 @@ fs_status fs_slice_fwd(const fs_shape* s, const void* x_mid, const void* fx,
                        const float* W_slice, const float* bias, const float* tau,
                        float* tokens, float* wsum, float* lse, int finalize,
                        void* ws, size_t ws_bytes, fs_stream_t stream);
+
+/* The statistics pass alone (App. G.1, the per-point statistic of the G-blocked
+ * kernels): lse [B,H,N] (natural log) of the logits of these weights, exactly as
+ * fs_slice_fwd writes it.  With fs_slice_fwd_lse it splits fs_slice_fwd in two,
+ * so that fx can still be on its way to the device while the statistics run;
+ * it also gives an untied deslice or a FrozenSlice layer its statistics.
+ * ws: FS_OP_STATS's workspace. */
+fs_status fs_stats(const fs_shape* s, const void* x_mid, const float* W_slice,
+                   const float* bias, const float* tau, float* lse, void* ws,
+                   size_t ws_bytes, fs_stream_t stream);
 
 /* Slice given its statistics: fs_slice_fwd with lse [B,H,N] an input (as
  * fs_slice_fwd writes it, natural log) and no statistics pass.  For the

@@ -81,6 +81,9 @@ Regions regions(const Shape& s, int op) {
       r.stats = take(pts * sizeof(float));
       r.tc = take(tc_deslice_prep_bytes(s));
       break;
+    case FS_OP_STATS:
+      r.tc = take(tc_deslice_prep_bytes(s));
+      break;
     case FS_OP_DESLICE_BWD:
       if (tc_backward_supported(s)) {
         r.stats = take(pts * sizeof(float));
@@ -237,6 +240,21 @@ fs_status fs_slice_fwd(const fs_shape* s, const void* x_mid, const void* fx, con
   FS_CUDA(simt_slice_partials(sh, P, x_mid, fx, W_slice, bias, tau, lse_buf, part, status, st));
   FS_CUDA(simt_reduce_tokens(sh, P, part, sh.G, tokens, wsum, finalize, st));
   return FS_OK;
+}
+
+fs_status fs_stats(const fs_shape* s, const void* x_mid, const float* W_slice, const float* bias, const float* tau,
+                   float* lse, void* ws, size_t ws_bytes, fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(x_mid); FS_CHECK_PTR(W_slice); FS_CHECK_PTR(bias); FS_CHECK_PTR(tau); FS_CHECK_PTR(lse);
+  const Shape sh = to_shape(s);
+  if (fs_status e = check_ws(sh, FS_OP_STATS, ws, ws_bytes)) return e;
+  const Regions r = regions(sh, FS_OP_STATS);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  uint32_t* status = at<uint32_t>(ws, r.status);
+  FS_CUDA(reset_status(ws, st));
+  if (tc_forward_supported(sh))
+    return cuda_status(tc_stats(sh, x_mid, W_slice, bias, tau, lse, at<void>(ws, r.tc), status, st));
+  return cuda_status(simt_stats(sh, x_mid, W_slice, bias, tau, lse, status, st));
 }
 
 fs_status fs_slice_fwd_lse(const fs_shape* s, const void* x_mid, const void* fx, const float* W_slice,

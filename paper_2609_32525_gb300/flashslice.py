@@ -29,12 +29,12 @@ FS_OK, FS_ERR_INVALID, FS_ERR_UNSUPPORTED, FS_ERR_CUDA, FS_ERR_TIMEOUT, FS_ERR_B
 FS_NOALLOC_SCRATCH_BYTES = 16 << 20
 FS_F32, FS_BF16 = 0, 1
 FS_DOT_BF16, FS_DOT_BF16X2 = 0, 1
-FS_OP_SLICE_FWD, FS_OP_DESLICE_FWD, FS_OP_DESLICE_BWD, FS_OP_SLICE_BWD = range(4)
+FS_OP_SLICE_FWD, FS_OP_DESLICE_FWD, FS_OP_DESLICE_BWD, FS_OP_SLICE_BWD, FS_OP_STATS = range(5)
 
 EXPORTED = ("fs_workspace_bytes", "fs_slice_fwd", "fs_slice_finalize", "fs_mix", "fs_deslice_fwd",
             "fs_deslice_bwd", "fs_mix_bwd", "fs_slice_bwd", "fs_device_status", "fs_status_string",
             "fs_path_for_shape", "fs_backward_path_for_shape", "fs_forward_launch_count", "fs_slice_fwd_noalloc",
-            "fs_slice_fwd_lse", "fs_mix_channels", "fs_mix_channels_bwd")
+            "fs_slice_fwd_lse", "fs_mix_channels", "fs_mix_channels_bwd", "fs_stats")
 
 
 class fs_shape(ctypes.Structure):
@@ -57,6 +57,7 @@ _sig = {
     "fs_slice_fwd": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _Z, _P]),
     "fs_slice_fwd_lse": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _I, _P, _Z, _P]),
     "fs_slice_finalize": (_I, [_S, _P, _P, _P]),
+    "fs_stats": (_I, [_S, _P, _P, _P, _P, _P, _P, _Z, _P]),
     "fs_mix_channels": (_I, [_S, _P, _P, _P, _P]),
     "fs_mix_channels_bwd": (_I, [_S, _P, _P, _P, _P, _P, _P]),
     "fs_mix": (_I, [_S, _P, _P, _P, _P]),
@@ -139,6 +140,12 @@ def fs_slice_fwd(shape, x_mid, fx, W_slice, bias, tau, tokens, wsum, lse, finali
                            _ptr(tokens), _ptr(wsum), _ptr(lse), int(bool(finalize)), _ptr(ws), ws.numel(),
                            _stream(stream))
     _check("fs_slice_fwd", st)
+
+
+def fs_stats(shape, x_mid, W_slice, bias, tau, lse, ws, stream=None):
+    st = _lib.fs_stats(ctypes.byref(shape), _ptr(x_mid), _ptr(W_slice), _ptr(bias), _ptr(tau), _ptr(lse), _ptr(ws),
+                       ws.numel(), _stream(stream))
+    _check("fs_stats", st)
 
 
 def fs_slice_fwd_lse(shape, x_mid, fx, W_slice, bias, tau, lse, tokens, wsum, finalize, ws, stream=None):

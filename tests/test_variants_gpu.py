@@ -114,3 +114,27 @@ def test_frozen_slice_with_layer1_statistics(lib, case):
     # the weight sums do not depend on fx: the same as layer 1's
     _check("wsum vs layer 1", host(wsum2), host(ws1), dt)
     _check("tokens vs fs_slice_fwd", host(tok2), host(tok2b), dt)
+
+
+@pytest.mark.parametrize("case", CASES, ids=IDS)
+def test_stats_alone_matches_the_slice_call(lib, case):
+    """fs_stats writes the same lse as fs_slice_fwd (the same kernels), and
+    fs_stats + fs_slice_fwd_lse gives the same tokens as fs_slice_fwd."""
+    B, N, H, d, G, dt = case
+    wl = make_case(B, N, H, d, G, dtype=dt, seed=960 + G, backward=False)
+    dev = upload(wl)
+    s = lib.shape_of(dev["x_mid"], G, wl.eps)
+    f32 = dict(dtype=torch.float32, device="cuda")
+    ws, ws_st = lib.workspace(s, lib.FS_OP_SLICE_FWD), lib.workspace(s, lib.FS_OP_STATS)
+    tok, wsum, lse = torch.empty(B, H, G, d, **f32), torch.empty(B, H, G, **f32), torch.empty(B, H, N, **f32)
+    lib.fs_slice_fwd(s, dev["x_mid"], dev["fx"], dev["W_slice"], dev["bias"], dev["tau"], tok, wsum, lse, True, ws)
+    lse2 = torch.full_like(lse, float("nan"))
+    lib.fs_stats(s, dev["x_mid"], dev["W_slice"], dev["bias"], dev["tau"], lse2, ws_st)
+    tok2, wsum2 = torch.empty_like(tok), torch.empty_like(wsum)
+    lib.fs_slice_fwd_lse(s, dev["x_mid"], dev["fx"], dev["W_slice"], dev["bias"], dev["tau"], lse2, tok2, wsum2, True,
+                         ws)
+    torch.cuda.synchronize()
+    assert lib.fs_device_status(ws_st) == lib.FS_OK and lib.fs_device_status(ws) == lib.FS_OK
+    assert torch.equal(lse, lse2)
+    _check("tokens", host(tok2), host(tok), dt)
+    _check("wsum", host(wsum2), host(wsum), dt)
