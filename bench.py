@@ -380,6 +380,99 @@ def run_train(args, wl, dev, world, rank):
         dist.destroy_process_group()
 
 
+VARIANTS = ("tied", "untied", "frozen", "notokenattn")
+
+
+def run_variant(args, wl, dev, world, rank):
+    """One coupling forward of a variant of Sec. 3 (the variants table) on a forward
+    workload, through the same C-ABI calls:
+      untied      fs_slice_fwd, fs_mix, fs_deslice_fwd with its own (W', beta', tau')
+                  and lse = NULL (the deslice computes its own statistics);
+      frozen      a later layer slicing its own features fx2 with the layer-1 weights
+                  and statistics: fs_slice_fwd_lse (no statistics pass), fs_mix,
+                  fs_deslice_fwd with the layer-1 lse;
+      notokenattn fs_slice_fwd, fs_mix_channels (a d x d map per head), fs_deslice_fwd.
+    Timed like the default line (CUDA events on the launching stream, max over
+    ranks); its work is the tied step's (8*C*G flops per point: the statistics a
+    call recomputes are not algorithmic work)."""
+    import torch
+
+    from paper_2609_32525_gb300 import flashslice as fs
+    from paper_2609_32525_gb300 import sharding
+
+    tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+
+    def put(a, dt):
+        return torch.from_numpy(a).to(device=dev, dtype=dt).contiguous()
+
+    x, fx = put(wl.x_mid, tdt), put(wl.fx, tdt)
+    W, b, t, M = (put(getattr(wl, k), torch.float32) for k in ("W_slice", "bias", "tau", "M"))
+    c = fs.Coupling(wl.B, wl.N, wl.H, wl.d, wl.G, tdt, wl.eps, device=dev)
+    s = c.shape
+    stream = torch.cuda.current_stream()
+    g = torch.Generator(device=dev)
+    g.manual_seed(2609)
+    f32 = dict(dtype=torch.float32, device=dev)
+    # the second weight set, the later layer's features and the channel map, seeded:
+    # W' ~ N(0, 1/d), beta' = 0, tau' = 0.7; fx2 ~ N(0, 1); Wc = I + N(0, 0.01)
+    W2 = torch.randn(W.shape, generator=g, **f32) / wl.d ** 0.5
+    b2, t2 = torch.zeros_like(b), torch.full_like(t, 0.7)
+    fx2 = torch.randn(fx.shape, generator=g, **f32).to(tdt)
+    Wc = torch.eye(wl.d, **f32).expand(wl.H, wl.d, wl.d) + 0.1 * torch.randn(wl.H, wl.d, wl.d, generator=g, **f32)
+    Wc = Wc.contiguous()
+    lse1 = torch.empty_like(c.lse)
+    fs.fs_slice_fwd(s, x, fx, W, b, t, c.tokens, c.wsum, lse1, True, c.ws_slice)  # layer 1's statistics
+
+    def step():
+        if args.variant == "untied":
+            fs.fs_slice_fwd(s, x, fx, W, b, t, c.tokens, c.wsum, c.lse, True, c.ws_slice)
+            fs.fs_mix(s, M, c.tokens, c.tokens_mixed)
+            fs.fs_deslice_fwd(s, x, W2, b2, t2, c.tokens_mixed, None, c.out, c.ws_deslice)
+        elif args.variant == "frozen":
+            fs.fs_slice_fwd_lse(s, x, fx2, W, b, t, lse1, c.tokens, c.wsum, True, c.ws_slice)
+            fs.fs_mix(s, M, c.tokens, c.tokens_mixed)
+            fs.fs_deslice_fwd(s, x, W, b, t, c.tokens_mixed, lse1, c.out, c.ws_deslice)
+        elif args.variant == "notokenattn":
+            fs.fs_slice_fwd(s, x, fx, W, b, t, c.tokens, c.wsum, c.lse, True, c.ws_slice)
+            fs.fs_mix_channels(s, Wc, c.tokens, c.tokens_mixed)
+            fs.fs_deslice_fwd(s, x, W, b, t, c.tokens_mixed, c.lse, c.out, c.ws_deslice)
+        else:
+            fs.fs_slice_fwd(s, x, fx, W, b, t, c.tokens, c.wsum, c.lse, True, c.ws_slice)
+            fs.fs_mix(s, M, c.tokens, c.tokens_mixed)
+            fs.fs_deslice_fwd(s, x, W, b, t, c.tokens_mixed, c.lse, c.out, c.ws_deslice)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if c.device_status() != fs.FS_OK:
+        raise RuntimeError("device status after warm-up: " + fs.status_string(c.device_status()))
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(None)
+    time.sleep(0.3)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        step()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = sharding.job_time_ms(t0.elapsed_time(t1), dev) / args.steps
+    assert c.device_status() == fs.FS_OK
+    alg, peaks = _algorithmic(wl), _peaks()
+    roof_t = max(alg["flops"] / (peaks["bf16_tflops"] * 1e12), alg["bytes"] / (peaks["hbm_gbs"] * 1e9))
+    line = {"metric": "coupling forward Mpoints/s, variant " + args.variant, "value": sharding.job_rate(wl.points, world, ms),
+            "unit": UNIT, "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
+            "data": "synthetic (seeded; " + wl.recipe + ")",
+            "config": {"workload": wl.name, "variant": args.variant, "B": wl.B, "N": wl.N, "H": wl.H, "d": wl.d,
+                       "G": wl.G, "parallelism": f"replicas x{world}"},
+            "clocks": clocks, "step_frac": roof_t / (ms * 1e-3)}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -387,6 +480,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="large_g_bf16")
+    ap.add_argument("--variant", default=None, choices=VARIANTS,
+                    help="time one coupling variant of the forward workload instead (Sec. 3 variants table)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--ref-points", type=int, default=16384)
@@ -423,6 +518,8 @@ def main():
     wl = make_named(args.workload, n_override=args.points)
     if wl.dout is not None:
         return run_train(args, wl, dev, world, rank)
+    if args.variant is not None:
+        return run_variant(args, wl, dev, world, rank)
     tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
 
     def put(a, dt):

@@ -7,8 +7,15 @@ point_range(N, r, R) of every batch:
   2. allreduce_partials(U, S): the sums over all points (the one exchange step,
      B*H*G*(d+1) floats: 33 KB at H = 8, G = 32, d = 32);
   3. fs_slice_finalize, fs_mix, then fs_deslice_fwd on the local points.
-The backward exchanges d_tokens_mixed the same way before fs_mix_bwd and
-fs_slice_bwd, and sums the parameter gradients at the end.
+The point-sharded backward, given each rank's dO of its points:
+  4. fs_deslice_bwd on the local points: a partial d_tokens_mixed (its points'
+     share of the sum over n), the local dx_mid and partial dW, dbias, dtau;
+  5. allreduce_sums(d_tokens_mixed): the second exchange, B*H*G*d floats;
+  6. fs_mix_bwd (the same on every rank: its inputs are now global, so dM is the
+     whole gradient and is not exchanged), then fs_slice_bwd on the local
+     points with the global tokens and weight sums: dfx, and dx_mid, dW, dbias,
+     dtau added;
+  7. allreduce_sums(dW, dbias, dtau): the parameter gradients of all points.
 """
 from __future__ import annotations
 
@@ -28,6 +35,13 @@ def allreduce_partials(U: torch.Tensor, S: torch.Tensor, group=None) -> None:
     all ranks in place (before fs_slice_finalize)."""
     dist.all_reduce(U, op=dist.ReduceOp.SUM, group=group)
     dist.all_reduce(S, op=dist.ReduceOp.SUM, group=group)
+
+
+def allreduce_sums(*tensors: torch.Tensor, group=None) -> None:
+    """Sum each tensor over all ranks in place: the backward's partial
+    d_tokens_mixed, and the parameter gradients dW, dbias, dtau at the end."""
+    for t in tensors:
+        dist.all_reduce(t, op=dist.ReduceOp.SUM, group=group)
 
 
 def job_time_ms(local_ms: float, device=None) -> float:

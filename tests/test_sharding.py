@@ -6,6 +6,11 @@
   sharding.allreduce_partials, then finalised. The result must equal the
   unsharded oracle, and so must each rank's deslice of its own points with
   the reduced tokens.
+* The sharded backward: each rank's deslice backward of its points gives a
+  partial d_tokens_mixed, summed across ranks (sharding.allreduce_sums); the mix
+  backward then runs on the global tokens, the slice backward on the rank's
+  points, and dW, dbias, dtau are summed at the end.  Every gradient must equal
+  the unsharded oracle's (dx_mid and dfx on the rank's own points).
 * Job timing: the job time is the maximum of the ranks' times, and the
   job rate counts every rank's points.
 """
@@ -37,7 +42,7 @@ def _worker(rank, port, results):
         from oracle import flashslice_oracle as orc
         from paper_2609_32525_gb300.workloads import make_case
 
-        wl = make_case(2, 1001, 3, 8, 7, dtype="f32", seed=41, backward=False)
+        wl = make_case(2, 1001, 3, 8, 7, dtype="f32", seed=41, backward=True)
         n0, n1 = sharding.point_range(wl.N, rank, WORLD)
         local = orc.slice_fwd(wl.x_mid[:, n0:n1], wl.fx[:, n0:n1], wl.W_slice, wl.bias, wl.tau, eps=wl.eps,
                               finalize=False)
@@ -52,8 +57,27 @@ def _worker(rank, port, results):
         ok_tokens = np.allclose(tokens, ref["tokens"], rtol=1e-12, atol=1e-14)
         ok_wsum = np.allclose(S.numpy(), ref["wsum"], rtol=1e-12, atol=1e-14)
         ok_out = np.allclose(out_local, ref["out"][:, n0:n1], rtol=1e-12, atol=1e-14)
+
+        # backward: exchange the partial d_tokens_mixed, then the parameter gradients
+        x_l, f_l = wl.x_mid[:, n0:n1], wl.fx[:, n0:n1]
+        rd = orc.deslice_bwd(x_l, wl.W_slice, wl.bias, wl.tau, zp, wl.dout[:, n0:n1])
+        dzm = torch.from_numpy(np.ascontiguousarray(rd["d_tokens_mixed"]))
+        sharding.allreduce_sums(dzm)
+        rm = orc.mix_bwd(wl.M, tokens, dzm.numpy())
+        rs = orc.slice_bwd(x_l, f_l, wl.W_slice, wl.bias, wl.tau, tokens, S.numpy(), rm["d_tokens"], eps=wl.eps)
+        grads = [torch.from_numpy(np.ascontiguousarray(rd[k] + rs[k])) for k in ("dW", "dbias", "dtau")]
+        sharding.allreduce_sums(*grads)
+        rb = orc.backward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, wl.dout, eps=wl.eps)
+
+        def close(a, b):
+            return np.allclose(a, b, rtol=1e-10, atol=1e-12)
+
+        ok_bwd = {"dM": close(rm["dM"], rb["dM"]),
+                  "dx_mid": close(rd["dx_mid"] + rs["dx_mid"], rb["dx_mid"][:, n0:n1]),
+                  "dfx": close(rs["dfx"], rb["dfx"][:, n0:n1]),
+                  **{k: close(g.numpy(), rb[k]) for k, g in zip(("dW", "dbias", "dtau"), grads)}}
         t = sharding.job_time_ms(1.0 + rank)
-        results[rank] = (ok_tokens, ok_wsum, ok_out, t, (n0, n1))
+        results[rank] = (ok_tokens, ok_wsum, ok_out, t, (n0, n1), ok_bwd)
     finally:
         dist.destroy_process_group()
 
@@ -75,15 +99,17 @@ def test_single_process_job_time_and_rate():
     assert sharding.job_rate(1_000_000, 4, 10.0) == pytest.approx(400.0)
 
 
-def test_two_gloo_ranks_shard_points_and_time_the_job():
+def test_two_gloo_ranks_shard_points_forward_backward_and_time_the_job():
     port = _free_port()
     with mp.Manager() as mgr:
         results = mgr.dict()
         mp.spawn(_worker, args=(port, results), nprocs=WORLD, join=True)
         res = dict(results)
     assert sorted(res) == list(range(WORLD))
-    for rank, (ok_tokens, ok_wsum, ok_out, t, rng) in res.items():
+    for rank, (ok_tokens, ok_wsum, ok_out, t, rng, ok_bwd) in res.items():
         assert ok_tokens and ok_wsum, f"rank {rank}: reduced tokens differ from the unsharded oracle"
         assert ok_out, f"rank {rank}: local deslice differs"
+        bad = [k for k, ok in ok_bwd.items() if not ok]
+        assert not bad, f"rank {rank}: sharded gradients differ from the unsharded oracle: {bad}"
         assert t == float(WORLD)  # max over ranks of 1 + rank
     assert res[0][4][1] == res[1][4][0]
