@@ -51,7 +51,7 @@ def test_status_strings(fs):
 
 def test_workspace_sizes(fs):
     s = fs.make_shape(1, 4096, 8, 32, 32)
-    for op in range(4):
+    for op in (fs.FS_OP_SLICE_FWD, fs.FS_OP_DESLICE_FWD, fs.FS_OP_DESLICE_BWD, fs.FS_OP_SLICE_BWD, fs.FS_OP_STATS):
         assert fs.workspace_bytes(s, op) >= 256
     assert fs.workspace_bytes(fs.make_shape(1, 4096, 8, 32, 32), 99) == 0
     assert fs.workspace_bytes(fs.make_shape(0, 4096, 8, 32, 32), 0) == 0       # invalid
@@ -85,6 +85,23 @@ def test_validation_rejects_bad_arguments_without_launching(fs):
     # workspace missing or too small
     assert _call_slice(fs, s, good, ws_ptr=0) == fs.FS_ERR_INVALID
     assert _call_slice(fs, s, good, ws_bytes=8) == fs.FS_ERR_INVALID
+
+
+def test_stats_validation(fs):
+    """fs_stats checks its pointers, shape and workspace before any launch."""
+    lib, P = fs._lib, ctypes.c_void_p
+    s = fs.make_shape(1, 100, 2, 32, 8)
+    ptrs = [P(16 * (i + 1)) for i in range(5)]  # fake aligned addresses, never dereferenced
+
+    def call(shape, args, ws=P(16), ws_bytes=1 << 30):
+        return lib.fs_stats(ctypes.byref(shape), *args, ws, ws_bytes, None)
+
+    for i in range(5):
+        assert call(s, ptrs[:i] + [None] + ptrs[i + 1:]) == fs.FS_ERR_INVALID
+    assert call(fs.make_shape(1, 0, 2, 32, 8), ptrs) == fs.FS_ERR_INVALID
+    assert call(fs.make_shape(1, 100, 2, 48, 8), ptrs) == fs.FS_ERR_UNSUPPORTED
+    assert call(s, ptrs, ws=None) == fs.FS_ERR_INVALID
+    assert call(s, ptrs, ws_bytes=fs.workspace_bytes(s, fs.FS_OP_STATS) - 1) == fs.FS_ERR_INVALID
 
 
 def test_mix_rejects_in_place(fs):
