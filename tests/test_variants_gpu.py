@@ -9,7 +9,8 @@ the fp64 oracle:
   input, weights and statistics: fs_slice_fwd_lse with the layer-1 lse, against the
   oracle's slice of fx2 with the layer-1 weights, and against fs_slice_fwd.
 
-Shapes: tensor-core (bf16, d = 32; G = 256 and a padded G = 100) and SIMT (fp32).
+Shapes: tensor-core bf16 (d = 32; G = 256 and a padded G = 100), the fp32 tensor-core
+path (d = 32, G = 128, B*N*H*G >= 2^24: split bf16 halves) and SIMT (fp32, d = 16).
 Tolerances as everywhere: fp32 normwise max relative 1e-4; bf16 relative L2 1e-2.
 """
 import numpy as np
@@ -23,8 +24,9 @@ from _parity import error, host, tol, upload
 
 pytestmark = pytest.mark.gpu
 
-CASES = [(2, 1500, 2, 32, 256, "bf16"), (1, 900, 2, 32, 100, "bf16"), (2, 700, 2, 16, 40, "f32")]
-IDS = ["tc-G256", "tc-G100-padded", "simt-f32"]
+CASES = [(2, 1500, 2, 32, 256, "bf16"), (1, 900, 2, 32, 100, "bf16"), (1, 70000, 2, 32, 128, "f32"),
+         (2, 700, 2, 16, 40, "f32")]
+IDS = ["tc-G256", "tc-G100-padded", "tc-f32-split", "simt-f32"]
 
 
 def _f32(a):
