@@ -349,17 +349,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 // the point-extra row [1, 1, -lse2_hi, -lse2_lo, 0 x 4] (lse2 = lse*log2(e)) to
 // px[bh*Np + n] (Np = N rounded up to a whole tile; padded points get -1e30 so
 // that their weights vanish).
-// Two logits issuers and two softmax warpgroups: block q (tile q / nb, slot block
-// q % nb) goes through S buffer q % 2, issuer 1 + q % 2 and warpgroup q % 2.  Each
-// warpgroup keeps a running (max, sum) over the blocks it took; the two shares of
-// a tile are combined through shared memory by the one that took its last block.
+// Two logits issuers and four softmax warpgroups (640 threads): block q (tile
+// q / nb, slot block q % nb) goes through S buffer p = q % 2, issuer 1 + p and
+// warpgroups 2p and 2p + 1, each of which takes one half (64 slots) of every row,
+// so that each SM sub-partition holds four softmax warps whose exponentials and
+// reductions interleave.  Each warpgroup keeps a running (max, sum) over the slots
+// it took; the four shares of a tile are combined through shared memory by half 0
+// of the pair that took the tile's last block.
 // smem: [W img G*96][x stages][constant extra][ml exchange][barriers]
 // TMEM: two S buffers [0, 256).
 // =========================================================================================
 // X3 (fp32 inputs): x arrives as bf16 hi and residual tiles (xmap, xrmap), one stage
 // holding both, and the logits add x_r W'_hi.
+constexpr int kStatsThreads = 640;
 template <bool split, bool X3>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kStatsThreads, 1)
     k_stats(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap xrmap,
             const uint8_t* __restrict__ wimg, float* __restrict__ lse, uint4* __restrict__ px, int64_t N,
             int64_t Np, int H, int G, int splits, uint32_t* status) {
@@ -371,15 +375,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* s_w = smem;
   uint8_t* s_x = s_w + wbytes;
   uint8_t* s_ex = s_x + kStages * kXSt;
-  float2* s_ml = reinterpret_cast<float2*>(s_ex + kExBytes);  // [2][128] warpgroup-1 partials
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_ml + 2 * kTile);
+  float2* s_ml = reinterpret_cast<float2*>(s_ex + kExBytes);  // [2 tile parities][3 partials][128 rows]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_ml + 6 * kTile);
   uint64_t* w_full = bars;
   uint64_t* x_full = bars + 1;
   uint64_t* x_empty = x_full + kStages;
   uint64_t* s_full = x_empty + kStages;
   uint64_t* s_free = s_full + 2;
-  uint64_t* ml_full = s_free + 2;   // warpgroup 1 partials written   (per tile parity)
-  uint64_t* ml_empty = ml_full + 2; // warpgroup 0 has read them
+  uint64_t* ml_full = s_free + 2;   // the other three warpgroups' partials written (per tile parity)
+  uint64_t* ml_empty = ml_full + 2; // the finalising warpgroup has read them
   uint64_t* drain = ml_empty + 2;   // one per issuing warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 2);
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
@@ -398,8 +402,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < 2; i++) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&s_free[i], 4);
-      mbar_init(&ml_full[i], 4);
+      mbar_init(&s_free[i], 8);
+      mbar_init(&ml_full[i], nch >= 2 ? 12 : 4);
       mbar_init(&ml_empty[i], 4);
     }
     mbar_init(&drain[0], 1);
@@ -462,52 +466,45 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= kSoftmaxWarp0) {
     const int wg = (warp - kSoftmaxWarp0) >> 2;
+    const int pr = wg >> 1, hf = wg & 1;  // S buffer (block parity) and the half of each row
     const int wq = warp & 3;
     const int r = wq * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     const int total = wk.ntiles * nch;
     bool ok = true;
     float m = -INFINITY, l = 0.f;
-    // Warpgroup wg takes the whole blocks q with q % 2 == wg (always S buffer wg), so
-    // the two run out of phase.  A tile's last block is taken by the warpgroup that
-    // finalises the tile; with two or more blocks per tile the other warpgroup hands
-    // over its (max, sum) over the blocks it took.
-    BlockPos pos(wg, nch);
-    for (int q = wg; ok && q < total; q += 2, pos.step(2, nch)) {
+    // The pair of warpgroups of S buffer pr takes the whole blocks q with q % 2 == pr,
+    // warpgroup hf the slots [64 hf, 64 hf + 64) of each.  A tile's last block is taken
+    // by the pair that finalises the tile; there half 0 finalises, and the other three
+    // warpgroups hand over their (max, sum) over the slots they took: the other pair
+    // (with two or more blocks per tile) at its last block of the tile, half 1 at the
+    // tile's last block.
+    BlockPos pos(pr, nch);
+    for (int q = pr; ok && q < total; q += 2, pos.step(2, nch)) {
       const int i = pos.i, c = pos.c;
-      if (!(ok = mbar_wait(&s_full[wg], (uint32_t)((q >> 1) & 1), ab, status))) break;
+      if (!(ok = mbar_wait(&s_full[pr], (uint32_t)((q >> 1) & 1), ab, status))) break;
       tc_fence_after();
-      // The whole row of the block (128 logits) into registers, then S goes back to
-      // the issuer at once; the maximum, the 128 exponentials (independent, issued
-      // back to back) and a pairwise sum follow.
-      const uint32_t tS = tmem + lane_addr + (uint32_t)wg * kGC;
-      uint32_t v[4][32];
+      const uint32_t tS = tmem + lane_addr + (uint32_t)pr * kGC + (uint32_t)hf * 64;
+      uint32_t v[2][32];
       tmem_ld32(tS, v[0]);
       tmem_ld32(tS + 32, v[1]);
-      tmem_ld32(tS + 64, v[2]);
-      tmem_ld32(tS + 96, v[3]);
       tmem_wait_ld2(v[0], v[1]);
-      tmem_wait_ld2(v[2], v[3]);  // ties the other half's registers after the (already complete) wait
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&s_free[wg]);
-      float t[43];
+      if (lane == 0) mbar_arrive(&s_free[pr]);
+      float t[22];
 #pragma unroll
-      for (int k = 0; k < 42; k++)
+      for (int k = 0; k < 21; k++)
         t[k] = max3(__uint_as_float(v[(3 * k) >> 5][(3 * k) & 31]), __uint_as_float(v[(3 * k + 1) >> 5][(3 * k + 1) & 31]),
                     __uint_as_float(v[(3 * k + 2) >> 5][(3 * k + 2) & 31]));
-      t[42] = max3(__uint_as_float(v[3][30]), __uint_as_float(v[3][31]), m);
+      t[21] = fmaxf(__uint_as_float(v[1][31]), m);
 #pragma unroll
-      for (int k = 0; k < 14; k++) t[k] = max3(t[3 * k], t[3 * k + 1], t[3 * k + 2]);
-      t[14] = t[42];
-#pragma unroll
-      for (int k = 0; k < 5; k++) t[k] = max3(t[3 * k], t[3 * k + 1], t[3 * k + 2]);
-      const float mn = max3(max3(t[0], t[1], t[2]), t[3], t[4]);
+      for (int k = 0; k < 7; k++) t[k] = max3(t[3 * k], t[3 * k + 1], t[3 * k + 2]);
+      const float mn = max3(max3(t[0], t[1], t[2]), max3(t[3], t[4], t[5]), fmaxf(t[6], t[21]));
       const uint32_t nmb = __float_as_uint(-mn);
       const uint64_t nm2 = pack2(nmb, nmb);
-      // Paired (f32x2) subtraction, then every exponential, then a pairwise f32x2 sum.
 #pragma unroll
-      for (int j = 0; j < 4; j++)
+      for (int j = 0; j < 2; j++)
 #pragma unroll
         for (int k = 0; k < 16; k++) {
           const uint64_t a = add2(pack2(v[j][2 * k], v[j][2 * k + 1]), nm2);
@@ -517,8 +514,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint64_t acc[16];
 #pragma unroll
       for (int k = 0; k < 16; k++)
-        acc[k] = add2(add2(pack2(v[0][2 * k], v[0][2 * k + 1]), pack2(v[1][2 * k], v[1][2 * k + 1])),
-                      add2(pack2(v[2][2 * k], v[2][2 * k + 1]), pack2(v[3][2 * k], v[3][2 * k + 1])));
+        acc[k] = add2(pack2(v[0][2 * k], v[0][2 * k + 1]), pack2(v[1][2 * k], v[1][2 * k + 1]));
 #pragma unroll
       for (int w = 8; w >= 1; w >>= 1)
 #pragma unroll
@@ -527,24 +523,28 @@ __global__ void __launch_bounds__(kThreads, 1)
       l = l * ex2(m - mn) + sum;
       m = mn;
       const int pb = i & 1;
-      if (c == nch - 2) {
-        // Hand over this warpgroup's share of tile i.
+      const bool last = c == nch - 1;
+      if ((c == nch - 2) || (last && hf == 1)) {
+        // Hand over this warpgroup's share of tile i: slot hf from the other pair,
+        // slot 2 from half 1 of the finalising pair.
         if (i >= 2 && !(ok = mbar_wait(&ml_empty[pb], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
-        s_ml[pb * kTile + r] = make_float2(m, l);
+        s_ml[(pb * 3 + (last ? 2 : hf)) * kTile + r] = make_float2(m, l);
         __syncwarp();
         if (lane == 0) mbar_arrive(&ml_full[pb]);
         m = -INFINITY;
         l = 0.f;
-      } else if (c == nch - 1) {
-        float M = m, L = l;
+      } else if (last) {
+        if (!(ok = mbar_wait(&ml_full[pb], (uint32_t)((i >> 1) & 1), ab, status))) break;
+        const float2 o2 = s_ml[(pb * 3 + 2) * kTile + r];
+        float2 o0 = make_float2(-INFINITY, 0.f), o1 = o0;
         if (nch >= 2) {
-          if (!(ok = mbar_wait(&ml_full[pb], (uint32_t)((i >> 1) & 1), ab, status))) break;
-          const float2 o = s_ml[pb * kTile + r];
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&ml_empty[pb]);
-          M = fmaxf(m, o.x);
-          L = l * ex2(m - M) + o.y * ex2(o.x - M);
+          o0 = s_ml[(pb * 3 + 0) * kTile + r];
+          o1 = s_ml[(pb * 3 + 1) * kTile + r];
         }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&ml_empty[pb]);
+        const float M = fmaxf(fmaxf(m, o2.x), fmaxf(o0.x, o1.x));
+        const float L = l * ex2(m - M) + o2.y * ex2(o2.x - M) + o0.y * ex2(o0.x - M) + o1.y * ex2(o1.x - M);
         m = -INFINITY;
         l = 0.f;
         const int64_t n = (wk.tile0 + i) * kTile + r;
@@ -823,7 +823,7 @@ size_t smem_deslice(int G, bool hilo, int mode = 0, bool ps = false, bool x3 = f
          kStages * (kDStage + (x3 ? kXBytes : 0)) + 512;
 }
 size_t smem_stats(int G, bool split, bool x3 = false) {
-  return 1024 + (size_t)G * (split ? kWRow : 96) + kStages * kXBytes * (x3 ? 2 : 1) + kExBytes + 2 * kTile * 8 + 512;
+  return 1024 + (size_t)G * (split ? kWRow : 96) + kStages * kXBytes * (x3 ? 2 : 1) + kExBytes + 6 * kTile * 8 + 512;
 }
 size_t smem_slice(bool x3 = false) {
   return 1024 + (size_t)kWBlock +
@@ -854,7 +854,7 @@ cudaError_t run_stats(const Shape& s, const void* x, const void* xr, const uint8
   const auto kernel = x3 ? k_stats<true, true> : (split ? k_stats<true, false> : k_stats<false, false>);
   cudaError_t e = set_smem(kernel, sm);
   if (e != cudaSuccess) return e;
-  kernel<<<dim3((unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(xmap, xrmap, wimg, lse, static_cast<uint4*>(px),
+  kernel<<<dim3((unsigned)P, (unsigned)s.BH()), kStatsThreads, sm, st>>>(xmap, xrmap, wimg, lse, static_cast<uint4*>(px),
                                                                     s.N, padded_n(s), s.H, s.G, P, status);
   return cudaGetLastError();
 }
