@@ -310,6 +310,20 @@ __device__ __forceinline__ void weights_in_halves(uint32_t tS) {
   }
 }
 
+// One 64-slot half of the row: the log2-weights in columns [0, 64) from tS -> bf16
+// weights packed in pairs into columns [0, 32) from tS, which this thread has read.
+__device__ __forceinline__ void weights_half(uint32_t tS) {
+  uint32_t v0[32], v1[32];
+  tmem_ld32(tS, v0);
+  tmem_ld32(tS + 32, v1);
+  tmem_wait_ld2(v0, v1);
+  uint32_t pk0[16], pk1[16];
+  weights32(v0, pk0);
+  weights32(v1, pk1);
+  tmem_st16(tS, pk0);
+  tmem_st16(tS + 16, pk1);
+}
+
 // The weight helpers above, plus acc += sum over the block's 128 slots of w_g ds[g]
 // (ds: the block's slice of a per-slot array in shared memory; every lane reads
 // the same address, a broadcast).  The backward of the slice needs this sum for

@@ -82,8 +82,16 @@ constexpr uint32_t kDStage = kXBytes + 2 * kPxBytes;  // x tile, point extra (bo
 
 // X3 (fp32 inputs, MODE 0 with PS): each stage also holds x's residual tile
 // (xrmap), the logits add x_r W'_hi, and out is fp32.
+// The forward with single-level products (MODE 0, !PS) runs four softmax
+// warpgroups (640 threads): warpgroups 2p and 2p + 1 take the blocks q with
+// q % 2 == p, each one 64-slot half of every row, and half j's packed weights go to
+// columns [64 j, 64 j + 32) of the S buffer, where product issuer j reads them as
+// soon as half j is ready.  The other modes keep two warpgroups on whole rows.
+template <int MODE, bool PS>
+constexpr bool desl_wg4() { return MODE == 0 && !PS; }
+constexpr int kDesl4Threads = 640;
 template <int MODE, bool PS, bool X3 = false>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThreads, 1)
     k_deslice(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap pmap,
               const __grid_constant__ CUtensorMap xrmap,
               const uint8_t* __restrict__ wimg, const uint8_t* __restrict__ zimg, __nv_bfloat16* __restrict__ out,
@@ -106,8 +114,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* x_full = bars + 1;
   uint64_t* x_empty = x_full + kStages;
   uint64_t* s_full = x_empty + kStages;
-  uint64_t* p_ready = s_full + kSBuf;
-  uint64_t* pv_done = p_ready + kSBuf;
+  constexpr bool kWG4 = desl_wg4<MODE, PS>();
+  uint64_t* p_ready = s_full + kSBuf;  // [kSBuf][2 halves] with four warpgroups, else [kSBuf]
+  uint64_t* pv_done = p_ready + 2 * kSBuf;
   uint64_t* o_full = pv_done + kSBuf;
   uint64_t* o_free = o_full + 2;
   uint64_t* drain = o_free + 2;  // one per issuing warp
@@ -130,7 +139,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < kSBuf; i++) {
       mbar_init(&s_full[i], 1);
-      mbar_init(&p_ready[i], 4);  // the four warps of the warpgroup that owns the block
+      mbar_init(&p_ready[2 * i], 4);  // the four warps of the warpgroup that owns the block (half)
+      mbar_init(&p_ready[2 * i + 1], 4);
       mbar_init(&pv_done[i], 2);
     }
     for (int i = 0; i < 2; i++) {
@@ -212,9 +222,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int ob = i & 1;
         const int bb = q % kSBuf;
         if (c == 0 && i >= 2 && !(ok = mbar_wait_w(&o_free[ob], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
-        if (!(ok = mbar_wait_w(&p_ready[bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
+        if (!(ok = mbar_wait_w(&p_ready[kWG4 ? 2 * bb + j : 2 * bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t tP = tmem + (uint32_t)bb * kGC + (uint32_t)j * 32;  // weights of slots 64j.. (packed pairs)
+        // weights of slots 64j.. (packed pairs)
+        const uint32_t tP = tmem + (uint32_t)bb * kGC + (uint32_t)j * (kWG4 ? 64 : 32);
         const uint32_t tO = tmem + kO + (uint32_t)(j * 2 + ob) * kD;
 #pragma unroll
         for (int kk = 0; kk < 4; kk++) {
@@ -234,7 +245,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp >= kSoftmaxWarp0) {
     // ------------------------------ softmax warpgroups ------------------------------
-    const int wg = (warp - kSoftmaxWarp0) >> 2;
+    const int wg4 = (warp - kSoftmaxWarp0) >> 2;
+    const int wg = kWG4 ? wg4 >> 1 : wg4;  // the block parity this warpgroup takes
+    const int hf = kWG4 ? wg4 & 1 : 0;     // four warpgroups: the half of each row
     const int wq = warp & 3;  // TMEM sub-partition of this warp
     const int r = wq * 32 + lane;
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
@@ -324,18 +337,21 @@ __global__ void __launch_bounds__(kThreads, 1)
           weights_in_halves_ds(tmem + lane_addr + (uint32_t)bb * kGC, s_ds + c * kGC, wds_acc);
       } else if (PS) {
         weights_hilo_in_place(tmem + lane_addr + (uint32_t)bb * kGC);
+      } else if (kWG4) {
+        weights_half(tmem + lane_addr + (uint32_t)bb * kGC + (uint32_t)hf * 64);
       } else {
         weights_in_halves(tmem + lane_addr + (uint32_t)bb * kGC);
       }
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&p_ready[bb]);
-      // The output of the previous tile is drained by the warpgroup that took the
-      // first block of this tile, when the last products of that tile have long finished.
-      if (c == 0 && i > 0 && !(ok = epilogue(i - 1))) break;
+      if (lane == 0) mbar_arrive(&p_ready[2 * bb + hf]);
+      // The output of the previous tile is drained by the warpgroup (half 0 of the
+      // pair) that took the first block of this tile, when the last products of that
+      // tile have long finished.
+      if (c == 0 && i > 0 && hf == 0 && !(ok = epilogue(i - 1))) break;
     }
-    if (ok && total > 0 && total % 2 == wg) epilogue(wk.ntiles - 1);
+    if (ok && total > 0 && total % 2 == wg && hf == 0) epilogue(wk.ntiles - 1);
     if (ok) flush_wds();
   }
   tc_fence_before();
@@ -1025,7 +1041,7 @@ cudaError_t tc_deslice_fwd(const Shape& s0, const void* x, const float* W, const
   dim3 grid((unsigned)P, (unsigned)s.BH());
   const auto kernel = x3 ? k_deslice<0, true, true> : k_deslice<0, false>;
   if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
-  kernel<<<grid, kThreads, sm, st>>>(xmap, pmap, xrmap, wimg, zimg, static_cast<__nv_bfloat16*>(out), nullptr,
+  kernel<<<grid, x3 ? kThreads : kDesl4Threads, sm, st>>>(xmap, pmap, xrmap, wimg, zimg, static_cast<__nv_bfloat16*>(out), nullptr,
                                      nullptr, nullptr, nullptr, s.N, Np, s.H, s.G, P, hilo ? 1 : 0,
                                      (uint32_t)s.G * (ps ? 128 : 64), status);
   return cudaGetLastError();
