@@ -163,7 +163,8 @@ fs_status fs_slice_finalize(const fs_shape* s, float* tokens, const float* wsum,
                             fs_stream_t stream);
 
 /* Constant token mix, the core of Eq. (1) acting on the slot index:
- * tokens_mixed[b,h,g,:] = sum_k M[h,g,k] tokens[b,h,k,:].  Out-of-place only. */
+ * tokens_mixed[b,h,g,:] = sum_k M[h,g,k] tokens[b,h,k,:].  Out-of-place only: an
+ * output that shares any byte with an input is rejected (FS_ERR_INVALID). */
 fs_status fs_mix(const fs_shape* s, const float* M, const float* tokens,
                  float* tokens_mixed, fs_stream_t stream);
 
@@ -171,13 +172,15 @@ fs_status fs_mix(const fs_shape* s, const float* M, const float* tokens,
  * variants table): A is the identity, so the tokens do not interact, and a
  * learned linear map acts on the channels of each token, one per head:
  * tokens_mixed[b,h,g,c] = sum_k Wc[h,c,k] tokens[b,h,g,k].  Wc [H,d,d] fp32.
- * Out-of-place only.  It may replace fs_mix, or follow it (the two commute). */
+ * Out-of-place only (overlapping input and output: FS_ERR_INVALID).  It may
+ * replace fs_mix, or follow it (the two commute). */
 fs_status fs_mix_channels(const fs_shape* s, const float* Wc, const float* tokens,
                           float* tokens_mixed, fs_stream_t stream);
 
 /* Backward of fs_mix_channels: d_tokens[b,h,g,k] = sum_c Wc[h,c,k]
  * d_tokens_mixed[b,h,g,c] (overwritten); dWc [H,d,d] = sum over b and g of
- * d_tokens_mixed tokens^T (overwritten). */
+ * d_tokens_mixed tokens^T (overwritten).  Outputs that overlap an input or each
+ * other: FS_ERR_INVALID. */
 fs_status fs_mix_channels_bwd(const fs_shape* s, const float* Wc, const float* tokens,
                               const float* d_tokens_mixed, float* d_tokens, float* dWc,
                               fs_stream_t stream);
@@ -210,7 +213,8 @@ fs_status fs_deslice_bwd(const fs_shape* s, const void* x_mid, const float* W_sl
                          int accumulate, void* ws, size_t ws_bytes, fs_stream_t stream);
 
 /* Backward of the mix: d_tokens = M^T d_tokens_mixed per (b,h) (overwritten);
- * dM [H,G,G] = sum_b d_tokens_mixed tokens^T (overwritten). */
+ * dM [H,G,G] = sum_b d_tokens_mixed tokens^T (overwritten).  Outputs that overlap
+ * an input or each other: FS_ERR_INVALID. */
 fs_status fs_mix_bwd(const fs_shape* s, const float* M, const float* tokens,
                      const float* d_tokens_mixed, float* d_tokens, float* dM,
                      fs_stream_t stream);
@@ -244,7 +248,10 @@ fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx,
  *     unsupported shapes give fs_slice_fwd's errors.
  *   - The first call on a device (with that device current) looks up the
  *     scratch's device address through the CUDA runtime; later calls on that
- *     device reuse it.  Make that first call before any stream capture begins.
+ *     device reuse it while the device's context stays the same.  After a
+ *     cudaDeviceReset, or with another context current, the next call looks the
+ *     address up again.  Make each call that does the lookup (the first one, and
+ *     the first after a reset or context change) before any stream capture.
  *   - Each call clears the status word at the start of the scratch; nothing
  *     else in the scratch has to start at zero.
  *   - There is ONE scratch per device.  Calls that can overlap in time (on

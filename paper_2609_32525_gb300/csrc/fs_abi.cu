@@ -6,6 +6,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstring>
+#include <initializer_list>
 
 namespace fs {
 
@@ -49,6 +50,28 @@ bool supported_shape(const fs_shape* s) {
 Shape to_shape(const fs_shape* s) { return Shape{s->B, s->N, s->H, s->d, s->G, s->dtype, s->eps, s->dot}; }
 
 bool aligned(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// A byte range [p, p + n) of a caller buffer.
+struct Span {
+  const void* p;
+  size_t n;
+};
+// True when two ranges share a byte.
+bool overlap(Span a, Span b) {
+  const uintptr_t a0 = reinterpret_cast<uintptr_t>(a.p), b0 = reinterpret_cast<uintptr_t>(b.p);
+  return a.n && b.n && a0 < b0 + b.n && b0 < a0 + a.n;
+}
+// The out-of-place calls (the mixes and their backward) read every input while
+// they write: no output may share a byte with an input or with another output.
+bool disjoint(std::initializer_list<Span> ins, std::initializer_list<Span> outs) {
+  for (const Span& o : outs) {
+    for (const Span& i : ins)
+      if (overlap(o, i)) return false;
+    for (const Span& o2 : outs)
+      if (&o2 != &o && overlap(o, o2)) return false;
+  }
+  return true;
+}
 
 // Byte sizes of the regions each op places in `ws` (each 256-byte aligned).
 struct Regions {
@@ -289,7 +312,8 @@ fs_status fs_mix(const fs_shape* s, const float* M, const float* tokens, float* 
                  fs_stream_t stream) {
   FS_CHECK_SHAPE(s);
   FS_CHECK_PTR(M); FS_CHECK_PTR(tokens); FS_CHECK_PTR(tokens_mixed);
-  if (tokens == tokens_mixed) return FS_ERR_INVALID;
+  const size_t tb = (size_t)s->B * s->H * s->G * s->d * 4, mb = (size_t)s->H * s->G * s->G * 4;
+  if (!disjoint({{M, mb}, {tokens, tb}}, {{tokens_mixed, tb}})) return FS_ERR_INVALID;
   return cuda_status(simt_mix(to_shape(s), M, tokens, tokens_mixed, reinterpret_cast<cudaStream_t>(stream)));
 }
 
@@ -297,7 +321,8 @@ fs_status fs_mix_channels(const fs_shape* s, const float* Wc, const float* token
                           fs_stream_t stream) {
   FS_CHECK_SHAPE(s);
   FS_CHECK_PTR(Wc); FS_CHECK_PTR(tokens); FS_CHECK_PTR(tokens_mixed);
-  if (tokens == tokens_mixed) return FS_ERR_INVALID;
+  const size_t tb = (size_t)s->B * s->H * s->G * s->d * 4, wb = (size_t)s->H * s->d * s->d * 4;
+  if (!disjoint({{Wc, wb}, {tokens, tb}}, {{tokens_mixed, tb}})) return FS_ERR_INVALID;
   return cuda_status(simt_mix_channels(to_shape(s), Wc, tokens, tokens_mixed, reinterpret_cast<cudaStream_t>(stream)));
 }
 
@@ -305,7 +330,8 @@ fs_status fs_mix_channels_bwd(const fs_shape* s, const float* Wc, const float* t
                               float* d_tokens, float* dWc, fs_stream_t stream) {
   FS_CHECK_SHAPE(s);
   FS_CHECK_PTR(Wc); FS_CHECK_PTR(tokens); FS_CHECK_PTR(d_tokens_mixed); FS_CHECK_PTR(d_tokens); FS_CHECK_PTR(dWc);
-  if (d_tokens == d_tokens_mixed) return FS_ERR_INVALID;
+  const size_t tb = (size_t)s->B * s->H * s->G * s->d * 4, wb = (size_t)s->H * s->d * s->d * 4;
+  if (!disjoint({{Wc, wb}, {tokens, tb}, {d_tokens_mixed, tb}}, {{d_tokens, tb}, {dWc, wb}})) return FS_ERR_INVALID;
   return cuda_status(simt_mix_channels_bwd(to_shape(s), Wc, tokens, d_tokens_mixed, d_tokens, dWc,
                                            reinterpret_cast<cudaStream_t>(stream)));
 }
@@ -366,7 +392,8 @@ fs_status fs_mix_bwd(const fs_shape* s, const float* M, const float* tokens, con
                      float* d_tokens, float* dM, fs_stream_t stream) {
   FS_CHECK_SHAPE(s);
   FS_CHECK_PTR(M); FS_CHECK_PTR(tokens); FS_CHECK_PTR(d_tokens_mixed); FS_CHECK_PTR(d_tokens); FS_CHECK_PTR(dM);
-  if (d_tokens == d_tokens_mixed) return FS_ERR_INVALID;
+  const size_t tb = (size_t)s->B * s->H * s->G * s->d * 4, mb = (size_t)s->H * s->G * s->G * 4;
+  if (!disjoint({{M, mb}, {tokens, tb}, {d_tokens_mixed, tb}}, {{d_tokens, tb}, {dM, mb}})) return FS_ERR_INVALID;
   return cuda_status(simt_mix_bwd(to_shape(s), M, tokens, d_tokens_mixed, d_tokens, dM,
                                   reinterpret_cast<cudaStream_t>(stream)));
 }

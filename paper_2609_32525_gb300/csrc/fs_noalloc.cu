@@ -6,6 +6,7 @@
 // kernels as fs_slice_fwd with that array as its workspace.
 #include "flashslice.h"
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -17,22 +18,62 @@ namespace {
 
 constexpr int kMaxDevices = 64;
 std::mutex g_mutex;
-void* g_scratch_addr[kMaxDevices] = {};
 
-// Device address of the scratch on the current device.  The lookup (a CUDA
-// runtime call) runs on the first call per device only; later calls read the
-// cached address.
+// The scratch address looked up on a device, and the unique id of the context it
+// was looked up in: a device reset, or another context made current, gives a new
+// id, and the address is looked up again.
+struct Entry {
+  unsigned long long ctx_id;
+  void* addr;
+};
+Entry g_entry[kMaxDevices] = {};
+
+using CtxGetCurrent = CUresult (*)(CUcontext*);
+using CtxGetId = CUresult (*)(CUcontext, unsigned long long*);
+CtxGetCurrent g_get_current = nullptr;
+CtxGetId g_get_id = nullptr;
+std::once_flag g_once;
+
+// Unique id (for the life of the process) of the calling thread's current context.
+bool current_context_id(unsigned long long* id) {
+  std::call_once(g_once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_get_current = reinterpret_cast<CtxGetCurrent>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_get_id = reinterpret_cast<CtxGetId>(p);
+  });
+  CUcontext c = nullptr;
+  return g_get_current && g_get_id && g_get_current(&c) == CUDA_SUCCESS && c != nullptr &&
+         g_get_id(c, id) == CUDA_SUCCESS;
+}
+
+// Device address of the scratch on the current device, in the current context.
+// The lookup (a CUDA runtime call) runs on the first call per device and again
+// after the device's context has changed; other calls read the cached address.
 fs_status scratch_address(void** out) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return FS_ERR_CUDA;
   if (dev < 0 || dev >= kMaxDevices) return FS_ERR_UNSUPPORTED;
   std::lock_guard<std::mutex> lock(g_mutex);
-  if (g_scratch_addr[dev] == nullptr) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return FS_ERR_CUDA;
-    g_scratch_addr[dev] = p;
+  unsigned long long id = 0;
+  const bool have_id = current_context_id(&id);
+  if (have_id && g_entry[dev].addr != nullptr && g_entry[dev].ctx_id == id) {
+    *out = g_entry[dev].addr;
+    return FS_OK;
   }
-  *out = g_scratch_addr[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return FS_ERR_CUDA;
+  // The lookup makes the device's primary context current if none was: its id now.
+  if (current_context_id(&id))
+    g_entry[dev] = Entry{id, p};
+  else
+    g_entry[dev] = Entry{0, nullptr};  // no context id available: look up again next time
+  *out = p;
   return FS_OK;
 }
 

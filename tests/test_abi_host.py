@@ -111,6 +111,33 @@ def test_mix_rejects_in_place(fs):
     assert fs._lib.fs_device_status(None, None) == fs.FS_ERR_INVALID
 
 
+def test_mix_calls_reject_partly_overlapping_buffers(fs):
+    """The mixes and their backward read every input while writing: an output that
+    shares any byte with an input (or another output) is rejected before any
+    launch.  Fake 16-byte-aligned addresses, never dereferenced: every call below
+    fails validation."""
+    lib, P = fs._lib, ctypes.c_void_p
+    B, H, d, G = 1, 2, 32, 8
+    s = fs.make_shape(B, 100, H, d, G)
+    tb = B * H * G * d * 4        # tokens [B,H,G,d] fp32
+    mb = H * G * G * 4            # M [H,G,G]
+    wb = H * d * d * 4            # Wc [H,d,d]
+    base = 1 << 20
+    M, tok = base, base + 4 * tb
+    # the output starts inside tokens (tail overlap) or ends inside it (head overlap)
+    for out in (tok + 16, tok - tb + 16):
+        assert lib.fs_mix(ctypes.byref(s), P(M), P(tok), P(out), None) == fs.FS_ERR_INVALID
+        assert lib.fs_mix_channels(ctypes.byref(s), P(M), P(tok), P(out), None) == fs.FS_ERR_INVALID
+    # the output overlaps M / Wc
+    assert lib.fs_mix(ctypes.byref(s), P(M), P(tok), P(M + mb - 16), None) == fs.FS_ERR_INVALID
+    assert lib.fs_mix_channels(ctypes.byref(s), P(M), P(tok), P(M + wb - 16), None) == fs.FS_ERR_INVALID
+    # backward: d_tokens over d_tokens_mixed, dM over tokens, the two outputs over each other
+    dzp, dz, dM = base + 8 * tb, base + 12 * tb, base + 16 * tb
+    for args in ((M, tok, dzp, dzp + 16, dM), (M, tok, dzp, dz, tok + 16), (M, tok, dzp, dz, dz + 16)):
+        assert lib.fs_mix_bwd(ctypes.byref(s), *[P(a) for a in args], None) == fs.FS_ERR_INVALID
+        assert lib.fs_mix_channels_bwd(ctypes.byref(s), *[P(a) for a in args], None) == fs.FS_ERR_INVALID
+
+
 def test_path_query(fs):
     assert fs.path_for_shape(fs.make_shape(1, 100, 2, 48, 8)) == -1
     assert fs.path_for_shape(fs.make_shape(1, 100, 2, 32, 8, dtype=fs.FS_F32)) == 0

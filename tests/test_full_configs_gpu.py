@@ -36,8 +36,10 @@ def _points(N, seed, k=4096):
     return np.unique(pts)
 
 
-def _check(name, got, ref, dtype):
+def _check(name, got, ref, dtype, workload=""):
     e = error(got, ref, dtype)
+    # One line per tensor (shown with pytest -s): the parity margin of each workload.
+    print(f"PARITY {workload} {name} {e:.3e} tol {tol(dtype):.0e} ({'max rel' if dtype == 'f32' else 'rel L2'})")
     assert e <= tol(dtype), f"{name}: error {e:.3e} > {tol(dtype):.0e}"
 
 
@@ -64,11 +66,11 @@ def test_full_size_parity(lib, name):
 
     ref = orc.forward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, eps=wl.eps, heads=heads, points=pts)
     hs = np.array(heads)
-    _check("tokens", host(c.tokens)[:, hs], ref["tokens"][:, hs], wl.dtype)
-    _check("wsum", host(c.wsum)[:, hs], ref["wsum"][:, hs], wl.dtype)
-    _check("tokens_mixed", host(c.tokens_mixed)[:, hs], ref["tokens_mixed"][:, hs], wl.dtype)
+    _check("tokens", host(c.tokens)[:, hs], ref["tokens"][:, hs], wl.dtype, name)
+    _check("wsum", host(c.wsum)[:, hs], ref["wsum"][:, hs], wl.dtype, name)
+    _check("tokens_mixed", host(c.tokens_mixed)[:, hs], ref["tokens_mixed"][:, hs], wl.dtype, name)
     out = host(c.out)
-    _check("out", out[:, pts][:, :, hs], ref["out"][:, pts][:, :, hs], wl.dtype)
+    _check("out", out[:, pts][:, :, hs], ref["out"][:, pts][:, :, hs], wl.dtype, name)
     lse = host(c.lse)  # [B, H, N]
     for b in range(wl.B):
         for h in heads:
@@ -79,9 +81,9 @@ def test_full_size_parity(lib, name):
     if wl.dout is None:
         return
     rb = orc.backward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, wl.dout, eps=wl.eps, heads=heads)
-    _check("d_tokens_mixed", host(c.d_tokens_mixed)[:, hs], rb["d_tokens_mixed"][:, hs], wl.dtype)
+    _check("d_tokens_mixed", host(c.d_tokens_mixed)[:, hs], rb["d_tokens_mixed"][:, hs], wl.dtype, name)
     for k in ("dW", "dbias", "dM"):
-        _check(k, host(g[k])[hs], rb[k][hs], wl.dtype)
-    _check("dtau", host(g["dtau"])[hs], rb["dtau"][hs], wl.dtype)
+        _check(k, host(g[k])[hs], rb[k][hs], wl.dtype, name)
+    _check("dtau", host(g["dtau"])[hs], rb["dtau"][hs], wl.dtype, name)
     for k in ("dx_mid", "dfx"):
-        _check(k, host(g[k])[:, pts][:, :, hs], rb[k][:, pts][:, :, hs], wl.dtype)
+        _check(k, host(g[k])[:, pts][:, :, hs], rb[k][:, pts][:, :, hs], wl.dtype, name)
