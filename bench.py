@@ -17,7 +17,10 @@ step's Mpoints/s on its own line (metric "train step ...").
 
 Multi-GPU: the workload is replicated (each rank runs its own full copy; no
 collective on the data path), so scaling is weak.  Launched with torchrun for
-N > 1; rank 0 prints the line.
+N > 1; rank 0 prints the line.  --shard instead splits one coupling's points
+over the ranks, with NCCL all-reduces of the slice partials (and, with an
+upstream gradient, of d_tokens_mixed and the parameter gradients): strong
+scaling (App. G.4).
 
 --impl reference times the fp64 CPU oracle (the only reference this method
 has) on the host cores, on a bounded sample of the same workload.
@@ -347,15 +350,24 @@ def run_train(args, wl, dev, world, rank):
     flops, bytes_ = 24.0 * C * wl.G * P, 11.0 * C * e * P
     per_call = {"fs_slice_fwd": 4.0 * C * wl.G * P, "fs_deslice_fwd": 4.0 * C * wl.G * P,
                 "fs_deslice_bwd": 8.0 * C * wl.G * P, "fs_slice_bwd": 8.0 * C * wl.G * P}
+    per_call_bytes = {"fs_slice_fwd": 2.0 * C * e * P, "fs_deslice_fwd": 2.0 * C * e * P,
+                      "fs_deslice_bwd": 3.0 * C * e * P, "fs_slice_bwd": 4.0 * C * e * P}
     peaks = _peaks()
     dom = max(per_call, key=lambda k: call_ms[k])
-    achieved = per_call[dom] / (call_ms[dom] * 1e-3) / 1e12
-    roof_t = max(flops / (peaks["bf16_tflops"] * 1e12), bytes_ / (peaks["hbm_gbs"] * 1e9))
-    roofline = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
-                "frac": achieved / peaks["bf16_tflops"], "traffic": None, "kernel": dom,
-                "peak_source": peaks["source"] + " bf16 burst", "step_frac": roof_t / (ms_per_step * 1e-3),
+    t_tensor, t_hbm = flops / (peaks["bf16_tflops"] * 1e12), bytes_ / (peaks["hbm_gbs"] * 1e9)
+    roof_t = max(t_tensor, t_hbm)
+    if t_tensor >= t_hbm:
+        achieved = per_call[dom] / (call_ms[dom] * 1e-3) / 1e12
+        bound = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                 "frac": achieved / peaks["bf16_tflops"], "peak_source": peaks["source"] + " bf16 burst"}
+    else:
+        achieved = per_call_bytes[dom] / (call_ms[dom] * 1e-3) / 1e9
+        bound = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                 "frac": achieved / peaks["hbm_gbs"], "peak_source": peaks["source"] + " HBM copy"}
+    roofline = {**bound, "traffic": None, "kernel": dom, "step_frac": roof_t / (ms_per_step * 1e-3),
                 "call_ms": call_ms,
-                "per_call_work": "forward calls 4*C*G flops per point each, backward calls 8*C*G (C=256)"}
+                "per_call_work": "forward calls 4*C*G flops and 2*C*e bytes per point each; backward calls "
+                                 "8*C*G flops, 3*C*e (deslice) and 4*C*e (slice) bytes"}
     line = {"metric": TRAIN_METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
@@ -368,6 +380,7 @@ def run_train(args, wl, dev, world, rank):
                        **({"points_override": "N reduced for profiling; not the benchmark workload"}
                           if args.points else {})},
             "clocks": clocks, "roofline": roofline,
+            "gpu_launches": (fs.forward_launch_count(s) + fs.backward_launch_count(s, True)) * args.steps,
             "e2e": {"value": sharding.job_rate(wl.points, world, e2e_ms), "unit": UNIT,
                     "h2d_bytes_per_step": 3 * hx.numel() * hx.element_size(),
                     "d2h_bytes_per_step": sum(h_.numel() * h_.element_size() for h_ in hout), "ms_per_step": e2e_ms}}
@@ -381,6 +394,83 @@ def run_train(args, wl, dev, world, rank):
 
 
 VARIANTS = ("tied", "untied", "frozen", "notokenattn")
+
+
+def run_shard(args, wl, dev, world, rank):
+    """--shard: one coupling point-sharded over the ranks (App. G.4).  Rank r holds
+    points sharding.point_range(N, r, world) of every batch; a step is
+    sharding.sharded_forward (the slice's unnormalised partials summed over ranks
+    by NCCL, then finalize, mix, deslice of the local points) and, for a workload
+    with an upstream gradient, sharding.sharded_backward (d_tokens_mixed summed,
+    mix backward, slice backward, dW, dbias, dtau summed).  The total work is the
+    workload's, whatever the number of ranks: scaling is strong."""
+    import torch
+
+    from paper_2609_32525_gb300 import flashslice as fs
+    from paper_2609_32525_gb300 import sharding
+
+    n0, n1 = sharding.point_range(wl.N, rank, world)
+    tdt = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+
+    def put(a, dt):
+        return torch.from_numpy(np.ascontiguousarray(a)).to(device=dev, dtype=dt).contiguous()
+
+    x, fx = put(wl.x_mid[:, n0:n1], tdt), put(wl.fx[:, n0:n1], tdt)
+    dout = put(wl.dout[:, n0:n1], tdt) if wl.dout is not None else None
+    W, b, t, M = (put(getattr(wl, k), torch.float32) for k in ("W_slice", "bias", "tau", "M"))
+    ops = fs.ShardedCoupling(wl.B, n1 - n0, wl.H, wl.d, wl.G, x, fx, W, b, t, M, tdt, wl.eps, dout=dout, device=dev)
+    train = dout is not None
+    stream = torch.cuda.current_stream()
+
+    def step():
+        sharding.sharded_forward(ops)
+        if train:
+            sharding.sharded_backward(ops)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    if ops.c.device_status() != fs.FS_OK:
+        raise RuntimeError("device status after warm-up: " + fs.status_string(ops.c.device_status()))
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+    except Exception:
+        pass
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(uuid)
+    time.sleep(0.3)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    ms = sharding.job_time_ms(e0.elapsed_time(e1) / args.steps, dev)
+    assert ops.c.device_status() == fs.FS_OK
+    # the forward's kernels and the finalize of the summed partials; the backward's
+    # calls all get the forward's lse
+    per_step = fs.forward_launch_count(ops.c.shape) + 1 + (fs.backward_launch_count(ops.c.shape, True) if train else 0)
+    line = {"metric": ("train step" if train else "coupling forward") + " Mpoints/s, point-sharded",
+            "value": wl.points / (ms * 1e-3) / 1e6, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "strong",
+            "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
+            "data": "synthetic (seeded; " + wl.recipe + ")",
+            "config": {"workload": wl.name, "B": wl.B, "N": wl.N, "H": wl.H, "d": wl.d, "G": wl.G,
+                       "points_per_rank": n1 - n0, "parallelism": f"point-sharded x{world}",
+                       "exchange": "NCCL all-reduce of (U, S)" + (", d_tokens_mixed, dW, dbias, dtau" if train else ""),
+                       "path": ["simt", "tcgen05"][fs.path_for_shape(ops.c.shape)]},
+            "clocks": clocks, "gpu_launches": per_step * args.steps}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
 
 
 def run_variant(args, wl, dev, world, rank):
@@ -482,6 +572,9 @@ def main():
     ap.add_argument("--workload", default="large_g_bf16")
     ap.add_argument("--variant", default=None, choices=VARIANTS,
                     help="time one coupling variant of the forward workload instead (Sec. 3 variants table)")
+    ap.add_argument("--shard", action="store_true",
+                    help="one coupling point-sharded over the ranks with NCCL all-reduces (App. G.4), "
+                         "strong scaling, instead of one replica per rank")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--ref-points", type=int, default=16384)
@@ -516,6 +609,11 @@ def main():
     from paper_2609_32525_gb300.workloads import make_named
 
     wl = make_named(args.workload, n_override=args.points)
+    if args.shard:
+        run_shard(args, wl, dev, world, rank)
+        if world > 1:
+            dist.destroy_process_group()
+        return
     if wl.dout is not None:
         return run_train(args, wl, dev, world, rank)
     if args.variant is not None:
@@ -614,16 +712,23 @@ def main():
     peaks = _peaks()
     alg = _algorithmic(wl)
     dom_name, dom_ms = ("fs_slice_fwd", slice_ms) if slice_ms >= desl_ms else ("fs_deslice_fwd", desl_ms)
-    achieved_tf = alg["flops_per_call"] / (dom_ms * 1e-3) / 1e12
-    roof_t = max(alg["flops"] / (peaks["bf16_tflops"] * 1e12), alg["bytes"] / (peaks["hbm_gbs"] * 1e9))
-    roofline = {"bound": "tensor", "achieved": achieved_tf, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
-                "frac": achieved_tf / peaks["bf16_tflops"], "traffic": _traffic(wl, dom_name), "kernel": dom_name,
+    t_tensor = alg["flops"] / (peaks["bf16_tflops"] * 1e12)
+    t_hbm = alg["bytes"] / (peaks["hbm_gbs"] * 1e9)
+    roof_t = max(t_tensor, t_hbm)
+    if t_tensor >= t_hbm:
+        achieved = alg["flops_per_call"] / (dom_ms * 1e-3) / 1e12
+        bound = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                 "frac": achieved / peaks["bf16_tflops"], "peak_source": peaks["source"] + " bf16 burst",
+                 "frac_sustained": achieved / peaks["bf16_tflops_sustained"]}
+    else:
+        achieved = alg["bytes_per_call"] / (dom_ms * 1e-3) / 1e9
+        bound = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                 "frac": achieved / peaks["hbm_gbs"], "peak_source": peaks["source"] + " HBM copy"}
+    roofline = {**bound, "traffic": _traffic(wl, dom_name), "kernel": dom_name,
                 "traffic_unit": "bytes per call (ncu DRAM read + write)",
-                "peak_source": peaks["source"] + " bf16 burst",
-                "frac_sustained": achieved_tf / peaks["bf16_tflops_sustained"],
                 "step_frac": roof_t / (ms_per_step * 1e-3),
                 "call_ms": {"fs_slice_fwd": slice_ms, "fs_mix": mix_ms, "fs_deslice_fwd": desl_ms},
-                "per_call_work": "4*C*G flops per point for each of slice and deslice (C=256)"}
+                "per_call_work": "4*C*G flops and 2*C*e bytes per point for each of slice and deslice"}
 
     # Each of the three sweeps (statistics, slice, deslice) makes one exponential per
     # point, head and slot; at 32 ex2 per clock per SM (measured on GB300) that floor

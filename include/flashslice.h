@@ -285,6 +285,12 @@ int fs_backward_path_for_shape(const fs_shape* s);
 /* Number of kernels the forward (slice + mix + deslice) launches for this shape. */
 int fs_forward_launch_count(const fs_shape* s);
 
+/* Number of kernels the backward (fs_deslice_bwd + fs_mix_bwd + fs_slice_bwd)
+ * launches for this shape.  lse_given: nonzero when both backward calls get the
+ * forward's lse (each call that must recompute the statistics launches that pass
+ * again).  Memsets are not counted.  -1 for an invalid or unsupported shape. */
+int fs_backward_launch_count(const fs_shape* s, int lse_given);
+
 #ifdef __cplusplus
 }
 #endif

@@ -239,6 +239,23 @@ int fs_forward_launch_count(const fs_shape* s) {
   return 3 /*stats, partials, reduce*/ + 1 /*mix*/ + 1 /*deslice*/;
 }
 
+int fs_backward_launch_count(const fs_shape* s, int lse_given) {
+  if (!valid_shape(s) || !supported_shape(s)) return -1;
+  const Shape sh = to_shape(s);
+  // Each backward call recomputes the statistics unless backward_stats takes the caller's lse.
+  const bool tc = tc_forward_supported(sh) && sh.dtype == FS_BF16;
+  const bool fp32_tc = tc_forward_supported(sh) && sh.dtype == FS_F32;
+  int stats = 0;
+  if (!(lse_given && !fp32_tc && (!tc || sh.dot == FS_DOT_BF16X2))) {
+    Shape split = sh;
+    split.dot = FS_DOT_BF16X2;
+    stats = tc ? tc_stats_launch_count(split) : 1;
+  }
+  const int mix_bwd = 2;  // d_tokens, dM
+  if (tc_backward_supported(sh)) return 2 * stats + tc_backward_launch_count(1) + mix_bwd + tc_backward_launch_count(2);
+  return 2 * stats + 5 /*point, slot, three reductions*/ + mix_bwd + 5 /*prologue, point, slot, two reductions*/;
+}
+
 fs_status fs_slice_fwd(const fs_shape* s, const void* x_mid, const void* fx, const float* W_slice,
                        const float* bias, const float* tau, float* tokens, float* wsum, float* lse,
                        int finalize, void* ws, size_t ws_bytes, fs_stream_t stream) {

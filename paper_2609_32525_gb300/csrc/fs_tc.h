@@ -9,6 +9,8 @@ namespace fs {
 bool tc_forward_supported(const Shape& s);
 // Kernels launched by tc_slice_fwd + tc_deslice_fwd (the mix is not counted).
 int tc_forward_launch_count(const Shape& s);
+// Kernels launched by tc_stats.
+int tc_stats_launch_count(const Shape& s);
 // Workspace the tensor-core slice needs for its split-N partials and its
 // prepared operand images; the deslice needs only the latter.
 size_t tc_slice_partials_bytes(const Shape& s);
@@ -44,6 +46,8 @@ size_t tc_rows_smem(const Shape& s, int mode, bool ps, bool hilo);
 bool tc_backward_supported(const Shape& s);
 // Workspace of one tensor-core backward call (mode 1 deslice, 2 slice).
 size_t tc_backward_bytes(const Shape& s, int mode);
+// Kernels launched by tc_deslice_bwd (mode 1) or tc_slice_bwd (mode 2).
+int tc_backward_launch_count(int mode);
 cudaError_t tc_deslice_bwd(const Shape& s, const void* x, const float* W, const float* bias, const float* tau,
                            const float* zp, const float* lse, const void* dout, float* dzp, void* dx, float* dW,
                            float* db, float* dtau, int accumulate, void* ws_tc, uint32_t* status, cudaStream_t st);

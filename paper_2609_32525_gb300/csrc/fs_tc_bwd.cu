@@ -784,6 +784,11 @@ size_t tc_backward_bytes(const Shape& s, int mode) {
 
 int tc_backward_slot_splits(const Shape& s) { return bwd_slot_splits(s); }
 
+// prep_t, prep_z2; prep_w, prep_wt, prep_px, rows, prep_dpx, slot, dx; the
+// reductions of the parameters and dtau (and of dz' in mode 1); in mode 2 also
+// the slice backward's dU/dS prologue.
+int tc_backward_launch_count(int mode) { return 2 + 7 + (mode == 1 ? 3 : 2 + 1); }
+
 // The backward forms every weight with split products whatever the forward's
 // arithmetic: its lse comes from split products (recomputed when the forward's
 // did not), and weights from bf16 logits would not sum to one against it; the

@@ -893,6 +893,8 @@ bool tc_forward_supported(const Shape& s) {
          s.BH() * np < (int64_t(1) << 31) && encode_fn() != nullptr;
 }
 
+int tc_stats_launch_count(const Shape& s) { return 2 /*prep_w, stats*/ + (x3_shape(s) ? 1 : 0); }
+
 int tc_forward_launch_count(const Shape& s) {
   return 4 /*prep_w, stats, slice, reduce*/ + 4 /*prep_w, prep_z, prep_px, deslice*/ +
          (x3_shape(s) ? 3 /*splits of x, fx; of x*/ : 0);

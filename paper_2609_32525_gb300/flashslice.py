@@ -33,8 +33,8 @@ FS_OP_SLICE_FWD, FS_OP_DESLICE_FWD, FS_OP_DESLICE_BWD, FS_OP_SLICE_BWD, FS_OP_ST
 
 EXPORTED = ("fs_workspace_bytes", "fs_slice_fwd", "fs_slice_finalize", "fs_mix", "fs_deslice_fwd",
             "fs_deslice_bwd", "fs_mix_bwd", "fs_slice_bwd", "fs_device_status", "fs_status_string",
-            "fs_path_for_shape", "fs_backward_path_for_shape", "fs_forward_launch_count", "fs_slice_fwd_noalloc",
-            "fs_slice_fwd_lse", "fs_mix_channels", "fs_mix_channels_bwd", "fs_stats")
+            "fs_path_for_shape", "fs_backward_path_for_shape", "fs_forward_launch_count", "fs_backward_launch_count",
+            "fs_slice_fwd_noalloc", "fs_slice_fwd_lse", "fs_mix_channels", "fs_mix_channels_bwd", "fs_stats")
 
 
 class fs_shape(ctypes.Structure):
@@ -70,6 +70,7 @@ _sig = {
     "fs_path_for_shape": (_I, [_S]),
     "fs_backward_path_for_shape": (_I, [_S]),
     "fs_forward_launch_count": (_I, [_S]),
+    "fs_backward_launch_count": (_I, [_S, _I]),
     "fs_slice_fwd_noalloc": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _I, ctypes.POINTER(_P), _P]),
 }
 for _name, (_res, _args) in _sig.items():
@@ -129,6 +130,10 @@ def backward_path_for_shape(shape: fs_shape) -> int:
 
 def forward_launch_count(shape: fs_shape) -> int:
     return int(_lib.fs_forward_launch_count(ctypes.byref(shape)))
+
+
+def backward_launch_count(shape: fs_shape, lse_given: bool = True) -> int:
+    return int(_lib.fs_backward_launch_count(ctypes.byref(shape), int(bool(lse_given))))
 
 
 def status_string(st: int) -> str:
@@ -282,3 +287,52 @@ class Coupling:
             st = fs_device_status(ws, stream)
             worst = worst or st
         return worst
+
+
+class ShardedCoupling:
+    """The local compute of a point-sharded coupling (App. G.4) for
+    sharding.sharded_forward / sharding.sharded_backward: this rank's points of
+    every batch, x_mid and fx [B, n_local, H, d], through the C ABI.  The slice
+    keeps its numerators unnormalised (finalize = 0) until they are summed over
+    ranks; the backward's two calls add into the same dx_mid, dW, dbias, dtau."""
+
+    def __init__(self, B, n_local, H, d, G, x_mid, fx, W_slice, bias, tau, M, dtype=torch.bfloat16, eps=1e-5,
+                 dout=None, device="cuda", dot=None):
+        self.c = Coupling(B, n_local, H, d, G, dtype, eps, backward=dout is not None, device=device, dot=dot)
+        self.x, self.fx, self.W, self.bias, self.tau, self.M, self.dout = x_mid, fx, W_slice, bias, tau, M, dout
+
+    def slice_partials(self):
+        c = self.c
+        fs_slice_fwd(c.shape, self.x, self.fx, self.W, self.bias, self.tau, c.tokens, c.wsum, c.lse, False,
+                     c.ws_slice)
+        return c.tokens, c.wsum
+
+    def finalize(self, U, S):
+        fs_slice_finalize(self.c.shape, U, S)
+        return U
+
+    def mix(self, tokens):
+        fs_mix(self.c.shape, self.M, tokens, self.c.tokens_mixed)
+        return self.c.tokens_mixed
+
+    def deslice(self, tokens_mixed):
+        c = self.c
+        fs_deslice_fwd(c.shape, self.x, self.W, self.bias, self.tau, tokens_mixed, c.lse, c.out, c.ws_deslice)
+        return c.out
+
+    def deslice_bwd(self):
+        c = self.c
+        fs_deslice_bwd(c.shape, self.x, self.W, self.bias, self.tau, c.tokens_mixed, c.lse, self.dout,
+                       c.d_tokens_mixed, c.dx_mid, c.dW, c.dbias, c.dtau, False, c.ws_dbwd)
+        return c.d_tokens_mixed
+
+    def mix_bwd(self, d_tokens_mixed):
+        c = self.c
+        fs_mix_bwd(c.shape, self.M, c.tokens, d_tokens_mixed, c.d_tokens, c.dM)
+        return c.d_tokens, c.dM
+
+    def slice_bwd(self, d_tokens):
+        c = self.c
+        fs_slice_bwd(c.shape, self.x, self.fx, self.W, self.bias, self.tau, c.tokens, c.wsum, c.lse, d_tokens,
+                     c.dx_mid, c.dfx, c.dW, c.dbias, c.dtau, True, c.ws_sbwd)
+        return c.dW, c.dbias, c.dtau

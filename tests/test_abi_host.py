@@ -142,3 +142,12 @@ def test_path_query(fs):
     assert fs.path_for_shape(fs.make_shape(1, 100, 2, 48, 8)) == -1
     assert fs.path_for_shape(fs.make_shape(1, 100, 2, 32, 8, dtype=fs.FS_F32)) == 0
     assert fs.forward_launch_count(fs.make_shape(1, 100, 2, 32, 8)) >= 3
+
+
+def test_backward_launch_count(fs):
+    assert fs.backward_launch_count(fs.make_shape(1, 100, 2, 48, 8)) == -1
+    # the fp32 SIMT backward: 5 + 2 + 5 kernels, and the statistics pass once per
+    # backward call when no lse is given
+    s = fs.make_shape(1, 100, 2, 32, 8, dtype=fs.FS_F32)
+    assert fs.backward_launch_count(s, True) == 12
+    assert fs.backward_launch_count(s, False) == 14

@@ -82,6 +82,94 @@ def _worker(rank, port, results):
         dist.destroy_process_group()
 
 
+class _OracleOps:
+    """The local compute of sharding.sharded_forward / sharded_backward on a CPU rank:
+    the fp64 oracle on this rank's points, standing in for flashslice.ShardedCoupling
+    (the same call sequence the C ABI runs on a GPU)."""
+
+    def __init__(self, wl, n0, n1):
+        from oracle import flashslice_oracle as orc
+
+        self.orc, self.wl = orc, wl
+        self.x, self.f, self.do = wl.x_mid[:, n0:n1], wl.fx[:, n0:n1], wl.dout[:, n0:n1]
+
+    def slice_partials(self):
+        wl = self.wl
+        r = self.orc.slice_fwd(self.x, self.f, wl.W_slice, wl.bias, wl.tau, eps=wl.eps, finalize=False)
+        return torch.from_numpy(r["tokens"].copy()), torch.from_numpy(r["wsum"].copy())
+
+    def finalize(self, U, S):
+        self.S = S.numpy()
+        self.tokens = self.orc.slice_finalize(U.numpy(), self.S, self.wl.eps)
+        return self.tokens
+
+    def mix(self, tokens):
+        self.zp = self.orc.mix(self.wl.M, tokens)
+        return self.zp
+
+    def deslice(self, zp):
+        wl = self.wl
+        self.out = self.orc.deslice_fwd(self.x, wl.W_slice, wl.bias, wl.tau, zp)
+        return self.out
+
+    def deslice_bwd(self):
+        wl = self.wl
+        self.rd = self.orc.deslice_bwd(self.x, wl.W_slice, wl.bias, wl.tau, self.zp, self.do)
+        return torch.from_numpy(np.ascontiguousarray(self.rd["d_tokens_mixed"]))
+
+    def mix_bwd(self, dzp):
+        rm = self.orc.mix_bwd(self.wl.M, self.tokens, dzp.numpy())
+        return rm["d_tokens"], rm["dM"]
+
+    def slice_bwd(self, dz):
+        wl = self.wl
+        self.rs = self.orc.slice_bwd(self.x, self.f, wl.W_slice, wl.bias, wl.tau, self.tokens, self.S, dz, eps=wl.eps)
+        return tuple(torch.from_numpy(np.ascontiguousarray(self.rd[k] + self.rs[k])) for k in ("dW", "dbias", "dtau"))
+
+
+def _orchestration_worker(rank, port, results):
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=WORLD)
+    try:
+        from oracle import flashslice_oracle as orc
+        from paper_2609_32525_gb300.workloads import make_case
+
+        wl = make_case(2, 777, 2, 8, 6, dtype="f32", seed=43, backward=True)
+        n0, n1 = sharding.point_range(wl.N, rank, WORLD)
+        ops = _OracleOps(wl, n0, n1)
+        out = sharding.sharded_forward(ops)
+        dM, (dW, db, dt) = sharding.sharded_backward(ops)
+        ref = orc.forward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, eps=wl.eps)
+        rb = orc.backward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, wl.dout, eps=wl.eps)
+
+        def close(a, b):
+            return bool(np.allclose(a, b, rtol=1e-10, atol=1e-12))
+
+        results[rank] = {"out": close(out, ref["out"][:, n0:n1]), "tokens": close(ops.tokens, ref["tokens"]),
+                         "dM": close(dM, rb["dM"]), "dW": close(dW.numpy(), rb["dW"]),
+                         "dbias": close(db.numpy(), rb["dbias"]), "dtau": close(dt.numpy(), rb["dtau"]),
+                         "dx_mid": close(ops.rd["dx_mid"] + ops.rs["dx_mid"], rb["dx_mid"][:, n0:n1]),
+                         "dfx": close(ops.rs["dfx"], rb["dfx"][:, n0:n1])}
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_gloo_ranks_run_the_sharded_orchestration():
+    """sharding.sharded_forward and sharded_backward, the functions bench.py --shard
+    runs over NCCL, on two gloo ranks with the oracle as each rank's compute: every
+    output and gradient equals the unsharded oracle's."""
+    port = _free_port()
+    with mp.Manager() as mgr:
+        results = mgr.dict()
+        mp.spawn(_orchestration_worker, args=(port, results), nprocs=WORLD, join=True)
+        res = dict(results)
+    assert sorted(res) == list(range(WORLD))
+    for rank, oks in res.items():
+        bad = [k for k, ok in oks.items() if not ok]
+        assert not bad, f"rank {rank}: sharded results differ from the unsharded oracle: {bad}"
+
+
 def test_point_range_partitions_the_points():
     for N in (1, 7, 1000, 1001):
         for world in (1, 2, 3, 8):
