@@ -61,8 +61,18 @@ def _peaks():
 # deslice) are scaled x4; the W/Z' images and the split-partial reduction are not.
 # Valid only for the kernel sources it was measured on, identified by their SHA-1.
 # When the sources change the figure is reported as null.
-_TRAFFIC = {"sources_sha1": "b11a36dcf5c3113643144473f0046db55c82d7fb", "workload": "large_g_bf16", "N": 1048576,
-            "fs_slice_fwd": 2.5238e9, "fs_deslice_fwd": 1.0602e9}
+_TRAFFIC = {"sources_sha1": "560992d440d7587167df7a918cc4bd88921b958b", "workload": "large_g_bf16", "N": 1048576,
+            "fs_slice_fwd": 2.4290e9, "fs_deslice_fwd": 1.0601e9}
+
+
+def _overrides(args):
+    """Config entries that mark a run on a changed recipe."""
+    o = {}
+    if args.points:
+        o["points_override"] = "N reduced for profiling; not the benchmark workload"
+    if args.slots:
+        o["slots_override"] = "G set to %d; not one of the named configurations" % args.slots
+    return o
 
 
 def _pipelined_e2e(K, stream, dev, ins, outs, compute):
@@ -377,8 +387,7 @@ def run_train(args, wl, dev, world, rank):
                        "dot": ["bf16", "bf16x2"][s.dot],
                        "path": {"forward": ["simt", "tcgen05"][fs.path_for_shape(s)],
                                 "backward": ["simt", "tcgen05"][fs.backward_path_for_shape(s)]},
-                       **({"points_override": "N reduced for profiling; not the benchmark workload"}
-                          if args.points else {})},
+                       **_overrides(args)},
             "clocks": clocks, "roofline": roofline,
             "gpu_launches": (fs.forward_launch_count(s) + fs.backward_launch_count(s, True)) * args.steps,
             "e2e": {"value": sharding.job_rate(wl.points, world, e2e_ms), "unit": UNIT,
@@ -467,7 +476,7 @@ def run_shard(args, wl, dev, world, rank):
             "config": {"workload": wl.name, "B": wl.B, "N": wl.N, "H": wl.H, "d": wl.d, "G": wl.G,
                        "points_per_rank": n1 - n0, "parallelism": f"point-sharded x{world}",
                        "exchange": "NCCL all-reduce of (U, S)" + (", d_tokens_mixed, dW, dbias, dtau" if train else ""),
-                       "path": ["simt", "tcgen05"][fs.path_for_shape(ops.c.shape)]},
+                       "path": ["simt", "tcgen05"][fs.path_for_shape(ops.c.shape)], **_overrides(args)},
             "clocks": clocks, "gpu_launches": per_step * args.steps}
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -557,7 +566,7 @@ def run_variant(args, wl, dev, world, rank):
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype,
             "data": "synthetic (seeded; " + wl.recipe + ")",
             "config": {"workload": wl.name, "variant": args.variant, "B": wl.B, "N": wl.N, "H": wl.H, "d": wl.d,
-                       "G": wl.G, "parallelism": f"replicas x{world}"},
+                       "G": wl.G, "parallelism": f"replicas x{world}", **_overrides(args)},
             "clocks": clocks, "step_frac": roof_t / (ms * 1e-3)}
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -580,6 +589,8 @@ def main():
     ap.add_argument("--ref-points", type=int, default=16384)
     ap.add_argument("--points", type=int, default=None,
                     help="profiling runs only: the workload's recipe at a smaller N (the line says so)")
+    ap.add_argument("--slots", type=int, default=None,
+                    help="the workload's recipe at another slot count G (the line says so)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -608,7 +619,7 @@ def main():
     from paper_2609_32525_gb300 import sharding
     from paper_2609_32525_gb300.workloads import make_named
 
-    wl = make_named(args.workload, n_override=args.points)
+    wl = make_named(args.workload, n_override=args.points, g_override=args.slots)
     if args.shard:
         run_shard(args, wl, dev, world, rank)
         if world > 1:
@@ -752,8 +763,7 @@ def main():
                        "step": "fs_slice_fwd + fs_mix + fs_deslice_fwd", "parallelism": f"replicas x{world}",
                        "l2": "inputs 2 x %d MiB > 129 MB L2, no flush" % (hx.numel() * hx.element_size() >> 20),
                        "path": ["simt", "tcgen05"][fs.path_for_shape(s)],
-                       **({"points_override": "N reduced for profiling; not the benchmark workload"}
-                          if args.points else {})},
+                       **_overrides(args)},
             "clocks": clocks, "gpu_launches": launches, "roofline": roofline,
             "e2e": {"value": e2e_val, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "ms_per_step": e2e_ms}}

@@ -252,7 +252,8 @@ int fs_backward_launch_count(const fs_shape* s, int lse_given) {
     stats = tc ? tc_stats_launch_count(split) : 1;
   }
   const int mix_bwd = 2;  // d_tokens, dM
-  if (tc_backward_supported(sh)) return 2 * stats + tc_backward_launch_count(1) + mix_bwd + tc_backward_launch_count(2);
+  if (tc_backward_supported(sh))
+    return 2 * stats + tc_backward_launch_count(sh, 1) + mix_bwd + tc_backward_launch_count(sh, 2);
   return 2 * stats + 5 /*point, slot, three reductions*/ + mix_bwd + 5 /*prologue, point, slot, two reductions*/;
 }
 

@@ -249,51 +249,156 @@ __global__ void k_finalize(float* __restrict__ tokens, const float* __restrict__
 
 // ---- mix and its backward ------------------------------------------------------------
 // out[bh][g][c] = sum_k A_h(g, k) in[bh][k][c] per (b, h), with A_h = M[h] (the mix,
-// z' = M z) or A_h = M[h]^T (its backward, dz = M^T dz').  Blocks of 16 rows g x 32
-// channels (16 x 16 threads, 2 outputs each; many blocks, so that the short K
-// loop's latency overlaps) stage A and `in` 64 k at a time in shared memory; the
-// sum over k runs in a fixed order.
+// z' = M z) or A_h = M[h]^T (its backward, dz = M^T dz').
+//
+// A block of 8 warps owns a tile of 16 rows g x 32 channels and sweeps k in chunks of
+// 64.  A and `in` chunks are staged in shared memory by cp.async, three chunks deep,
+// so that two chunks' loads are in flight while one is multiplied.  Warp w takes k
+// = 8w .. 8w + 7 of every chunk; each lane keeps a 4 x 4 register tile (4 rows g, 4
+// channels), so that two 16-byte shared loads feed 16 FMAs.  The eight warps'
+// partial sums are added at the end in warp order: the sum over k has a fixed order.
+// kVec: G % 4 == 0, so rows of M move as 16-byte pieces; otherwise as 4-byte words.
+constexpr int kMixTG = 16, kMixTC = 32, kMixKC = 64, kMixStages = 3;
+// A tile: g-major [16][64 + 4] for the mix (the pad puts the four rows a lane reads,
+// g = q, q + 4, q + 8, q + 12, on different banks); k-major [64][16] for the transpose,
+// as M[k][g] lies in memory.
 template <bool kTrans>
+__host__ __device__ constexpr int mix_a_words() { return kTrans ? kMixKC * kMixTG : kMixTG * (kMixKC + 4); }
+
+__device__ __forceinline__ void cp_async16(float* dst, const float* src, bool valid) {
+  const unsigned d = static_cast<unsigned>(__cvta_generic_to_shared(dst));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(src), "r"(valid ? 16 : 0) : "memory");
+}
+__device__ __forceinline__ void cp_async4(float* dst, const float* src, bool valid) {
+  const unsigned d = static_cast<unsigned>(__cvta_generic_to_shared(dst));
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n" ::"r"(d), "l"(src), "r"(valid ? 4 : 0) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory"); }
+
+template <bool kTrans, bool kVec>
 __global__ void __launch_bounds__(256) k_mix_tiled(const float* __restrict__ M, const float* __restrict__ in,
                                                    float* __restrict__ out, int H, int G, int D) {
-  constexpr int TG = 16, TC = 32, KC = 64;
-  __shared__ float sa[KC][TG + 1];
-  __shared__ float sb[KC][TC + 1];
+  constexpr int TG = kMixTG, TC = kMixTC, KC = kMixKC, S = kMixStages;
+  constexpr int AW = mix_a_words<kTrans>(), BW = KC * TC, SW = AW + BW;
+  __shared__ __align__(16) float sm[S * SW];
   const int64_t bh = blockIdx.y;
   const int h = (int)(bh % H);
   const int g0 = blockIdx.x * TG, c0 = blockIdx.z * TC;
-  const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+  const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const float* Mh = M + (int64_t)h * G * G;
   const float* X = in + bh * (int64_t)G * D;
-  float acc0 = 0.f, acc1 = 0.f;
-  for (int k0 = 0; k0 < G; k0 += KC) {
-    __syncthreads();
-    for (int i = threadIdx.x; i < TG * KC; i += 256) {
-      // consecutive threads read consecutive addresses of M: k for the mix, g for its transpose
-      const int g = kTrans ? i % TG : i / KC, k = kTrans ? i / TG : i % KC;
-      float v = 0.f;
-      if (g0 + g < G && k0 + k < G)
-        v = kTrans ? Mh[(int64_t)(k0 + k) * G + g0 + g] : Mh[(int64_t)(g0 + g) * G + k0 + k];
-      sa[k][g] = v;
+  const int nch = (G + KC - 1) / KC;
+
+  // Stage chunk `ch` (k = ch * KC ...) into buffer `buf`; out-of-range words are zero-filled.
+  auto issue = [&](int ch, int buf) {
+    if (ch < nch) {
+      const int k0 = ch * KC;
+      float* sa = sm + buf * SW;
+      float* sb = sa + AW;
+      if (kVec) {
+        if (kTrans) {  // A(g, k) = M[k][g]: row k, 4 consecutive g
+          const int k = t >> 2, gg = (t & 3) * 4;
+          const bool v = k0 + k < G && g0 + gg < G;
+          cp_async16(sa + k * TG + gg, v ? Mh + (int64_t)(k0 + k) * G + g0 + gg : Mh, v);
+        } else {  // A(g, k) = M[g][k]: row g, 4 consecutive k
+          const int g = t >> 4, kk = (t & 15) * 4;
+          const bool v = g0 + g < G && k0 + kk < G;
+          cp_async16(sa + g * (KC + 4) + kk, v ? Mh + (int64_t)(g0 + g) * G + k0 + kk : Mh, v);
+        }
+      } else {
+#pragma unroll
+        for (int r = 0; r < 4; r++) {
+          const int e = t + 256 * r;
+          if (kTrans) {
+            const int k = e / TG, gg = e % TG;
+            const bool v = k0 + k < G && g0 + gg < G;
+            cp_async4(sa + k * TG + gg, v ? Mh + (int64_t)(k0 + k) * G + g0 + gg : Mh, v);
+          } else {
+            const int g = e / KC, kk = e % KC;
+            const bool v = g0 + g < G && k0 + kk < G;
+            cp_async4(sa + g * (KC + 4) + kk, v ? Mh + (int64_t)(g0 + g) * G + k0 + kk : Mh, v);
+          }
+        }
+      }
+#pragma unroll
+      for (int r = 0; r < 2; r++) {  // `in` rows k, 4 consecutive channels (D % 4 == 0)
+        const int e = t + 256 * r, k = e >> 3, cc = (e & 7) * 4;
+        const bool v = k0 + k < G && c0 + cc < D;
+        cp_async16(sb + k * TC + cc, v ? X + (int64_t)(k0 + k) * D + c0 + cc : X, v);
+      }
     }
-    for (int i = threadIdx.x; i < KC * TC; i += 256) {
-      const int k = i / TC, c = i % TC;
-      sb[k][c] = (k0 + k < G && c0 + c < D) ? X[(int64_t)(k0 + k) * D + c0 + c] : 0.f;
-    }
-    __syncthreads();
-#pragma unroll 16
-    for (int k = 0; k < KC; k++) {
-      const float a = sa[k][ty];
-      acc0 = fmaf(a, sb[k][tx], acc0);
-      acc1 = fmaf(a, sb[k][tx + 16], acc1);
+    cp_async_commit();
+  };
+
+  // Lane (gq, cq): channels 4cq .. 4cq + 3; rows g = gq + 4i (mix) or 4gq + i (transpose).
+  const int gq = lane >> 3, cq = lane & 7;
+  float acc[4][4] = {};
+#pragma unroll
+  for (int st = 0; st < S - 1; st++) issue(st, st);
+  for (int ch = 0; ch < nch; ch++) {
+    cp_async_wait<S - 2>();
+    __syncthreads();  // chunk ch is visible; every warp is done with chunk ch - 1's buffer
+    issue(ch + S - 1, (ch + S - 1) % S);
+    const float* sa = sm + (ch % S) * SW;
+    const float* sb = sa + AW;
+    if (kTrans) {
+#pragma unroll
+      for (int kk = 0; kk < 8; kk++) {
+        const int k = warp * 8 + kk;
+        const float4 a = *reinterpret_cast<const float4*>(sa + k * TG + 4 * gq);
+        const float4 b = *reinterpret_cast<const float4*>(sb + k * TC + 4 * cq);
+        const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+        for (int i = 0; i < 4; i++)
+#pragma unroll
+          for (int j = 0; j < 4; j++) acc[i][j] = fmaf(av[i], bv[j], acc[i][j]);
+      }
+    } else {
+#pragma unroll
+      for (int half = 0; half < 2; half++) {
+        const int kb = warp * 8 + half * 4;
+        float av[4][4], bv[4][4];
+#pragma unroll
+        for (int i = 0; i < 4; i++) {
+          const float4 a = *reinterpret_cast<const float4*>(sa + (gq + 4 * i) * (KC + 4) + kb);
+          av[i][0] = a.x; av[i][1] = a.y; av[i][2] = a.z; av[i][3] = a.w;
+        }
+#pragma unroll
+        for (int kk = 0; kk < 4; kk++) {
+          const float4 b = *reinterpret_cast<const float4*>(sb + (kb + kk) * TC + 4 * cq);
+          bv[kk][0] = b.x; bv[kk][1] = b.y; bv[kk][2] = b.z; bv[kk][3] = b.w;
+        }
+#pragma unroll
+        for (int kk = 0; kk < 4; kk++)
+#pragma unroll
+          for (int i = 0; i < 4; i++)
+#pragma unroll
+            for (int j = 0; j < 4; j++) acc[i][j] = fmaf(av[i][kk], bv[kk][j], acc[i][j]);
+      }
     }
   }
-  const int g = g0 + ty;
-  if (g < G) {
-    if (c0 + tx < D) out[(bh * G + g) * (int64_t)D + c0 + tx] = acc0;
-    if (c0 + tx + 16 < D) out[(bh * G + g) * (int64_t)D + c0 + tx + 16] = acc1;
+  cp_async_wait<0>();
+  __syncthreads();  // the staging buffers become the eight warps' partial tiles
+  float* red = sm;  // [8][TG][TC]
+#pragma unroll
+  for (int i = 0; i < 4; i++) {
+    const int g = kTrans ? 4 * gq + i : gq + 4 * i;
+    *reinterpret_cast<float4*>(red + (warp * TG + g) * TC + 4 * cq) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+  }
+  __syncthreads();
+#pragma unroll
+  for (int r = 0; r < 2; r++) {
+    const int o = t + 256 * r, g = o / TC, c = o % TC;
+    float v = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; w++) v += red[(w * TG + g) * TC + c];
+    if (g0 + g < G && c0 + c < D) out[(bh * G + g0 + g) * (int64_t)D + c0 + c] = v;
   }
 }
+static_assert(8 * kMixTG * kMixTC <= kMixStages * (kMixKC * kMixTC + kMixTG * (kMixKC + 4)),
+              "the partial tiles fit in the staging buffers");
 
 // Per-token channel map (the attention-free core): out[bh][g][c] = sum_k A(c, k)
 // in[bh][g][k], with A = Wc[h] (forward) or Wc[h]^T (its token backward); one
@@ -827,15 +932,21 @@ cudaError_t simt_finalize(const Shape& s, float* tokens, const float* wsum, cuda
 }
 
 cudaError_t simt_mix(const Shape& s, const float* M, const float* z, float* zp, cudaStream_t st) {
-  const dim3 grid((unsigned)((s.G + 15) / 16), (unsigned)s.BH(), (unsigned)((s.d + 31) / 32));
-  k_mix_tiled<false><<<grid, 256, 0, st>>>(M, z, zp, s.H, s.G, s.d);
+  const dim3 grid((unsigned)((s.G + kMixTG - 1) / kMixTG), (unsigned)s.BH(), (unsigned)((s.d + kMixTC - 1) / kMixTC));
+  if (s.G % 4 == 0)
+    k_mix_tiled<false, true><<<grid, 256, 0, st>>>(M, z, zp, s.H, s.G, s.d);
+  else
+    k_mix_tiled<false, false><<<grid, 256, 0, st>>>(M, z, zp, s.H, s.G, s.d);
   return cudaGetLastError();
 }
 
 cudaError_t simt_mix_bwd(const Shape& s, const float* M, const float* z, const float* dzp, float* dz, float* dM,
                          cudaStream_t st) {
-  const dim3 grid((unsigned)((s.G + 15) / 16), (unsigned)s.BH(), (unsigned)((s.d + 31) / 32));
-  k_mix_tiled<true><<<grid, 256, 0, st>>>(M, dzp, dz, s.H, s.G, s.d);
+  const dim3 grid((unsigned)((s.G + kMixTG - 1) / kMixTG), (unsigned)s.BH(), (unsigned)((s.d + kMixTC - 1) / kMixTC));
+  if (s.G % 4 == 0)
+    k_mix_tiled<true, true><<<grid, 256, 0, st>>>(M, dzp, dz, s.H, s.G, s.d);
+  else
+    k_mix_tiled<true, false><<<grid, 256, 0, st>>>(M, dzp, dz, s.H, s.G, s.d);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   const dim3 tiles((unsigned)((s.G + 63) / 64), (unsigned)((s.G + 63) / 64), (unsigned)s.H);

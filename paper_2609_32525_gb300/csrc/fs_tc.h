@@ -32,22 +32,23 @@ cudaError_t tc_deslice_fwd(const Shape& s, const void* x, const float* W, const 
 
 // Rows pass of the backward (the deslice kernel in backward mode 1 or 2) on
 // prepared operands: W image, Z-layout image of t (hi then lo, G*128 bytes per
-// (b,h)), lse point-extra rows; writes delta (and, mode 2, dfx and the two
-// per-warpgroup partials wds of sum_g w dS, which must start at zero).
+// (b,h)), lse point-extra rows; writes delta (and, mode 2, dfx), or adds to them
+// when accumulate != 0 (a later slot range of the same points), and adds the two
+// per-warpgroup partials of sum_g w dS to wds (which must start at zero).
 cudaError_t tc_rows_bwd(const Shape& s, int mode, const void* x, const uint8_t* wimg, const uint8_t* zimg,
                         const void* px, const void* v, void* dfx, float* delta, float* wds, const float* dS,
-                        uint32_t* status, cudaStream_t st);
+                        int accumulate, uint32_t* status, cudaStream_t st);
 size_t tc_rows_smem(const Shape& s, int mode, bool ps, bool hilo);
 
 // ---- tensor-core backward (fs_tc_bwd.cu) ----
-// True when the tensor-core backward implements this shape (the forward's
-// shapes with N >= 2 whose operand images fit in shared memory: G <= 640, padded
-// like the forward's to whole 128-slot blocks).
+// True when the tensor-core backward implements this shape: bf16, d = 32, N >= 2,
+// G <= 4096.  Its passes hold the operand images of at most 640 slots (padded to
+// whole 128-slot blocks); a larger G runs them over slot ranges.
 bool tc_backward_supported(const Shape& s);
 // Workspace of one tensor-core backward call (mode 1 deslice, 2 slice).
 size_t tc_backward_bytes(const Shape& s, int mode);
 // Kernels launched by tc_deslice_bwd (mode 1) or tc_slice_bwd (mode 2).
-int tc_backward_launch_count(int mode);
+int tc_backward_launch_count(const Shape& s, int mode);
 cudaError_t tc_deslice_bwd(const Shape& s, const void* x, const float* W, const float* bias, const float* tau,
                            const float* zp, const float* lse, const void* dout, float* dzp, void* dx, float* dW,
                            float* db, float* dtau, int accumulate, void* ws_tc, uint32_t* status, cudaStream_t st);

@@ -663,11 +663,51 @@ size_t smem_bwd_dx(int G, bool hilo) {
 int bwd_slot_blocks(const Shape& s) { return s.G / kGC; }
 int bwd_slot_splits(const Shape& s) { return point_splits(s, (int)(s.BH() * bwd_slot_blocks(s))); }
 
-// Workspace layout of one tensor-core backward call (offsets from the tc region).
-struct BwdLayout {
-  size_t wimg, wtimg, timg, zimg, px, dpx, delta, wds, ds, dtp, part, total;
+// Slot ranges.  The point pass holds three images of its slots in shared memory,
+// which fits up to kBwdSlotsMax slots.  A larger G runs every pass over ranges of
+// `size` slots (a multiple of 128; the last range may hold fewer real slots), all
+// with the full problem's lse, so that the weights of a range are those of the
+// softmax over all G.  The sums over slots (delta, dfx, dx) add up over the
+// ranges; the slot-owned gradients of a range are its own.  `size` is the
+// largest that minimises the padded slot count n * size.
+constexpr int kBwdSlotsMax = 640;
+struct SlotRanges {
+  int n, size;
 };
-BwdLayout bwd_layout(const Shape& s, int mode) {
+SlotRanges slot_ranges(int G) {
+  if (G <= kBwdSlotsMax) return {1, (G + kGC - 1) / kGC * kGC};
+  SlotRanges best{0, 0};
+  for (int size = kGC; size <= kBwdSlotsMax; size += kGC) {
+    const int n = (G + size - 1) / size;
+    if (best.n == 0 || (int64_t)n * size <= (int64_t)best.n * best.size) best = {n, size};
+  }
+  return best;
+}
+
+// The backward forms every weight with split products whatever the forward's
+// arithmetic: its lse comes from split products (recomputed when the forward's
+// did not), and weights from bf16 logits would not sum to one against it; the
+// excess would bias the gradients that are sums of cancelling terms (dbias, dtau).
+Shape split_shape(const Shape& s) {
+  Shape r = s;
+  r.dot = FS_DOT_BF16X2;
+  return r;
+}
+
+// The shape the passes see: split products, G = the slot range.
+Shape pass_shape(const Shape& s0) {
+  Shape s = split_shape(s0);
+  s.G = slot_ranges(s0.G).size;
+  return s;
+}
+
+// Workspace layout of one tensor-core backward call (offsets from the tc region).
+// With several slot ranges it also holds a range's slice of W, bias and t (wc, bc,
+// tc) and its slot-owned gradients (dwc, dbc, dzc) before they go to their places.
+struct BwdLayout {
+  size_t wimg, wtimg, timg, zimg, px, dpx, delta, wds, ds, dtp, part, wc, bc, tc, dwc, dbc, dzc, total;
+};
+BwdLayout bwd_layout(const Shape& s0, int mode) {
   BwdLayout L{};
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -675,6 +715,7 @@ BwdLayout bwd_layout(const Shape& s, int mode) {
     off = align_up(off + bytes, 256);
     return o;
   };
+  const Shape s = pass_shape(s0);
   const size_t BHG = (size_t)s.BH() * s.G;
   const size_t pts = (size_t)s.BH() * s.N;
   const int P = bwd_slot_splits(s), R = bwd_slot_blocks(s);
@@ -689,6 +730,13 @@ BwdLayout bwd_layout(const Shape& s, int mode) {
   L.ds = take(BHG * sizeof(float));
   L.dtp = take((size_t)s.BH() * P * R * sizeof(float));
   L.part = take((size_t)P * BHG * (mode == 1 ? 2 * kD + 2 : kD + 2) * sizeof(float));
+  const size_t rs = slot_ranges(s0.G).n > 1 ? (size_t)s.G : 0;
+  L.wc = take((size_t)s.H * kD * rs * sizeof(float));
+  L.bc = take((size_t)s.H * rs * sizeof(float));
+  L.tc = take((size_t)s.BH() * rs * (kD + 1) * sizeof(float));
+  L.dwc = take((size_t)s.H * kD * rs * sizeof(float));
+  L.dbc = take((size_t)s.H * rs * sizeof(float));
+  L.dzc = take(mode == 1 ? (size_t)s.BH() * rs * kD * sizeof(float) : 0);
   L.total = off;
   return L;
 }
@@ -701,60 +749,14 @@ bool make_maps(const Shape& s, const void* x, const void* v, const void* px, con
          make_px_map(dmap, dpx, s.BH(), Np);
 }
 
-// The common part of both backward calls, after the T and Z images are written:
-// the W images and lse rows, the rows pass, delta's rows, the slot and the point passes.
-// s: the padded shape (s.G a whole number of 128-slot blocks); G: the caller's.
-cudaError_t run_backward(const Shape& s, int G, int mode, const void* x, const void* v, const float* W,
-                         const float* bias, const float* tau, const float* lse, void* dfx, void* dx, int accumulate,
-                         uint8_t* ws, const BwdLayout& L, uint32_t* status, cudaStream_t st) {
-  const int64_t Np = padded_n(s);
-  cudaError_t e = prep_w(s, G, W, bias, tau, ws + L.wimg, status, st);
-  if (e != cudaSuccess) return e;
-  const int64_t nwt = (int64_t)s.H * kD * s.G;
-  k_prep_wt<<<(unsigned)((nwt + 255) / 256), 256, 0, st>>>(W, tau, ws + L.wtimg, s.H, G, s.G, status);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  const int64_t npx = s.BH() * Np;
-  k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(ws + L.px), s.BH(), s.N,
-                                                             Np);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  float* delta = reinterpret_cast<float*>(ws + L.delta);
-  float* wds = mode == 2 ? reinterpret_cast<float*>(ws + L.wds) : nullptr;
-  if (wds && (e = cudaMemsetAsync(wds, 0, 2 * (size_t)s.BH() * s.N * sizeof(float), st)) != cudaSuccess) return e;
-  if ((e = tc_rows_bwd(s, mode, x, ws + L.wimg, ws + L.zimg, ws + L.px, v, dfx, delta, wds,
-                       reinterpret_cast<const float*>(ws + L.ds), status, st)) != cudaSuccess)
-    return e;
-  k_prep_dpx<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(delta, wds, reinterpret_cast<uint4*>(ws + L.dpx),
-                                                              s.BH(), s.N, Np);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
-
-  CUtensorMap xmap, vmap, pmap, dmap;
-  if (!make_maps(s, x, v, ws + L.px, ws + L.dpx, &xmap, &vmap, &pmap, &dmap)) return cudaErrorInvalidValue;
-  const bool split = s.dot == FS_DOT_BF16X2;
-  {
-    const int R = bwd_slot_blocks(s), P = bwd_slot_splits(s);
-    const size_t sm = smem_bwd_slot();
-    const auto kernel = mode == 1 ? (split ? k_bwd_slot_tc<1, true> : k_bwd_slot_tc<1, false>)
-                                  : (split ? k_bwd_slot_tc<2, true> : k_bwd_slot_tc<2, false>);
-    if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
-    kernel<<<dim3((unsigned)R, (unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(
-        xmap, vmap, pmap, dmap, ws + L.wimg, ws + L.timg, reinterpret_cast<float*>(ws + L.part),
-        reinterpret_cast<float*>(ws + L.dtp), s.N, Np, s.H, s.G, P, status);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  }
-  {
-    const bool hilo = split && smem_bwd_dx(s.G, true) <= kMaxSmem;
-    const size_t sm = smem_bwd_dx(s.G, hilo);
-    const int P = point_splits(s, (int)s.BH());
-    const auto kernel = split ? k_bwd_dx_tc<true> : k_bwd_dx_tc<false>;
-    if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
-    kernel<<<dim3((unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(
-        xmap, vmap, pmap, dmap, ws + L.wimg, ws + L.timg, ws + L.wtimg, static_cast<__nv_bfloat16*>(dx), s.N, Np,
-        s.H, s.G, P, hilo ? 1 : 0, accumulate, status);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  }
-  return cudaSuccess;
+// rows x cols floats from src (row pitch spitch floats) to dst (row pitch dpitch floats).
+cudaError_t copy_rows(float* dst, int64_t dpitch, const float* src, int64_t spitch, int64_t cols, int64_t rows,
+                      cudaStream_t st) {
+  return cudaMemcpy2DAsync(dst, (size_t)dpitch * sizeof(float), src, (size_t)spitch * sizeof(float),
+                           (size_t)cols * sizeof(float), (size_t)rows, cudaMemcpyDeviceToDevice, st);
 }
 
+// Slot-side images of t (T image, its c column, Z-layout image) for G slots.
 cudaError_t prep_t_images(const Shape& s, int G, const float* t, int tstride, int has_c, uint8_t* ws,
                           const BwdLayout& L, cudaStream_t st) {
   const int64_t BHG = s.BH() * s.G;
@@ -766,6 +768,135 @@ cudaError_t prep_t_images(const Shape& s, int G, const float* t, int tstride, in
   return cudaGetLastError();
 }
 
+// One backward call: mode 1 (deslice; t = z', v = dO, writes dzp) or 2 (slice; t =
+// dU | dS with tstride 33, v = fx, writes dfx).  t: [BH][G][tstride] fp32.
+//   1. lse rows; for each slot range: its images, then the rows pass (delta, dfx
+//      and the wds partials add up over the ranges);
+//   2. delta's rows; for each slot range: the slot pass, its reduction into the
+//      range's dW, dbias, dtau (and dz') partials, and the point pass (dx).
+cudaError_t run_backward(const Shape& s0, int mode, const void* x, const void* v, const float* W,
+                         const float* bias, const float* tau, const float* t, int tstride, const float* lse,
+                         void* dfx, void* dx, float* dzp, float* dW, float* db, float* dtau, int accumulate,
+                         uint8_t* ws, uint32_t* status, cudaStream_t st) {
+  const SlotRanges sr = slot_ranges(s0.G);
+  const Shape s = pass_shape(s0);
+  const BwdLayout L = bwd_layout(s0, mode);
+  const bool ranged = sr.n > 1;
+  const int64_t Np = padded_n(s);
+  const int64_t npx = s.BH() * Np;
+  const int has_c = mode == 2 ? 1 : 0;
+  cudaError_t e;
+  auto range_g = [&](int k) { return k < sr.n - 1 ? sr.size : s0.G - (sr.n - 1) * sr.size; };
+
+  // Images of range k: t's, W's (and W'^T's when wt).
+  auto prep_range = [&](int k, bool wt) -> cudaError_t {
+    const int g0 = k * sr.size, G = range_g(k);
+    const float *Wk = W, *bk = bias, *tk = t;
+    cudaError_t r;
+    if (ranged) {
+      float* wc = reinterpret_cast<float*>(ws + L.wc);
+      float* bc = reinterpret_cast<float*>(ws + L.bc);
+      float* tc = reinterpret_cast<float*>(ws + L.tc);
+      if ((r = copy_rows(wc, G, W + g0, s0.G, G, (int64_t)s.H * kD, st)) != cudaSuccess) return r;
+      if ((r = copy_rows(bc, G, bias + g0, s0.G, G, s.H, st)) != cudaSuccess) return r;
+      if ((r = copy_rows(tc, (int64_t)G * tstride, t + (int64_t)g0 * tstride, (int64_t)s0.G * tstride,
+                         (int64_t)G * tstride, s.BH(), st)) != cudaSuccess)
+        return r;
+      Wk = wc, bk = bc, tk = tc;
+    }
+    if ((r = prep_t_images(s, G, tk, tstride, has_c, ws, L, st)) != cudaSuccess) return r;
+    if ((r = prep_w(s, G, Wk, bk, tau, ws + L.wimg, status, st)) != cudaSuccess) return r;
+    if (wt) {
+      const int64_t nwt = (int64_t)s.H * kD * s.G;
+      k_prep_wt<<<(unsigned)((nwt + 255) / 256), 256, 0, st>>>(Wk, tau, ws + L.wtimg, s.H, G, s.G, status);
+      r = cudaGetLastError();
+    }
+    return r;
+  };
+
+  k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(ws + L.px), s.BH(), s.N,
+                                                             Np);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  float* delta = reinterpret_cast<float*>(ws + L.delta);
+  float* wds = mode == 2 ? reinterpret_cast<float*>(ws + L.wds) : nullptr;
+  if (wds && (e = cudaMemsetAsync(wds, 0, 2 * (size_t)s.BH() * s.N * sizeof(float), st)) != cudaSuccess) return e;
+  for (int k = 0; k < sr.n; k++) {
+    if ((e = prep_range(k, false)) != cudaSuccess) return e;
+    if ((e = tc_rows_bwd(s, mode, x, ws + L.wimg, ws + L.zimg, ws + L.px, v, dfx, delta, wds,
+                         reinterpret_cast<const float*>(ws + L.ds), k > 0 ? 1 : 0, status, st)) != cudaSuccess)
+      return e;
+  }
+  k_prep_dpx<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(delta, wds, reinterpret_cast<uint4*>(ws + L.dpx),
+                                                              s.BH(), s.N, Np);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+
+  CUtensorMap xmap, vmap, pmap, dmap;
+  if (!make_maps(s, x, v, ws + L.px, ws + L.dpx, &xmap, &vmap, &pmap, &dmap)) return cudaErrorInvalidValue;
+  const int R = bwd_slot_blocks(s), P = bwd_slot_splits(s);
+  for (int k = 0; k < sr.n; k++) {
+    const int g0 = k * sr.size, G = range_g(k);
+    // The images of the last range are still in place after the rows passes; W'^T is not.
+    if (ranged) {
+      if ((e = prep_range(k, true)) != cudaSuccess) return e;
+    } else {
+      const int64_t nwt = (int64_t)s.H * kD * s.G;
+      k_prep_wt<<<(unsigned)((nwt + 255) / 256), 256, 0, st>>>(W, tau, ws + L.wtimg, s.H, G, s.G, status);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    {
+      const size_t sm = smem_bwd_slot();
+      const auto kernel = mode == 1 ? k_bwd_slot_tc<1, true> : k_bwd_slot_tc<2, true>;
+      if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
+      kernel<<<dim3((unsigned)R, (unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(
+          xmap, vmap, pmap, dmap, ws + L.wimg, ws + L.timg, reinterpret_cast<float*>(ws + L.part),
+          reinterpret_cast<float*>(ws + L.dtp), s.N, Np, s.H, s.G, P, status);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    // The slot-owned gradients of range k: straight into dW, dbias (and dz') with
+    // one range; else into the range's buffers (holding dW, dbias's values when
+    // they are added to), then to their places.  dtau sums over the ranges.
+    const int acc = accumulate || k > 0;
+    Shape sk = s0;
+    sk.G = G;
+    float *dWk = dW, *dbk = db, *dzk = dzp;
+    if (ranged) {
+      dWk = reinterpret_cast<float*>(ws + L.dwc);
+      dbk = reinterpret_cast<float*>(ws + L.dbc);
+      dzk = mode == 1 ? reinterpret_cast<float*>(ws + L.dzc) : nullptr;
+      if (accumulate) {
+        if ((e = copy_rows(dWk, G, dW + g0, s0.G, G, (int64_t)s.H * kD, st)) != cudaSuccess) return e;
+        if ((e = copy_rows(dbk, G, db + g0, s0.G, G, s.H, st)) != cudaSuccess) return e;
+      } else if (acc) {
+        if ((e = cudaMemsetAsync(dWk, 0, (size_t)s.H * kD * G * sizeof(float), st)) != cudaSuccess) return e;
+        if ((e = cudaMemsetAsync(dbk, 0, (size_t)s.H * G * sizeof(float), st)) != cudaSuccess) return e;
+      }
+    }
+    if ((e = simt_reduce_bwd(sk, P, reinterpret_cast<const float*>(ws + L.part), s.G,
+                             mode == 1 ? 2 * kD + 2 : kD + 2, mode == 1 ? 1 : 0, tau, dzk, dWk, dbk, dtau,
+                             reinterpret_cast<const float*>(ws + L.dtp), (int64_t)P * R, acc, st)) != cudaSuccess)
+      return e;
+    if (ranged) {
+      if ((e = copy_rows(dW + g0, s0.G, dWk, G, G, (int64_t)s.H * kD, st)) != cudaSuccess) return e;
+      if ((e = copy_rows(db + g0, s0.G, dbk, G, G, s.H, st)) != cudaSuccess) return e;
+      if (mode == 1 && (e = copy_rows(dzp + (int64_t)g0 * kD, (int64_t)s0.G * kD, dzk, (int64_t)G * kD,
+                                      (int64_t)G * kD, s.BH(), st)) != cudaSuccess)
+        return e;
+    }
+    {
+      const bool hilo = smem_bwd_dx(s.G, true) <= kMaxSmem;
+      const size_t sm = smem_bwd_dx(s.G, hilo);
+      const int Pd = point_splits(s, (int)s.BH());
+      const auto kernel = k_bwd_dx_tc<true>;
+      if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
+      kernel<<<dim3((unsigned)Pd, (unsigned)s.BH()), kThreads, sm, st>>>(
+          xmap, vmap, pmap, dmap, ws + L.wimg, ws + L.timg, ws + L.wtimg, static_cast<__nv_bfloat16*>(dx), s.N, Np,
+          s.H, s.G, Pd, hilo ? 1 : 0, acc, status);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+  }
+  return cudaSuccess;
+}
+
 }  // namespace
 
 // A single point (N = 1) takes the fp32 SIMT backward: every token is then that
@@ -773,65 +904,41 @@ cudaError_t prep_t_images(const Shape& s, int G, const float* t, int tstride, in
 // cancelling terms of size |dz||fx|/(S + eps) that split bf16 products resolve only
 // to ~2^-17 of that size.
 bool tc_backward_supported(const Shape& s0) {
-  if (s0.dtype != FS_BF16 || !tc_forward_supported(s0) || s0.N < 2) return false;
-  const Shape s = tc_padded(s0);
-  return smem_bwd_dx(s.G, false) <= kMaxSmem && tc_rows_smem(s, 2, false, false) <= kMaxSmem;
+  if (s0.dtype != FS_BF16 || s0.d != kD || s0.N < 2 || s0.G > 4096) return false;
+  const Shape s = pass_shape(s0);
+  return tc_forward_supported(s) && smem_bwd_dx(s.G, false) <= kMaxSmem &&
+         tc_rows_smem(s, 2, false, false) <= kMaxSmem;
 }
 
 size_t tc_backward_bytes(const Shape& s, int mode) {
-  return tc_backward_supported(s) ? bwd_layout(tc_padded(s), mode).total : 0;
+  return tc_backward_supported(s) ? bwd_layout(s, mode).total : 0;
 }
 
-int tc_backward_slot_splits(const Shape& s) { return bwd_slot_splits(s); }
-
-// prep_t, prep_z2; prep_w, prep_wt, prep_px, rows, prep_dpx, slot, dx; the
-// reductions of the parameters and dtau (and of dz' in mode 1); in mode 2 also
-// the slice backward's dU/dS prologue.
-int tc_backward_launch_count(int mode) { return 2 + 7 + (mode == 1 ? 3 : 2 + 1); }
-
-// The backward forms every weight with split products whatever the forward's
-// arithmetic: its lse comes from split products (recomputed when the forward's
-// did not), and weights from bf16 logits would not sum to one against it; the
-// excess would bias the gradients that are sums of cancelling terms (dbias, dtau).
-Shape split_shape(const Shape& s) {
-  Shape r = s;
-  r.dot = FS_DOT_BF16X2;
-  return r;
+int tc_backward_launch_count(const Shape& s, int mode) {
+  const SlotRanges sr = slot_ranges(s.G);
+  // per range: prep_t, prep_z2, prep_w, rows; then prep_px, prep_dpx; per range: the
+  // images again (or prep_wt alone with one range), slot, dx and the reductions of
+  // the parameters and dtau (and of dz' in mode 1); mode 2 also the dU/dS prologue.
+  const int images = sr.n > 1 ? 4 : 1;
+  const int reduce = mode == 1 ? 3 : 2;
+  return 4 * sr.n + 2 + sr.n * (images + 2 + reduce) + (mode == 2 ? 1 : 0);
 }
 
 cudaError_t tc_deslice_bwd(const Shape& s0, const void* x, const float* W, const float* bias, const float* tau,
                            const float* zp, const float* lse, const void* dout, float* dzp, void* dx, float* dW,
                            float* db, float* dtau, int accumulate, void* ws_tc, uint32_t* status, cudaStream_t st) {
-  const Shape s = tc_padded(split_shape(s0));
-  const BwdLayout L = bwd_layout(s, 1);
-  uint8_t* ws = static_cast<uint8_t*>(ws_tc);
-  cudaError_t e = prep_t_images(s, s0.G, zp, kD, 0, ws, L, st);
-  if (e != cudaSuccess) return e;
-  if ((e = run_backward(s, s0.G, 1, x, dout, W, bias, tau, lse, nullptr, dx, accumulate, ws, L, status, st)) !=
-      cudaSuccess)
-    return e;
-  const int P = bwd_slot_splits(s);
-  return simt_reduce_bwd(s0, P, reinterpret_cast<const float*>(ws + L.part), s.G, 2 * kD + 2, 1, tau, dzp, dW, db,
-                         dtau, reinterpret_cast<const float*>(ws + L.dtp), (int64_t)P * bwd_slot_blocks(s),
-                         accumulate, st);
+  return run_backward(s0, 1, x, dout, W, bias, tau, zp, kD, lse, nullptr, dx, dzp, dW, db, dtau, accumulate,
+                      static_cast<uint8_t*>(ws_tc), status, st);
 }
 
 cudaError_t tc_slice_bwd(const Shape& s0, const void* x, const void* f, const float* W, const float* bias,
                          const float* tau, const float* z, const float* wsum, const float* lse, const float* dz,
                          void* dx, void* dfx, float* dW, float* db, float* dtau, int accumulate, float* dUS,
                          void* ws_tc, uint32_t* status, cudaStream_t st) {
-  const Shape s = tc_padded(split_shape(s0));
-  const BwdLayout L = bwd_layout(s, 2);
-  uint8_t* ws = static_cast<uint8_t*>(ws_tc);
   cudaError_t e = simt_slice_bwd_prep(s0, z, wsum, dz, dUS, st);
   if (e != cudaSuccess) return e;
-  if ((e = prep_t_images(s, s0.G, dUS, kD + 1, 1, ws, L, st)) != cudaSuccess) return e;
-  if ((e = run_backward(s, s0.G, 2, x, f, W, bias, tau, lse, dfx, dx, accumulate, ws, L, status, st)) != cudaSuccess)
-    return e;
-  const int P = bwd_slot_splits(s);
-  return simt_reduce_bwd(s0, P, reinterpret_cast<const float*>(ws + L.part), s.G, kD + 2, 0, tau, nullptr, dW, db,
-                         dtau, reinterpret_cast<const float*>(ws + L.dtp), (int64_t)P * bwd_slot_blocks(s),
-                         accumulate, st);
+  return run_backward(s0, 2, x, f, W, bias, tau, dUS, kD + 1, lse, dfx, dx, nullptr, dW, db, dtau, accumulate,
+                      static_cast<uint8_t*>(ws_tc), status, st);
 }
 
 }  // namespace fs

@@ -73,8 +73,10 @@ using namespace tc;
 //   MODE 1 (deslice backward, t = z', v = dO): delta_n = dO_n . R_n (fp32);
 //   MODE 2 (slice backward, t = dU, v = fx): dfx_n = R_n (bf16, into out) and
 //     delta_n = fx_n . R_n + sum_g w_ng dS_g.  The second sum is formed by the
-//     softmax warpgroups from the fp32 weights; each warpgroup stores its own
-//     partial per point (wds[wg][bh][n], cleared beforehand) and the consumer adds them.
+//     softmax warpgroups from the fp32 weights; each warpgroup adds its own
+//     partial per point to wds[wg][bh][n] (cleared beforehand) and the consumer adds them.
+// accumulate (MODES 1, 2): the pass covers a later range of the slots, whose
+// contributions to delta and dfx are added to those of the earlier ranges.
 // PS (split products): the weights and t as bf16 hi + lo halves, P t = Phi thi +
 // Plo thi + Phi tlo; the image then holds t's residual half after its bf16 half.
 // =========================================================================================
@@ -97,7 +99,7 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
               const uint8_t* __restrict__ wimg, const uint8_t* __restrict__ zimg, __nv_bfloat16* __restrict__ out,
               const __nv_bfloat16* __restrict__ v, float* __restrict__ delta, float* __restrict__ wds,
               const float* __restrict__ dS, int64_t N, int64_t Np, int H, int G, int splits, int hilo,
-              uint32_t zstride, uint32_t* status) {
+              uint32_t zstride, int accumulate, uint32_t* status) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   // hilo: the residual half of W' fits in shared memory too (K = 80 logits, as in
@@ -279,11 +281,17 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
           uint4* dst = reinterpret_cast<uint4*>(out + row);
 #pragma unroll
           for (int k = 0; k < 4; k++) {
+            // MODE 2 over a later slot range: add the dfx of the earlier ranges
+            uint4 p4 = make_uint4(0u, 0u, 0u, 0u);
+            if (MODE == 2 && accumulate) p4 = dst[k];
+            const uint32_t pw[4] = {p4.x, p4.y, p4.z, p4.w};
             uint32_t w[4];
 #pragma unroll
             for (int e = 0; e < 4; e++)
-              w[e] = pack_bf16(__uint_as_float(o0[8 * k + 2 * e]) + __uint_as_float(o1[8 * k + 2 * e]),
-                               __uint_as_float(o0[8 * k + 2 * e + 1]) + __uint_as_float(o1[8 * k + 2 * e + 1]));
+              w[e] = pack_bf16(__uint_as_float(o0[8 * k + 2 * e]) + __uint_as_float(o1[8 * k + 2 * e]) +
+                                   __uint_as_float(pw[e] << 16),
+                               __uint_as_float(o0[8 * k + 2 * e + 1]) + __uint_as_float(o1[8 * k + 2 * e + 1]) +
+                                   __uint_as_float(pw[e] & 0xFFFF0000u));
             dst[k] = make_uint4(w[0], w[1], w[2], w[3]);
           }
         }
@@ -303,7 +311,7 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
                          acc);
             }
           }
-          delta[wk.bh * N + n] = acc;
+          delta[wk.bh * N + n] = accumulate ? delta[wk.bh * N + n] + acc : acc;
         }
       }
       return true;
@@ -314,7 +322,7 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
     auto flush_wds = [&]() {
       if (MODE == 2 && wds_tile >= 0) {
         const int64_t n = (wk.tile0 + wds_tile) * kTile + r;
-        if (n < N) wds[((int64_t)wg * gridDim.y + wk.bh) * N + n] = wds_acc;
+        if (n < N) wds[((int64_t)wg * gridDim.y + wk.bh) * N + n] += wds_acc;
       }
       wds_acc = 0.f;
     };
@@ -1045,7 +1053,7 @@ cudaError_t tc_deslice_fwd(const Shape& s0, const void* x, const float* W, const
   if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
   kernel<<<grid, x3 ? kThreads : kDesl4Threads, sm, st>>>(xmap, pmap, xrmap, wimg, zimg, static_cast<__nv_bfloat16*>(out), nullptr,
                                      nullptr, nullptr, nullptr, s.N, Np, s.H, s.G, P, hilo ? 1 : 0,
-                                     (uint32_t)s.G * (ps ? 128 : 64), status);
+                                     (uint32_t)s.G * (ps ? 128 : 64), 0, status);
   return cudaGetLastError();
 }
 
@@ -1053,7 +1061,7 @@ size_t tc_rows_smem(const Shape& s, int mode, bool ps, bool hilo) { return smem_
 
 cudaError_t tc_rows_bwd(const Shape& s, int mode, const void* x, const uint8_t* wimg, const uint8_t* zimg,
                         const void* px, const void* v, void* dfx, float* delta, float* wds, const float* dS,
-                        uint32_t* status, cudaStream_t st) {
+                        int accumulate, uint32_t* status, cudaStream_t st) {
   const bool split = s.dot == FS_DOT_BF16X2;
   const bool ps = split && smem_deslice(s.G, false, mode, true) <= kMaxSmem;
   const bool hilo = split && smem_deslice(s.G, true, mode, ps) <= kMaxSmem;
@@ -1071,7 +1079,7 @@ cudaError_t tc_rows_bwd(const Shape& s, int mode, const void* x, const uint8_t* 
   if (e != cudaSuccess) return e;
   kernel<<<grid, kThreads, sm, st>>>(xmap, pmap, xmap, wimg, zimg, static_cast<__nv_bfloat16*>(dfx),
                                      static_cast<const __nv_bfloat16*>(v), delta, wds, dS, s.N, Np, s.H, s.G, P,
-                                     hilo ? 1 : 0, (uint32_t)s.G * 128, status);
+                                     hilo ? 1 : 0, (uint32_t)s.G * 128, accumulate, status);
   return cudaGetLastError();
 }
 

@@ -82,8 +82,9 @@ def _mixer_identity_noise(rng, H, G, std=0.1):
 NAMED = ("tiny_f32", "surface_bf16", "batched_bf16", "large_g_bf16", "train_bf16")
 
 
-def make_named(name: str, n_override: Optional[int] = None) -> Workload:
-    """One of the five named workloads; `n_override` shrinks N (same recipe)."""
+def make_named(name: str, n_override: Optional[int] = None, g_override: Optional[int] = None) -> Workload:
+    """One of the five named workloads; `n_override` changes N and `g_override`
+    the slot count G (same recipe otherwise)."""
     idx = NAMED.index(name) + 1
     rng = np.random.Generator(np.random.PCG64(1000 + idx))
     H, d = 8, 32
@@ -100,6 +101,8 @@ def make_named(name: str, n_override: Optional[int] = None) -> Workload:
         B, N, G, dtype, bwd = 2, 524288, 512, "bf16", True
     if n_override is not None:
         N = int(n_override)
+    if g_override is not None:
+        G = int(g_override)
     mixture = name in ("batched_bf16", "train_bf16")
     if mixture:
         x = _gmm_points(rng, B, N, C).reshape(B, N, H, d)

@@ -1,6 +1,6 @@
-"""GPU parity of the tcgen05 tensor-core backward (bf16, d = 32, G up to 640,
-padded inside the kernels to whole 128-slot blocks) against the fp64 oracle, at
-both product arithmetics.
+"""GPU parity of the tcgen05 tensor-core backward (bf16, d = 32, G up to 4096,
+padded inside the kernels to whole 128-slot blocks; past 640 slots every pass runs
+over slot ranges) against the fp64 oracle, at both product arithmetics.
 
 Each backward call runs in isolation, fed with the ORACLE's forward values
 (mixed tokens, tokens, weight sums and lse), so that only the backward kernels
@@ -35,6 +35,14 @@ SHAPES = [
     (2, 2049, 2, 256),
     (1, 1000, 2, 100),  # G padded to 128 inside the kernels
     (2, 777, 1, 48),
+]
+# G past 640: the passes run over 2, 2, 3 and 8 slot ranges (the last one ragged
+# for G = 700 and 1500).
+RANGED = [
+    (1, 300, 2, 700),
+    (1, 2000, 2, 1024),
+    (2, 129, 1, 1500),
+    (1, 257, 1, 4096),
 ]
 TOL = 1e-2
 
@@ -85,7 +93,7 @@ def _run(lib, wl, dev, dot, accumulate=False, path=1):
 
 
 @pytest.mark.parametrize("dot", ["bf16", "bf16x2"])
-@pytest.mark.parametrize("shp", SHAPES, ids=lambda s: "B{}N{}H{}G{}".format(*s))
+@pytest.mark.parametrize("shp", SHAPES + RANGED, ids=lambda s: "B{}N{}H{}G{}".format(*s))
 def test_tc_backward_calls(lib, shp, dot):
     B, N, H, G = shp
     wl = make_case(B, N, H, 32, G, dtype="bf16", seed=600 + N + G, backward=True)
@@ -101,8 +109,9 @@ def test_tc_backward_calls(lib, shp, dot):
     assert not bad, "rel L2 above {:.0e}: {}".format(TOL, {k: "{:.3e}".format(e) for k, e in bad.items()})
 
 
-def test_tc_backward_accumulates(lib):
-    wl = make_case(2, 1500, 2, 32, 256, dtype="bf16", seed=611, backward=True)
+@pytest.mark.parametrize("G", [256, 1024])
+def test_tc_backward_accumulates(lib, G):
+    wl = make_case(2, 1500, 2, 32, G, dtype="bf16", seed=611 + G, backward=True)
     dev = upload(wl)
     got, ref = _run(lib, wl, dev, lib.FS_DOT_BF16X2, accumulate=True)
     for k in ("dx_mid", "dW", "dbias", "dtau"):
@@ -123,7 +132,10 @@ def test_single_point_takes_the_simt_backward(lib):
             assert e <= TOL, f"{call}.{k}: {e:.3e}"
 
 
-def test_tc_backward_shapes_beyond_its_images_take_the_simt_path(lib):
-    s = lib.make_shape(1, 4096, 2, 32, 1024, lib.FS_BF16)
-    assert lib.path_for_shape(s) == 1
-    assert lib.backward_path_for_shape(s) == 0
+def test_backward_path_by_shape(lib):
+    """bf16, d = 32: the tensor-core backward up to the header's G = 4096 (slot
+    ranges past 640), the SIMT backward for other head widths."""
+    assert lib.backward_path_for_shape(lib.make_shape(1, 4096, 2, 32, 1024, lib.FS_BF16)) == 1
+    assert lib.backward_path_for_shape(lib.make_shape(1, 4096, 2, 32, 4096, lib.FS_BF16)) == 1
+    assert lib.path_for_shape(lib.make_shape(1, 4096, 2, 32, 4096, lib.FS_BF16)) == 0
+    assert lib.backward_path_for_shape(lib.make_shape(1, 4096, 2, 64, 1024, lib.FS_BF16)) == 0
