@@ -45,9 +45,11 @@
  *    device agree bit for bit.
  *  - Supported: d in {16, 32, 64}; G in [1, 4096]; B*H <= 65535; B*N*H*d < 2^40.
  *    Kernels (fs_path_for_shape, fs_backward_path_for_shape say which):
- *      FS_BF16, d = 32, G <= 1024: tcgen05 tensor cores, fp32 accumulation, at
- *        the dot level of fs_shape.dot (below); the backward on tensor cores for
- *        G <= 640 (always with split products), else in fp32 FMA.
+ *      FS_BF16, d = 32, G <= 1024: the forward on tcgen05 tensor cores, fp32
+ *        accumulation, at the dot level of fs_shape.dot (below).
+ *      FS_BF16, d = 32, N >= 2 (any supported G): the backward on tensor cores,
+ *        always with split products; past G = 640 its passes run over ranges of
+ *        at most 640 slots, whose dx_mid and dfx contributions are summed in bf16.
  *      FS_F32, d = 32, G <= 512, B*N*H*G >= 2^24: the forward on tensor cores
  *        with every operand split into two bf16 halves (normwise relative error
  *        ~1e-5); the backward in fp32 FMA.
@@ -278,7 +280,8 @@ int fs_path_for_shape(const fs_shape* s);
 
 /* Kernel path of the backward (fs_deslice_bwd, fs_slice_bwd) for this shape:
  * 0 = SIMT fp32 kernels, 1 = tcgen05 tensor-core kernels (bf16, d = 32,
- * G <= 640, N >= 2; the weights with split products whatever s->dot says).
+ * N >= 2, any supported G, over slot ranges past G = 640; the weights with split
+ * products whatever s->dot says).
  * For tests and benchmarks. */
 int fs_backward_path_for_shape(const fs_shape* s);
 
