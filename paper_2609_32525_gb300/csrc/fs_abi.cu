@@ -21,7 +21,7 @@ int slot_splits(const Shape& s) {
   const int64_t gblocks = (s.G + 127) / 128;
   const int64_t units = s.BH() * gblocks;
   int64_t P = (2LL * num_sms() + units - 1) / units;
-  const int64_t max_by_n = (s.N + 255) / 256;
+  const int64_t max_by_n = (s.N + 63) / 64;
   if (P > max_by_n) P = max_by_n;
   if (P < 1) P = 1;
   if (P > 1024) P = 1024;

@@ -191,15 +191,24 @@ __global__ void __launch_bounds__(kThreads) k_slice_partial(
       sl[i] = (n < n_end) ? lse[bh * N + n] * kLog2e : CUDART_INF_F;
     }
     __syncthreads();
-#pragma unroll 4
-    for (int j = 0; j < PT; j++) {
-      float a = bb;
+    // Four points at a time: their logits are independent chains; the sums take
+    // the points in order.
+#pragma unroll 1
+    for (int j = 0; j < PT; j += 4) {
+      float a[4] = {bb, bb, bb, bb};
 #pragma unroll
-      for (int k = 0; k < D; k++) a = fmaf(sx[j][k], wc[k], a);
-      const float w = exp2f(a - sl[j]);
-      S += w;
+      for (int k = 0; k < D; k++)
 #pragma unroll
-      for (int k = 0; k < D; k++) U[k] = fmaf(w, sf[j][k], U[k]);
+        for (int q = 0; q < 4; q++) a[q] = fmaf(sx[j + q][k], wc[k], a[q]);
+      float w[4];
+#pragma unroll
+      for (int q = 0; q < 4; q++) w[q] = exp2f(a[q] - sl[j + q]);
+#pragma unroll
+      for (int q = 0; q < 4; q++) {
+        S += w[q];
+#pragma unroll
+        for (int k = 0; k < D; k++) U[k] = fmaf(w[q], sf[j + q][k], U[k]);
+      }
     }
   }
   if (g < G) {
@@ -210,34 +219,44 @@ __global__ void __launch_bounds__(kThreads) k_slice_partial(
   }
 }
 
-// Fixed-order sum of the P partials, then (optionally) the normalisation.
-// One thread per (slot, column) of the partials [P, BHG, D+1]: consecutive threads
-// read consecutive words of every split.  The sum over splits runs in split order.
-// Partials hold Gs >= G slot rows per (b, h) (the tensor-core path pads G to whole
-// 128-slot blocks); only the first G are reduced.
+// Fixed-order sum of the P partials [P, BHG, D+1], then (optionally) the
+// normalisation.  The sum over splits runs in split order.  Partials hold Gs >= G
+// slot rows per (b, h) (the tensor-core path pads G to whole 128-slot blocks);
+// only the first G are reduced.
 __global__ void k_reduce_tokens(const float* __restrict__ part, int P, int64_t BH, int G, int Gs, int D,
                                 float* __restrict__ tokens, float* __restrict__ wsum, int finalize,
                                 float eps) {
-  const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (idx >= BH * G * (D + 1)) return;
-  const int64_t i = idx / (D + 1);  // output row bh * G + g
-  const int c = (int)(idx % (D + 1));
+  // One warp per output row bh * G + g; lane l sums columns l, l + 32, l + 64 (<= D)
+  // of its partial row over the splits, loads four splits ahead.
+  const int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  if (i >= BH * G) return;  // whole warps
   const int64_t row = (i / G) * Gs + i % G;  // its partial row
   const int64_t stride = BH * Gs * (D + 1);
-  const int64_t at = row * (D + 1) + c;
-  float v = 0.f;
-  for (int p = 0; p < P; p++) v += part[(int64_t)p * stride + at];
-  if (c == D) {
-    wsum[i] = v;
-    return;
+  const float* src = part + row * (D + 1);
+  float v[3] = {0.f, 0.f, 0.f};
+#pragma unroll
+  for (int j = 0; j < 3; j++) {
+    const int c = lane + 32 * j;
+    if (c > D) continue;
+    int p = 0;
+    for (; p + 4 <= P; p += 4) {
+      const float a0 = src[(int64_t)p * stride + c], a1 = src[(int64_t)(p + 1) * stride + c];
+      const float a2 = src[(int64_t)(p + 2) * stride + c], a3 = src[(int64_t)(p + 3) * stride + c];
+      v[j] = (((v[j] + a0) + a1) + a2) + a3;
+    }
+    for (; p < P; p++) v[j] += src[(int64_t)p * stride + c];
   }
-  if (!finalize) {
-    tokens[i * D + c] = v;
-    return;
+  const int jS = D >> 5;  // column D (the weight sum) is lane D % 32's entry jS
+  const float S = __shfl_sync(0xffffffffu, jS == 0 ? v[0] : (jS == 1 ? v[1] : v[2]), D & 31);
+#pragma unroll
+  for (int j = 0; j < 3; j++) {
+    const int c = lane + 32 * j;
+    if (c < D)
+      tokens[i * D + c] = finalize ? v[j] / (S + eps) : v[j];
+    else if (c == D)
+      wsum[i] = v[j];
   }
-  float S = 0.f;
-  for (int p = 0; p < P; p++) S += part[(int64_t)p * stride + row * (D + 1) + D];
-  tokens[i * D + c] = v / (S + eps);
 }
 
 __global__ void k_finalize(float* __restrict__ tokens, const float* __restrict__ wsum, int64_t BHG,
@@ -520,13 +539,24 @@ __global__ void __launch_bounds__(kThreads) k_deslice(const T* __restrict__ x, c
     }
     __syncthreads();
     const int gn = min(GC, G - g0);
-    for (int g = 0; g < gn; g++) {
-      float a = sB[g];
+    // Four slots at a time (independent logit chains); the output sums the slots in
+    // order.  Slots past gn have zero z' rows and add exact zeros.
+#pragma unroll 1
+    for (int g = 0; g < gn; g += 4) {
+      float a[4];
 #pragma unroll
-      for (int k = 0; k < D; k++) a = fmaf(xr[k], sW[g][k], a);
-      const float w = exp2f(a - l2);
+      for (int q = 0; q < 4; q++) a[q] = sB[g + q];
 #pragma unroll
-      for (int k = 0; k < D; k++) acc[k] = fmaf(w, sZ[g][k], acc[k]);
+      for (int k = 0; k < D; k++)
+#pragma unroll
+        for (int q = 0; q < 4; q++) a[q] = fmaf(xr[k], sW[g + q][k], a[q]);
+#pragma unroll
+      for (int q = 0; q < 4; q++) {
+        if (g + q >= gn) break;
+        const float w = exp2f(a[q] - l2);
+#pragma unroll
+        for (int k = 0; k < D; k++) acc[k] = fmaf(w, sZ[g + q][k], acc[k]);
+      }
     }
   }
   if (valid) store_row<D>(out + row_index(b, n, h, N, H) * D, acc);
@@ -919,7 +949,7 @@ cudaError_t simt_slice_partials(const Shape& s, int P, const void* x, const void
 
 cudaError_t simt_reduce_tokens(const Shape& s, int P, const float* part, int Gs, float* tokens, float* wsum,
                                int finalize, cudaStream_t st) {
-  const int64_t n = s.BH() * s.G * (s.d + 1);
+  const int64_t n = s.BH() * s.G * 32;  // a warp per output row
   k_reduce_tokens<<<(unsigned)((n + 255) / 256), 256, 0, st>>>(part, P, s.BH(), s.G, Gs, s.d, tokens, wsum, finalize,
                                                                s.eps);
   return cudaGetLastError();

@@ -55,12 +55,16 @@ __device__ __forceinline__ uint32_t off_z(int c, int g) {
 
 // Slots [G, Gp) pad the image to whole 128-slot blocks: W' = 0 and b' = -1e30, so
 // their logits are -1e30 and their weights exactly 0 in every pass.
+// Thread (h, q, g): for q < 4 the 16-byte pieces of channels [8q, 8q + 8) of slot g
+// in both halves of W'; for q = 4 the slot's extra row.  Consecutive threads take
+// consecutive slots, so the reads of W [H, d, G] coalesce.
 __global__ void k_prep_w(const float* __restrict__ W, const float* __restrict__ bias, const float* __restrict__ tau,
                          uint8_t* __restrict__ img, int H, int G, int Gp, uint32_t* status) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t total = (int64_t)H * Gp;
-  if (i >= total) return;
-  const int h = (int)(i / Gp), g = (int)(i % Gp);
+  if (i >= (int64_t)H * 5 * Gp) return;
+  const int g = (int)(i % Gp);
+  const int q = (int)((i / Gp) % 5);
+  const int h = (int)(i / ((int64_t)5 * Gp));
   const float t = tau[h];
   if (!(t > 0.f && t < INFINITY)) {
     atomicCAS(status, 0u, (uint32_t)FS_ERR_BAD_TAU);
@@ -69,22 +73,31 @@ __global__ void k_prep_w(const float* __restrict__ W, const float* __restrict__ 
   const float scale = kLog2e / t;
   const bool real = g < G;
   uint8_t* base = img + (size_t)h * Gp * kWRow;
-  __nv_bfloat16* wp = reinterpret_cast<__nv_bfloat16*>(base);
-  __nv_bfloat16* wl = reinterpret_cast<__nv_bfloat16*>(base + (size_t)Gp * 96);
-  for (int k = 0; k < kD; k++) {
-    const float w2 = real ? W[((int64_t)h * kD + k) * G + g] * scale : 0.f;
-    const __nv_bfloat16 whi = __float2bfloat16_rn(w2);
-    wp[off_sw64(g, k) / 2] = whi;
-    wl[off_sw64(g, k) / 2] = __float2bfloat16_rn(w2 - __bfloat162float(whi));
+  if (q < 4) {
+    uint32_t hi[4], lo[4];
+#pragma unroll
+    for (int e = 0; e < 4; e++) {
+      const int k = 8 * q + 2 * e;
+      const float w0 = real ? W[((int64_t)h * kD + k) * G + g] * scale : 0.f;
+      const float w1 = real ? W[((int64_t)h * kD + k + 1) * G + g] * scale : 0.f;
+      const uint32_t p = pack_bf16(w0, w1);
+      hi[e] = p;
+      lo[e] = pack_bf16(w0 - __uint_as_float(p << 16), w1 - __uint_as_float(p & 0xFFFF0000u));
+    }
+    const uint32_t off = off_sw64(g, 8 * q);
+    *reinterpret_cast<uint4*>(base + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+    *reinterpret_cast<uint4*>(base + (size_t)Gp * 96 + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+    return;
   }
-  __nv_bfloat16* ep = reinterpret_cast<__nv_bfloat16*>(base + (size_t)Gp * 64);
+  // The extra row [b'_hi, b'_lo, 1, 1, 0 ...]; k = 2, 3 multiply the point side's
+  // -lse2 halves (zero in the statistics pass).
   const float b2 = real ? bias[(int64_t)h * G + g] * scale : -1e30f;
-  const __nv_bfloat16 hi = __float2bfloat16_rn(b2);
-  const __nv_bfloat16 lo = __float2bfloat16_rn(b2 - __bfloat162float(hi));
-  // k = 2, 3 multiply the point side's -lse2 halves (zero in the statistics pass).
-  for (int k = 0; k < 16; k++)
-    ep[off_sw32(g, k) / 2] =
-        k == 0 ? hi : (k == 1 ? lo : __float2bfloat16_rn((k == 2 || k == 3) ? 1.f : 0.f));
+  const uint32_t bp = pack_bf16(b2, 0.f) & 0xFFFFu;
+  const float bhi = __uint_as_float(bp << 16);
+  const uint32_t blo = pack_bf16(b2 - bhi, 0.f) & 0xFFFFu;
+  uint8_t* ep = base + (size_t)Gp * 64;
+  *reinterpret_cast<uint4*>(ep + off_sw32(g, 0)) = make_uint4(bp | (blo << 16), 0x3F803F80u, 0u, 0u);
+  *reinterpret_cast<uint4*>(ep + off_sw32(g, 8)) = make_uint4(0u, 0u, 0u, 0u);
 }
 
 // Padding slots [G, Gp) get zero rows (their weights are 0, and 0 * 0 stays 0).
@@ -504,7 +517,7 @@ cudaError_t set_smem(K kernel, size_t bytes) {
 // W image of the padded shape sp (sp.G = G rounded up) from W [H, d, G].
 cudaError_t prep_w(const Shape& sp, int G, const float* W, const float* bias, const float* tau, uint8_t* img,
                    uint32_t* status, cudaStream_t st) {
-  const int64_t n = (int64_t)sp.H * sp.G;
+  const int64_t n = (int64_t)sp.H * 5 * sp.G;
   k_prep_w<<<(unsigned)((n + 127) / 128), 128, 0, st>>>(W, bias, tau, img, sp.H, G, sp.G, status);
   return cudaGetLastError();
 }
