@@ -50,7 +50,7 @@
  *      FS_BF16, d = 32, N >= 2 (any supported G): the backward on tensor cores,
  *        always with split products; past G = 640 its passes run over ranges of
  *        at most 640 slots, whose dx_mid and dfx contributions are summed in bf16.
- *      FS_F32, d = 32, G <= 512, B*N*H*G >= 2^24: the forward on tensor cores
+ *      FS_F32, d = 32, G <= 1024, B*N*H*G >= 2^24: the forward on tensor cores
  *        with every operand split into two bf16 halves (normwise relative error
  *        ~1e-5); the backward in fp32 FMA.
  *      everything else: fp32 FMA (SIMT) kernels.

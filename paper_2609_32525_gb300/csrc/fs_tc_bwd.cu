@@ -668,8 +668,9 @@ int bwd_slot_splits(const Shape& s) { return point_splits(s, (int)(s.BH() * bwd_
 // `size` slots (a multiple of 128; the last range may hold fewer real slots), all
 // with the full problem's lse, so that the weights of a range are those of the
 // softmax over all G.  The sums over slots (delta, dfx, dx) add up over the
-// ranges; the slot-owned gradients of a range are its own.  `size` is the
-// largest that minimises the padded slot count n * size.
+// ranges; the slot-owned gradients of a range are its own.  `size` minimises the
+// padded slots plus half a block per range (a range re-reads x and v); ties go to
+// the larger size.
 constexpr int kBwdSlotsMax = 640;
 struct SlotRanges {
   int n, size;
@@ -679,7 +680,7 @@ SlotRanges slot_ranges(int G) {
   SlotRanges best{0, 0};
   for (int size = kGC; size <= kBwdSlotsMax; size += kGC) {
     const int n = (G + size - 1) / size;
-    if (best.n == 0 || (int64_t)n * size <= (int64_t)best.n * best.size) best = {n, size};
+    if (best.n == 0 || (int64_t)n * (size + kGC / 2) <= (int64_t)best.n * (best.size + kGC / 2)) best = {n, size};
   }
   return best;
 }
@@ -747,13 +748,6 @@ bool make_maps(const Shape& s, const void* x, const void* v, const void* px, con
   return make_point_map(xmap, x, s, kD, CU_TENSOR_MAP_SWIZZLE_64B) &&
          make_point_map(vmap, v, s, kD, CU_TENSOR_MAP_SWIZZLE_64B) && make_px_map(pmap, px, s.BH(), Np) &&
          make_px_map(dmap, dpx, s.BH(), Np);
-}
-
-// rows x cols floats from src (row pitch spitch floats) to dst (row pitch dpitch floats).
-cudaError_t copy_rows(float* dst, int64_t dpitch, const float* src, int64_t spitch, int64_t cols, int64_t rows,
-                      cudaStream_t st) {
-  return cudaMemcpy2DAsync(dst, (size_t)dpitch * sizeof(float), src, (size_t)spitch * sizeof(float),
-                           (size_t)cols * sizeof(float), (size_t)rows, cudaMemcpyDeviceToDevice, st);
 }
 
 // Slot-side images of t (T image, its c column, Z-layout image) for G slots.

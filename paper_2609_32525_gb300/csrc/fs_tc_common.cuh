@@ -508,6 +508,14 @@ int point_splits(const Shape& s, int units) {
   return (int)best;
 }
 
+// rows x cols floats from src (row pitch spitch floats) to dst (row pitch dpitch
+// floats): a slot range's slice of W [H, d, G], bias [H, G] or a per-slot tensor.
+cudaError_t copy_rows(float* dst, int64_t dpitch, const float* src, int64_t spitch, int64_t cols, int64_t rows,
+                      cudaStream_t st) {
+  return cudaMemcpy2DAsync(dst, (size_t)dpitch * sizeof(float), src, (size_t)spitch * sizeof(float),
+                           (size_t)cols * sizeof(float), (size_t)rows, cudaMemcpyDeviceToDevice, st);
+}
+
 constexpr size_t kMaxSmem = 232448;  // opt-in shared memory per block on sm_103
 template <typename K>
 cudaError_t set_smem(K kernel, size_t bytes) {

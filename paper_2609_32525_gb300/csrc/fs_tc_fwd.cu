@@ -75,8 +75,9 @@ using namespace tc;
 //     delta_n = fx_n . R_n + sum_g w_ng dS_g.  The second sum is formed by the
 //     softmax warpgroups from the fp32 weights; each warpgroup adds its own
 //     partial per point to wds[wg][bh][n] (cleared beforehand) and the consumer adds them.
-// accumulate (MODES 1, 2): the pass covers a later range of the slots, whose
-// contributions to delta and dfx are added to those of the earlier ranges.
+// accumulate (MODES 1, 2, and MODE 0 with X3): the pass covers a later range of the
+// slots, whose contributions to delta and dfx (to the fp32 out) are added to those of
+// the earlier ranges.
 // PS (split products): the weights and t as bf16 hi + lo halves, P t = Phi thi +
 // Plo thi + Phi tlo; the image then holds t's residual half after its bf16 half.
 // =========================================================================================
@@ -270,13 +271,16 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
       if (n < N) {
         const int64_t row = ((b * N + n) * H + h) * kD;
         if (X3) {
+          // accumulate: a later slot range, added to the earlier ranges' output
           float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(out) + row);
 #pragma unroll
-          for (int k = 0; k < 8; k++)
-            dst[k] = make_float4(__uint_as_float(o0[4 * k]) + __uint_as_float(o1[4 * k]),
-                                 __uint_as_float(o0[4 * k + 1]) + __uint_as_float(o1[4 * k + 1]),
-                                 __uint_as_float(o0[4 * k + 2]) + __uint_as_float(o1[4 * k + 2]),
-                                 __uint_as_float(o0[4 * k + 3]) + __uint_as_float(o1[4 * k + 3]));
+          for (int k = 0; k < 8; k++) {
+            const float4 p = accumulate ? dst[k] : make_float4(0.f, 0.f, 0.f, 0.f);
+            dst[k] = make_float4(p.x + (__uint_as_float(o0[4 * k]) + __uint_as_float(o1[4 * k])),
+                                 p.y + (__uint_as_float(o0[4 * k + 1]) + __uint_as_float(o1[4 * k + 1])),
+                                 p.z + (__uint_as_float(o0[4 * k + 2]) + __uint_as_float(o1[4 * k + 2])),
+                                 p.w + (__uint_as_float(o0[4 * k + 3]) + __uint_as_float(o1[4 * k + 3])));
+          }
         } else if (MODE != 1) {
           uint4* dst = reinterpret_cast<uint4*>(out + row);
 #pragma unroll
@@ -840,6 +844,26 @@ int slice_splits(const Shape& s) { return point_splits(s, (int)(s.BH() * slice_b
 // (x, fx and W', the weights, z'): the X3 kernels.  Their inputs are first split
 // into bf16 hi and residual tensors in the workspace (k_split_bf16).
 bool x3_shape(const Shape& s) { return s.dtype == FS_F32; }
+
+// The X3 deslice holds both halves of W' and of z' in shared memory, which fits up to
+// 512 slots; past that it runs over ranges of `size` slots (a multiple of 128), each
+// with the full lse, adding its output to the earlier ranges'.  `size` minimises the
+// padded slots plus half a block per range (a range re-reads x); ties go to the
+// larger size.
+constexpr int kX3SlotsMax = 512;
+struct X3Ranges {
+  int n, size;
+};
+X3Ranges x3_ranges(const Shape& s0) {
+  const int Gp = (s0.G + kGC - 1) / kGC * kGC;
+  if (s0.dtype != FS_F32 || s0.G <= kX3SlotsMax) return {1, Gp};
+  X3Ranges best{0, 0};
+  for (int size = kGC; size <= kX3SlotsMax; size += kGC) {
+    const int n = (s0.G + size - 1) / size;
+    if (best.n == 0 || (int64_t)n * (size + kGC / 2) <= (int64_t)best.n * (best.size + kGC / 2)) best = {n, size};
+  }
+  return best;
+}
 size_t half_bytes(const Shape& s) { return align_up((size_t)s.B * s.N * s.H * s.d * 2, 256); }
 
 size_t smem_deslice(int G, bool hilo, int mode = 0, bool ps = false, bool x3 = false) {
@@ -893,10 +917,10 @@ cudaError_t run_slice(const Shape& s, int G, const void* x, const void* f, const
 bool tc_forward_supported(const Shape& s) {
   // TMA coordinates and the kernels' block counters are 32-bit.
   const int64_t np = (s.N + kTile - 1) / kTile * kTile;
-  // fp32 inputs need the residual half of W' in the deslice's shared memory (G <= 512),
-  // and take the tensor cores only when there is enough work to pay for splitting
-  // their inputs: B*N*H*G >= 2^24 (smaller problems keep the exact fp32 SIMT kernels).
-  const bool fp32_ok = s.dtype == FS_F32 && s.G <= 512 && (double)s.BH() * s.N * s.G >= 16777216.0;
+  // fp32 inputs take the tensor cores only when there is enough work to pay for
+  // splitting their inputs: B*N*H*G >= 2^24 (smaller problems keep the exact fp32
+  // SIMT kernels).  Their deslice runs over slot ranges past 512 slots (X3 ranges).
+  const bool fp32_ok = s.dtype == FS_F32 && (double)s.BH() * s.N * s.G >= 16777216.0;
   return (s.dtype == FS_BF16 || fp32_ok) && s.d == kD && s.G <= 1024 && s.N >= 1 &&
          s.BH() * np < (int64_t(1) << 31) && encode_fn() != nullptr;
 }
@@ -904,7 +928,7 @@ bool tc_forward_supported(const Shape& s) {
 int tc_stats_launch_count(const Shape& s) { return 2 /*prep_w, stats*/ + (x3_shape(s) ? 1 : 0); }
 
 int tc_forward_launch_count(const Shape& s) {
-  return 4 /*prep_w, stats, slice, reduce*/ + 4 /*prep_w, prep_z, prep_px, deslice*/ +
+  return 4 /*prep_w, stats, slice, reduce*/ + 1 /*prep_px*/ + 3 * x3_ranges(s).n /*prep_w, prep_z, deslice*/ +
          (x3_shape(s) ? 3 /*splits of x, fx; of x*/ : 0);
 }
 
@@ -923,8 +947,13 @@ size_t tc_slice_prep_bytes(const Shape& s0) {
 }
 size_t tc_deslice_prep_bytes(const Shape& s0) {
   const Shape s = tc_padded(s0);
+  const X3Ranges xr = x3_ranges(s0);
+  // with several X3 ranges, a range's slices of W, bias and z' too
+  const size_t gather = xr.n > 1 ? align_up((size_t)s.H * (kD + 1) * xr.size * sizeof(float), 256) +
+                                       align_up((size_t)s.BH() * xr.size * kD * sizeof(float), 256)
+                                 : 0;
   return tc_forward_supported(s0) ? align_up(w_image_bytes(s), 256) + align_up(z_image_bytes(s), 256) +
-                                        align_up(px_bytes(s), 256) + (x3_shape(s) ? 2 * half_bytes(s) : 0)
+                                        align_up(px_bytes(s), 256) + (x3_shape(s) ? 2 * half_bytes(s) : 0) + gather
                                   : 0;
 }
 
@@ -1018,22 +1047,21 @@ cudaError_t tc_slice_fwd_lse(const Shape& s0, const void* x, const void* f, cons
 cudaError_t tc_deslice_fwd(const Shape& s0, const void* x, const float* W, const float* bias, const float* tau,
                            const float* zp, const float* lse, void* out, void* prep, uint32_t* status,
                            cudaStream_t st) {
-  const Shape s = tc_padded(s0);
-  const bool x3 = x3_shape(s);
+  const Shape sf = tc_padded(s0);  // the whole problem (layout of the workspace)
+  const bool x3 = x3_shape(sf);
+  const X3Ranges xr = x3_ranges(s0);
+  const bool ranged = xr.n > 1;
+  Shape s = sf;  // the shape the kernel sees: G = the range's slots
+  s.G = xr.size;
   uint8_t* wimg = static_cast<uint8_t*>(prep);
-  uint8_t* zimg = wimg + align_up(w_image_bytes(s), 256);
-  uint8_t* px = zimg + align_up(z_image_bytes(s), 256);
-  uint8_t* xh = px + align_up(px_bytes(s), 256);
-  cudaError_t e = prep_w(s, s0.G, W, bias, tau, wimg, status, st);
-  if (e != cudaSuccess) return e;
-  const int64_t nz = s.BH() * s.G * kD;
-  // With split products the image holds z' hi then its residual (G*128 bytes per (b,h)).
-  const bool ps = x3;
-  if (ps)
-    k_prep_z2<<<(unsigned)((nz + 255) / 256), 256, 0, st>>>(zp, kD, zimg, s.BH(), s0.G, s.G);
-  else
-    k_prep_z<<<(unsigned)((nz + 255) / 256), 256, 0, st>>>(zp, zimg, s.BH(), s0.G, s.G);
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  uint8_t* zimg = wimg + align_up(w_image_bytes(sf), 256);
+  uint8_t* px = zimg + align_up(z_image_bytes(sf), 256);
+  uint8_t* xh = px + align_up(px_bytes(sf), 256);
+  float* wc = reinterpret_cast<float*>(xh + (x3 ? 2 * half_bytes(sf) : 0));  // range slices (ranged only)
+  float* bc = wc + (size_t)s.H * kD * xr.size;
+  float* zc = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(wc) +
+                                       align_up((size_t)s.H * (kD + 1) * xr.size * sizeof(float), 256));
+  cudaError_t e;
   const int64_t Np = padded_n(s), npx = s.BH() * Np;
   k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(px), s.BH(), s.N, Np);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
@@ -1045,16 +1073,37 @@ cudaError_t tc_deslice_fwd(const Shape& s0, const void* x, const float* W, const
   if (!make_px_map(&pmap, px, s.BH(), Np)) return cudaErrorInvalidValue;
   const int P = point_splits(s, (int)s.BH());
   const bool split = s.dot == FS_DOT_BF16X2 || x3;
+  // With split products the image holds z' hi then its residual (G*128 bytes per (b,h)).
+  const bool ps = x3;
   const bool hilo = split && smem_deslice(s.G, true, 0, ps, x3) <= kMaxSmem;  // up to G = 768 (bf16)
   const size_t sm = smem_deslice(s.G, hilo, 0, ps, x3);
   if (sm > kMaxSmem) return cudaErrorInvalidValue;
-  dim3 grid((unsigned)P, (unsigned)s.BH());
   const auto kernel = x3 ? k_deslice<0, true, true> : k_deslice<0, false>;
   if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
-  kernel<<<grid, x3 ? kThreads : kDesl4Threads, sm, st>>>(xmap, pmap, xrmap, wimg, zimg, static_cast<__nv_bfloat16*>(out), nullptr,
-                                     nullptr, nullptr, nullptr, s.N, Np, s.H, s.G, P, hilo ? 1 : 0,
-                                     (uint32_t)s.G * (ps ? 128 : 64), 0, status);
-  return cudaGetLastError();
+  for (int k = 0; k < xr.n; k++) {
+    const int g0 = k * xr.size, G = ranged ? std::min(xr.size, s0.G - g0) : s0.G;
+    const float *Wk = W, *bk = bias, *zk = zp;
+    if (ranged) {
+      if ((e = copy_rows(wc, G, W + g0, s0.G, G, (int64_t)s.H * kD, st)) != cudaSuccess) return e;
+      if ((e = copy_rows(bc, G, bias + g0, s0.G, G, s.H, st)) != cudaSuccess) return e;
+      if ((e = copy_rows(zc, (int64_t)G * kD, zp + (int64_t)g0 * kD, (int64_t)s0.G * kD, (int64_t)G * kD, s.BH(),
+                         st)) != cudaSuccess)
+        return e;
+      Wk = wc, bk = bc, zk = zc;
+    }
+    if ((e = prep_w(s, G, Wk, bk, tau, wimg, status, st)) != cudaSuccess) return e;
+    const int64_t nz = s.BH() * s.G * kD;
+    if (ps)
+      k_prep_z2<<<(unsigned)((nz + 255) / 256), 256, 0, st>>>(zk, kD, zimg, s.BH(), G, s.G);
+    else
+      k_prep_z<<<(unsigned)((nz + 255) / 256), 256, 0, st>>>(zk, zimg, s.BH(), G, s.G);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    kernel<<<dim3((unsigned)P, (unsigned)s.BH()), x3 ? kThreads : kDesl4Threads, sm, st>>>(
+        xmap, pmap, xrmap, wimg, zimg, static_cast<__nv_bfloat16*>(out), nullptr, nullptr, nullptr, nullptr, s.N, Np,
+        s.H, s.G, P, hilo ? 1 : 0, (uint32_t)s.G * (ps ? 128 : 64), k > 0 ? 1 : 0, status);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 size_t tc_rows_smem(const Shape& s, int mode, bool ps, bool hilo) { return smem_deslice(s.G, hilo, mode, ps); }

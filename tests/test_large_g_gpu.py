@@ -3,8 +3,7 @@ the header's limit of 4096 (forward and backward, fp32 and bf16 inputs, every
 supported head width; the forward on the fp32 SIMT kernels, the bf16 d = 32
 backward on the tensor cores over slot ranges), the bf16 backward beyond G = 640
 after a tensor-core forward, and fp32 inputs at G = 768 and 1024 (the fp32
-tensor-core forward stops at G = 512; larger G takes the SIMT kernels whatever
-the problem size).
+tensor-core forward, its deslice over slot ranges past 512 slots).
 
 Tolerances (tests/_parity.py): fp32 inputs normwise max relative error <= 1e-4
 per tensor; bf16 inputs relative L2 error <= 1e-2 per tensor.
@@ -71,15 +70,15 @@ def test_bf16_backward_over_slot_ranges(lib, G):
 
 
 @pytest.mark.parametrize("G", [768, 1024])
-def test_fp32_above_512_slots_takes_the_simt_kernels(lib, G):
-    """fp32 inputs with B*N*H*G >= 2^24 take the tensor cores only up to G = 512;
-    at G = 768 and 1024 the SIMT kernels run, at the fp32 bar."""
+def test_fp32_above_512_slots_on_tensor_cores(lib, G):
+    """fp32 inputs with B*N*H*G >= 2^24 at G = 768 and 1024: the tensor-core
+    forward, its deslice over slot ranges, at the fp32 bar."""
     N = 3000
     assert N * 8 * G >= 1 << 24
     wl = make_case(1, N, 8, 32, G, dtype="f32", seed=1500 + G, backward=False)
     dev = upload(wl)
     c = gpu_forward(lib, wl, dev)
-    assert lib.path_for_shape(c.shape) == 0
+    assert lib.path_for_shape(c.shape) == 1
     torch.cuda.synchronize()
     assert c.device_status() == lib.FS_OK
     ref = oracle_forward(wl)

@@ -1,8 +1,9 @@
-"""GPU parity of the tensor-core forward for fp32 inputs (d = 32, G <= 512,
+"""GPU parity of the tensor-core forward for fp32 inputs (d = 32, G <= 1024,
 B*N*H*G >= 2^24; smaller fp32 problems keep the exact SIMT kernels): every
 operand as two bf16 halves (x, fx, W' = W log2(e)/tau, the weights, z'), the
-paper's three-product level for fp32 data (App. G.2 dot levels).  Against the
-fp64 oracle at the fp32 bar: normwise max relative error <= 1e-4 for tokens, wsum,
+paper's three-product level for fp32 data (App. G.2 dot levels); past 512 slots
+the deslice runs over slot ranges whose fp32 outputs add up.  Against the fp64
+oracle at the fp32 bar: normwise max relative error <= 1e-4 for tokens, wsum,
 tokens_mixed, out and lse.  The backward of these shapes runs on the fp32 SIMT
 kernels with exact fp32 statistics; it is checked too.
 """
@@ -17,7 +18,10 @@ from _parity import host, max_rel, upload
 
 pytestmark = pytest.mark.gpu
 
-SHAPES = [(1, 20001, 8, 128), (1, 33000, 8, 100), (2, 9000, 8, 256), (1, 5000, 8, 512), (1, 70000, 8, 32)]
+# G = 640, 700 and 1024 run the deslice over slot ranges: 384 + 256, 384 + 316 and
+# 2 x 512.
+SHAPES = [(1, 20001, 8, 128), (1, 33000, 8, 100), (2, 9000, 8, 256), (1, 5000, 8, 512), (1, 70000, 8, 32),
+          (1, 4000, 8, 640), (1, 3001, 8, 700), (1, 2500, 8, 1024)]
 TOL = 1e-4
 
 
@@ -36,6 +40,7 @@ def test_fp32_tensor_core_forward(lib, shp):
             "tokens_mixed": max_rel(host(c.tokens_mixed), ref["tokens_mixed"]),
             "out": max_rel(host(c.out), ref["out"]),
             "lse": max_rel(host(c.lse), ref["lse"].transpose(0, 2, 1))}
+    print(shp, " ".join("{}={:.2e}".format(k, e) for k, e in errs.items()))
     bad = {k: e for k, e in errs.items() if not e <= TOL}
     assert not bad, {k: "{:.2e}".format(e) for k, e in bad.items()}
 
@@ -43,7 +48,9 @@ def test_fp32_tensor_core_forward(lib, shp):
 def test_small_fp32_problems_keep_the_simt_kernels(lib):
     assert lib.path_for_shape(lib.make_shape(1, 4096, 8, 32, 32, lib.FS_F32)) == 0
     assert lib.path_for_shape(lib.make_shape(1, 70000, 8, 32, 32, lib.FS_F32)) == 1
-    assert lib.path_for_shape(lib.make_shape(1, 70000, 8, 32, 640, lib.FS_F32)) == 0
+    assert lib.path_for_shape(lib.make_shape(1, 70000, 8, 32, 640, lib.FS_F32)) == 1
+    assert lib.path_for_shape(lib.make_shape(1, 70000, 8, 32, 1024, lib.FS_F32)) == 1
+    assert lib.path_for_shape(lib.make_shape(1, 70000, 8, 32, 1025, lib.FS_F32)) == 0
 
 
 def test_fp32_backward_after_tensor_core_forward(lib):
