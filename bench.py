@@ -277,7 +277,9 @@ def run_train(args, wl, dev, world, rank):
     c = fs.Coupling(wl.B, wl.N, wl.H, wl.d, wl.G, tdt, wl.eps, device=dev, backward=True)
     s = c.shape
     stream = torch.cuda.current_stream()
-    names = ("fs_slice_fwd", "fs_mix", "fs_deslice_fwd", "fs_deslice_bwd", "fs_mix_bwd", "fs_slice_bwd")
+    sep = args.separate_backward
+    names = ("fs_slice_fwd", "fs_mix", "fs_deslice_fwd") + (
+        ("fs_deslice_bwd", "fs_mix_bwd", "fs_slice_bwd") if sep else ("fs_coupling_bwd",))
 
     def step(ev=None, xs=x, fs_=fx, ds=dO, outs=None):
         out, dx, dfx = outs or (c.out, c.dx_mid, c.dfx)
@@ -285,12 +287,21 @@ def run_train(args, wl, dev, world, rank):
             lambda: fs.fs_slice_fwd(s, xs, fs_, W, b, t, c.tokens, c.wsum, c.lse, True, c.ws_slice),
             lambda: fs.fs_mix(s, M, c.tokens, c.tokens_mixed),
             lambda: fs.fs_deslice_fwd(s, xs, W, b, t, c.tokens_mixed, c.lse, out, c.ws_deslice),
-            lambda: fs.fs_deslice_bwd(s, xs, W, b, t, c.tokens_mixed, c.lse, ds, c.d_tokens_mixed, dx, c.dW,
-                                      c.dbias, c.dtau, False, c.ws_dbwd),
-            lambda: fs.fs_mix_bwd(s, M, c.tokens, c.d_tokens_mixed, c.d_tokens, c.dM),
-            lambda: fs.fs_slice_bwd(s, xs, fs_, W, b, t, c.tokens, c.wsum, c.lse, c.d_tokens, dx, dfx, c.dW,
-                                    c.dbias, c.dtau, True, c.ws_sbwd),
         )
+        if sep:
+            calls += (
+                lambda: fs.fs_deslice_bwd(s, xs, W, b, t, c.tokens_mixed, c.lse, ds, c.d_tokens_mixed, dx, c.dW,
+                                          c.dbias, c.dtau, False, c.ws_dbwd),
+                lambda: fs.fs_mix_bwd(s, M, c.tokens, c.d_tokens_mixed, c.d_tokens, c.dM),
+                lambda: fs.fs_slice_bwd(s, xs, fs_, W, b, t, c.tokens, c.wsum, c.lse, c.d_tokens, dx, dfx, c.dW,
+                                        c.dbias, c.dtau, True, c.ws_sbwd),
+            )
+        else:
+            calls += (
+                lambda: fs.fs_coupling_bwd(s, xs, fs_, W, b, t, M, c.tokens, c.wsum, c.tokens_mixed, c.lse, ds,
+                                           c.d_tokens_mixed, c.d_tokens, dx, dfx, c.dW, c.dbias, c.dtau, c.dM, False,
+                                           c.ws_cbwd),
+            )
         for i, call in enumerate(calls):
             if ev is not None:
                 ev[i].record(stream)
@@ -359,9 +370,13 @@ def run_train(args, wl, dev, world, rank):
     P = wl.B * wl.N
     flops, bytes_ = 24.0 * C * wl.G * P, 11.0 * C * e * P
     per_call = {"fs_slice_fwd": 4.0 * C * wl.G * P, "fs_deslice_fwd": 4.0 * C * wl.G * P,
-                "fs_deslice_bwd": 8.0 * C * wl.G * P, "fs_slice_bwd": 8.0 * C * wl.G * P}
+                "fs_deslice_bwd": 8.0 * C * wl.G * P, "fs_slice_bwd": 8.0 * C * wl.G * P,
+                "fs_coupling_bwd": 16.0 * C * wl.G * P}
     per_call_bytes = {"fs_slice_fwd": 2.0 * C * e * P, "fs_deslice_fwd": 2.0 * C * e * P,
-                      "fs_deslice_bwd": 3.0 * C * e * P, "fs_slice_bwd": 4.0 * C * e * P}
+                      "fs_deslice_bwd": 3.0 * C * e * P, "fs_slice_bwd": 4.0 * C * e * P,
+                      "fs_coupling_bwd": 7.0 * C * e * P}
+    per_call = {k: v for k, v in per_call.items() if k in call_ms}
+    per_call_bytes = {k: v for k, v in per_call_bytes.items() if k in call_ms}
     peaks = _peaks()
     dom = max(per_call, key=lambda k: call_ms[k])
     t_tensor, t_hbm = flops / (peaks["bf16_tflops"] * 1e12), bytes_ / (peaks["hbm_gbs"] * 1e9)
@@ -376,8 +391,9 @@ def run_train(args, wl, dev, world, rank):
                  "frac": achieved / peaks["hbm_gbs"], "peak_source": peaks["source"] + " HBM copy"}
     roofline = {**bound, "traffic": None, "kernel": dom, "step_frac": roof_t / (ms_per_step * 1e-3),
                 "call_ms": call_ms,
-                "per_call_work": "forward calls 4*C*G flops and 2*C*e bytes per point each; backward calls "
-                                 "8*C*G flops, 3*C*e (deslice) and 4*C*e (slice) bytes"}
+                "per_call_work": "forward calls 4*C*G flops and 2*C*e bytes per point each; the backward "
+                                 "16*C*G flops and 7*C*e bytes (deslice backward 8*C*G and 3*C*e, slice "
+                                 "backward 8*C*G and 4*C*e)"}
     line = {"metric": TRAIN_METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
@@ -389,7 +405,8 @@ def run_train(args, wl, dev, world, rank):
                                 "backward": ["simt", "tcgen05"][fs.backward_path_for_shape(s)]},
                        **_overrides(args)},
             "clocks": clocks, "roofline": roofline,
-            "gpu_launches": (fs.forward_launch_count(s) + fs.backward_launch_count(s, True)) * args.steps,
+            "gpu_launches": (fs.forward_launch_count(s) + (fs.backward_launch_count(s, True) if sep else
+                                                           fs.coupling_bwd_launch_count(s, True))) * args.steps,
             "e2e": {"value": sharding.job_rate(wl.points, world, e2e_ms), "unit": UNIT,
                     "h2d_bytes_per_step": 3 * hx.numel() * hx.element_size(),
                     "d2h_bytes_per_step": sum(h_.numel() * h_.element_size() for h_ in hout), "ms_per_step": e2e_ms}}
@@ -589,6 +606,9 @@ def main():
     ap.add_argument("--ref-points", type=int, default=16384)
     ap.add_argument("--points", type=int, default=None,
                     help="profiling runs only: the workload's recipe at a smaller N (the line says so)")
+    ap.add_argument("--separate-backward", action="store_true",
+                    help="training: the backward as fs_deslice_bwd, fs_mix_bwd, fs_slice_bwd instead of "
+                         "fs_coupling_bwd")
     ap.add_argument("--slots", type=int, default=None,
                     help="the workload's recipe at another slot count G (the line says so)")
     args = ap.parse_args()

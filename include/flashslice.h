@@ -120,7 +120,8 @@ typedef enum fs_op {
   FS_OP_DESLICE_FWD = 1,
   FS_OP_DESLICE_BWD = 2,
   FS_OP_SLICE_BWD = 3,
-  FS_OP_STATS = 4
+  FS_OP_STATS = 4,
+  FS_OP_COUPLING_BWD = 5
 } fs_op;
 
 /* Bytes of scratch `ws` that entry point `op` needs for this shape on the
@@ -234,6 +235,29 @@ fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx,
                        float* dbias, float* dtau, int accumulate, void* ws,
                        size_t ws_bytes, fs_stream_t stream);
 
+/* The whole backward of one coupling in one call: the results of
+ *   fs_deslice_bwd(..., accumulate) ; fs_mix_bwd ; fs_slice_bwd(..., accumulate = 1)
+ * (App. G.1 backward; App. G.2 temperature gradient; the mix backward of Eq. (1)).
+ *   d_tokens_mixed, d_tokens [B,H,G,d], dfx [B,N,H,d], dM [H,G,G]: overwritten;
+ *   dx_mid [B,N,H,d], dW [H,d,G], dbias [H,G], dtau [H]: the sum of both calls'
+ *   contributions, written if accumulate == 0, added if accumulate != 0.
+ *   tokens, wsum, tokens_mixed, lse: the forward's (lse may be NULL, as in the
+ *   separate calls).  ws: fs_workspace_bytes(s, FS_OP_COUPLING_BWD).
+ * On the tensor-core backward (fs_backward_path_for_shape == 1) the two calls'
+ * dx come from one point pass: their da_ng share the weights, so one pass over
+ * (point, slot) forms da_D + da_S and dx from it, instead of one pass per call.
+ * Results agree with the separate calls to rounding (dx is summed before its one
+ * bf16 rounding instead of after each call's).  Elsewhere it makes the three
+ * calls.  M, tokens and tokens_mixed overlapping an output, or two outputs
+ * overlapping each other: FS_ERR_INVALID. */
+fs_status fs_coupling_bwd(const fs_shape* s, const void* x_mid, const void* fx,
+                          const float* W_slice, const float* bias, const float* tau,
+                          const float* M, const float* tokens, const float* wsum,
+                          const float* tokens_mixed, const float* lse, const void* dout,
+                          float* d_tokens_mixed, float* d_tokens, void* dx_mid, void* dfx,
+                          float* dW, float* dbias, float* dtau, float* dM, int accumulate,
+                          void* ws, size_t ws_bytes, fs_stream_t stream);
+
 /* Fixed-scratch variant of fs_slice_fwd.  The paper has no counterpart.
  *
  * For callers that cannot give the library device memory at the call site: a
@@ -293,6 +317,11 @@ int fs_forward_launch_count(const fs_shape* s);
  * forward's lse (each call that must recompute the statistics launches that pass
  * again).  Memsets are not counted.  -1 for an invalid or unsupported shape. */
 int fs_backward_launch_count(const fs_shape* s, int lse_given);
+
+/* Number of kernels fs_coupling_bwd launches for this shape (lse_given as above;
+ * the one call recomputes the statistics at most once).  -1 for an invalid or
+ * unsupported shape. */
+int fs_coupling_bwd_launch_count(const fs_shape* s, int lse_given);
 
 #ifdef __cplusplus
 }

@@ -132,6 +132,16 @@ Regions regions(const Shape& s, int op) {
       r.stats = take(pts * sizeof(float));
       r.tc = take(tc_deslice_prep_bytes(s));
       break;
+    case FS_OP_COUPLING_BWD:
+      if (tc_backward_supported(s)) {
+        r.dus = take(BHG * (s.d + 1) * sizeof(float));
+        r.stats = take(pts * sizeof(float));
+        r.tc = take(std::max(tc_coupling_bwd_bytes(s), tc_deslice_prep_bytes(s)));
+        break;
+      }
+      // the three calls one after another on the same scratch
+      return Regions{0, 0, 0, 0, 0, 0, 0,
+                     std::max(regions(s, FS_OP_DESLICE_BWD).total, regions(s, FS_OP_SLICE_BWD).total)};
     default:
       return Regions{};
   }
@@ -255,6 +265,15 @@ int fs_backward_launch_count(const fs_shape* s, int lse_given) {
   if (tc_backward_supported(sh))
     return 2 * stats + tc_backward_launch_count(sh, 1) + mix_bwd + tc_backward_launch_count(sh, 2);
   return 2 * stats + 5 /*point, slot, three reductions*/ + mix_bwd + 5 /*prologue, point, slot, two reductions*/;
+}
+
+int fs_coupling_bwd_launch_count(const fs_shape* s, int lse_given) {
+  if (!valid_shape(s) || !supported_shape(s)) return -1;
+  const Shape sh = to_shape(s);
+  if (!tc_backward_supported(sh)) return fs_backward_launch_count(s, lse_given);
+  const bool tc = tc_forward_supported(sh);
+  const int stats = (lse_given && sh.dot == FS_DOT_BF16X2) ? 0 : (tc ? 2 : 1);  // the statistics once
+  return stats + tc_coupling_bwd_launch_count(sh);
 }
 
 fs_status fs_slice_fwd(const fs_shape* s, const void* x_mid, const void* fx, const float* W_slice,
@@ -440,6 +459,41 @@ fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx, con
                                     d_tokens, dx_mid, dfx, dW, dbias, dtau, accumulate, at<float>(ws, r.delta),
                                     at<float>(ws, r.dus), at<float>(ws, r.partials), at<float>(ws, r.dtau_p),
                                     at<uint32_t>(ws, r.status), st));
+}
+
+fs_status fs_coupling_bwd(const fs_shape* s, const void* x_mid, const void* fx, const float* W_slice,
+                          const float* bias, const float* tau, const float* M, const float* tokens,
+                          const float* wsum, const float* tokens_mixed, const float* lse, const void* dout,
+                          float* d_tokens_mixed, float* d_tokens, void* dx_mid, void* dfx, float* dW, float* dbias,
+                          float* dtau, float* dM, int accumulate, void* ws, size_t ws_bytes, fs_stream_t stream) {
+  FS_CHECK_SHAPE(s);
+  FS_CHECK_PTR(x_mid); FS_CHECK_PTR(fx); FS_CHECK_PTR(W_slice); FS_CHECK_PTR(bias); FS_CHECK_PTR(tau);
+  FS_CHECK_PTR(M); FS_CHECK_PTR(tokens); FS_CHECK_PTR(wsum); FS_CHECK_PTR(tokens_mixed); FS_CHECK_PTR(dout);
+  if (lse && !aligned(lse)) return FS_ERR_INVALID;
+  FS_CHECK_PTR(d_tokens_mixed); FS_CHECK_PTR(d_tokens); FS_CHECK_PTR(dx_mid); FS_CHECK_PTR(dfx);
+  FS_CHECK_PTR(dW); FS_CHECK_PTR(dbias); FS_CHECK_PTR(dtau); FS_CHECK_PTR(dM);
+  // the mix backward inside reads M, tokens and d_tokens_mixed while it writes d_tokens and dM
+  const size_t tb = (size_t)s->B * s->H * s->G * s->d * 4, mb = (size_t)s->H * s->G * s->G * 4;
+  if (!disjoint({{M, mb}, {tokens, tb}, {tokens_mixed, tb}}, {{d_tokens_mixed, tb}, {d_tokens, tb}, {dM, mb}}))
+    return FS_ERR_INVALID;
+  const Shape sh = to_shape(s);
+  if (fs_status e = check_ws(sh, FS_OP_COUPLING_BWD, ws, ws_bytes)) return e;
+  if (!tc_backward_supported(sh)) {
+    fs_status e = fs_deslice_bwd(s, x_mid, W_slice, bias, tau, tokens_mixed, lse, dout, d_tokens_mixed, dx_mid, dW,
+                                 dbias, dtau, accumulate, ws, ws_bytes, stream);
+    if (e != FS_OK) return e;
+    if ((e = fs_mix_bwd(s, M, tokens, d_tokens_mixed, d_tokens, dM, stream)) != FS_OK) return e;
+    return fs_slice_bwd(s, x_mid, fx, W_slice, bias, tau, tokens, wsum, lse, d_tokens, dx_mid, dfx, dW, dbias, dtau,
+                        1, ws, ws_bytes, stream);
+  }
+  const Regions r = regions(sh, FS_OP_COUPLING_BWD);
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  FS_CUDA(reset_status(ws, st));
+  const float* lse_use = nullptr;
+  FS_CUDA(backward_stats(sh, x_mid, W_slice, bias, tau, lse, ws, r, at<uint32_t>(ws, r.status), st, &lse_use));
+  return cuda_status(tc_coupling_bwd(sh, x_mid, fx, dout, W_slice, bias, tau, M, tokens, wsum, tokens_mixed, lse_use,
+                                     d_tokens_mixed, d_tokens, dM, dx_mid, dfx, dW, dbias, dtau, accumulate,
+                                     at<float>(ws, r.dus), at<void>(ws, r.tc), at<uint32_t>(ws, r.status), st));
 }
 
 fs_status fs_device_status(const void* ws, fs_stream_t stream) {

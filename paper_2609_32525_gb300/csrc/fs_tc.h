@@ -52,6 +52,15 @@ int tc_backward_launch_count(const Shape& s, int mode);
 cudaError_t tc_deslice_bwd(const Shape& s, const void* x, const float* W, const float* bias, const float* tau,
                            const float* zp, const float* lse, const void* dout, float* dzp, void* dx, float* dW,
                            float* db, float* dtau, int accumulate, void* ws_tc, uint32_t* status, cudaStream_t st);
+// The coupling's whole backward (deslice, mix, slice) with one point pass for both
+// calls' dx; workspace and kernel count.
+size_t tc_coupling_bwd_bytes(const Shape& s);
+int tc_coupling_bwd_launch_count(const Shape& s);
+cudaError_t tc_coupling_bwd(const Shape& s, const void* x, const void* f, const void* dout, const float* W,
+                            const float* bias, const float* tau, const float* M, const float* z, const float* wsum,
+                            const float* zp, const float* lse, float* dzp, float* dz, float* dM, void* dx, void* dfx,
+                            float* dW, float* db, float* dtau, int accumulate, float* dUS, void* ws_tc,
+                            uint32_t* status, cudaStream_t st);
 cudaError_t tc_slice_bwd(const Shape& s, const void* x, const void* f, const float* W, const float* bias,
                          const float* tau, const float* z, const float* wsum, const float* lse, const float* dz,
                          void* dx, void* dfx, float* dW, float* db, float* dtau, int accumulate, float* dUS,

@@ -84,15 +84,17 @@ __global__ void k_prep_wt(const float* __restrict__ W, const float* __restrict__
 }
 
 // delta's point-extra rows [1, 1, -delta_hi, -delta_lo, 0, 0, 0, 0] into dpx [BH, Np, 8];
-// delta_n = delta[bh][n] (+ wds[0][bh][n] + wds[1][bh][n] when wds is given).
-__global__ void k_prep_dpx(const float* __restrict__ delta, const float* __restrict__ wds, uint4* __restrict__ dpx,
-                           int64_t BH, int64_t N, int64_t Np) {
+// delta_n = delta[bh][n] (+ delta2[bh][n] when given, + wds[0][bh][n] + wds[1][bh][n]
+// when wds is given).
+__global__ void k_prep_dpx(const float* __restrict__ delta, const float* __restrict__ delta2,
+                           const float* __restrict__ wds, uint4* __restrict__ dpx, int64_t BH, int64_t N, int64_t Np) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= BH * Np) return;
   const int64_t bh = i / Np, n = i % Np;
   float d = 0.f;
   if (n < N) {
     d = delta[bh * N + n];
+    if (delta2) d += delta2[bh * N + n];
     if (wds) d += wds[bh * N + n] + wds[(BH + bh) * N + n];
   }
   const __nv_bfloat16 hi = __float2bfloat16_rn(-d);
@@ -105,11 +107,12 @@ __global__ void k_prep_dpx(const float* __restrict__ delta, const float* __restr
 
 // M = 128 x N = 64 product with K = 48 (80 with the residual half, lo_a or lo_b):
 // a0/b0 are the K-major 64B-swizzled 32-channel blocks, ae/be the extra blocks.
+// acc0: add to what d holds (a second chain into the same accumulator).
 template <bool kLoA>
 __device__ __forceinline__ void issue_dot64(uint32_t d, uint32_t a, uint32_t b, uint64_t ae, uint64_t be,
-                                            uint32_t lo) {
+                                            uint32_t lo, uint32_t acc0 = 0) {
   constexpr uint32_t idesc = idesc_bf16(128, 64, false, false);
-  mma_ss_w(d, sdesc(a, 16, 512, kSw64), sdesc(b, 16, 512, kSw64), idesc, 0);
+  mma_ss_w(d, sdesc(a, 16, 512, kSw64), sdesc(b, 16, 512, kSw64), idesc, acc0);
   mma_ss_w(d, sdesc(a + 32, 16, 512, kSw64), sdesc(b + 32, 16, 512, kSw64), idesc, 1);
   if (lo) {
     if (kLoA) {
@@ -431,24 +434,34 @@ __global__ void __launch_bounds__(kThreads, 1)
 // N = 64 slots, into set q % 3; softmax warpgroup q % 2 writes da in place (hi, lo
 // pairs); warp 2 + j issues K-steps [2 j, 2 j + 2) of the chunk into O_j:
 //   O_j += da W'^T (B: the W'^T image, channel rows, slots along K).
-// smem: [W img G x (96 | 160)][T img G x 96][W'^T img G x 64][stages][zero 2K][bars]
+// kComb (the whole coupling's backward): da is the sum of the deslice's and the
+// slice's, which share the weights, so one pass serves both: dw - delta is two chains
+// into the same accumulator, [dO | 1, 1, -delta] against the deslice's T image (c = 0)
+// and [fx | 1, 1, 0 ...] (a constant extra block) against the slice's (t = dU, c = dS),
+// with delta = delta_D + delta_S in the point rows.  Each stage also holds the fx tile.
+// smem: [W img G x (96 | 160)][T img G x 96][kComb: T2 img G x 96][W'^T img G x 64]
+//       [kComb: constant extra 4K][stages][zero 2K][bars]
 // TMEM: sets [0, 384) of (L 64 | dw 64); O_(j, tile parity) at [384 + 32 (2 j + parity)).
 // =========================================================================================
-template <bool split>
+template <bool split, bool kComb = false>
 __global__ void __launch_bounds__(kThreads, 1)
     k_bwd_dx_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap vmap,
                 const __grid_constant__ CUtensorMap pmap, const __grid_constant__ CUtensorMap dmap,
-                const uint8_t* __restrict__ wimg, const uint8_t* __restrict__ timg,
+                const __grid_constant__ CUtensorMap fmap, const uint8_t* __restrict__ wimg,
+                const uint8_t* __restrict__ timg, const uint8_t* __restrict__ timg2,
                 const uint8_t* __restrict__ wtimg, __nv_bfloat16* __restrict__ dx, int64_t N, int64_t Np, int H,
                 int G, int splits, int hilo, int accumulate, uint32_t* status) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  constexpr uint32_t kStg = kBStage + (kComb ? kXBytes : 0u);  // x | v | px | dpx [| fx]
   const uint32_t wbytes = (uint32_t)G * (hilo ? kWRow : 96);
   uint8_t* s_w = smem;
   uint8_t* s_t = s_w + wbytes;
-  uint8_t* s_wt = s_t + (uint32_t)G * 96;
-  uint8_t* s_st = s_wt + (uint32_t)G * 64;
-  uint8_t* s_zero = s_st + kDxStages * kBStage;
+  uint8_t* s_t2 = s_t + (uint32_t)G * 96;
+  uint8_t* s_wt = s_t2 + (kComb ? (uint32_t)G * 96 : 0u);
+  uint8_t* s_ex = s_wt + (uint32_t)G * 64;
+  uint8_t* s_st = s_ex + (kComb ? kExBytes : 0u);
+  uint8_t* s_zero = s_st + kDxStages * kStg;
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_zero + kPxZero);
   uint64_t* wz_full = bars;
   uint64_t* x_full = bars + 1;
@@ -491,6 +504,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_mbar_init();
   }
   zero_smem(s_zero, kPxZero);
+  if (kComb) write_const_extra(s_ex);
   fence_proxy_async_smem();
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
@@ -504,21 +518,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&vmap);
       prefetch_tmap(&pmap);
       prefetch_tmap(&dmap);
-      mbar_expect_tx(wz_full, wbytes + (uint32_t)G * 96 + (uint32_t)G * 64);
+      if (kComb) prefetch_tmap(&fmap);
+      mbar_expect_tx(wz_full, wbytes + (uint32_t)G * 96 * (kComb ? 2u : 1u) + (uint32_t)G * 64);
       load_images(s_w, wimg + (size_t)h * G * kWRow, wbytes, wz_full);
       load_images(s_t, timg + (size_t)wk.bh * G * kWRow, (uint32_t)G * 96, wz_full);
+      if (kComb) load_images(s_t2, timg2 + (size_t)wk.bh * G * kWRow, (uint32_t)G * 96, wz_full);
       load_images(s_wt, wtimg + (size_t)h * G * 128, (uint32_t)G * 64, wz_full);
       int i = 0;
       for (; i < wk.ntiles; i++) {
         const int s = i % kDxStages;
         if (i >= kDxStages && !mbar_wait(&x_empty[s], (uint32_t)(((i / kDxStages) - 1) & 1), ab, status)) break;
-        uint8_t* st = s_st + s * kBStage;
+        uint8_t* st = s_st + s * kStg;
         const int n0 = (int)((wk.tile0 + i) * kTile);
-        mbar_expect_tx(&x_full[s], kBStage);
+        mbar_expect_tx(&x_full[s], kStg);
         tma_load_3d(st, &xmap, h * kD, n0, (int)b, &x_full[s]);
         tma_load_3d(st + kVOff, &vmap, h * kD, n0, (int)b, &x_full[s]);
         tma_load_2d(st + kPOff, &pmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
         tma_load_2d(st + kDOff, &dmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
+        if (kComb) tma_load_3d(st + kBStage, &fmap, h * kD, n0, (int)b, &x_full[s]);
       }
       for (int j = (i > kDxStages ? i - kDxStages : 0); j < i; j++)
         mbar_wait(&x_full[j % kDxStages], (uint32_t)((j / kDxStages) & 1), ab, nullptr, kWaitNs);
@@ -526,7 +543,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     if (wk.ntiles > 0) {
-      const uint32_t sw = smem_u32(s_w), stt = smem_u32(s_t), sz = smem_u32(s_zero);
+      const uint32_t sw = smem_u32(s_w), stt = smem_u32(s_t), stt2 = smem_u32(s_t2), sz = smem_u32(s_zero);
       bool ok = mbar_wait_w(wz_full, 0, ab, status);
       BlockPos pos(0, nch);
       for (int q = 0; ok && q < total; q++, pos.step(1, nch)) {
@@ -536,7 +553,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (c == 0 && !(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kDxStages) & 1), ab, status))) break;
         if (q >= kSBuf && !(ok = mbar_wait_w(&pv_done[bb], (uint32_t)(((q / kSBuf) - 1) & 1), ab, status))) break;
         tc_fence_after();
-        const uint32_t st = smem_u32(s_st + s * kBStage);
+        const uint32_t st = smem_u32(s_st + s * kStg);
         const uint32_t tL = tmem + (uint32_t)bb * kGC;
         const uint32_t rows = (uint32_t)c * 64 * 64, erows = (uint32_t)c * 64 * 32;
         issue_dot64<false>(tL, st, sw + rows, px_desc(st + kPOff, sz),
@@ -544,6 +561,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                            hilo ? sw + (uint32_t)G * 96 + rows : 0u);
         issue_dot64<false>(tL + 64, st + kVOff, stt + rows, px_desc(st + kDOff, sz),
                            sdesc(stt + (uint32_t)G * 64 + erows, 16, 256, kSw32), 0u);
+        if (kComb)
+          issue_dot64<false>(tL + 64, st + kBStage, stt2 + rows, const_extra_desc(smem_u32(s_ex)),
+                             sdesc(stt2 + (uint32_t)G * 64 + erows, 16, 256, kSw32), 0u, 1u);
         mma_commit_w(&s_full[bb]);
         if (c == nch - 1) mma_commit_w(&x_empty[s]);
       }
@@ -656,8 +676,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 size_t smem_bwd_slot() {
   return 1024 + 2 * (size_t)kWBlockB + kBStages * (size_t)kBStage + kPxZero + 3 * kGC * 4 + 512;
 }
-size_t smem_bwd_dx(int G, bool hilo) {
-  return 1024 + (size_t)G * ((hilo ? kWRow : 96) + 96 + 64) + kDxStages * (size_t)kBStage + kPxZero + 512;
+size_t smem_bwd_dx(int G, bool hilo, bool comb = false) {
+  return 1024 + (size_t)G * ((hilo ? kWRow : 96) + 96 * (comb ? 2 : 1) + 64) + (comb ? kExBytes : 0) +
+         kDxStages * (size_t)(kBStage + (comb ? kXBytes : 0)) + kPxZero + 512;
 }
 
 int bwd_slot_blocks(const Shape& s) { return s.G / kGC; }
@@ -767,11 +788,13 @@ cudaError_t prep_t_images(const Shape& s, int G, const float* t, int tstride, in
 //   1. lse rows; for each slot range: its images, then the rows pass (delta, dfx
 //      and the wds partials add up over the ranges);
 //   2. delta's rows; for each slot range: the slot pass, its reduction into the
-//      range's dW, dbias, dtau (and dz') partials, and the point pass (dx).
+//      range's dW, dbias, dtau (and dz') partials, and the point pass (dx; skipped
+//      when dx is null).
+// delta_out: where delta goes (null: the layout's own buffer).
 cudaError_t run_backward(const Shape& s0, int mode, const void* x, const void* v, const float* W,
                          const float* bias, const float* tau, const float* t, int tstride, const float* lse,
                          void* dfx, void* dx, float* dzp, float* dW, float* db, float* dtau, int accumulate,
-                         uint8_t* ws, uint32_t* status, cudaStream_t st) {
+                         uint8_t* ws, uint32_t* status, cudaStream_t st, float* delta_out = nullptr) {
   const SlotRanges sr = slot_ranges(s0.G);
   const Shape s = pass_shape(s0);
   const BwdLayout L = bwd_layout(s0, mode);
@@ -811,7 +834,7 @@ cudaError_t run_backward(const Shape& s0, int mode, const void* x, const void* v
   k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(ws + L.px), s.BH(), s.N,
                                                              Np);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  float* delta = reinterpret_cast<float*>(ws + L.delta);
+  float* delta = delta_out ? delta_out : reinterpret_cast<float*>(ws + L.delta);
   float* wds = mode == 2 ? reinterpret_cast<float*>(ws + L.wds) : nullptr;
   if (wds && (e = cudaMemsetAsync(wds, 0, 2 * (size_t)s.BH() * s.N * sizeof(float), st)) != cudaSuccess) return e;
   for (int k = 0; k < sr.n; k++) {
@@ -820,8 +843,8 @@ cudaError_t run_backward(const Shape& s0, int mode, const void* x, const void* v
                          reinterpret_cast<const float*>(ws + L.ds), k > 0 ? 1 : 0, status, st)) != cudaSuccess)
       return e;
   }
-  k_prep_dpx<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(delta, wds, reinterpret_cast<uint4*>(ws + L.dpx),
-                                                              s.BH(), s.N, Np);
+  k_prep_dpx<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(delta, nullptr, wds,
+                                                              reinterpret_cast<uint4*>(ws + L.dpx), s.BH(), s.N, Np);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
 
   CUtensorMap xmap, vmap, pmap, dmap;
@@ -829,10 +852,11 @@ cudaError_t run_backward(const Shape& s0, int mode, const void* x, const void* v
   const int R = bwd_slot_blocks(s), P = bwd_slot_splits(s);
   for (int k = 0; k < sr.n; k++) {
     const int g0 = k * sr.size, G = range_g(k);
-    // The images of the last range are still in place after the rows passes; W'^T is not.
+    // The images of the last range are still in place after the rows passes; W'^T
+    // (for the point pass, when dx is wanted) is not.
     if (ranged) {
-      if ((e = prep_range(k, true)) != cudaSuccess) return e;
-    } else {
+      if ((e = prep_range(k, dx != nullptr)) != cudaSuccess) return e;
+    } else if (dx) {
       const int64_t nwt = (int64_t)s.H * kD * s.G;
       k_prep_wt<<<(unsigned)((nwt + 255) / 256), 256, 0, st>>>(W, tau, ws + L.wtimg, s.H, G, s.G, status);
       if ((e = cudaGetLastError()) != cudaSuccess) return e;
@@ -876,17 +900,135 @@ cudaError_t run_backward(const Shape& s0, int mode, const void* x, const void* v
                                       (int64_t)G * kD, s.BH(), st)) != cudaSuccess)
         return e;
     }
-    {
+    if (dx) {
       const bool hilo = smem_bwd_dx(s.G, true) <= kMaxSmem;
       const size_t sm = smem_bwd_dx(s.G, hilo);
       const int Pd = point_splits(s, (int)s.BH());
       const auto kernel = k_bwd_dx_tc<true>;
       if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
       kernel<<<dim3((unsigned)Pd, (unsigned)s.BH()), kThreads, sm, st>>>(
-          xmap, vmap, pmap, dmap, ws + L.wimg, ws + L.timg, ws + L.wtimg, static_cast<__nv_bfloat16*>(dx), s.N, Np,
-          s.H, s.G, Pd, hilo ? 1 : 0, acc, status);
+          xmap, vmap, pmap, dmap, xmap, ws + L.wimg, ws + L.timg, nullptr, ws + L.wtimg,
+          static_cast<__nv_bfloat16*>(dx), s.N, Np, s.H, s.G, Pd, hilo ? 1 : 0, acc, status);
       if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
+  }
+  return cudaSuccess;
+}
+
+// The coupling's backward in one call (fs_coupling_bwd): the deslice's and the slice's
+// passes as in the two calls but without their point passes, the mix backward between
+// them, then ONE point pass for dx = ln2 sum_g (da_D + da_S)_ng W'_g: the two calls'
+// da share the weights, so their dw - delta add up (k_bwd_dx_tc<·, true>).  That pass
+// holds two T images besides W' and W'^T and runs over slot ranges of at most 256.
+constexpr int kCombSlotsMax = 256;
+SlotRanges comb_ranges(const Shape& s0) {
+  const int cap = std::min(kCombSlotsMax, pass_shape(s0).G);
+  const int Gp = (s0.G + kGC - 1) / kGC * kGC;
+  if (Gp <= cap) return {1, Gp};
+  SlotRanges best{0, 0};
+  for (int size = kGC; size <= cap; size += kGC) {
+    const int n = (s0.G + size - 1) / size;
+    if (best.n == 0 || (int64_t)n * (size + kGC / 2) <= (int64_t)best.n * (best.size + kGC / 2)) best = {n, size};
+  }
+  return best;
+}
+
+// Workspace of the coupling backward: the larger of the two calls' layouts, then the
+// deslice's delta, the slice's T image for the point pass, and (with several point-pass
+// ranges) a range's slices of W, bias, z' and dU | dS.
+struct CoupLayout {
+  size_t deltaD, timg2, wc, bc, zc, uc, total;
+};
+CoupLayout coup_layout(const Shape& s0) {
+  CoupLayout C{};
+  size_t off = std::max(bwd_layout(s0, 1).total, bwd_layout(s0, 2).total);
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  const Shape s = pass_shape(s0);
+  const SlotRanges cr = comb_ranges(s0);
+  const size_t rs = cr.n > 1 ? (size_t)cr.size : 0;
+  C.deltaD = take((size_t)s.BH() * s.N * sizeof(float));
+  C.timg2 = take((size_t)s.BH() * cr.size * kWRow);
+  C.wc = take((size_t)s.H * kD * rs * sizeof(float));
+  C.bc = take((size_t)s.H * rs * sizeof(float));
+  C.zc = take((size_t)s.BH() * rs * kD * sizeof(float));
+  C.uc = take((size_t)s.BH() * rs * (kD + 1) * sizeof(float));
+  C.total = off;
+  return C;
+}
+
+cudaError_t run_coupling_bwd(const Shape& s0, const void* x, const void* f, const void* dout, const float* W,
+                             const float* bias, const float* tau, const float* M, const float* z, const float* wsum,
+                             const float* zp, const float* lse, float* dzp, float* dz, float* dM, void* dx, void* dfx,
+                             float* dW, float* db, float* dtau, int accumulate, float* dUS, uint8_t* ws,
+                             uint32_t* status, cudaStream_t st) {
+  const CoupLayout C = coup_layout(s0);
+  const BwdLayout L = bwd_layout(s0, 2);
+  float* deltaD = reinterpret_cast<float*>(ws + C.deltaD);
+  cudaError_t e;
+  if ((e = run_backward(s0, 1, x, dout, W, bias, tau, zp, kD, lse, nullptr, nullptr, dzp, dW, db, dtau, accumulate,
+                        ws, status, st, deltaD)) != cudaSuccess)
+    return e;
+  if ((e = simt_mix_bwd(s0, M, z, dzp, dz, dM, st)) != cudaSuccess) return e;
+  if ((e = simt_slice_bwd_prep(s0, z, wsum, dz, dUS, st)) != cudaSuccess) return e;
+  if ((e = run_backward(s0, 2, x, f, W, bias, tau, dUS, kD + 1, lse, dfx, nullptr, nullptr, dW, db, dtau, 1, ws,
+                        status, st)) != cudaSuccess)
+    return e;
+  // delta = delta_S + delta_D + the slice's sum_g w dS, into the point rows; the lse
+  // rows are still in place from the slice's passes.
+  const SlotRanges cr = comb_ranges(s0);
+  Shape s = pass_shape(s0);
+  s.G = cr.size;
+  const int64_t Np = padded_n(s), npx = s.BH() * Np;
+  k_prep_dpx<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(
+      reinterpret_cast<const float*>(ws + L.delta), deltaD, reinterpret_cast<const float*>(ws + L.wds),
+      reinterpret_cast<uint4*>(ws + L.dpx), s.BH(), s.N, Np);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  CUtensorMap xmap, vmap, pmap, dmap, fmap;
+  if (!make_maps(s, x, dout, ws + L.px, ws + L.dpx, &xmap, &vmap, &pmap, &dmap) ||
+      !make_point_map(&fmap, f, s, kD, CU_TENSOR_MAP_SWIZZLE_64B))
+    return cudaErrorInvalidValue;
+  const bool hilo = smem_bwd_dx(s.G, true, true) <= kMaxSmem;
+  const size_t sm = smem_bwd_dx(s.G, hilo, true);
+  if (sm > kMaxSmem) return cudaErrorInvalidValue;
+  const auto kernel = k_bwd_dx_tc<true, true>;
+  if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
+  const int Pd = point_splits(s, (int)s.BH());
+  const bool ranged = cr.n > 1;
+  for (int k = 0; k < cr.n; k++) {
+    const int g0 = k * cr.size, G = k < cr.n - 1 ? cr.size : s0.G - (cr.n - 1) * cr.size;
+    const float *Wk = W, *bk = bias, *zk = zp, *uk = dUS;
+    if (ranged) {
+      float* wc = reinterpret_cast<float*>(ws + C.wc);
+      float* bc = reinterpret_cast<float*>(ws + C.bc);
+      float* zc = reinterpret_cast<float*>(ws + C.zc);
+      float* uc = reinterpret_cast<float*>(ws + C.uc);
+      if ((e = copy_rows(wc, G, W + g0, s0.G, G, (int64_t)s.H * kD, st)) != cudaSuccess) return e;
+      if ((e = copy_rows(bc, G, bias + g0, s0.G, G, s.H, st)) != cudaSuccess) return e;
+      if ((e = copy_rows(zc, (int64_t)G * kD, zp + (int64_t)g0 * kD, (int64_t)s0.G * kD, (int64_t)G * kD, s.BH(),
+                         st)) != cudaSuccess)
+        return e;
+      if ((e = copy_rows(uc, (int64_t)G * (kD + 1), dUS + (int64_t)g0 * (kD + 1), (int64_t)s0.G * (kD + 1),
+                         (int64_t)G * (kD + 1), s.BH(), st)) != cudaSuccess)
+        return e;
+      Wk = wc, bk = bc, zk = zc, uk = uc;
+    }
+    if ((e = prep_w(s, G, Wk, bk, tau, ws + L.wimg, status, st)) != cudaSuccess) return e;
+    const int64_t nwt = (int64_t)s.H * kD * s.G, BHG = s.BH() * s.G;
+    k_prep_wt<<<(unsigned)((nwt + 255) / 256), 256, 0, st>>>(Wk, tau, ws + L.wtimg, s.H, G, s.G, status);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    k_prep_t<<<(unsigned)((BHG + 127) / 128), 128, 0, st>>>(zk, kD, 0, ws + L.timg, nullptr, s.BH(), G, s.G);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    k_prep_t<<<(unsigned)((BHG + 127) / 128), 128, 0, st>>>(uk, kD + 1, 1, ws + C.timg2, nullptr, s.BH(), G, s.G);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    kernel<<<dim3((unsigned)Pd, (unsigned)s.BH()), kThreads, sm, st>>>(
+        xmap, vmap, pmap, dmap, fmap, ws + L.wimg, ws + L.timg, ws + C.timg2, ws + L.wtimg,
+        static_cast<__nv_bfloat16*>(dx), s.N, Np, s.H, s.G, Pd, hilo ? 1 : 0, (accumulate || k > 0) ? 1 : 0,
+        status);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
   return cudaSuccess;
 }
@@ -923,6 +1065,28 @@ cudaError_t tc_deslice_bwd(const Shape& s0, const void* x, const float* W, const
                            float* db, float* dtau, int accumulate, void* ws_tc, uint32_t* status, cudaStream_t st) {
   return run_backward(s0, 1, x, dout, W, bias, tau, zp, kD, lse, nullptr, dx, dzp, dW, db, dtau, accumulate,
                       static_cast<uint8_t*>(ws_tc), status, st);
+}
+
+size_t tc_coupling_bwd_bytes(const Shape& s) { return tc_backward_supported(s) ? coup_layout(s).total : 0; }
+
+int tc_coupling_bwd_launch_count(const Shape& s) {
+  const SlotRanges sr = slot_ranges(s.G), cr = comb_ranges(s);
+  // each call's passes without its point pass (and without W'^T's image when it has
+  // one range), the mix backward, the dU/dS prologue, the combined delta rows, and per
+  // point-pass range its four images and the pass
+  const int images = sr.n > 1 ? 3 : 0;
+  const int call1 = 4 * sr.n + 2 + sr.n * (images + 1 + 3);
+  const int call2 = 4 * sr.n + 2 + sr.n * (images + 1 + 2);
+  return call1 + 2 + 1 + call2 + 1 + 5 * cr.n;
+}
+
+cudaError_t tc_coupling_bwd(const Shape& s0, const void* x, const void* f, const void* dout, const float* W,
+                            const float* bias, const float* tau, const float* M, const float* z, const float* wsum,
+                            const float* zp, const float* lse, float* dzp, float* dz, float* dM, void* dx, void* dfx,
+                            float* dW, float* db, float* dtau, int accumulate, float* dUS, void* ws_tc,
+                            uint32_t* status, cudaStream_t st) {
+  return run_coupling_bwd(s0, x, f, dout, W, bias, tau, M, z, wsum, zp, lse, dzp, dz, dM, dx, dfx, dW, db, dtau,
+                          accumulate, dUS, static_cast<uint8_t*>(ws_tc), status, st);
 }
 
 cudaError_t tc_slice_bwd(const Shape& s0, const void* x, const void* f, const float* W, const float* bias,

@@ -29,12 +29,13 @@ FS_OK, FS_ERR_INVALID, FS_ERR_UNSUPPORTED, FS_ERR_CUDA, FS_ERR_TIMEOUT, FS_ERR_B
 FS_NOALLOC_SCRATCH_BYTES = 16 << 20
 FS_F32, FS_BF16 = 0, 1
 FS_DOT_BF16, FS_DOT_BF16X2 = 0, 1
-FS_OP_SLICE_FWD, FS_OP_DESLICE_FWD, FS_OP_DESLICE_BWD, FS_OP_SLICE_BWD, FS_OP_STATS = range(5)
+FS_OP_SLICE_FWD, FS_OP_DESLICE_FWD, FS_OP_DESLICE_BWD, FS_OP_SLICE_BWD, FS_OP_STATS, FS_OP_COUPLING_BWD = range(6)
 
 EXPORTED = ("fs_workspace_bytes", "fs_slice_fwd", "fs_slice_finalize", "fs_mix", "fs_deslice_fwd",
             "fs_deslice_bwd", "fs_mix_bwd", "fs_slice_bwd", "fs_device_status", "fs_status_string",
             "fs_path_for_shape", "fs_backward_path_for_shape", "fs_forward_launch_count", "fs_backward_launch_count",
-            "fs_slice_fwd_noalloc", "fs_slice_fwd_lse", "fs_mix_channels", "fs_mix_channels_bwd", "fs_stats")
+            "fs_slice_fwd_noalloc", "fs_slice_fwd_lse", "fs_mix_channels", "fs_mix_channels_bwd", "fs_stats",
+            "fs_coupling_bwd", "fs_coupling_bwd_launch_count")
 
 
 class fs_shape(ctypes.Structure):
@@ -71,6 +72,8 @@ _sig = {
     "fs_backward_path_for_shape": (_I, [_S]),
     "fs_forward_launch_count": (_I, [_S]),
     "fs_backward_launch_count": (_I, [_S, _I]),
+    "fs_coupling_bwd_launch_count": (_I, [_S, _I]),
+    "fs_coupling_bwd": (_I, [_S] + [_P] * 11 + [_P] * 8 + [_I, _P, _Z, _P]),
     "fs_slice_fwd_noalloc": (_I, [_S, _P, _P, _P, _P, _P, _P, _P, _P, _I, ctypes.POINTER(_P), _P]),
 }
 for _name, (_res, _args) in _sig.items():
@@ -115,9 +118,12 @@ def workspace_bytes(shape: fs_shape, op: int) -> int:
 
 
 def workspace(shape: fs_shape, op: int, device="cuda") -> torch.Tensor:
-    """Scratch for one op, allocated through torch (the library never allocates)."""
+    """Scratch for one op, allocated through torch (the library never allocates).
+    Its status word starts at FS_OK, so a scratch no call has used yet reads clean."""
     n = max(16, workspace_bytes(shape, op))
-    return torch.empty(n, dtype=torch.uint8, device=device)
+    ws = torch.empty(n, dtype=torch.uint8, device=device)
+    ws[:16].zero_()
+    return ws
 
 
 def path_for_shape(shape: fs_shape) -> int:
@@ -134,6 +140,10 @@ def forward_launch_count(shape: fs_shape) -> int:
 
 def backward_launch_count(shape: fs_shape, lse_given: bool = True) -> int:
     return int(_lib.fs_backward_launch_count(ctypes.byref(shape), int(bool(lse_given))))
+
+
+def coupling_bwd_launch_count(shape: fs_shape, lse_given: bool = True) -> int:
+    return int(_lib.fs_coupling_bwd_launch_count(ctypes.byref(shape), int(bool(lse_given))))
 
 
 def status_string(st: int) -> str:
@@ -209,6 +219,15 @@ def fs_slice_bwd(shape, x_mid, fx, W_slice, bias, tau, tokens, wsum, lse, d_toke
     _check("fs_slice_bwd", st)
 
 
+def fs_coupling_bwd(shape, x_mid, fx, W_slice, bias, tau, M, tokens, wsum, tokens_mixed, lse, dout, d_tokens_mixed,
+                    d_tokens, dx_mid, dfx, dW, dbias, dtau, dM, accumulate, ws, stream=None):
+    st = _lib.fs_coupling_bwd(ctypes.byref(shape), _ptr(x_mid), _ptr(fx), _ptr(W_slice), _ptr(bias), _ptr(tau),
+                              _ptr(M), _ptr(tokens), _ptr(wsum), _ptr(tokens_mixed), _ptr(lse), _ptr(dout),
+                              _ptr(d_tokens_mixed), _ptr(d_tokens), _ptr(dx_mid), _ptr(dfx), _ptr(dW), _ptr(dbias),
+                              _ptr(dtau), _ptr(dM), int(bool(accumulate)), _ptr(ws), ws.numel(), _stream(stream))
+    _check("fs_coupling_bwd", st)
+
+
 def fs_device_status(ws, stream=None) -> int:
     return int(_lib.fs_device_status(_ptr(ws), _stream(stream)))
 
@@ -263,6 +282,7 @@ class Coupling:
             self.dM = torch.empty(H, G, G, **f32)
             self.ws_dbwd = workspace(self.shape, FS_OP_DESLICE_BWD, device)
             self.ws_sbwd = workspace(self.shape, FS_OP_SLICE_BWD, device)
+            self.ws_cbwd = workspace(self.shape, FS_OP_COUPLING_BWD, device)
 
     def forward(self, x_mid, fx, W_slice, bias, tau, M, stream=None):
         s = self.shape
@@ -271,19 +291,26 @@ class Coupling:
         fs_deslice_fwd(s, x_mid, W_slice, bias, tau, self.tokens_mixed, self.lse, self.out, self.ws_deslice, stream)
         return self.out
 
-    def backward(self, x_mid, fx, W_slice, bias, tau, M, dout, stream=None):
+    def backward(self, x_mid, fx, W_slice, bias, tau, M, dout, stream=None, fused=True):
+        """fused: one fs_coupling_bwd call; else fs_deslice_bwd, fs_mix_bwd, fs_slice_bwd."""
         s = self.shape
-        fs_deslice_bwd(s, x_mid, W_slice, bias, tau, self.tokens_mixed, self.lse, dout, self.d_tokens_mixed,
-                       self.dx_mid, self.dW, self.dbias, self.dtau, False, self.ws_dbwd, stream)
-        fs_mix_bwd(s, M, self.tokens, self.d_tokens_mixed, self.d_tokens, self.dM, stream)
-        fs_slice_bwd(s, x_mid, fx, W_slice, bias, tau, self.tokens, self.wsum, self.lse, self.d_tokens, self.dx_mid,
-                     self.dfx, self.dW, self.dbias, self.dtau, True, self.ws_sbwd, stream)
+        if fused:
+            fs_coupling_bwd(s, x_mid, fx, W_slice, bias, tau, M, self.tokens, self.wsum, self.tokens_mixed, self.lse,
+                            dout, self.d_tokens_mixed, self.d_tokens, self.dx_mid, self.dfx, self.dW, self.dbias,
+                            self.dtau, self.dM, False, self.ws_cbwd, stream)
+        else:
+            fs_deslice_bwd(s, x_mid, W_slice, bias, tau, self.tokens_mixed, self.lse, dout, self.d_tokens_mixed,
+                           self.dx_mid, self.dW, self.dbias, self.dtau, False, self.ws_dbwd, stream)
+            fs_mix_bwd(s, M, self.tokens, self.d_tokens_mixed, self.d_tokens, self.dM, stream)
+            fs_slice_bwd(s, x_mid, fx, W_slice, bias, tau, self.tokens, self.wsum, self.lse, self.d_tokens,
+                         self.dx_mid, self.dfx, self.dW, self.dbias, self.dtau, True, self.ws_sbwd, stream)
         return {"dx_mid": self.dx_mid, "dfx": self.dfx, "dW": self.dW, "dbias": self.dbias, "dtau": self.dtau,
                 "dM": self.dM}
 
     def device_status(self, stream=None):
         worst = FS_OK
-        for ws in (self.ws_slice, self.ws_deslice) + ((self.ws_dbwd, self.ws_sbwd) if hasattr(self, "ws_dbwd") else ()):
+        for ws in (self.ws_slice, self.ws_deslice) + (
+                (self.ws_dbwd, self.ws_sbwd, self.ws_cbwd) if hasattr(self, "ws_dbwd") else ()):
             st = fs_device_status(ws, stream)
             worst = worst or st
         return worst

@@ -151,3 +151,36 @@ def test_backward_launch_count(fs):
     s = fs.make_shape(1, 100, 2, 32, 8, dtype=fs.FS_F32)
     assert fs.backward_launch_count(s, True) == 12
     assert fs.backward_launch_count(s, False) == 14
+
+
+def test_coupling_bwd_launch_count_and_overlap_checks(fs):
+    """fs_coupling_bwd: on the SIMT backward it makes the three calls, so it
+    launches what they launch; outputs overlapping M, tokens, tokens_mixed or each
+    other are rejected before any launch (fake aligned addresses, never read)."""
+    s = fs.make_shape(1, 100, 2, 32, 8, dtype=fs.FS_F32)
+    assert fs.coupling_bwd_launch_count(s, True) == fs.backward_launch_count(s, True)
+    assert fs.coupling_bwd_launch_count(fs.make_shape(1, 100, 2, 48, 8)) == -1
+    lib, P = fs._lib, ctypes.c_void_p
+    B, N, H, d, G = 1, 100, 2, 32, 8
+    tb, mb, pb = B * H * G * d * 4, H * G * G * 4, B * N * H * d * 4
+    base = 1 << 24
+    addr = [base + i * (1 << 20) for i in range(20)]
+    ws = 1 << 30
+    nbytes = fs.workspace_bytes(s, fs.FS_OP_COUPLING_BWD)
+    assert nbytes >= max(fs.workspace_bytes(s, fs.FS_OP_DESLICE_BWD), fs.workspace_bytes(s, fs.FS_OP_SLICE_BWD))
+    # x, fx, W, bias, tau, M, tokens, wsum, tokens_mixed, lse, dout | dzm, dz, dx, dfx, dW, db, dt, dM
+    ins, outs = addr[:11], addr[11:19]
+    M, tokens, tokens_mixed = ins[5], ins[6], ins[8]
+
+    def call(o):
+        return lib.fs_coupling_bwd(ctypes.byref(s), *[P(a) for a in ins], *[P(a) for a in o], 0, P(ws), nbytes, None)
+
+    for k, target in ((0, tokens), (1, tokens_mixed), (7, M)):  # d_tokens_mixed, d_tokens, dM over an input
+        o = list(outs)
+        o[k] = target + 16
+        assert call(o) == fs.FS_ERR_INVALID
+    o = list(outs)
+    o[1] = o[0] + 16  # d_tokens over d_tokens_mixed
+    assert call(o) == fs.FS_ERR_INVALID
+    assert lib.fs_coupling_bwd(ctypes.byref(s), *[P(a) for a in ins], *[P(a) for a in outs], 0, P(ws), nbytes - 1,
+                               None) == fs.FS_ERR_INVALID
