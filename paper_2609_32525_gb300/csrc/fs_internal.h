@@ -71,6 +71,8 @@ cudaError_t simt_slice_bwd_prep(const Shape& s, const float* z, const float* wsu
 cudaError_t simt_reduce_bwd(const Shape& s, int P, const float* part, int Gs, int PS, int has_dzp, const float* tau,
                             float* dzp, float* dW, float* db, float* dtau, const float* dt_part, int64_t nblk,
                             int accumulate, cudaStream_t st);
+// The token gradient alone from partials whose first d words per slot are dz'.
+cudaError_t simt_reduce_dzp(const Shape& s, int P, const float* part, int Gs, int PS, float* dzp, cudaStream_t st);
 cudaError_t simt_slice_bwd(const Shape& s, int P, const void* x, const void* f, const float* W,
                            const float* bias, const float* tau, const float* z,
                            const float* wsum, const float* lse, const float* dz, void* dx,

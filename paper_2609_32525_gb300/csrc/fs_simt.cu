@@ -927,6 +927,12 @@ cudaError_t simt_reduce_bwd(const Shape& s, int P, const float* part, int Gs, in
   return cudaGetLastError();
 }
 
+cudaError_t simt_reduce_dzp(const Shape& s, int P, const float* part, int Gs, int PS, float* dzp, cudaStream_t st) {
+  const int64_t BHG = s.BH() * s.G;
+  k_reduce_bwd_tokens<<<(unsigned)((BHG * s.d + 255) / 256), 256, 0, st>>>(part, P, s.BH(), s.G, Gs, s.d, PS, dzp);
+  return cudaGetLastError();
+}
+
 cudaError_t simt_slice_bwd_prep(const Shape& s, const float* z, const float* wsum, const float* dz, float* dUS,
                                 cudaStream_t st) {
   const int64_t BHG = s.BH() * s.G;

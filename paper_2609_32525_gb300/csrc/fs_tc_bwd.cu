@@ -186,6 +186,33 @@ __device__ __forceinline__ void da_unit(uint32_t tL, uint32_t tD, float& dt, flo
 // TMEM column (within a unit) of the hi pairs of K-step kk (16 entries).
 __device__ __forceinline__ uint32_t da_col(int kk) { return (uint32_t)(32 * (kk >> 1) + 8 * (kk & 1)); }
 
+// One 64-column unit of a TMEM lane: L (log2 weights) -> w = 2^L in place, as bf16
+// pairs in da_unit's layout (hi pairs, then their residuals with kSplit).
+template <bool kSplit>
+__device__ __forceinline__ void w_unit(uint32_t tL) {
+  const uint64_t neg1 = pack2(__float_as_uint(-1.f), __float_as_uint(-1.f));
+#pragma unroll 1
+  for (int h2 = 0; h2 < 2; h2++) {
+    uint32_t l[32];
+    tmem_ld32(tL + 32 * h2, l);
+    tmem_wait_ld(l);
+    uint32_t wh[16], wl[16];
+#pragma unroll
+    for (int k = 0; k < 16; k++) {
+      const uint64_t w2 = pack2(__float_as_uint(ex2(__uint_as_float(l[2 * k]))),
+                                __float_as_uint(ex2(__uint_as_float(l[2 * k + 1]))));
+      const uint32_t q = pack_bf16(lo_f(w2), hi_f(w2));
+      wh[k] = q;
+      if (kSplit) {
+        const uint64_t r2 = fma2(pack2(q << 16, q & 0xFFFF0000u), neg1, w2);
+        wl[k] = pack_bf16(lo_f(r2), hi_f(r2));
+      }
+    }
+    tmem_st16(tL + 32 * h2, wh);
+    if (kSplit) tmem_st16(tL + 32 * h2 + 16, wl);
+  }
+}
+
 // =========================================================================================
 // Slot pass: CTA (slot block, point split p, bh) owns 128 slots.  Unit u is half
 // u & 1 (64 points) of point tile u >> 1.  Per unit, warp 1 forms, transposed
@@ -197,6 +224,11 @@ __device__ __forceinline__ uint32_t da_col(int kk) { return (uint32_t)(32 * (kk 
 //   MODE 1: dZ += w^T dO (the token gradient), from dO's tile the same way.
 // Writes part[p][bh][g] = MODE 1: (dZ(32), dWx(32), sum da, 0); MODE 2: (dWx, sum da, 0)
 // and dt_part[bh][p * R + block] = ln2 * sum over the block's slots of sum da (a2 - lse2).
+// Two more modes serve fs_coupling_bwd:
+//   MODE 0: the token gradient alone, dZ += w^T dO (no dw chain, no da): part = dZ(32);
+//   MODE 3: da = da_D + da_S as in the combined point pass (dw - delta as two chains:
+//     the deslice's T block against [dO | 1, 1, -delta], the slice's T2 block against
+//     [fx | 1, 1, 0 ...], delta = delta_D + delta_S), written like MODE 2.
 // smem: [W block: hi 8K | extra 4K | lo 8K][T block: same][stages][zero 2K][red 1.5K][bars]
 // TMEM: unit u uses set u % 3: L [128 s, +64), dw [128 s + 64, +64); accumulators
 // dWx_j [384 + 32 j), dZ_j [448 + 32 j).
@@ -205,22 +237,29 @@ template <int MODE, bool split>
 __global__ void __launch_bounds__(kThreads, 1)
     k_bwd_slot_tc(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap vmap,
                   const __grid_constant__ CUtensorMap pmap, const __grid_constant__ CUtensorMap dmap,
-                  const uint8_t* __restrict__ wimg, const uint8_t* __restrict__ timg, float* __restrict__ part,
+                  const __grid_constant__ CUtensorMap fmap, const uint8_t* __restrict__ wimg,
+                  const uint8_t* __restrict__ timg, const uint8_t* __restrict__ timg2, float* __restrict__ part,
                   float* __restrict__ dt_part, int64_t N, int64_t Np, int H, int G, int splits,
                   uint32_t* status) {
+  constexpr int kNSt = MODE == 3 ? kBStages - 1 : kBStages;    // stages (MODE 3's are larger)
+  constexpr uint32_t kStgS = kBStage + (MODE == 3 ? kXBytes : 0u);  // x | v | px | dpx [| fx]
   const int g_base = blockIdx.x * kGC;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* s_w = smem;               // W block
   uint8_t* s_t = s_w + kWBlockB;     // T block
-  uint8_t* s_st = s_t + kWBlockB;    // stages
-  uint8_t* s_zero = s_st + kBStages * kBStage;
+  uint8_t* s_t2 = s_t + kWBlockB;    // MODE 3: the slice's T block
+  uint8_t* s_st = s_t2 + (MODE == 3 ? kWBlockB : 0u);  // stages
+  // MODE 3: point rows [1, 1, 0 ...] (no delta).  Like the stages' point rows it lies
+  // below the zero block, which its descriptor reaches at a positive offset.
+  uint8_t* s_ones = s_st + kNSt * kStgS;
+  uint8_t* s_zero = s_ones + (MODE == 3 ? kPxBytes : 0u);
   float* s_red = reinterpret_cast<float*>(s_zero + kPxZero);  // 3 x 128 floats
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_red + 3 * kGC);
   uint64_t* w_full = bars;
   uint64_t* x_full = bars + 1;
-  uint64_t* st_empty = x_full + kBStages;
-  uint64_t* s_full = st_empty + kBStages;
+  uint64_t* st_empty = x_full + kNSt;
+  uint64_t* s_full = st_empty + kNSt;
   uint64_t* p_ready = s_full + kSBuf;  // [issuer][set]
   uint64_t* pv_done = p_ready + 2 * kSBuf;
   uint64_t* acc_full = pv_done + kSBuf;
@@ -238,7 +277,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (threadIdx.x == 0) {
     mbar_init(w_full, 1);
-    for (int s = 0; s < kBStages; s++) {
+    for (int s = 0; s < kNSt; s++) {
       mbar_init(&x_full[s], 1);
       mbar_init(&st_empty[s], 3);  // the logits issuer and both product issuers
     }
@@ -254,6 +293,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_mbar_init();
   }
   zero_smem(s_zero, kPxZero);
+  if (MODE == 3)
+    for (int r = threadIdx.x; r < kTile; r += blockDim.x)
+      st_shared_v4(smem_u32(s_ones) + (uint32_t)r * 16, 0x3F803F80u, 0u, 0u, 0u);
   fence_proxy_async_smem();
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
@@ -267,52 +309,60 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&xmap);
       prefetch_tmap(&vmap);
       prefetch_tmap(&pmap);
-      prefetch_tmap(&dmap);
-      mbar_expect_tx(w_full, 2 * kWBlockB);
+      if (MODE != 0) prefetch_tmap(&dmap);
+      if (MODE == 3) prefetch_tmap(&fmap);
+      constexpr int kImages = MODE == 0 ? 1 : (MODE == 3 ? 3 : 2);  // W [, T [, T2]]
+      mbar_expect_tx(w_full, kImages * kWBlockB);
       const uint8_t* ws = wimg + (size_t)h * G * kWRow;
       const uint8_t* ts = timg + (size_t)wk.bh * G * kWRow;
-      for (int im = 0; im < 2; im++) {
-        const uint8_t* src = im ? ts : ws;
-        uint8_t* dst = im ? s_t : s_w;
+      const uint8_t* ts2 = MODE == 3 ? timg2 + (size_t)wk.bh * G * kWRow : nullptr;
+      for (int im = 0; im < kImages; im++) {
+        const uint8_t* src = im == 0 ? ws : (im == 1 ? ts : ts2);
+        uint8_t* dst = im == 0 ? s_w : (im == 1 ? s_t : s_t2);
         load_images(dst, src + (size_t)g_base * 64, kGC * 64, w_full);
         load_images(dst + kGC * 64, src + (size_t)G * 64 + (size_t)g_base * 32, kGC * 32, w_full);
         load_images(dst + kGC * 96, src + (size_t)G * 96 + (size_t)g_base * 64, kGC * 64, w_full);
       }
       int i = 0;
       for (; i < wk.ntiles; i++) {
-        const int s = i % kBStages;
-        if (i >= kBStages && !mbar_wait(&st_empty[s], (uint32_t)(((i / kBStages) - 1) & 1), ab, status)) break;
-        uint8_t* st = s_st + s * kBStage;
+        const int s = i % kNSt;
+        if (i >= kNSt && !mbar_wait(&st_empty[s], (uint32_t)(((i / kNSt) - 1) & 1), ab, status)) break;
+        uint8_t* st = s_st + s * kStgS;
         const int n0 = (int)((wk.tile0 + i) * kTile);
-        mbar_expect_tx(&x_full[s], kBStage);
+        mbar_expect_tx(&x_full[s], MODE == 0 ? kBStage - kPxBytes : kStgS);
         tma_load_3d(st, &xmap, h * kD, n0, (int)b, &x_full[s]);
         tma_load_3d(st + kVOff, &vmap, h * kD, n0, (int)b, &x_full[s]);
         tma_load_2d(st + kPOff, &pmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
-        tma_load_2d(st + kDOff, &dmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
+        if (MODE != 0) tma_load_2d(st + kDOff, &dmap, 0, (int)(wk.bh * Np + n0), &x_full[s]);
+        if (MODE == 3) tma_load_3d(st + kBStage, &fmap, h * kD, n0, (int)b, &x_full[s]);
       }
-      for (int j = (i > kBStages ? i - kBStages : 0); j < i; j++)
-        mbar_wait(&x_full[j % kBStages], (uint32_t)((j / kBStages) & 1), ab, nullptr, kWaitNs);
+      for (int j = (i > kNSt ? i - kNSt : 0); j < i; j++)
+        mbar_wait(&x_full[j % kNSt], (uint32_t)((j / kNSt) & 1), ab, nullptr, kWaitNs);
       mbar_wait(w_full, 0, ab, nullptr, kWaitNs);
     }
   } else if (warp == 1) {
     // ------------------------------ logits and dw issuer ------------------------------
-    const uint32_t sw = smem_u32(s_w), stt = smem_u32(s_t), sz = smem_u32(s_zero);
+    const uint32_t sw = smem_u32(s_w), stt = smem_u32(s_t), stt2 = smem_u32(s_t2), sz = smem_u32(s_zero);
     bool ok = mbar_wait_w(w_full, 0, ab, status);
     for (int u = 0; ok && u < units; u++) {
       const int i = u >> 1, half = u & 1;
-      const int s = i % kBStages;
+      const int s = i % kNSt;
       const int bb = u % kSBuf;
-      if (half == 0 && !(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kBStages) & 1), ab, status))) break;
+      if (half == 0 && !(ok = mbar_wait_w(&x_full[s], (uint32_t)((i / kNSt) & 1), ab, status))) break;
       if (u >= kSBuf && !(ok = mbar_wait_w(&pv_done[bb], (uint32_t)(((u / kSBuf) - 1) & 1), ab, status))) break;
       tc_fence_after();
-      const uint32_t st = smem_u32(s_st + s * kBStage);
+      const uint32_t st = smem_u32(s_st + s * kStgS);
       const uint32_t rows = (uint32_t)half * 64 * 64;     // the unit's 64 points in the 64-byte-row tiles
       const uint32_t prow = (uint32_t)half * 64 * 16;     // ... and in the 16-byte extra rows
       const uint32_t tL = tmem + (uint32_t)bb * kGC;
       issue_dot64<true>(tL, sw, st + rows, sdesc(sw + kGC * 64, 16, 256, kSw32), px_desc(st + kPOff + prow, sz),
                         split ? sw + kGC * 96 : 0u);
-      issue_dot64<true>(tL + 64, stt, st + kVOff + rows, sdesc(stt + kGC * 64, 16, 256, kSw32),
-                        px_desc(st + kDOff + prow, sz), split ? stt + kGC * 96 : 0u);
+      if (MODE != 0)
+        issue_dot64<true>(tL + 64, stt, st + kVOff + rows, sdesc(stt + kGC * 64, 16, 256, kSw32),
+                          px_desc(st + kDOff + prow, sz), split ? stt + kGC * 96 : 0u);
+      if (MODE == 3)
+        issue_dot64<true>(tL + 64, stt2, st + kBStage + rows, sdesc(stt2 + kGC * 64, 16, 256, kSw32),
+                          px_desc(smem_u32(s_ones) + prow, sz), split ? stt2 + kGC * 96 : 0u, 1u);
       mma_commit_w(&s_full[bb]);
       if (half == 1) mma_commit_w(&st_empty[s]);
     }
@@ -325,18 +375,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     bool ok = true;
     for (int u = j; ok && u < units; u += 2) {
       const int i = u >> 1;
-      const int s = i % kBStages;
+      const int s = i % kNSt;
       const int bb = u % kSBuf;
       // This issuer's units on set bb are 2 kSBuf apart.
       if (!(ok = mbar_wait_w(&p_ready[j * kSBuf + bb], (uint32_t)((u / (2 * kSBuf)) & 1), ab, status))) break;
       tc_fence_after();
-      const uint32_t st = smem_u32(s_st + s * kBStage) + (uint32_t)j * 64 * 64;
+      const uint32_t st = smem_u32(s_st + s * kStgS) + (uint32_t)j * 64 * 64;
       const uint32_t tL = tmem + (uint32_t)bb * kGC, tD = tL + 64;
 #pragma unroll
       for (int kk = 0; kk < 4; kk++) {
         // 16 points: two 8-row groups of the 64B-swizzled tile (MN-major: channels contiguous).
         const uint64_t xd = sdesc(st + (uint32_t)kk * 1024, 4096, 512, kSw64);
         const uint32_t acc = (u >= 2 || kk > 0) ? 1u : 0u;
+        if (MODE == 0) {  // the weights are in the L columns: dZ += w^T dO
+          const uint64_t vd = sdesc(st + kVOff + (uint32_t)kk * 1024, 4096, 512, kSw64);
+          mma_ts_w(tmem + kAccZ + (uint32_t)j * 32, tL + da_col(kk), vd, idesc, acc);
+          if (split) mma_ts_w(tmem + kAccZ + (uint32_t)j * 32, tL + da_col(kk) + 16, vd, idesc, 1u);
+          continue;
+        }
         mma_ts_w(tmem + kAccW + (uint32_t)j * 32, tL + da_col(kk), xd, idesc, acc);
         if (split) mma_ts_w(tmem + kAccW + (uint32_t)j * 32, tL + da_col(kk) + 16, xd, idesc, 1u);
         if (MODE == 1) {
@@ -364,20 +420,40 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((u / kSBuf) & 1), ab, status))) break;
       tc_fence_after();
       const uint32_t tL = tmem + lane_addr + (uint32_t)bb * kGC;
-      float t = 0.f, sb = 0.f;
-      da_unit<split, MODE == 1, true>(tL, tL + 64, t, sb);
-      dt += t;
-      db += sb;
+      if (MODE == 0) {
+        w_unit<split>(tL);
+      } else {
+        float t = 0.f, sb = 0.f;
+        da_unit<split, MODE == 1, true>(tL, tL + 64, t, sb);
+        dt += t;
+        db += sb;
+      }
       tmem_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_ready[wg * kSBuf + bb]);
     }
     // Epilogue: warpgroup 1 hands its sums to warpgroup 0, which writes dWx and the
-    // sums; warpgroup 1 writes dZ (MODE 1).
+    // sums; warpgroup 1 writes dZ (MODE 1; MODE 0 writes dZ alone).
     const int64_t BH = gridDim.z;
-    const int PS = MODE == 1 ? 2 * kD + 2 : kD + 2;
+    const int PS = MODE == 1 ? 2 * kD + 2 : (MODE == 0 ? kD : kD + 2);
     float* o = part + (((int64_t)blockIdx.y * BH + wk.bh) * G + g_base + r) * PS;
+    if (MODE == 0) {
+      const bool have0 = ok && wk.ntiles > 0 && mbar_wait(acc_full, 0, ab, status);
+      if (have0) tc_fence_after();
+      if (wg == 1) {
+        if (have0) {
+          uint32_t z0[32], z1[32];
+          tmem_ld32(tmem + lane_addr + kAccZ, z0);
+          tmem_ld32(tmem + lane_addr + kAccZ + 32, z1);
+          tmem_wait_ld2(z0, z1);
+#pragma unroll
+          for (int k = 0; k < kD; k++) o[k] = __uint_as_float(z0[k]) + __uint_as_float(z1[k]);
+        } else {
+          for (int k = 0; k < kD; k++) o[k] = 0.f;
+        }
+      }
+    } else {
     if (wg == 1) {
       s_red[r] = dt;
       s_red[kGC + r] = db;
@@ -419,6 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       } else {
         for (int k = 0; k < kD; k++) o[k] = 0.f;
       }
+    }
     }
   }
   tc_fence_before();
@@ -673,8 +750,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ---- host side ---------------------------------------------------------------------------------
 
-size_t smem_bwd_slot() {
-  return 1024 + 2 * (size_t)kWBlockB + kBStages * (size_t)kBStage + kPxZero + 3 * kGC * 4 + 512;
+size_t smem_bwd_slot(int mode = 1) {
+  const bool m3 = mode == 3;
+  return 1024 + (m3 ? 3 : 2) * (size_t)kWBlockB + (m3 ? kBStages - 1 : kBStages) * (size_t)(kBStage + (m3 ? kXBytes : 0)) +
+         kPxZero + (m3 ? kPxBytes : 0) + 3 * kGC * 4 + 512;
 }
 size_t smem_bwd_dx(int G, bool hilo, bool comb = false) {
   return 1024 + (size_t)G * ((hilo ? kWRow : 96) + 96 * (comb ? 2 : 1) + 64) + (comb ? kExBytes : 0) +
@@ -862,11 +941,11 @@ cudaError_t run_backward(const Shape& s0, int mode, const void* x, const void* v
       if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     {
-      const size_t sm = smem_bwd_slot();
+      const size_t sm = smem_bwd_slot(mode);
       const auto kernel = mode == 1 ? k_bwd_slot_tc<1, true> : k_bwd_slot_tc<2, true>;
       if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
       kernel<<<dim3((unsigned)R, (unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(
-          xmap, vmap, pmap, dmap, ws + L.wimg, ws + L.timg, reinterpret_cast<float*>(ws + L.part),
+          xmap, vmap, pmap, dmap, xmap, ws + L.wimg, ws + L.timg, nullptr, reinterpret_cast<float*>(ws + L.part),
           reinterpret_cast<float*>(ws + L.dtp), s.N, Np, s.H, s.G, P, status);
       if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
@@ -915,11 +994,19 @@ cudaError_t run_backward(const Shape& s0, int mode, const void* x, const void* v
   return cudaSuccess;
 }
 
-// The coupling's backward in one call (fs_coupling_bwd): the deslice's and the slice's
-// passes as in the two calls but without their point passes, the mix backward between
-// them, then ONE point pass for dx = ln2 sum_g (da_D + da_S)_ng W'_g: the two calls'
-// da share the weights, so their dw - delta add up (k_bwd_dx_tc<·, true>).  That pass
-// holds two T images besides W' and W'^T and runs over slot ranges of at most 256.
+// The coupling's backward in one call (fs_coupling_bwd).  The deslice's and the
+// slice's da share the weights, so their slot-owned and point-owned products can be
+// formed once from da_D + da_S; what has to come first is d z' (it feeds the mix
+// backward, and so dU, dS and the slice's part).  Per slot range (as in the separate
+// calls):
+//   1. the deslice part's rows pass: delta_D;
+//   2. the slot pass in mode 0: d z' from the weights alone;
+//   3. the mix backward and the dU | dS prologue;
+//   4. the slice part's rows pass: delta_S, dfx, the sum_g w dS partials;
+//   5. delta = delta_S + delta_D + sum_g w dS into the point rows;
+//   6. the slot pass in mode 3: dW, dbias, dtau of da_D + da_S;
+//   7. one point pass (k_bwd_dx_tc<., true>) for dx, over ranges of at most 256
+//      slots (it holds two T images besides W' and W'^T).
 constexpr int kCombSlotsMax = 256;
 SlotRanges comb_ranges(const Shape& s0) {
   const int cap = std::min(kCombSlotsMax, pass_shape(s0).G);
@@ -933,25 +1020,28 @@ SlotRanges comb_ranges(const Shape& s0) {
   return best;
 }
 
-// Workspace of the coupling backward: the larger of the two calls' layouts, then the
-// deslice's delta, the slice's T image for the point pass, and (with several point-pass
-// ranges) a range's slices of W, bias, z' and dU | dS.
+// Workspace of the coupling backward: the slice backward's layout, then delta_D, a
+// second T image (the slice's, beside the deslice's), the ranges' d z' slices, and a
+// range's slices of W, bias, z' and dU | dS (for the passes' ranges and the point
+// pass's, whichever are larger).
 struct CoupLayout {
-  size_t deltaD, timg2, wc, bc, zc, uc, total;
+  size_t deltaD, timg2, dzc, wc, bc, zc, uc, total;
 };
 CoupLayout coup_layout(const Shape& s0) {
   CoupLayout C{};
-  size_t off = std::max(bwd_layout(s0, 1).total, bwd_layout(s0, 2).total);
+  size_t off = bwd_layout(s0, 2).total;
   auto take = [&](size_t bytes) {
     const size_t o = off;
     off = align_up(off + bytes, 256);
     return o;
   };
   const Shape s = pass_shape(s0);
-  const SlotRanges cr = comb_ranges(s0);
-  const size_t rs = cr.n > 1 ? (size_t)cr.size : 0;
+  const SlotRanges sr = slot_ranges(s0.G), cr = comb_ranges(s0);
+  const size_t rp = sr.n > 1 ? (size_t)sr.size : 0;
+  const size_t rs = std::max(rp, cr.n > 1 ? (size_t)cr.size : 0);
   C.deltaD = take((size_t)s.BH() * s.N * sizeof(float));
-  C.timg2 = take((size_t)s.BH() * cr.size * kWRow);
+  C.timg2 = take((size_t)s.BH() * std::max(s.G, cr.size) * kWRow);
+  C.dzc = take((size_t)s.BH() * rp * kD * sizeof(float));
   C.wc = take((size_t)s.H * kD * rs * sizeof(float));
   C.bc = take((size_t)s.H * rs * sizeof(float));
   C.zc = take((size_t)s.BH() * rs * kD * sizeof(float));
@@ -965,68 +1055,182 @@ cudaError_t run_coupling_bwd(const Shape& s0, const void* x, const void* f, cons
                              const float* zp, const float* lse, float* dzp, float* dz, float* dM, void* dx, void* dfx,
                              float* dW, float* db, float* dtau, int accumulate, float* dUS, uint8_t* ws,
                              uint32_t* status, cudaStream_t st) {
-  const CoupLayout C = coup_layout(s0);
+  const SlotRanges sr = slot_ranges(s0.G);
+  const Shape s = pass_shape(s0);
   const BwdLayout L = bwd_layout(s0, 2);
-  float* deltaD = reinterpret_cast<float*>(ws + C.deltaD);
-  cudaError_t e;
-  if ((e = run_backward(s0, 1, x, dout, W, bias, tau, zp, kD, lse, nullptr, nullptr, dzp, dW, db, dtau, accumulate,
-                        ws, status, st, deltaD)) != cudaSuccess)
-    return e;
-  if ((e = simt_mix_bwd(s0, M, z, dzp, dz, dM, st)) != cudaSuccess) return e;
-  if ((e = simt_slice_bwd_prep(s0, z, wsum, dz, dUS, st)) != cudaSuccess) return e;
-  if ((e = run_backward(s0, 2, x, f, W, bias, tau, dUS, kD + 1, lse, dfx, nullptr, nullptr, dW, db, dtau, 1, ws,
-                        status, st)) != cudaSuccess)
-    return e;
-  // delta = delta_S + delta_D + the slice's sum_g w dS, into the point rows; the lse
-  // rows are still in place from the slice's passes.
-  const SlotRanges cr = comb_ranges(s0);
-  Shape s = pass_shape(s0);
-  s.G = cr.size;
+  const CoupLayout C = coup_layout(s0);
+  const bool ranged = sr.n > 1;
   const int64_t Np = padded_n(s), npx = s.BH() * Np;
-  k_prep_dpx<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(
-      reinterpret_cast<const float*>(ws + L.delta), deltaD, reinterpret_cast<const float*>(ws + L.wds),
-      reinterpret_cast<uint4*>(ws + L.dpx), s.BH(), s.N, Np);
+  float* deltaD = reinterpret_cast<float*>(ws + C.deltaD);
+  float* deltaS = reinterpret_cast<float*>(ws + L.delta);
+  float* wds = reinterpret_cast<float*>(ws + L.wds);
+  float* wc = reinterpret_cast<float*>(ws + C.wc);
+  float* bc = reinterpret_cast<float*>(ws + C.bc);
+  float* zc = reinterpret_cast<float*>(ws + C.zc);
+  float* uc = reinterpret_cast<float*>(ws + C.uc);
+  cudaError_t e;
+  // Slices [g0, g0 + G) of W, bias, z' and dU | dS (the gathered ones when `slice`).
+  struct Src {
+    const float *W, *b, *z, *u;
+  };
+  auto gather = [&](int g0, int G, bool slice, bool wz, bool zt, bool ut, Src* o) -> cudaError_t {
+    *o = {W, bias, zp, dUS};
+    if (!slice) return cudaSuccess;
+    cudaError_t r;
+    if (wz) {
+      if ((r = copy_rows(wc, G, W + g0, s0.G, G, (int64_t)s.H * kD, st)) != cudaSuccess) return r;
+      if ((r = copy_rows(bc, G, bias + g0, s0.G, G, s.H, st)) != cudaSuccess) return r;
+      o->W = wc, o->b = bc;
+    }
+    if (zt) {
+      if ((r = copy_rows(zc, (int64_t)G * kD, zp + (int64_t)g0 * kD, (int64_t)s0.G * kD, (int64_t)G * kD, s.BH(),
+                         st)) != cudaSuccess)
+        return r;
+      o->z = zc;
+    }
+    if (ut) {
+      if ((r = copy_rows(uc, (int64_t)G * (kD + 1), dUS + (int64_t)g0 * (kD + 1), (int64_t)s0.G * (kD + 1),
+                         (int64_t)G * (kD + 1), s.BH(), st)) != cudaSuccess)
+        return r;
+      o->u = uc;
+    }
+    return cudaSuccess;
+  };
+  auto range_g = [&](int k) { return k < sr.n - 1 ? sr.size : s0.G - (sr.n - 1) * sr.size; };
+
+  k_prep_px<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(lse, reinterpret_cast<uint4*>(ws + L.px), s.BH(), s.N,
+                                                             Np);
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  // 1. delta_D
+  for (int k = 0; k < sr.n; k++) {
+    const int g0 = k * sr.size, G = range_g(k);
+    Src a;
+    if ((e = gather(g0, G, ranged, true, true, false, &a)) != cudaSuccess) return e;
+    if ((e = prep_w(s, G, a.W, a.b, tau, ws + L.wimg, status, st)) != cudaSuccess) return e;
+    if ((e = prep_t_images(s, G, a.z, kD, 0, ws, L, st)) != cudaSuccess) return e;
+    if ((e = tc_rows_bwd(s, 1, x, ws + L.wimg, ws + L.zimg, ws + L.px, dout, nullptr, deltaD, nullptr,
+                         reinterpret_cast<const float*>(ws + L.ds), k > 0 ? 1 : 0, status, st)) != cudaSuccess)
+      return e;
+  }
+  const int R = bwd_slot_blocks(s), P = bwd_slot_splits(s);
   CUtensorMap xmap, vmap, pmap, dmap, fmap;
   if (!make_maps(s, x, dout, ws + L.px, ws + L.dpx, &xmap, &vmap, &pmap, &dmap) ||
       !make_point_map(&fmap, f, s, kD, CU_TENSOR_MAP_SWIZZLE_64B))
     return cudaErrorInvalidValue;
-  const bool hilo = smem_bwd_dx(s.G, true, true) <= kMaxSmem;
-  const size_t sm = smem_bwd_dx(s.G, hilo, true);
+  // 2. d z' (the W image of the last range is in place)
+  {
+    const size_t sm = smem_bwd_slot(0);
+    const auto kernel = k_bwd_slot_tc<0, true>;
+    if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
+    for (int k = 0; k < sr.n; k++) {
+      const int g0 = k * sr.size, G = range_g(k);
+      if (ranged) {
+        Src a;
+        if ((e = gather(g0, G, true, true, false, false, &a)) != cudaSuccess) return e;
+        if ((e = prep_w(s, G, a.W, a.b, tau, ws + L.wimg, status, st)) != cudaSuccess) return e;
+      }
+      kernel<<<dim3((unsigned)R, (unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(
+          xmap, vmap, pmap, pmap, xmap, ws + L.wimg, ws + L.timg, nullptr, reinterpret_cast<float*>(ws + L.part),
+          reinterpret_cast<float*>(ws + L.dtp), s.N, Np, s.H, s.G, P, status);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      Shape sk = s0;
+      sk.G = G;
+      float* dzk = ranged ? reinterpret_cast<float*>(ws + C.dzc) : dzp;
+      if ((e = simt_reduce_dzp(sk, P, reinterpret_cast<const float*>(ws + L.part), s.G, kD, dzk, st)) != cudaSuccess)
+        return e;
+      if (ranged && (e = copy_rows(dzp + (int64_t)g0 * kD, (int64_t)s0.G * kD, dzk, (int64_t)G * kD, (int64_t)G * kD,
+                                   s.BH(), st)) != cudaSuccess)
+        return e;
+    }
+  }
+  // 3. the mix backward and dU | dS
+  if ((e = simt_mix_bwd(s0, M, z, dzp, dz, dM, st)) != cudaSuccess) return e;
+  if ((e = simt_slice_bwd_prep(s0, z, wsum, dz, dUS, st)) != cudaSuccess) return e;
+  // 4. delta_S, dfx, sum_g w dS
+  if ((e = cudaMemsetAsync(wds, 0, 2 * (size_t)s.BH() * s.N * sizeof(float), st)) != cudaSuccess) return e;
+  for (int k = 0; k < sr.n; k++) {
+    const int g0 = k * sr.size, G = range_g(k);
+    Src a;
+    if ((e = gather(g0, G, ranged, true, false, true, &a)) != cudaSuccess) return e;
+    if ((e = prep_w(s, G, a.W, a.b, tau, ws + L.wimg, status, st)) != cudaSuccess) return e;
+    if ((e = prep_t_images(s, G, a.u, kD + 1, 1, ws, L, st)) != cudaSuccess) return e;
+    if ((e = tc_rows_bwd(s, 2, x, ws + L.wimg, ws + L.zimg, ws + L.px, f, dfx, deltaS, wds,
+                         reinterpret_cast<const float*>(ws + L.ds), k > 0 ? 1 : 0, status, st)) != cudaSuccess)
+      return e;
+  }
+  // 5. delta's point rows
+  k_prep_dpx<<<(unsigned)((npx + 255) / 256), 256, 0, st>>>(deltaS, deltaD, wds, reinterpret_cast<uint4*>(ws + L.dpx),
+                                                              s.BH(), s.N, Np);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  // 6. dW, dbias, dtau of da_D + da_S
+  {
+    const size_t sm = smem_bwd_slot(3);
+    const auto kernel = k_bwd_slot_tc<3, true>;
+    if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
+    for (int k = 0; k < sr.n; k++) {
+      const int g0 = k * sr.size, G = range_g(k);
+      Src a;
+      if ((e = gather(g0, G, ranged, true, true, true, &a)) != cudaSuccess) return e;
+      if ((e = prep_w(s, G, a.W, a.b, tau, ws + L.wimg, status, st)) != cudaSuccess) return e;
+      const int64_t BHG = s.BH() * s.G;
+      k_prep_t<<<(unsigned)((BHG + 127) / 128), 128, 0, st>>>(a.z, kD, 0, ws + L.timg, nullptr, s.BH(), G, s.G);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      k_prep_t<<<(unsigned)((BHG + 127) / 128), 128, 0, st>>>(a.u, kD + 1, 1, ws + C.timg2, nullptr, s.BH(), G, s.G);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      kernel<<<dim3((unsigned)R, (unsigned)P, (unsigned)s.BH()), kThreads, sm, st>>>(
+          xmap, vmap, pmap, dmap, fmap, ws + L.wimg, ws + L.timg, ws + C.timg2, reinterpret_cast<float*>(ws + L.part),
+          reinterpret_cast<float*>(ws + L.dtp), s.N, Np, s.H, s.G, P, status);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+      const int acc = accumulate || k > 0;
+      Shape sk = s0;
+      sk.G = G;
+      float *dWk = dW, *dbk = db;
+      if (ranged) {
+        dWk = reinterpret_cast<float*>(ws + L.dwc);
+        dbk = reinterpret_cast<float*>(ws + L.dbc);
+        if (accumulate) {
+          if ((e = copy_rows(dWk, G, dW + g0, s0.G, G, (int64_t)s.H * kD, st)) != cudaSuccess) return e;
+          if ((e = copy_rows(dbk, G, db + g0, s0.G, G, s.H, st)) != cudaSuccess) return e;
+        } else if (acc) {
+          if ((e = cudaMemsetAsync(dWk, 0, (size_t)s.H * kD * G * sizeof(float), st)) != cudaSuccess) return e;
+          if ((e = cudaMemsetAsync(dbk, 0, (size_t)s.H * G * sizeof(float), st)) != cudaSuccess) return e;
+        }
+      }
+      if ((e = simt_reduce_bwd(sk, P, reinterpret_cast<const float*>(ws + L.part), s.G, kD + 2, 0, tau, nullptr, dWk,
+                               dbk, dtau, reinterpret_cast<const float*>(ws + L.dtp), (int64_t)P * R, acc, st)) !=
+          cudaSuccess)
+        return e;
+      if (ranged) {
+        if ((e = copy_rows(dW + g0, s0.G, dWk, G, G, (int64_t)s.H * kD, st)) != cudaSuccess) return e;
+        if ((e = copy_rows(db + g0, s0.G, dbk, G, G, s.H, st)) != cudaSuccess) return e;
+      }
+    }
+  }
+  // 7. dx from da_D + da_S
+  const SlotRanges cr = comb_ranges(s0);
+  Shape sc = s;
+  sc.G = cr.size;
+  const bool hilo = smem_bwd_dx(sc.G, true, true) <= kMaxSmem;
+  const size_t sm = smem_bwd_dx(sc.G, hilo, true);
   if (sm > kMaxSmem) return cudaErrorInvalidValue;
   const auto kernel = k_bwd_dx_tc<true, true>;
   if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
-  const int Pd = point_splits(s, (int)s.BH());
-  const bool ranged = cr.n > 1;
+  const int Pd = point_splits(sc, (int)sc.BH());
   for (int k = 0; k < cr.n; k++) {
     const int g0 = k * cr.size, G = k < cr.n - 1 ? cr.size : s0.G - (cr.n - 1) * cr.size;
-    const float *Wk = W, *bk = bias, *zk = zp, *uk = dUS;
-    if (ranged) {
-      float* wc = reinterpret_cast<float*>(ws + C.wc);
-      float* bc = reinterpret_cast<float*>(ws + C.bc);
-      float* zc = reinterpret_cast<float*>(ws + C.zc);
-      float* uc = reinterpret_cast<float*>(ws + C.uc);
-      if ((e = copy_rows(wc, G, W + g0, s0.G, G, (int64_t)s.H * kD, st)) != cudaSuccess) return e;
-      if ((e = copy_rows(bc, G, bias + g0, s0.G, G, s.H, st)) != cudaSuccess) return e;
-      if ((e = copy_rows(zc, (int64_t)G * kD, zp + (int64_t)g0 * kD, (int64_t)s0.G * kD, (int64_t)G * kD, s.BH(),
-                         st)) != cudaSuccess)
-        return e;
-      if ((e = copy_rows(uc, (int64_t)G * (kD + 1), dUS + (int64_t)g0 * (kD + 1), (int64_t)s0.G * (kD + 1),
-                         (int64_t)G * (kD + 1), s.BH(), st)) != cudaSuccess)
-        return e;
-      Wk = wc, bk = bc, zk = zc, uk = uc;
-    }
-    if ((e = prep_w(s, G, Wk, bk, tau, ws + L.wimg, status, st)) != cudaSuccess) return e;
-    const int64_t nwt = (int64_t)s.H * kD * s.G, BHG = s.BH() * s.G;
-    k_prep_wt<<<(unsigned)((nwt + 255) / 256), 256, 0, st>>>(Wk, tau, ws + L.wtimg, s.H, G, s.G, status);
+    Src a;
+    if ((e = gather(g0, G, cr.n > 1, true, true, true, &a)) != cudaSuccess) return e;
+    if ((e = prep_w(sc, G, a.W, a.b, tau, ws + L.wimg, status, st)) != cudaSuccess) return e;
+    const int64_t nwt = (int64_t)sc.H * kD * sc.G, BHG = sc.BH() * sc.G;
+    k_prep_wt<<<(unsigned)((nwt + 255) / 256), 256, 0, st>>>(a.W, tau, ws + L.wtimg, sc.H, G, sc.G, status);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    k_prep_t<<<(unsigned)((BHG + 127) / 128), 128, 0, st>>>(zk, kD, 0, ws + L.timg, nullptr, s.BH(), G, s.G);
+    k_prep_t<<<(unsigned)((BHG + 127) / 128), 128, 0, st>>>(a.z, kD, 0, ws + L.timg, nullptr, sc.BH(), G, sc.G);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    k_prep_t<<<(unsigned)((BHG + 127) / 128), 128, 0, st>>>(uk, kD + 1, 1, ws + C.timg2, nullptr, s.BH(), G, s.G);
+    k_prep_t<<<(unsigned)((BHG + 127) / 128), 128, 0, st>>>(a.u, kD + 1, 1, ws + C.timg2, nullptr, sc.BH(), G, sc.G);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    kernel<<<dim3((unsigned)Pd, (unsigned)s.BH()), kThreads, sm, st>>>(
+    kernel<<<dim3((unsigned)Pd, (unsigned)sc.BH()), kThreads, sm, st>>>(
         xmap, vmap, pmap, dmap, fmap, ws + L.wimg, ws + L.timg, ws + C.timg2, ws + L.wtimg,
-        static_cast<__nv_bfloat16*>(dx), s.N, Np, s.H, s.G, Pd, hilo ? 1 : 0, (accumulate || k > 0) ? 1 : 0,
+        static_cast<__nv_bfloat16*>(dx), sc.N, Np, sc.H, sc.G, Pd, hilo ? 1 : 0, (accumulate || k > 0) ? 1 : 0,
         status);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
   }
@@ -1071,13 +1275,13 @@ size_t tc_coupling_bwd_bytes(const Shape& s) { return tc_backward_supported(s) ?
 
 int tc_coupling_bwd_launch_count(const Shape& s) {
   const SlotRanges sr = slot_ranges(s.G), cr = comb_ranges(s);
-  // each call's passes without its point pass (and without W'^T's image when it has
-  // one range), the mix backward, the dU/dS prologue, the combined delta rows, and per
-  // point-pass range its four images and the pass
-  const int images = sr.n > 1 ? 3 : 0;
-  const int call1 = 4 * sr.n + 2 + sr.n * (images + 1 + 3);
-  const int call2 = 4 * sr.n + 2 + sr.n * (images + 1 + 2);
-  return call1 + 2 + 1 + call2 + 1 + 5 * cr.n;
+  const int n = sr.n, r = n > 1 ? 1 : 0;
+  // lse rows; per range: the deslice rows pass with its images (4), the d z' slot
+  // pass with its reduction (2, and the W image again with several ranges); the mix
+  // backward (2) and the dU | dS prologue; per range the slice rows pass with its
+  // images (4); delta's rows; per range the combined slot pass with its images and
+  // reductions (6); per point-pass range its images and the pass (5)
+  return 1 + 4 * n + n * (2 + r) + 3 + 4 * n + 1 + 6 * n + 5 * cr.n;
 }
 
 cudaError_t tc_coupling_bwd(const Shape& s0, const void* x, const void* f, const void* dout, const float* W,
