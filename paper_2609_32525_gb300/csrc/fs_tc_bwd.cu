@@ -1000,7 +1000,9 @@ cudaError_t run_backward(const Shape& s0, int mode, const void* x, const void* v
 // backward, and so dU, dS and the slice's part).  Per slot range (as in the separate
 // calls):
 //   1. the deslice part's rows pass: delta_D;
-//   2. the slot pass in mode 0: d z' from the weights alone;
+//   2. d z' = sum_n w_ng dO_n: the forward's slice with dO for fx (its unnormalised
+//      numerators) where the forward's kernels take the shape, else the slot pass in
+//      mode 0 (the weights alone);
 //   3. the mix backward and the dU | dS prologue;
 //   4. the slice part's rows pass: delta_S, dfx, the sum_g w dS partials;
 //   5. delta = delta_S + delta_D + sum_g w dS into the point rows;
@@ -1025,7 +1027,7 @@ SlotRanges comb_ranges(const Shape& s0) {
 // range's slices of W, bias, z' and dU | dS (for the passes' ranges and the point
 // pass's, whichever are larger).
 struct CoupLayout {
-  size_t deltaD, timg2, dzc, wc, bc, zc, uc, total;
+  size_t deltaD, timg2, dzc, wc, bc, zc, uc, sl_part, sl_prep, sl_wsum, total;
 };
 CoupLayout coup_layout(const Shape& s0) {
   CoupLayout C{};
@@ -1046,6 +1048,12 @@ CoupLayout coup_layout(const Shape& s0) {
   C.bc = take((size_t)s.H * rs * sizeof(float));
   C.zc = take((size_t)s.BH() * rs * kD * sizeof(float));
   C.uc = take((size_t)s.BH() * rs * (kD + 1) * sizeof(float));
+  // d z' through the forward's slice (split products, as the backward's weights)
+  const Shape ss = split_shape(s0);
+  const bool via_slice = tc_forward_supported(ss);
+  C.sl_part = take(via_slice ? tc_slice_partials_bytes(ss) : 0);
+  C.sl_prep = take(via_slice ? tc_slice_prep_bytes(ss) : 0);
+  C.sl_wsum = take(via_slice ? (size_t)s.BH() * s0.G * sizeof(float) : 0);
   C.total = off;
   return C;
 }
@@ -1117,8 +1125,13 @@ cudaError_t run_coupling_bwd(const Shape& s0, const void* x, const void* f, cons
   if (!make_maps(s, x, dout, ws + L.px, ws + L.dpx, &xmap, &vmap, &pmap, &dmap) ||
       !make_point_map(&fmap, f, s, kD, CU_TENSOR_MAP_SWIZZLE_64B))
     return cudaErrorInvalidValue;
-  // 2. d z' (the W image of the last range is in place)
-  {
+  // 2. d z'
+  const Shape ssl = split_shape(s0);
+  if (tc_forward_supported(ssl)) {
+    if ((e = tc_slice_fwd_lse(ssl, x, dout, W, bias, tau, lse, dzp, reinterpret_cast<float*>(ws + C.sl_wsum), 0,
+                              reinterpret_cast<float*>(ws + C.sl_part), ws + C.sl_prep, status, st)) != cudaSuccess)
+      return e;
+  } else {  // the slot pass in mode 0 (the W image of the last range is in place)
     const size_t sm = smem_bwd_slot(0);
     const auto kernel = k_bwd_slot_tc<0, true>;
     if ((e = set_smem(kernel, sm)) != cudaSuccess) return e;
@@ -1281,7 +1294,8 @@ int tc_coupling_bwd_launch_count(const Shape& s) {
   // backward (2) and the dU | dS prologue; per range the slice rows pass with its
   // images (4); delta's rows; per range the combined slot pass with its images and
   // reductions (6); per point-pass range its images and the pass (5)
-  return 1 + 4 * n + n * (2 + r) + 3 + 4 * n + 1 + 6 * n + 5 * cr.n;
+  const int dz = tc_forward_supported(split_shape(s)) ? 4 /*prep_w, prep_px, slice, reduce*/ : n * (2 + r);
+  return 1 + 4 * n + dz + 3 + 4 * n + 1 + 6 * n + 5 * cr.n;
 }
 
 cudaError_t tc_coupling_bwd(const Shape& s0, const void* x, const void* f, const void* dout, const float* W,
