@@ -3,7 +3,7 @@ against the fp64 oracle, and against the three separate calls (fs_deslice_bwd,
 fs_mix_bwd, fs_slice_bwd).  On the tensor-core backward its single point pass
 forms dx from the sum of both calls' da; it runs over slot ranges of at most 256
 (G = 384 as three of 128, G = 512 as two of 256, G = 1024 as four of 256 beside
-the other passes' two of 512).  Tolerances as in tests/_parity.py: bf16 inputs
+the other passes' two of 512), on shapes with one and with many point tiles per CTA.  Tolerances as in tests/_parity.py: bf16 inputs
 relative L2 <= 1e-2, fp32 inputs normwise max relative <= 1e-4."""
 import numpy as np
 import pytest
@@ -23,6 +23,9 @@ SHAPES = [
     (2, 777, 1, 32, 384, "bf16", "bf16x2"),
     (1, 2049, 2, 32, 512, "bf16", "bf16x2"),
     (1, 1500, 1, 32, 1024, "bf16", "bf16x2"),
+    # many point tiles per CTA (the passes' pipelines wrap around their buffers)
+    (1, 20000, 8, 32, 256, "bf16", "bf16x2"),
+    (2, 9000, 4, 32, 512, "bf16", "bf16x2"),
     (1, 900, 2, 32, 48, "f32", "bf16"),
     (1, 500, 2, 16, 40, "bf16", "bf16"),
 ]
