@@ -13,8 +13,8 @@
 //   slot  (slot-owned, split over points): dW, dbias, dtau (and d z') partials;
 //   point (point-owned): dx.
 // dw - delta is one more MMA chain of the logits' shape: the slot side carries
-// [t_g | c_g halves, 1, 1] (the T image, laid out as the W image) and the point
-// side [v_n | 1, 1, -delta_n halves] (delta's point-extra rows).
+// [t_g | c_g halves, 1, 1, 1] (the T image, laid out as the W image) and the point
+// side [v_n | 1, 1, -delta_n in three bf16 parts] (delta's point-extra rows).
 #include "fs_tc_common.cuh"
 
 namespace fs {
@@ -31,7 +31,8 @@ constexpr uint32_t kWBlockB = kGC * kWRow;             // one 128-slot block of 
 // ---- prep kernels ------------------------------------------------------------------------------
 
 // T image of (b,h), in the W image's layout (kWRow bytes per slot): t_g rounded to
-// bf16, the extra rows [c_hi, c_lo, 1, 1, 0...], the residual t_g - bf16(t_g).
+// bf16, the extra rows [c_hi, c_lo, 1, 1, 1, 0...] (k = 2..4 meet -delta's three
+// parts), the residual t_g - bf16(t_g).
 // t: [BH][G][tstride] fp32, c_g = t[..][32] when has_c.  Also writes c_g to c_out
 // [BH][Gp].  Padding slots [G, Gp) get t = 0 and c = 0 (their weights are 0).
 __global__ void k_prep_t(const float* __restrict__ t, int tstride, int has_c, uint8_t* __restrict__ img,
@@ -57,7 +58,7 @@ __global__ void k_prep_t(const float* __restrict__ t, int tstride, int has_c, ui
   const __nv_bfloat16 clo = __float2bfloat16_rn(c - __bfloat162float(chi));
   __nv_bfloat16* ep = reinterpret_cast<__nv_bfloat16*>(base + (size_t)Gp * 64);
   for (int k = 0; k < 16; k++)
-    ep[off_sw32(g, k) / 2] = k == 0 ? chi : (k == 1 ? clo : __float2bfloat16_rn((k == 2 || k == 3) ? 1.f : 0.f));
+    ep[off_sw32(g, k) / 2] = k == 0 ? chi : (k == 1 ? clo : __float2bfloat16_rn((k >= 2 && k <= 4) ? 1.f : 0.f));
 }
 
 // W'^T image of head h in the Z layout (channel rows, slots along K), W' =
@@ -83,7 +84,7 @@ __global__ void k_prep_wt(const float* __restrict__ W, const float* __restrict__
   lp[off_z(c, g) / 2] = __float2bfloat16_rn(v - __bfloat162float(hi));
 }
 
-// delta's point-extra rows [1, 1, -delta_hi, -delta_lo, 0, 0, 0, 0] into dpx [BH, Np, 8];
+// delta's point-extra rows [1, 1, -delta in three bf16 parts, 0, 0, 0] into dpx [BH, Np, 8];
 // delta_n = delta[bh][n] (+ delta2[bh][n] when given, + wds[0][bh][n] + wds[1][bh][n]
 // when wds is given).
 __global__ void k_prep_dpx(const float* __restrict__ delta, const float* __restrict__ delta2,
@@ -97,10 +98,7 @@ __global__ void k_prep_dpx(const float* __restrict__ delta, const float* __restr
     if (delta2) d += delta2[bh * N + n];
     if (wds) d += wds[bh * N + n] + wds[(BH + bh) * N + n];
   }
-  const __nv_bfloat16 hi = __float2bfloat16_rn(-d);
-  const __nv_bfloat16 lo = __float2bfloat16_rn(-d - __bfloat162float(hi));
-  dpx[i] = make_uint4(0x3F803F80u, (uint32_t)__bfloat16_as_ushort(hi) | ((uint32_t)__bfloat16_as_ushort(lo) << 16),
-                      0u, 0u);
+  dpx[i] = extra_row3(-d);
 }
 
 // ---- device pieces -----------------------------------------------------------------------------

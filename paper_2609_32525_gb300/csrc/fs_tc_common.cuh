@@ -89,14 +89,14 @@ __global__ void k_prep_w(const float* __restrict__ W, const float* __restrict__ 
     *reinterpret_cast<uint4*>(base + (size_t)Gp * 96 + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
     return;
   }
-  // The extra row [b'_hi, b'_lo, 1, 1, 0 ...]; k = 2, 3 multiply the point side's
-  // -lse2 halves (zero in the statistics pass).
+  // The extra row [b'_hi, b'_lo, 1, 1, 1, 0 ...]; k = 2, 3, 4 multiply the three bf16
+  // parts of the point side's -lse2 (zero in the statistics pass).
   const float b2 = real ? bias[(int64_t)h * G + g] * scale : -1e30f;
   const uint32_t bp = pack_bf16(b2, 0.f) & 0xFFFFu;
   const float bhi = __uint_as_float(bp << 16);
   const uint32_t blo = pack_bf16(b2 - bhi, 0.f) & 0xFFFFu;
   uint8_t* ep = base + (size_t)Gp * 64;
-  *reinterpret_cast<uint4*>(ep + off_sw32(g, 0)) = make_uint4(bp | (blo << 16), 0x3F803F80u, 0u, 0u);
+  *reinterpret_cast<uint4*>(ep + off_sw32(g, 0)) = make_uint4(bp | (blo << 16), 0x3F803F80u, 0x3F80u, 0u);
   *reinterpret_cast<uint4*>(ep + off_sw32(g, 8)) = make_uint4(0u, 0u, 0u, 0u);
 }
 
@@ -420,17 +420,28 @@ __device__ __forceinline__ void weights_hilo_in_place_ds(uint32_t tS, const floa
   tmem_st16(tS + 112, lo1);
 }
 
-// Point-extra rows [1, 1, -lse2_hi, -lse2_lo, 0, 0, 0, 0] (bf16) from lse [B,H,N]
-// (natural log) into px [B*H, Np, 8]; padded points (n >= N) get -1e30 so that
-// their weights vanish.
+// A point-extra row [1, 1, -v_1, -v_2, -v_3, 0, 0, 0] (bf16): v = v_1 + v_2 + v_3 in
+// three bf16 parts, which hold v's 24 significant bits, so that the row adds -v to
+// fp32 precision against a slot side [.., .., 1, 1, 1, 0 ...].  (Two parts would
+// leave an error of ~2^-17 |v|: as -lse2, a per-point error of the weights'
+// normalisation, which the softmax backward's cancellation amplifies in dtau.)
+__device__ __forceinline__ uint4 extra_row3(float nv) {
+  const __nv_bfloat16 p1 = __float2bfloat16_rn(nv);
+  const float r1 = nv - __bfloat162float(p1);
+  const __nv_bfloat16 p2 = __float2bfloat16_rn(r1);
+  const __nv_bfloat16 p3 = __float2bfloat16_rn(r1 - __bfloat162float(p2));
+  return make_uint4(0x3F803F80u, (uint32_t)__bfloat16_as_ushort(p1) | ((uint32_t)__bfloat16_as_ushort(p2) << 16),
+                    (uint32_t)__bfloat16_as_ushort(p3), 0u);
+}
+
+// Point-extra rows [1, 1, -lse2 in three parts, 0, 0, 0] from lse [B,H,N] (natural
+// log) into px [B*H, Np, 8]; padded points (n >= N) get -1e30 so that their weights
+// vanish.
 __global__ void k_prep_px(const float* __restrict__ lse, uint4* __restrict__ px, int64_t BH, int64_t N, int64_t Np) {
   const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= BH * Np) return;
   const int64_t bh = i / Np, n = i % Np;
-  const float nl2 = n < N ? -lse[bh * N + n] * kLog2e : -1e30f;
-  const __nv_bfloat16 hi = __float2bfloat16_rn(nl2);
-  const __nv_bfloat16 lo = __float2bfloat16_rn(nl2 - __bfloat162float(hi));
-  px[i] = make_uint4(0x3F803F80u, (uint32_t)__bfloat16_as_ushort(hi) | ((uint32_t)__bfloat16_as_ushort(lo) << 16), 0u, 0u);
+  px[i] = extra_row3(n < N ? -lse[bh * N + n] * kLog2e : -1e30f);
 }
 
 // ---- host side -------------------------------------------------------------------------------

@@ -15,13 +15,13 @@
 //
 // Logits.  A 128-point x 128-slot block of base-2 logits a2 = a * log2(e) is one
 // tcgen05.mma chain with K = 48:
-//   point side [ x (32 bf16) | 1, 1, -lse2_hi, -lse2_lo, 0 ... ]  (stats: 1, 1, 0 ...)
-//   slot side  [ W*log2e/tau (32) | b'_hi, b'_lo, 1, 1, 0 ... ]  (b' = bias*log2e/tau in
-//                                                           two bf16 halves)
+//   point side [ x (32 bf16) | 1, 1, -lse2 (three bf16 parts), 0 ... ]  (stats: 1, 1, 0 ...)
+//   slot side  [ W*log2e/tau (32) | b'_hi, b'_lo, 1, 1, 1, 0 ... ]  (b' = bias*log2e/tau
+//                                                                 in two bf16 halves)
 // The point-major passes (stats, deslice) put points on the MMA's M (TMEM lane
 // = point); the slice swaps the operands, so its TMEM lane is a slot and its
 // column a point.  In the slice and the deslice the point side's extra block is
-// [1, 1, -lse2_hi, -lse2_lo, 0 ...], so the accumulator holds a2 - lse2, the
+// [1, 1, -lse2 in three parts, 0 ...], so the accumulator holds a2 - lse2, the
 // log2 of the slice weight itself.  The stats pass writes these 16-byte rows per
 // point to memory and the later passes load them by TMA with each tile: no
 // thread writes a tensor-core operand per tile (that would cost a generic ->
@@ -374,7 +374,7 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
 
 // =========================================================================================
 // Statistics: lse_n = log sum_g exp(a_ng) (natural log) to lse[bh*N + n], and
-// the point-extra row [1, 1, -lse2_hi, -lse2_lo, 0 x 4] (lse2 = lse*log2(e)) to
+// the point-extra row [1, 1, -lse2 in three bf16 parts, 0 x 3] (lse2 = lse*log2(e)) to
 // px[bh*Np + n] (Np = N rounded up to a whole tile; padded points get -1e30 so
 // that their weights vanish).
 // Two logits issuers and four softmax warpgroups (640 threads): block q (tile
@@ -578,12 +578,7 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
         const int64_t n = (wk.tile0 + i) * kTile + r;
         const float lse2 = M + log2f(L);
         if (n < Np) {
-          const float nl2 = n < N ? -lse2 : -1e30f;
-          const __nv_bfloat16 hi = __float2bfloat16_rn(nl2);
-          const __nv_bfloat16 lo = __float2bfloat16_rn(nl2 - __bfloat162float(hi));
-          px[wk.bh * Np + n] =
-              make_uint4(0x3F803F80u, (uint32_t)__bfloat16_as_ushort(hi) | ((uint32_t)__bfloat16_as_ushort(lo) << 16),
-                         0u, 0u);
+          px[wk.bh * Np + n] = extra_row3(n < N ? -lse2 : -1e30f);
           if (n < N) lse[wk.bh * N + n] = lse2 * kLn2;
         }
       }
