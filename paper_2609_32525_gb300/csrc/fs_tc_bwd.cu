@@ -211,6 +211,12 @@ __device__ __forceinline__ void w_unit(uint32_t tL) {
   }
 }
 
+// The slot pass's accumulators are flushed into registers every kSlotFlush of an
+// issuer's units (64 points each), for the reason the slice's are: the tensor cores'
+// fp32 accumulation drifts towards zero over a long chain of K steps.
+constexpr int kSlotFlush = 8;
+__device__ __forceinline__ bool slot_flush_at(int u) { return ((u >> 1) % kSlotFlush) == 0; }
+
 // =========================================================================================
 // Slot pass: CTA (slot block, point split p, bh) owns 128 slots.  Unit u is half
 // u & 1 (64 points) of point tile u >> 1.  Per unit, warp 1 forms, transposed
@@ -261,7 +267,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* p_ready = s_full + kSBuf;  // [issuer][set]
   uint64_t* pv_done = p_ready + 2 * kSBuf;
   uint64_t* acc_full = pv_done + kSBuf;
-  uint64_t* drain = acc_full + 1;
+  uint64_t* acc_done = acc_full + 1;  // [issuer]: products of each of its units complete
+  uint64_t* drain = acc_done + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 3);
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
 
@@ -270,7 +277,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int64_t b = wk.bh / H;
   const int h = (int)(wk.bh % H);
   const int units = 2 * wk.ntiles;
+  // Accumulator flushes (as in the slice): issuer j's chain restarts every
+  // kSlotFlush of its units after warpgroup j has added the accumulator into
+  // registers.  MODE 1 keeps two accumulators per issuer (dW, dZ) and no flushes.
+  constexpr bool kFl = MODE != 1;
   constexpr uint32_t kAccW = kSBuf * kGC, kAccZ = kAccW + 64;
+  constexpr uint32_t kAccF = MODE == 0 ? kAccZ : kAccW;  // the flushed accumulator
   constexpr uint32_t kVOff = kXBytes, kPOff = 2 * kXBytes, kDOff = 2 * kXBytes + kPxBytes;
 
   if (threadIdx.x == 0) {
@@ -286,6 +298,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&pv_done[i], 1);
     }
     mbar_init(acc_full, 2);
+    mbar_init(&acc_done[0], 1);
+    mbar_init(&acc_done[1], 1);
     for (int i = 0; i < 3; i++) mbar_init(&drain[i], 1);
     ab->flag = 0;
     fence_mbar_init();
@@ -384,7 +398,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int kk = 0; kk < 4; kk++) {
         // 16 points: two 8-row groups of the 64B-swizzled tile (MN-major: channels contiguous).
         const uint64_t xd = sdesc(st + (uint32_t)kk * 1024, 4096, 512, kSw64);
-        const uint32_t acc = (u >= 2 || kk > 0) ? 1u : 0u;
+        const bool fresh = u < 2 || (kFl && slot_flush_at(u));
+        const uint32_t acc = (!fresh || kk > 0) ? 1u : 0u;
         if (MODE == 0) {  // the weights are in the L columns: dZ += w^T dO
           const uint64_t vd = sdesc(st + kVOff + (uint32_t)kk * 1024, 4096, 512, kSw64);
           mma_ts_w(tmem + kAccZ + (uint32_t)j * 32, tL + da_col(kk), vd, idesc, acc);
@@ -401,6 +416,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       mma_commit_w(&pv_done[bb]);
       mma_commit_w(&st_empty[s]);
+      if (kFl) mma_commit_w(&acc_done[j]);
     }
     if (ok) mma_commit_w(acc_full);
     mma_commit_w(&drain[1 + j]);
@@ -413,6 +429,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     bool ok = true;
     float dt = 0.f, db = 0.f;
+    float acc[kD];  // this warpgroup's flushed share of dWx (MODE 0: dZ)
+#pragma unroll
+    for (int k = 0; k < kD; k++) acc[k] = 0.f;
+    auto add_acc = [&]() {
+      uint32_t a[32];
+      tmem_ld32(tmem + lane_addr + kAccF + (uint32_t)wg * 32, a);
+      tmem_wait_ld(a);
+#pragma unroll
+      for (int k = 0; k < kD; k++) acc[k] += __uint_as_float(a[k]);
+    };
     for (int u = wg; ok && u < units; u += 2) {
       const int bb = u % kSBuf;
       if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((u / kSBuf) & 1), ab, status))) break;
@@ -427,20 +453,87 @@ __global__ void __launch_bounds__(kThreads, 1)
         db += sb;
       }
       tmem_wait_st();
+      if (kFl && u >= 2 && slot_flush_at(u)) {
+        // This warpgroup's units up to u - 2 have completed their products.
+        if (!(ok = mbar_wait(&acc_done[wg], (uint32_t)(((u - 2) >> 1) & 1), ab, status))) break;
+        tc_fence_after();
+        add_acc();
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_ready[wg * kSBuf + bb]);
     }
-    // Epilogue: warpgroup 1 hands its sums to warpgroup 0, which writes dWx and the
-    // sums; warpgroup 1 writes dZ (MODE 1; MODE 0 writes dZ alone).
+    // Epilogue.  Warpgroup 1 hands its sums dt, db to warpgroup 0 through shared
+    // memory.  Flushed modes: each warpgroup adds what its accumulator holds since
+    // its last flush; warpgroup 1 passes its share through the partial row and
+    // warpgroup 0 adds the two in a fixed order (MODE 0: dZ; MODES 2, 3: dWx and the
+    // sums).  MODE 1: warpgroup 0 writes dWx (both accumulators) and the sums,
+    // warpgroup 1 dZ.
     const int64_t BH = gridDim.z;
     const int PS = MODE == 1 ? 2 * kD + 2 : (MODE == 0 ? kD : kD + 2);
     float* o = part + (((int64_t)blockIdx.y * BH + wk.bh) * G + g_base + r) * PS;
-    if (MODE == 0) {
-      const bool have0 = ok && wk.ntiles > 0 && mbar_wait(acc_full, 0, ab, status);
-      if (have0) tc_fence_after();
+    const bool have = ok && wk.ntiles > 0 && mbar_wait(acc_full, 0, ab, status);
+    if (have) tc_fence_after();
+    if (kFl) {
+      if (have) add_acc();
       if (wg == 1) {
-        if (have0) {
+#pragma unroll
+        for (int k = 0; k < kD; k++) o[k] = acc[k];
+        if (MODE != 0) {
+          s_red[r] = dt;
+          s_red[kGC + r] = db;
+        }
+      }
+      named_barrier(1, 256);
+      if (wg == 0) {
+#pragma unroll
+        for (int k = 0; k < kD; k++) o[k] = acc[k] + o[k];
+        if (MODE != 0) {
+          dt += s_red[r];
+          db += s_red[kGC + r];
+          o[kD] = db;
+          o[kD + 1] = 0.f;
+          s_red[2 * kGC + r] = dt;
+          named_barrier(2, 128);
+          if (r == 0) {
+            float sum = 0.f;
+            for (int k = 0; k < kGC; k++) sum += s_red[2 * kGC + k];
+            dt_part[wk.bh * ((int64_t)gridDim.x * gridDim.y) + (int64_t)blockIdx.y * gridDim.x + blockIdx.x] =
+                sum * kLn2;
+          }
+        }
+      }
+    } else {
+      if (wg == 1) {
+        s_red[r] = dt;
+        s_red[kGC + r] = db;
+      }
+      named_barrier(1, 256);
+      if (wg == 0) {
+        dt += s_red[r];
+        db += s_red[kGC + r];
+        constexpr int off = kD;
+        if (have) {
+          uint32_t a0[32], a1[32];
+          tmem_ld32(tmem + lane_addr + kAccW, a0);
+          tmem_ld32(tmem + lane_addr + kAccW + 32, a1);
+          tmem_wait_ld2(a0, a1);
+#pragma unroll
+          for (int k = 0; k < kD; k++) o[off + k] = __uint_as_float(a0[k]) + __uint_as_float(a1[k]);
+        } else {
+          for (int k = 0; k < kD; k++) o[off + k] = 0.f;
+        }
+        o[off + kD] = db;
+        o[off + kD + 1] = 0.f;
+        s_red[2 * kGC + r] = dt;
+        named_barrier(2, 128);
+        if (r == 0) {
+          float sum = 0.f;
+          for (int k = 0; k < kGC; k++) sum += s_red[2 * kGC + k];
+          dt_part[wk.bh * ((int64_t)gridDim.x * gridDim.y) + (int64_t)blockIdx.y * gridDim.x + blockIdx.x] = sum * kLn2;
+        }
+      } else {
+        if (have) {
           uint32_t z0[32], z1[32];
           tmem_ld32(tmem + lane_addr + kAccZ, z0);
           tmem_ld32(tmem + lane_addr + kAccZ + 32, z1);
@@ -451,49 +544,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int k = 0; k < kD; k++) o[k] = 0.f;
         }
       }
-    } else {
-    if (wg == 1) {
-      s_red[r] = dt;
-      s_red[kGC + r] = db;
-    }
-    named_barrier(1, 256);
-    const bool have = ok && wk.ntiles > 0 && mbar_wait(acc_full, 0, ab, status);
-    if (have) tc_fence_after();
-    if (wg == 0) {
-      dt += s_red[r];
-      db += s_red[kGC + r];
-      const int off = MODE == 1 ? kD : 0;
-      if (have) {
-        uint32_t a0[32], a1[32];
-        tmem_ld32(tmem + lane_addr + kAccW, a0);
-        tmem_ld32(tmem + lane_addr + kAccW + 32, a1);
-        tmem_wait_ld2(a0, a1);
-#pragma unroll
-        for (int k = 0; k < kD; k++) o[off + k] = __uint_as_float(a0[k]) + __uint_as_float(a1[k]);
-      } else {
-        for (int k = 0; k < kD; k++) o[off + k] = 0.f;
-      }
-      o[off + kD] = db;
-      o[off + kD + 1] = 0.f;
-      s_red[2 * kGC + r] = dt;
-      named_barrier(2, 128);
-      if (r == 0) {
-        float sum = 0.f;
-        for (int k = 0; k < kGC; k++) sum += s_red[2 * kGC + k];
-        dt_part[wk.bh * ((int64_t)gridDim.x * gridDim.y) + (int64_t)blockIdx.y * gridDim.x + blockIdx.x] = sum * kLn2;
-      }
-    } else if (MODE == 1) {
-      if (have) {
-        uint32_t z0[32], z1[32];
-        tmem_ld32(tmem + lane_addr + kAccZ, z0);
-        tmem_ld32(tmem + lane_addr + kAccZ + 32, z1);
-        tmem_wait_ld2(z0, z1);
-#pragma unroll
-        for (int k = 0; k < kD; k++) o[k] = __uint_as_float(z0[k]) + __uint_as_float(z1[k]);
-      } else {
-        for (int k = 0; k < kD; k++) o[k] = 0.f;
-      }
-    }
     }
   }
   tc_fence_before();

@@ -337,6 +337,24 @@ __device__ __forceinline__ void weights_half(uint32_t tS) {
   tmem_st16(tS + 16, pk1);
 }
 
+// One 64-column half with split products: the log2-weights in columns [0, 64) from tS
+// -> the bf16 weights packed in pairs into columns [0, 32) and the bf16 pairs of
+// their residuals into [32, 64).  The whole half is in registers before the first
+// store, so the stores may land on columns not yet converted.
+__device__ __forceinline__ void weights_hilo_half(uint32_t tS) {
+  uint32_t v0[32], v1[32];
+  tmem_ld32(tS, v0);
+  tmem_ld32(tS + 32, v1);
+  tmem_wait_ld2(v0, v1);
+  uint32_t hi[16], lo[16];
+  weights32_hilo(v0, hi, lo);
+  tmem_st16(tS, hi);
+  tmem_st16(tS + 32, lo);
+  weights32_hilo(v1, hi, lo);
+  tmem_st16(tS + 16, hi);
+  tmem_st16(tS + 48, lo);
+}
+
 // The weight helpers above, plus acc += sum over the block's 128 slots of w_g ds[g]
 // (ds: the block's slice of a per-slot array in shared memory; every lane reads
 // the same address, a broadcast).  The backward of the slice needs this sum for

@@ -610,6 +610,20 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
 constexpr uint32_t kStageBytes = kXBytes + 3 * kFBlock + 2 * kPxBytes;  // x, [F | 1], point extra
 constexpr uint32_t kWBlock = 128 * kWRow;                               // one 128-slot block of the W image
 
+// Flushes.  The tensor cores' fp32 accumulation over a CTA's long point range (a
+// thousand and more K steps into one accumulator) loses ~2^-25 of the running sum per
+// step, always towards zero: at 27,600 points 4e-5 relative, and the temperature
+// gradient magnifies errors of the token gradients many times over (its sum over
+// (n, g) cancels to ~1e-5 of its terms' magnitude).  So each accumulator's chain is
+// restarted every kSliceFlush of its issuer's tiles, after its warpgroup has added
+// what it holds into fp32 registers (round to nearest).  Only with split products
+// and fp32 inputs: with single bf16 products the weights' own rounding (~3e-3
+// relative in the tokens) dwarfs the drift (~1e-4 at 55,000 points per CTA), and
+// the waits on each flushed chain cost the plain slice 4%.
+constexpr int kSliceFlush = 4;
+template <bool kOn>
+__device__ __forceinline__ bool slice_flush_at(int i) { return kOn && ((i >> 1) % kSliceFlush) == 0; }
+
 // X3 (fp32 inputs): each stage also holds the residual tiles of x and fx (xrmap,
 // frmap); the logits add x_r W'_hi and the products add P_hi F_r (N = 32: U only).
 // Its stages are larger, so there are half as many.
@@ -640,7 +654,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* p_ready = s_full + kSBuf;   // [issuer][S buffer]
   uint64_t* pv_done = p_ready + 2 * kSBuf;
   uint64_t* acc_full = pv_done + kSBuf;
-  uint64_t* drain = acc_full + 1;  // one per issuing warp
+  uint64_t* acc_done = acc_full + 1;  // [issuer]: products of each of its tiles complete
+  uint64_t* drain = acc_done + 2;  // one per issuing warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 3);
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
 
@@ -664,6 +679,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&pv_done[i], 1);
     }
     mbar_init(acc_full, 2);
+    mbar_init(&acc_done[0], 1);
+    mbar_init(&acc_done[1], 1);
     for (int i = 0; i < 3; i++) mbar_init(&drain[i], 1);
     ab->flag = 0;
     fence_mbar_init();
@@ -759,18 +776,25 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t tE = tmem + (uint32_t)bb * kGC;  // packed weights of the 128 points
         const uint32_t fs = smem_u32(s_st + s * kStB) + kFOff;
         const uint32_t tacc = tmem + kA + (uint32_t)j * 48;
+        // A chain restarts at this issuer's first tile and at every flush tile (its
+        // warpgroup has moved the earlier tiles' sums to registers by then).
+        const bool fresh = i < 2 || slice_flush_at<split || X3>(i);
 #pragma unroll
         for (int kk = 0; kk < 8; kk++) {
           const uint64_t fdesc = sdesc(fs + (uint32_t)kk * 512, kFBlock, 256, kSw32);
-          mma_ts_w(tacc, tE + (uint32_t)kk * 8, fdesc, idesc_sl, (i >= 2 || kk > 0) ? 1u : 0u);
+          // 16 points' packed weights: columns kk * 8, or with split products the hi
+          // pairs of half kk / 4 at (kk / 4) * 64 + (kk % 4) * 8, their residuals 32 on
+          const uint32_t tw = tE + (split ? (uint32_t)(kk >> 2) * 64 + (uint32_t)(kk & 3) * 8 : (uint32_t)kk * 8);
+          mma_ts_w(tacc, tw, fdesc, idesc_sl, (!fresh || kk > 0) ? 1u : 0u);
           // The residual halves of the weights: U and S to ~2^-16.
-          if (split) mma_ts_w(tacc, tE + 64 + (uint32_t)kk * 8, fdesc, idesc_sl, 1u);
+          if (split) mma_ts_w(tacc, tw + 32, fdesc, idesc_sl, 1u);
           if (X3)  // the weights against fx's residual half (U only)
-            mma_ts_w(tacc, tE + (uint32_t)kk * 8, sdesc(fs - kFOff + kFROff + (uint32_t)kk * 512, kFBlock, 256, kSw32),
+            mma_ts_w(tacc, tw, sdesc(fs - kFOff + kFROff + (uint32_t)kk * 512, kFBlock, 256, kSw32),
                      idesc_bf16(128, 32, false, true), 1u);
         }
         mma_commit_w(&pv_done[bb]);
         mma_commit_w(&st_empty[s]);
+        if (split || X3) mma_commit_w(&acc_done[j]);
       }
       if (ok) mma_commit_w(acc_full);
       mma_commit_w(&drain[1 + j]);
@@ -782,25 +806,62 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = wq * 32 + lane;  // TMEM lane: slot g_base + r
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     bool ok = true;
+    // This warpgroup's share of (U, S) for slot r, moved out of A_wg at every flush.
+    float acc[kD + 1];
+#pragma unroll
+    for (int k = 0; k <= kD; k++) acc[k] = 0.f;
+    const uint32_t tA = tmem + lane_addr + kA + (uint32_t)wg * 48;
+    auto add_acc = [&]() {
+      uint32_t u[32], sv[16];
+      tmem_ld32(tA, u);
+      tmem_ld16(tA + 32, sv);
+      tmem_wait_ld(u, sv);
+#pragma unroll
+      for (int k = 0; k < kD; k++) acc[k] += __uint_as_float(u[k]);
+      acc[kD] += __uint_as_float(sv[0]);
+    };
     // Warpgroup wg takes the whole tiles i with i % 2 == wg (out of phase with the other).
     for (int i = wg; ok && i < wk.ntiles; i += 2) {
       const int bb = i % kSBuf;
       if (!(ok = mbar_wait(&s_full[bb], (uint32_t)((i / kSBuf) & 1), ab, status))) break;
       tc_fence_after();
-      if (split)
-        weights_hilo_in_place(tmem + lane_addr + (uint32_t)bb * kGC);
-      else
+      if (split) {
+        weights_hilo_half(tmem + lane_addr + (uint32_t)bb * kGC);
+        weights_hilo_half(tmem + lane_addr + (uint32_t)bb * kGC + 64);
+      } else {
         weights_in_halves(tmem + lane_addr + (uint32_t)bb * kGC);
+      }
       tmem_wait_st();
+      if (i >= 2 && slice_flush_at<split || X3>(i)) {
+        // The products of this warpgroup's tiles up to i - 2 are complete (acc_done
+        // cannot move past that phase before this warpgroup hands over tile i).
+        if (!(ok = mbar_wait(&acc_done[wg], (uint32_t)(((i - 2) >> 1) & 1), ab, status))) break;
+        tc_fence_after();
+        add_acc();
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&p_ready[wg * kSBuf + bb]);
     }
-    // Epilogue: the accumulators of this CTA's slot block -> partials
-    // (warpgroup 0 the numerators U, warpgroup 1 the weight sums S).
     const int64_t BH = gridDim.z;
     float* o = part + (((int64_t)blockIdx.y * BH + wk.bh) * G + g_base + r) * (kD + 1);
-    if (ok && wk.ntiles > 0 && mbar_wait(acc_full, 0, ab, status)) {
+    const bool have = ok && wk.ntiles > 0 && mbar_wait(acc_full, 0, ab, status);
+    if (split || X3) {
+      // Epilogue with flushes: what A_wg holds since the last flush, then the two
+      // warpgroups' shares added in a fixed order (warpgroup 1 passes its share
+      // through the partial row).
+      if (have && wg < wk.ntiles) {
+        tc_fence_after();
+        add_acc();
+      }
+      if (wg == 1)
+        for (int k = 0; k <= kD; k++) o[k] = acc[k];
+      named_barrier(1, 256);
+      if (wg == 0)
+        for (int k = 0; k <= kD; k++) o[k] = acc[k] + o[k];
+    } else if (have) {
+      // Without flushes: warpgroup 0 writes the numerators U (A_0 + A_1), warpgroup 1
+      // the weight sums S.
       tc_fence_after();
       const bool two = wk.ntiles >= 2;  // A_1 holds tiles only when there are two (else unwritten)
       if (wg == 0) {
