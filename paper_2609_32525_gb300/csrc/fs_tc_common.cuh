@@ -259,10 +259,6 @@ __device__ __forceinline__ void weights32(const uint32_t (&v)[32], uint32_t (&p)
   for (int k = 0; k < 16; k++) p[k] = pack_bf16(ex2(__uint_as_float(v[2 * k])), ex2(__uint_as_float(v[2 * k + 1])));
 }
 
-// The 128 log2-weights of one TMEM lane of an S buffer -> bf16 weights written back
-// in place, packed in pairs, into the first 64 columns, in two halves: columns
-// [64 h, 64 h + 64) -> packed weights in columns [32 h, 32 h + 32), which this
-// thread has already read.
 // 2^t for 32 log2-weights -> the bf16 pairs (hi) and the bf16 pairs of the
 // residuals w - hi (lo): w = hi + lo to ~2^-16 relative.
 __device__ __forceinline__ void weights32_hilo(const uint32_t (&v)[32], uint32_t (&hi)[16], uint32_t (&lo)[16]) {
@@ -276,38 +272,10 @@ __device__ __forceinline__ void weights32_hilo(const uint32_t (&v)[32], uint32_t
   }
 }
 
-// Slice weights of one TMEM lane (a slot) of an S buffer, 128 points: the hi
-// halves packed in pairs into columns [0, 64), the lo halves into [64, 128).
-// Half h reads columns [64 h, 64 h + 64); the lo pairs of half 0 wait in
-// registers until half 1 has read the columns they go to.
-__device__ __forceinline__ void weights_hilo_in_place(uint32_t tS) {
-  uint32_t lo0[16], lo1[16];
-  {
-    uint32_t v0[32], v1[32];
-    tmem_ld32(tS, v0);
-    tmem_ld32(tS + 32, v1);
-    tmem_wait_ld2(v0, v1);
-    uint32_t hi0[16], hi1[16];
-    weights32_hilo(v0, hi0, lo0);
-    weights32_hilo(v1, hi1, lo1);
-    tmem_st16(tS, hi0);
-    tmem_st16(tS + 16, hi1);
-  }
-  uint32_t v0[32], v1[32];
-  tmem_ld32(tS + 64, v0);
-  tmem_ld32(tS + 96, v1);
-  tmem_wait_ld2(v0, v1);
-  tmem_st16(tS + 64, lo0);
-  tmem_st16(tS + 80, lo1);
-  uint32_t hi0[16], hi1[16];
-  weights32_hilo(v0, hi0, lo0);
-  weights32_hilo(v1, hi1, lo1);
-  tmem_st16(tS + 32, hi0);
-  tmem_st16(tS + 48, hi1);
-  tmem_st16(tS + 96, lo0);
-  tmem_st16(tS + 112, lo1);
-}
-
+// The 128 log2-weights of one TMEM lane of an S buffer -> bf16 weights written back
+// in place, packed in pairs, into the first 64 columns, in two halves: columns
+// [64 h, 64 h + 64) -> packed weights in columns [32 h, 32 h + 32), which this
+// thread has already read.
 __device__ __forceinline__ void weights_in_halves(uint32_t tS) {
 #pragma unroll 1
   for (int half = 0; half < 2; half++) {
@@ -410,32 +378,19 @@ __device__ __forceinline__ void weights_in_halves_ds(uint32_t tS, const float* d
     tmem_st16(tS + half * 32 + 16, pk1);
   }
 }
-__device__ __forceinline__ void weights_hilo_in_place_ds(uint32_t tS, const float* ds, float& acc) {
-  uint32_t lo0[16], lo1[16];
-  {
-    uint32_t v0[32], v1[32];
-    tmem_ld32(tS, v0);
-    tmem_ld32(tS + 32, v1);
-    tmem_wait_ld2(v0, v1);
-    uint32_t hi0[16], hi1[16];
-    weights32_hilo_ds(v0, hi0, lo0, ds, acc);
-    weights32_hilo_ds(v1, hi1, lo1, ds + 32, acc);
-    tmem_st16(tS, hi0);
-    tmem_st16(tS + 16, hi1);
-  }
+// weights_hilo_half with the sum over the half's 64 slots.
+__device__ __forceinline__ void weights_hilo_half_ds(uint32_t tS, const float* ds, float& acc) {
   uint32_t v0[32], v1[32];
-  tmem_ld32(tS + 64, v0);
-  tmem_ld32(tS + 96, v1);
+  tmem_ld32(tS, v0);
+  tmem_ld32(tS + 32, v1);
   tmem_wait_ld2(v0, v1);
-  tmem_st16(tS + 64, lo0);
-  tmem_st16(tS + 80, lo1);
-  uint32_t hi0[16], hi1[16];
-  weights32_hilo_ds(v0, hi0, lo0, ds + 64, acc);
-  weights32_hilo_ds(v1, hi1, lo1, ds + 96, acc);
-  tmem_st16(tS + 32, hi0);
-  tmem_st16(tS + 48, hi1);
-  tmem_st16(tS + 96, lo0);
-  tmem_st16(tS + 112, lo1);
+  uint32_t hi[16], lo[16];
+  weights32_hilo_ds(v0, hi, lo, ds, acc);
+  tmem_st16(tS, hi);
+  tmem_st16(tS + 32, lo);
+  weights32_hilo_ds(v1, hi, lo, ds + 32, acc);
+  tmem_st16(tS + 16, hi);
+  tmem_st16(tS + 48, lo);
 }
 
 // A point-extra row [1, 1, -v_1, -v_2, -v_3, 0, 0, 0] (bf16): v = v_1 + v_2 + v_3 in

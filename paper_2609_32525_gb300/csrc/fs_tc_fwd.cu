@@ -80,6 +80,8 @@ using namespace tc;
 // the earlier ranges.
 // PS (split products): the weights and t as bf16 hi + lo halves, P t = Phi thi +
 // Plo thi + Phi tlo; the image then holds t's residual half after its bf16 half.
+// The split weights of slot half j (slots [64 j, 64 j + 64) of the block) go to
+// columns [64 j, 64 j + 64) of the S buffer: the hi pairs, then the lo pairs.
 // =========================================================================================
 constexpr uint32_t kDStage = kXBytes + 2 * kPxBytes;  // x tile, point extra (both halves)
 
@@ -227,8 +229,8 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
         if (c == 0 && i >= 2 && !(ok = mbar_wait_w(&o_free[ob], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
         if (!(ok = mbar_wait_w(&p_ready[kWG4 ? 2 * bb + j : 2 * bb], (uint32_t)((q / kSBuf) & 1), ab, status))) break;
         tc_fence_after();
-        // weights of slots 64j.. (packed pairs)
-        const uint32_t tP = tmem + (uint32_t)bb * kGC + (uint32_t)j * (kWG4 ? 64 : 32);
+        // weights of slots 64j.. (packed pairs; PS: hi pairs, then lo pairs 32 on)
+        const uint32_t tP = tmem + (uint32_t)bb * kGC + (uint32_t)j * ((kWG4 || PS) ? 64 : 32);
         const uint32_t tO = tmem + kO + (uint32_t)(j * 2 + ob) * kD;
 #pragma unroll
         for (int kk = 0; kk < 4; kk++) {
@@ -236,7 +238,7 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
           const uint32_t zaddr = sz + (uint32_t)((g0 >> 6) * 4096 + (g0 & 63) * 2);
           mma_ts_w(tO, tP + (uint32_t)kk * 8, sdesc(zaddr, 16, 1024, kSw128), idesc_pv, (c > 0 || kk > 0) ? 1u : 0u);
           if (PS) {
-            mma_ts_w(tO, tP + 64 + (uint32_t)kk * 8, sdesc(zaddr, 16, 1024, kSw128), idesc_pv, 1u);
+            mma_ts_w(tO, tP + 32 + (uint32_t)kk * 8, sdesc(zaddr, 16, 1024, kSw128), idesc_pv, 1u);
             mma_ts_w(tO, tP + (uint32_t)kk * 8, sdesc(zaddr + (uint32_t)G * 64, 16, 1024, kSw128), idesc_pv, 1u);
           }
         }
@@ -260,10 +262,15 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
       const int ob = (int)(t & 1);
       if (!mbar_wait(&o_full[ob], (uint32_t)((t >> 1) & 1), ab, status)) return false;
       tc_fence_after();
-      uint32_t o0[32], o1[32];
-      tmem_ld32(tmem + lane_addr + kO + (uint32_t)ob * kD, o0);
-      tmem_ld32(tmem + lane_addr + kO + (uint32_t)(2 + ob) * kD, o1);
-      tmem_wait_ld2(o0, o1);
+      float R[kD];  // O_0 + O_1, in that order
+      {
+        uint32_t o0[32], o1[32];
+        tmem_ld32(tmem + lane_addr + kO + (uint32_t)ob * kD, o0);
+        tmem_ld32(tmem + lane_addr + kO + (uint32_t)(2 + ob) * kD, o1);
+        tmem_wait_ld2(o0, o1);
+#pragma unroll
+        for (int k = 0; k < kD; k++) R[k] = __uint_as_float(o0[k]) + __uint_as_float(o1[k]);
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&o_free[ob]);
@@ -276,10 +283,7 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
 #pragma unroll
           for (int k = 0; k < 8; k++) {
             const float4 p = accumulate ? dst[k] : make_float4(0.f, 0.f, 0.f, 0.f);
-            dst[k] = make_float4(p.x + (__uint_as_float(o0[4 * k]) + __uint_as_float(o1[4 * k])),
-                                 p.y + (__uint_as_float(o0[4 * k + 1]) + __uint_as_float(o1[4 * k + 1])),
-                                 p.z + (__uint_as_float(o0[4 * k + 2]) + __uint_as_float(o1[4 * k + 2])),
-                                 p.w + (__uint_as_float(o0[4 * k + 3]) + __uint_as_float(o1[4 * k + 3])));
+            dst[k] = make_float4(p.x + R[4 * k], p.y + R[4 * k + 1], p.z + R[4 * k + 2], p.w + R[4 * k + 3]);
           }
         } else if (MODE != 1) {
           uint4* dst = reinterpret_cast<uint4*>(out + row);
@@ -292,10 +296,8 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
             uint32_t w[4];
 #pragma unroll
             for (int e = 0; e < 4; e++)
-              w[e] = pack_bf16(__uint_as_float(o0[8 * k + 2 * e]) + __uint_as_float(o1[8 * k + 2 * e]) +
-                                   __uint_as_float(pw[e] << 16),
-                               __uint_as_float(o0[8 * k + 2 * e + 1]) + __uint_as_float(o1[8 * k + 2 * e + 1]) +
-                                   __uint_as_float(pw[e] & 0xFFFF0000u));
+              w[e] = pack_bf16(R[8 * k + 2 * e] + __uint_as_float(pw[e] << 16),
+                               R[8 * k + 2 * e + 1] + __uint_as_float(pw[e] & 0xFFFF0000u));
             dst[k] = make_uint4(w[0], w[1], w[2], w[3]);
           }
         }
@@ -310,9 +312,8 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
 #pragma unroll
             for (int e = 0; e < 4; e++) {
               const int c0 = 8 * k + 2 * e;
-              acc = fmaf(__uint_as_float(w[e] << 16), __uint_as_float(o0[c0]) + __uint_as_float(o1[c0]), acc);
-              acc = fmaf(__uint_as_float(w[e] & 0xFFFF0000u), __uint_as_float(o0[c0 + 1]) + __uint_as_float(o1[c0 + 1]),
-                         acc);
+              acc = fmaf(__uint_as_float(w[e] << 16), R[c0], acc);
+              acc = fmaf(__uint_as_float(w[e] & 0xFFFF0000u), R[c0 + 1], acc);
             }
           }
           delta[wk.bh * N + n] = accumulate ? delta[wk.bh * N + n] + acc : acc;
@@ -343,12 +344,14 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
           flush_wds();
           wds_tile = i;
         }
-        if (PS)
-          weights_hilo_in_place_ds(tmem + lane_addr + (uint32_t)bb * kGC, s_ds + c * kGC, wds_acc);
-        else
+        if (PS) {
+          weights_hilo_half_ds(tmem + lane_addr + (uint32_t)bb * kGC, s_ds + c * kGC, wds_acc);
+          weights_hilo_half_ds(tmem + lane_addr + (uint32_t)bb * kGC + 64, s_ds + c * kGC + 64, wds_acc);
+        } else
           weights_in_halves_ds(tmem + lane_addr + (uint32_t)bb * kGC, s_ds + c * kGC, wds_acc);
       } else if (PS) {
-        weights_hilo_in_place(tmem + lane_addr + (uint32_t)bb * kGC);
+        weights_hilo_half(tmem + lane_addr + (uint32_t)bb * kGC);
+        weights_hilo_half(tmem + lane_addr + (uint32_t)bb * kGC + 64);
       } else if (kWG4) {
         weights_half(tmem + lane_addr + (uint32_t)bb * kGC + (uint32_t)hf * 64);
       } else {
