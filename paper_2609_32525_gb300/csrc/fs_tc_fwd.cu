@@ -385,8 +385,12 @@ __global__ void __launch_bounds__(desl_wg4<MODE, PS>() ? kDesl4Threads : kThread
 // warpgroups 2p and 2p + 1, each of which takes one half (64 slots) of every row,
 // so that each SM sub-partition holds four softmax warps whose exponentials and
 // reductions interleave.  Each warpgroup keeps a running (max, sum) over the slots
-// it took; the four shares of a tile are combined through shared memory by half 0
-// of the pair that took the tile's last block.
+// it took and hands it over through shared memory after its last block of the tile.
+// With two or more blocks per tile all four warpgroups take blocks of every tile and
+// warp 3 combines their shares and writes lse and the px rows, so no softmax warp
+// waits for the others.  With one block per tile (G <= 128) the pair that takes it
+// combines in place: half 1 hands its share to half 0, which writes (at two tiles or
+// so per CTA an extra hop to warp 3 would lengthen each CTA's tail).
 // smem: [W img G*96][x stages][constant extra][ml exchange][barriers]
 // TMEM: two S buffers [0, 256).
 // =========================================================================================
@@ -406,15 +410,15 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
   uint8_t* s_w = smem;
   uint8_t* s_x = s_w + wbytes;
   uint8_t* s_ex = s_x + kStages * kXSt;
-  float2* s_ml = reinterpret_cast<float2*>(s_ex + kExBytes);  // [2 tile parities][3 partials][128 rows]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(s_ml + 6 * kTile);
+  float2* s_ml = reinterpret_cast<float2*>(s_ex + kExBytes);  // [2 tile parities][4 warpgroups][128 rows]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(s_ml + 8 * kTile);
   uint64_t* w_full = bars;
   uint64_t* x_full = bars + 1;
   uint64_t* x_empty = x_full + kStages;
   uint64_t* s_full = x_empty + kStages;
   uint64_t* s_free = s_full + 2;
-  uint64_t* ml_full = s_free + 2;   // the other three warpgroups' partials written (per tile parity)
-  uint64_t* ml_empty = ml_full + 2; // the finalising warpgroup has read them
+  uint64_t* ml_full = s_free + 2;   // the warpgroups' shares of a tile written (per tile parity)
+  uint64_t* ml_empty = ml_full + 2; // warp 3 has read them
   uint64_t* drain = ml_empty + 2;   // one per issuing warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 2);
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
@@ -434,8 +438,8 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
     for (int i = 0; i < 2; i++) {
       mbar_init(&s_full[i], 1);
       mbar_init(&s_free[i], 8);
-      mbar_init(&ml_full[i], nch >= 2 ? 12 : 4);
-      mbar_init(&ml_empty[i], 4);
+      mbar_init(&ml_full[i], nch >= 2 ? 16 : 4);
+      mbar_init(&ml_empty[i], nch >= 2 ? 1 : 4);
     }
     mbar_init(&drain[0], 1);
     mbar_init(&drain[1], 1);
@@ -495,6 +499,35 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
       mma_commit_w(&drain[j]);
       mbar_wait_w(&drain[j], 0, ab, nullptr, kWaitNs);
     }
+  } else if (warp == 3) {
+    // ------------------------------ combiner ------------------------------
+    // Tile i: the four warpgroups' shares -> lse and px rows (two or more blocks per
+    // tile).  Lane l takes the points l, l + 32, l + 64, l + 96 of the tile.
+    bool ok = nch >= 2;
+    for (int i = 0; ok && i < wk.ntiles; i++) {
+      const int pb = i & 1;
+      if (!(ok = mbar_wait(&ml_full[pb], (uint32_t)((i >> 1) & 1), ab, status))) break;
+      float2 sh[4][4];
+#pragma unroll
+      for (int k = 0; k < 4; k++)
+#pragma unroll
+        for (int w = 0; w < 4; w++) sh[k][w] = s_ml[(pb * 4 + w) * kTile + lane + 32 * k];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ml_empty[pb]);
+#pragma unroll
+      for (int k = 0; k < 4; k++) {
+        const float M = fmaxf(fmaxf(sh[k][0].x, sh[k][1].x), fmaxf(sh[k][2].x, sh[k][3].x));
+        float L = 0.f;
+#pragma unroll
+        for (int w = 0; w < 4; w++) L += sh[k][w].y * ex2(sh[k][w].x - M);
+        const int64_t n = (wk.tile0 + i) * kTile + lane + 32 * k;
+        const float lse2 = M + log2f(L);
+        if (n < Np) {
+          px[wk.bh * Np + n] = extra_row3(n < N ? -lse2 : -1e30f);
+          if (n < N) lse[wk.bh * N + n] = lse2 * kLn2;
+        }
+      }
+    }
   } else if (warp >= kSoftmaxWarp0) {
     const int wg = (warp - kSoftmaxWarp0) >> 2;
     const int pr = wg >> 1, hf = wg & 1;  // S buffer (block parity) and the half of each row
@@ -505,11 +538,9 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
     bool ok = true;
     float m = -INFINITY, l = 0.f;
     // The pair of warpgroups of S buffer pr takes the whole blocks q with q % 2 == pr,
-    // warpgroup hf the slots [64 hf, 64 hf + 64) of each.  A tile's last block is taken
-    // by the pair that finalises the tile; there half 0 finalises, and the other three
-    // warpgroups hand over their (max, sum) over the slots they took: the other pair
-    // (with two or more blocks per tile) at its last block of the tile, half 1 at the
-    // tile's last block.
+    // warpgroup hf the slots [64 hf, 64 hf + 64) of each.  A pair's last block of a
+    // tile is one of its last two (c >= nch - 2); after it the warpgroup hands its
+    // (max, sum) over the slots it took to warp 3.
     BlockPos pos(pr, nch);
     for (int q = pr; ok && q < total; q += 2, pos.step(2, nch)) {
       const int i = pos.i, c = pos.c;
@@ -554,36 +585,31 @@ __global__ void __launch_bounds__(kStatsThreads, 1)
       l = l * ex2(m - mn) + sum;
       m = mn;
       const int pb = i & 1;
-      const bool last = c == nch - 1;
-      if ((c == nch - 2) || (last && hf == 1)) {
-        // Hand over this warpgroup's share of tile i: slot hf from the other pair,
-        // slot 2 from half 1 of the finalising pair.
-        if (i >= 2 && !(ok = mbar_wait(&ml_empty[pb], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
-        s_ml[(pb * 3 + (last ? 2 : hf)) * kTile + r] = make_float2(m, l);
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&ml_full[pb]);
-        m = -INFINITY;
-        l = 0.f;
-      } else if (last) {
+      if (nch == 1 && hf == 0) {
+        // One block per tile: combine with half 1's share and write.
         if (!(ok = mbar_wait(&ml_full[pb], (uint32_t)((i >> 1) & 1), ab, status))) break;
-        const float2 o2 = s_ml[(pb * 3 + 2) * kTile + r];
-        float2 o0 = make_float2(-INFINITY, 0.f), o1 = o0;
-        if (nch >= 2) {
-          o0 = s_ml[(pb * 3 + 0) * kTile + r];
-          o1 = s_ml[(pb * 3 + 1) * kTile + r];
-        }
+        const float2 o = s_ml[(pb * 4 + wg + 1) * kTile + r];
         __syncwarp();
         if (lane == 0) mbar_arrive(&ml_empty[pb]);
-        const float M = fmaxf(fmaxf(m, o2.x), fmaxf(o0.x, o1.x));
-        const float L = l * ex2(m - M) + o2.y * ex2(o2.x - M) + o0.y * ex2(o0.x - M) + o1.y * ex2(o1.x - M);
-        m = -INFINITY;
-        l = 0.f;
+        const float M = fmaxf(m, o.x);
+        const float L = l * ex2(m - M) + o.y * ex2(o.x - M);
         const int64_t n = (wk.tile0 + i) * kTile + r;
         const float lse2 = M + log2f(L);
         if (n < Np) {
           px[wk.bh * Np + n] = extra_row3(n < N ? -lse2 : -1e30f);
           if (n < N) lse[wk.bh * N + n] = lse2 * kLn2;
         }
+        m = -INFINITY;
+        l = 0.f;
+      } else if (c >= nch - 2) {
+        // This warpgroup's last block of the tile: hand the share over (to warp 3, or
+        // with one block per tile to half 0 of the pair).
+        if (i >= 2 && !(ok = mbar_wait(&ml_empty[pb], (uint32_t)(((i >> 1) - 1) & 1), ab, status))) break;
+        s_ml[(pb * 4 + wg) * kTile + r] = make_float2(m, l);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&ml_full[pb]);
+        m = -INFINITY;
+        l = 0.f;
       }
     }
   }
@@ -930,7 +956,7 @@ size_t smem_deslice(int G, bool hilo, int mode = 0, bool ps = false, bool x3 = f
          kStages * (kDStage + (x3 ? kXBytes : 0)) + 512;
 }
 size_t smem_stats(int G, bool split, bool x3 = false) {
-  return 1024 + (size_t)G * (split ? kWRow : 96) + kStages * kXBytes * (x3 ? 2 : 1) + kExBytes + 6 * kTile * 8 + 512;
+  return 1024 + (size_t)G * (split ? kWRow : 96) + kStages * kXBytes * (x3 ? 2 : 1) + kExBytes + 8 * kTile * 8 + 512;
 }
 size_t smem_slice(bool x3 = false) {
   return 1024 + (size_t)kWBlock +

@@ -28,6 +28,17 @@ pytestmark = pytest.mark.gpu
 HEAD = 3
 FULL_ORACLE_ELEMS = 1 << 26  # B*N*H*G up to which every head is checked
 
+# Tighter bounds for the training workload's split products (FS_DOT_BF16X2), which
+# guard the accumulation itself rather than the contract: a split product carries
+# ~2^-17 of its size, and the slot-owned sums over a CTA's point range (tokens, weight
+# sums, d z', dW, dbias, and dM after them) stay within a few 2^-17 only because the
+# tensor cores' accumulators are moved into registers every few tiles (one chain over
+# the whole range drifts towards zero with its length: 3.5e-5 to 9.8e-5 here).  dtau's
+# sum over (n, g) cancels to ~1e-5 of its terms and magnifies what is left (4.8e-3
+# with one chain).
+SPLIT_SUM_BOUND = 3e-5
+SPLIT_DTAU_BOUND = 2e-3
+
 
 def _points(N, seed, k=4096):
     rng = np.random.default_rng(seed)
@@ -41,6 +52,7 @@ def _check(name, got, ref, dtype, workload=""):
     # One line per tensor (shown with pytest -s): the parity margin of each workload.
     print(f"PARITY {workload} {name} {e:.3e} tol {tol(dtype):.0e} ({'max rel' if dtype == 'f32' else 'rel L2'})")
     assert e <= tol(dtype), f"{name}: error {e:.3e} > {tol(dtype):.0e}"
+    return e
 
 
 def _gpu_run(lib, wl, dev):
@@ -81,9 +93,16 @@ def test_full_size_parity(lib, name):
     if wl.dout is None:
         return
     rb = orc.backward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, wl.dout, eps=wl.eps, heads=heads)
-    _check("d_tokens_mixed", host(c.d_tokens_mixed)[:, hs], rb["d_tokens_mixed"][:, hs], wl.dtype, name)
+    sums = {"tokens": error(host(c.tokens)[:, hs], ref["tokens"][:, hs], wl.dtype),
+            "wsum": error(host(c.wsum)[:, hs], ref["wsum"][:, hs], wl.dtype)}
+    sums["d_tokens_mixed"] = _check("d_tokens_mixed", host(c.d_tokens_mixed)[:, hs], rb["d_tokens_mixed"][:, hs],
+                                    wl.dtype, name)
     for k in ("dW", "dbias", "dM"):
-        _check(k, host(g[k])[hs], rb[k][hs], wl.dtype, name)
-    _check("dtau", host(g["dtau"])[hs], rb["dtau"][hs], wl.dtype, name)
+        sums[k] = _check(k, host(g[k])[hs], rb[k][hs], wl.dtype, name)
+    e_dtau = _check("dtau", host(g["dtau"])[hs], rb["dtau"][hs], wl.dtype, name)
     for k in ("dx_mid", "dfx"):
         _check(k, host(g[k])[:, pts][:, :, hs], rb[k][:, pts][:, :, hs], wl.dtype, name)
+    if c.shape.dot == lib.FS_DOT_BF16X2:
+        bad = {k: e for k, e in sums.items() if not e <= SPLIT_SUM_BOUND}
+        assert not bad, {k: f"{e:.3e} > {SPLIT_SUM_BOUND:.0e}" for k, e in bad.items()}
+        assert e_dtau <= SPLIT_DTAU_BOUND, f"dtau {e_dtau:.3e} > {SPLIT_DTAU_BOUND:.0e}"
