@@ -72,6 +72,8 @@ def _overrides(args):
         o["points_override"] = "N reduced for profiling; not the benchmark workload"
     if args.slots:
         o["slots_override"] = "G set to %d; not one of the named configurations" % args.slots
+    if args.dtype:
+        o["dtype_override"] = "inputs in %s; not the named configuration's dtype" % args.dtype
     return o
 
 
@@ -231,7 +233,7 @@ def run_reference(args):
     from oracle import flashslice_oracle as orc
     from paper_2609_32525_gb300.workloads import make_named
 
-    wl = make_named(args.workload)
+    wl = make_named(args.workload, n_override=args.points, g_override=args.slots, dtype_override=args.dtype)
     n = int(args.ref_points)
     train = wl.dout is not None  # the training workload: forward and backward, as its GPU line
     times = []
@@ -611,6 +613,8 @@ def main():
                          "fs_coupling_bwd")
     ap.add_argument("--slots", type=int, default=None,
                     help="the workload's recipe at another slot count G (the line says so)")
+    ap.add_argument("--dtype", default=None, choices=["bf16", "f32"],
+                    help="the workload's recipe with inputs of this dtype (the line says so)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -639,7 +643,7 @@ def main():
     from paper_2609_32525_gb300 import sharding
     from paper_2609_32525_gb300.workloads import make_named
 
-    wl = make_named(args.workload, n_override=args.points, g_override=args.slots)
+    wl = make_named(args.workload, n_override=args.points, g_override=args.slots, dtype_override=args.dtype)
     if args.shard:
         run_shard(args, wl, dev, world, rank)
         if world > 1:

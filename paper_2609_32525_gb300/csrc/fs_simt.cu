@@ -84,9 +84,12 @@ __device__ __forceinline__ int64_t row_index(int64_t b, int64_t n, int h, int64_
   return (b * N + n) * H + h;
 }
 
-// Stage GC slots of W[h] (scaled by `scale`) as sW[g][k] plus the scaled bias.
+// Stage GC slots of W[h] (scaled by `scale`) as sW[g][k] plus the scaled bias.  The
+// rows are unpadded (16-byte aligned), so that the compute loops, in which every lane
+// reads the same row, take them four floats at a time; the staging stores are then
+// bank-conflicted, which costs little against the compute on each chunk.
 template <int D, int GC>
-__device__ __forceinline__ void stage_w(float (*sW)[D + 1], float* sB, const float* W,
+__device__ __forceinline__ void stage_w(float (*sW)[D], float* sB, const float* W,
                                         const float* bias, int h, int G, int g0, float scale) {
   for (int i = threadIdx.x; i < GC * D; i += kThreads) {
     const int g = i % GC, k = i / GC;
@@ -103,7 +106,7 @@ __global__ void __launch_bounds__(kThreads) k_stats(const T* __restrict__ x, con
                                                      const float* __restrict__ tau, float* __restrict__ lse,
                                                      int64_t N, int H, int G, uint32_t* status) {
   constexpr int GC = 32;
-  __shared__ float sW[GC][D + 1];
+  __shared__ __align__(16) float sW[GC][D];
   __shared__ float sB[GC];
   const int64_t bh = blockIdx.y;
   const int64_t b = bh / H;
@@ -152,7 +155,7 @@ __global__ void __launch_bounds__(kThreads) k_slice_partial(
     const float* __restrict__ bias, const float* __restrict__ tau, const float* __restrict__ lse,
     float* __restrict__ part, int64_t B, int64_t N, int H, int G, int64_t per_split, uint32_t* status) {
   constexpr int PT = 32;
-  __shared__ float sx[PT][D];
+  __shared__ __align__(16) float sx[PT][D];
   __shared__ float sf[PT][D];
   __shared__ float sl[PT];
   const int g = blockIdx.x * kThreads + threadIdx.x;
@@ -511,8 +514,8 @@ __global__ void __launch_bounds__(kThreads) k_deslice(const T* __restrict__ x, c
                                                        const float* __restrict__ lse, T* __restrict__ out,
                                                        int64_t N, int H, int G, uint32_t* status) {
   constexpr int GC = 32;
-  __shared__ float sW[GC][D + 1];
-  __shared__ float sZ[GC][D];
+  __shared__ __align__(16) float sW[GC][D];
+  __shared__ __align__(16) float sZ[GC][D];
   __shared__ float sB[GC];
   const int64_t bh = blockIdx.y;
   const int64_t b = bh / H;
@@ -577,9 +580,10 @@ __global__ void __launch_bounds__(kThreads) k_bwd_point(
     int accumulate, int64_t N, int H, int G, uint32_t* status) {
   constexpr int GC = 16;
   __shared__ float s_dt[kThreads];
-  constexpr int TS = (MODE == 0) ? D : D + 1;  // token row stride
-  __shared__ float sW[GC][D + 1];
-  __shared__ float sT[GC][TS];
+  constexpr int TS = (MODE == 0) ? D : D + 1;  // token row stride in memory
+  __shared__ __align__(16) float sW[GC][D];
+  __shared__ __align__(16) float sT[GC][D];  // t_g (z' or dU)
+  __shared__ float sS[GC];                    // MODE 1: dS_g
   __shared__ float sB[GC];
   const int64_t bh = blockIdx.y;
   const int64_t b = bh / H;
@@ -610,29 +614,49 @@ __global__ void __launch_bounds__(kThreads) k_bwd_point(
       stage_w<D, GC>(sW, sB, W, bias, h, G, g0, scale);
       for (int i = threadIdx.x; i < GC * TS; i += kThreads) {
         const int g = i / TS, k = i % TS;
-        sT[g][k] = (g0 + g < G) ? tb[(int64_t)(g0 + g) * TS + k] : 0.f;
+        const float t = (g0 + g < G) ? tb[(int64_t)(g0 + g) * TS + k] : 0.f;
+        if (k < D)
+          sT[g][k] = t;
+        else
+          sS[g] = t;
       }
       __syncthreads();
       const int gn = min(GC, G - g0);
-      for (int g = 0; g < gn; g++) {
-        float a = sB[g];
+      // Four slots at a time: their logit and dw dot products are independent chains
+      // (one 32-long chain per slot would leave the FMA pipe waiting on each result).
+      // The per-slot updates below run in slot order, as one slot at a time would.
+#pragma unroll 1
+      for (int g = 0; g < gn; g += 4) {
+        float a[4], dwq[4];
 #pragma unroll
-        for (int k = 0; k < D; k++) a = fmaf(xr[k], sW[g][k], a);
-        const float w = exp2f(a - l2);
-        float dw = (MODE == 0) ? 0.f : sT[g][D];
+        for (int q = 0; q < 4; q++) {
+          a[q] = sB[g + q];
+          dwq[q] = (MODE == 0) ? 0.f : sS[g + q];
+        }
 #pragma unroll
-        for (int k = 0; k < D; k++) dw = fmaf(vr[k], sT[g][k], dw);
-        if (sweep == 0) {
-          dl = fmaf(w, dw, dl);
-          if (MODE == 1) {
+        for (int k = 0; k < D; k++)
 #pragma unroll
-            for (int k = 0; k < D; k++) acc[k] = fmaf(w, sT[g][k], acc[k]);
+          for (int q = 0; q < 4; q++) {
+            a[q] = fmaf(xr[k], sW[g + q][k], a[q]);
+            dwq[q] = fmaf(vr[k], sT[g + q][k], dwq[q]);
           }
-        } else {
-          const float da = w * (dw - dl);
 #pragma unroll
-          for (int k = 0; k < D; k++) acc[k] = fmaf(da, sW[g][k], acc[k]);
-          if (valid) dtn = fmaf(da, a - l2, dtn);
+        for (int q = 0; q < 4; q++) {
+          if (g + q >= gn) break;
+          const float w = exp2f(a[q] - l2);
+          const float dw = dwq[q];
+          if (sweep == 0) {
+            dl = fmaf(w, dw, dl);
+            if (MODE == 1) {
+#pragma unroll
+              for (int k = 0; k < D; k++) acc[k] = fmaf(w, sT[g + q][k], acc[k]);
+            }
+          } else {
+            const float da = w * (dw - dl);
+#pragma unroll
+            for (int k = 0; k < D; k++) acc[k] = fmaf(da, sW[g + q][k], acc[k]);
+            if (valid) dtn = fmaf(da, a[q] - l2, dtn);
+          }
         }
       }
     }
@@ -678,8 +702,8 @@ __global__ void __launch_bounds__(kThreads) k_bwd_slot(
   constexpr int PT = 32;
   constexpr int TS = (MODE == 0) ? D : D + 1;
   constexpr int PS = (MODE == 0) ? 2 * D + 2 : D + 2;
-  __shared__ float sx[PT][D];
-  __shared__ float sv[PT][D];
+  __shared__ __align__(16) float sx[PT][D];
+  __shared__ __align__(16) float sv[PT][D];
   __shared__ float sl[PT];
   __shared__ float sd[PT];
   const int g = blockIdx.x * kThreads + threadIdx.x;
@@ -725,23 +749,35 @@ __global__ void __launch_bounds__(kThreads) k_bwd_slot(
       sd[i] = ok ? delta[bh * N + n] : 0.f;
     }
     __syncthreads();
-#pragma unroll 2
-    for (int j = 0; j < PT; j++) {
-      float a = bb;
+    // Four points at a time: independent logit and dw chains; the updates below run
+    // in point order, as one point at a time would.
+#pragma unroll 1
+    for (int j = 0; j < PT; j += 4) {
+      float a[4], dwq[4];
 #pragma unroll
-      for (int k = 0; k < D; k++) a = fmaf(sx[j][k], wc[k], a);
-      const float w = exp2f(a - sl[j]);
-      float dw = dSg;
-#pragma unroll
-      for (int k = 0; k < D; k++) dw = fmaf(sv[j][k], tg[k], dw);
-      const float da = w * (dw - sd[j]);
-      if (MODE == 0) {
-#pragma unroll
-        for (int k = 0; k < D; k++) dzp[k] = fmaf(w, sv[j][k], dzp[k]);
+      for (int q = 0; q < 4; q++) {
+        a[q] = bb;
+        dwq[q] = dSg;
       }
 #pragma unroll
-      for (int k = 0; k < D; k++) dWa[k] = fmaf(da, sx[j][k], dWa[k]);
-      dba += da;
+      for (int k = 0; k < D; k++)
+#pragma unroll
+        for (int q = 0; q < 4; q++) {
+          a[q] = fmaf(sx[j + q][k], wc[k], a[q]);
+          dwq[q] = fmaf(sv[j + q][k], tg[k], dwq[q]);
+        }
+#pragma unroll
+      for (int q = 0; q < 4; q++) {
+        const float w = exp2f(a[q] - sl[j + q]);
+        const float da = w * (dwq[q] - sd[j + q]);
+        if (MODE == 0) {
+#pragma unroll
+          for (int k = 0; k < D; k++) dzp[k] = fmaf(w, sv[j + q][k], dzp[k]);
+        }
+#pragma unroll
+        for (int k = 0; k < D; k++) dWa[k] = fmaf(da, sx[j + q][k], dWa[k]);
+        dba += da;
+      }
     }
   }
   if (g < G) {

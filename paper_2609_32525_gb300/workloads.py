@@ -82,9 +82,11 @@ def _mixer_identity_noise(rng, H, G, std=0.1):
 NAMED = ("tiny_f32", "surface_bf16", "batched_bf16", "large_g_bf16", "train_bf16")
 
 
-def make_named(name: str, n_override: Optional[int] = None, g_override: Optional[int] = None) -> Workload:
-    """One of the five named workloads; `n_override` changes N and `g_override`
-    the slot count G (same recipe otherwise)."""
+def make_named(name: str, n_override: Optional[int] = None, g_override: Optional[int] = None,
+               dtype_override: Optional[str] = None) -> Workload:
+    """One of the five named workloads; `n_override` changes N, `g_override` the slot
+    count G and `dtype_override` the input dtype ("f32" or "bf16"; same recipe
+    otherwise)."""
     idx = NAMED.index(name) + 1
     rng = np.random.Generator(np.random.PCG64(1000 + idx))
     H, d = 8, 32
@@ -103,6 +105,10 @@ def make_named(name: str, n_override: Optional[int] = None, g_override: Optional
         N = int(n_override)
     if g_override is not None:
         G = int(g_override)
+    if dtype_override is not None:
+        if dtype_override not in ("f32", "bf16"):
+            raise ValueError(f"dtype_override must be 'f32' or 'bf16', got {dtype_override!r}")
+        dtype = dtype_override
     mixture = name in ("batched_bf16", "train_bf16")
     if mixture:
         x = _gmm_points(rng, B, N, C).reshape(B, N, H, d)
