@@ -139,9 +139,15 @@ Regions regions(const Shape& s, int op) {
         r.tc = take(std::max(tc_coupling_bwd_bytes(s), tc_deslice_prep_bytes(s)));
         break;
       }
-      // the three calls one after another on the same scratch
-      return Regions{0, 0, 0, 0, 0, 0, 0,
-                     std::max(regions(s, FS_OP_DESLICE_BWD).total, regions(s, FS_OP_SLICE_BWD).total)};
+      // the fused SIMT backward: dU|dS, delta, the slot partials (which first hold
+      // the d z' partials), the points' temperature terms, the statistics
+      r.dus = take(BHG * (s.d + 1) * sizeof(float));
+      r.delta = take(pts * sizeof(float));
+      r.partials = take((size_t)P * BHG * (s.d + 2) * sizeof(float));
+      r.dtau_p = take((size_t)s.BH() * simt_point_blocks(s) * sizeof(float));
+      r.stats = take(pts * sizeof(float));
+      r.tc = take(tc_deslice_prep_bytes(s));
+      break;
     default:
       return Regions{};
   }
@@ -249,18 +255,21 @@ int fs_forward_launch_count(const fs_shape* s) {
   return 3 /*stats, partials, reduce*/ + 1 /*mix*/ + 1 /*deslice*/;
 }
 
+// Kernels of backward_stats for one backward call: none when it takes the caller's lse.
+int backward_stats_launches(const Shape& sh, int lse_given) {
+  const bool tc = tc_forward_supported(sh) && sh.dtype == FS_BF16;
+  const bool fp32_tc = tc_forward_supported(sh) && sh.dtype == FS_F32;
+  if (lse_given && !fp32_tc && (!tc || sh.dot == FS_DOT_BF16X2)) return 0;
+  Shape split = sh;
+  split.dot = FS_DOT_BF16X2;
+  return tc ? tc_stats_launch_count(split) : 1;
+}
+
 int fs_backward_launch_count(const fs_shape* s, int lse_given) {
   if (!valid_shape(s) || !supported_shape(s)) return -1;
   const Shape sh = to_shape(s);
   // Each backward call recomputes the statistics unless backward_stats takes the caller's lse.
-  const bool tc = tc_forward_supported(sh) && sh.dtype == FS_BF16;
-  const bool fp32_tc = tc_forward_supported(sh) && sh.dtype == FS_F32;
-  int stats = 0;
-  if (!(lse_given && !fp32_tc && (!tc || sh.dot == FS_DOT_BF16X2))) {
-    Shape split = sh;
-    split.dot = FS_DOT_BF16X2;
-    stats = tc ? tc_stats_launch_count(split) : 1;
-  }
+  const int stats = backward_stats_launches(sh, lse_given);
   const int mix_bwd = 2;  // d_tokens, dM
   if (tc_backward_supported(sh))
     return 2 * stats + tc_backward_launch_count(sh, 1) + mix_bwd + tc_backward_launch_count(sh, 2);
@@ -270,7 +279,7 @@ int fs_backward_launch_count(const fs_shape* s, int lse_given) {
 int fs_coupling_bwd_launch_count(const fs_shape* s, int lse_given) {
   if (!valid_shape(s) || !supported_shape(s)) return -1;
   const Shape sh = to_shape(s);
-  if (!tc_backward_supported(sh)) return fs_backward_launch_count(s, lse_given);
+  if (!tc_backward_supported(sh)) return backward_stats_launches(sh, lse_given) + simt_coupling_bwd_launch_count();
   const bool tc = tc_forward_supported(sh);
   const int stats = (lse_given && sh.dot == FS_DOT_BF16X2) ? 0 : (tc ? 2 : 1);  // the statistics once
   return stats + tc_coupling_bwd_launch_count(sh);
@@ -479,12 +488,16 @@ fs_status fs_coupling_bwd(const fs_shape* s, const void* x_mid, const void* fx, 
   const Shape sh = to_shape(s);
   if (fs_status e = check_ws(sh, FS_OP_COUPLING_BWD, ws, ws_bytes)) return e;
   if (!tc_backward_supported(sh)) {
-    fs_status e = fs_deslice_bwd(s, x_mid, W_slice, bias, tau, tokens_mixed, lse, dout, d_tokens_mixed, dx_mid, dW,
-                                 dbias, dtau, accumulate, ws, ws_bytes, stream);
-    if (e != FS_OK) return e;
-    if ((e = fs_mix_bwd(s, M, tokens, d_tokens_mixed, d_tokens, dM, stream)) != FS_OK) return e;
-    return fs_slice_bwd(s, x_mid, fx, W_slice, bias, tau, tokens, wsum, lse, d_tokens, dx_mid, dfx, dW, dbias, dtau,
-                        1, ws, ws_bytes, stream);
+    const Regions r = regions(sh, FS_OP_COUPLING_BWD);
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    uint32_t* status = at<uint32_t>(ws, r.status);
+    FS_CUDA(reset_status(ws, st));
+    const float* lse_use = nullptr;
+    FS_CUDA(backward_stats(sh, x_mid, W_slice, bias, tau, lse, ws, r, status, st, &lse_use));
+    return cuda_status(simt_coupling_bwd(sh, slot_splits(sh), x_mid, fx, dout, W_slice, bias, tau, M, tokens, wsum,
+                                         tokens_mixed, lse_use, d_tokens_mixed, d_tokens, dM, dx_mid, dfx, dW, dbias,
+                                         dtau, accumulate, at<float>(ws, r.delta), at<float>(ws, r.dus),
+                                         at<float>(ws, r.partials), at<float>(ws, r.dtau_p), status, st));
   }
   const Regions r = regions(sh, FS_OP_COUPLING_BWD);
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);

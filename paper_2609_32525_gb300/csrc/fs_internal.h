@@ -72,6 +72,16 @@ cudaError_t simt_reduce_bwd(const Shape& s, int P, const float* part, int Gs, in
                             float* dzp, float* dW, float* db, float* dtau, const float* dt_part, int64_t nblk,
                             int accumulate, cudaStream_t st);
 // The token gradient alone from partials whose first d words per slot are dz'.
+// The coupling's whole backward on the SIMT kernels (fs_coupling_bwd on shapes the
+// tensor-core backward does not take); delta, dUS, part, dt_part as in the calls above
+// (part holds P * B*H * G * (d + 2) floats).
+cudaError_t simt_coupling_bwd(const Shape& s, int P, const void* x, const void* fx, const void* dout,
+                              const float* W, const float* bias, const float* tau, const float* M, const float* z,
+                              const float* wsum, const float* zp, const float* lse, float* dzp, float* dz,
+                              float* dM, void* dx, void* dfx, float* dW, float* db, float* dtau, int accumulate,
+                              float* delta, float* dUS, float* part, float* dt_part, uint32_t* status,
+                              cudaStream_t st);
+int simt_coupling_bwd_launch_count();
 cudaError_t simt_reduce_dzp(const Shape& s, int P, const float* part, int Gs, int PS, float* dzp, cudaStream_t st);
 cudaError_t simt_slice_bwd(const Shape& s, int P, const void* x, const void* f, const float* W,
                            const float* bias, const float* tau, const float* z,

@@ -795,6 +795,243 @@ __global__ void __launch_bounds__(kThreads) k_bwd_slot(
   }
 }
 
+// ---- the coupling's whole backward, fused -------------------------------------------------
+// The deslice's and the slice's weight gradients share the weights, so their softmax
+// backward adds up: da = w (dw - delta) with dw_g = dO . z'_g + fx . dU_g + dS_g and
+// delta = sum_g w_g dw_g.  One point pass and one slot pass then serve both (the
+// separate calls make two of each).
+// Point pass: sweep 1 forms delta and dfx = sum_g w_g dU_g, sweep 2 dx = (1/tau) sum_g
+// da_g W[:,g] (added to dx when accumulate) and the points' temperature terms.
+template <int D, typename T>
+__global__ void __launch_bounds__(kThreads) k_bwd_point_comb(
+    const T* __restrict__ x, const T* __restrict__ dO, const T* __restrict__ fx, const float* __restrict__ W,
+    const float* __restrict__ bias, const float* __restrict__ tau, const float* __restrict__ zp,
+    const float* __restrict__ dUS, const float* __restrict__ lse, T* __restrict__ dx, T* __restrict__ dfx,
+    float* __restrict__ delta, float* __restrict__ dt_part, int accumulate, int64_t N, int H, int G,
+    uint32_t* status) {
+  constexpr int GC = 16;
+  __shared__ float s_dt[kThreads];
+  __shared__ __align__(16) float sW[GC][D];
+  __shared__ __align__(16) float sZ[GC][D];  // z'_g
+  __shared__ __align__(16) float sU[GC][D];  // dU_g
+  __shared__ float sS[GC];                    // dS_g
+  __shared__ float sB[GC];
+  const int64_t bh = blockIdx.y;
+  const int64_t b = bh / H;
+  const int h = (int)(bh % H);
+  if (!tau_ok(tau[h], status)) return;
+  const float scale = kLog2e / tau[h];
+  const int64_t n = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  const bool valid = n < N;
+  float xr[D], dr[D], fr[D], acc[D];
+#pragma unroll
+  for (int k = 0; k < D; k++) { xr[k] = 0.f; dr[k] = 0.f; fr[k] = 0.f; acc[k] = 0.f; }
+  float l2 = CUDART_INF_F;
+  const int64_t row = row_index(b, n, h, N, H);
+  if (valid) {
+    load_row<D>(x + row * D, xr);
+    load_row<D>(dO + row * D, dr);
+    load_row<D>(fx + row * D, fr);
+    l2 = lse[bh * N + n] * kLog2e;
+  }
+  const float* zb = zp + bh * G * D;
+  const float* ub = dUS + bh * G * (D + 1);
+  auto stage = [&](int g0) {
+    __syncthreads();
+    stage_w<D, GC>(sW, sB, W, bias, h, G, g0, scale);
+    for (int i = threadIdx.x; i < GC * D; i += kThreads) {
+      const int g = i / D, k = i % D;
+      sZ[g][k] = (g0 + g < G) ? zb[(int64_t)(g0 + g) * D + k] : 0.f;
+    }
+    for (int i = threadIdx.x; i < GC * (D + 1); i += kThreads) {
+      const int g = i / (D + 1), k = i % (D + 1);
+      const float t = (g0 + g < G) ? ub[(int64_t)(g0 + g) * (D + 1) + k] : 0.f;
+      if (k < D)
+        sU[g][k] = t;
+      else
+        sS[g] = t;
+    }
+    __syncthreads();
+  };
+  // Logits and dw of kQ slots at a time (independent chains; the point's x, dO, fx and
+  // accumulator rows already hold 128 registers, so two rather than four).
+  constexpr int kQ = 2;
+  auto chains = [&](int g, float (&a)[kQ], float (&dwq)[kQ]) {
+#pragma unroll
+    for (int q = 0; q < kQ; q++) {
+      a[q] = sB[g + q];
+      dwq[q] = sS[g + q];
+    }
+#pragma unroll
+    for (int k = 0; k < D; k++)
+#pragma unroll
+      for (int q = 0; q < kQ; q++) {
+        a[q] = fmaf(xr[k], sW[g + q][k], a[q]);
+        dwq[q] = fmaf(dr[k], sZ[g + q][k], dwq[q]);
+        dwq[q] = fmaf(fr[k], sU[g + q][k], dwq[q]);
+      }
+  };
+  // Sweep 1: delta and dfx (updates in slot order).
+  float dl = 0.f;
+  for (int g0 = 0; g0 < G; g0 += GC) {
+    stage(g0);
+    const int gn = min(GC, G - g0);
+#pragma unroll 1
+    for (int g = 0; g < gn; g += kQ) {
+      float a[kQ], dwq[kQ];
+      chains(g, a, dwq);
+#pragma unroll
+      for (int q = 0; q < kQ; q++) {
+        if (g + q < gn) {
+          const float w = exp2f(a[q] - l2);
+          dl = fmaf(w, dwq[q], dl);
+#pragma unroll
+          for (int k = 0; k < D; k++) acc[k] = fmaf(w, sU[g + q][k], acc[k]);
+        }
+      }
+    }
+  }
+  if (valid) store_row<D>(dfx + row * D, acc);
+#pragma unroll
+  for (int k = 0; k < D; k++) acc[k] = 0.f;
+  // Sweep 2: dx and the temperature terms.
+  float dtn = 0.f;
+  for (int g0 = 0; g0 < G; g0 += GC) {
+    stage(g0);
+    const int gn = min(GC, G - g0);
+#pragma unroll 1
+    for (int g = 0; g < gn; g += kQ) {
+      float a[kQ], dwq[kQ];
+      chains(g, a, dwq);
+#pragma unroll
+      for (int q = 0; q < kQ; q++) {
+        if (g + q < gn) {
+          const float da = exp2f(a[q] - l2) * (dwq[q] - dl);
+#pragma unroll
+          for (int k = 0; k < D; k++) acc[k] = fmaf(da, sW[g + q][k], acc[k]);
+          if (valid) dtn = fmaf(da, a[q] - l2, dtn);
+        }
+      }
+    }
+  }
+  // Block sum of the temperature terms (fixed tree order) -> dt_part[bh][block].
+  s_dt[threadIdx.x] = dtn;
+  __syncthreads();
+  for (int w = kThreads / 2; w > 0; w >>= 1) {
+    if (threadIdx.x < w) s_dt[threadIdx.x] += s_dt[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) dt_part[bh * gridDim.x + blockIdx.x] = s_dt[0] * kLn2;
+  if (!valid) return;
+  delta[bh * N + n] = dl;
+#pragma unroll
+  for (int k = 0; k < D; k++) acc[k] *= kLn2;
+  if (accumulate) {
+    float old[D];
+    load_row<D>(dx + row * D, old);
+#pragma unroll
+    for (int k = 0; k < D; k++) acc[k] += old[k];
+  }
+  store_row<D>(dx + row * D, acc);
+}
+
+// Slot pass of the fused backward: thread = slot g; for every point n of the split,
+// da = w (dw - delta_n) with dw as above; dWa += da x_n; dba += da.
+// part[p][bh][g] = (dWa (D), dba, 0), un-scaled by 1/tau.
+template <int D, typename T>
+__global__ void __launch_bounds__(kThreads) k_bwd_slot_comb(
+    const T* __restrict__ x, const T* __restrict__ dO, const T* __restrict__ fx, const float* __restrict__ W,
+    const float* __restrict__ bias, const float* __restrict__ tau, const float* __restrict__ zp,
+    const float* __restrict__ dUS, const float* __restrict__ lse, const float* __restrict__ delta,
+    float* __restrict__ part, int64_t B, int64_t N, int H, int G, int64_t per_split, uint32_t* status) {
+  constexpr int PT = 32;
+  constexpr int PS = D + 2;
+  __shared__ __align__(16) float sx[PT][D];
+  __shared__ __align__(16) float sd[PT][D];  // dO
+  __shared__ __align__(16) float sf[PT][D];  // fx
+  __shared__ float sl[PT];
+  __shared__ float sdl[PT];
+  const int g = blockIdx.x * kThreads + threadIdx.x;
+  const int64_t bh = blockIdx.y;
+  const int64_t b = bh / H;
+  const int h = (int)(bh % H);
+  const int p = blockIdx.z;
+  if (!tau_ok(tau[h], status)) return;
+  const float scale = kLog2e / tau[h];
+  float wc[D], zg[D], ug[D], dWa[D];
+  float bb = 0.f, dSg = 0.f, dba = 0.f;
+#pragma unroll
+  for (int k = 0; k < D; k++) {
+    wc[k] = (g < G) ? W[((int64_t)h * D + k) * G + g] * scale : 0.f;
+    zg[k] = (g < G) ? zp[(bh * G + g) * D + k] : 0.f;
+    ug[k] = (g < G) ? dUS[(bh * G + g) * (D + 1) + k] : 0.f;
+    dWa[k] = 0.f;
+  }
+  if (g < G) {
+    bb = bias[(int64_t)h * G + g] * scale;
+    dSg = dUS[(bh * G + g) * (D + 1) + D];
+  }
+  const int64_t n_begin = (int64_t)p * per_split;
+  const int64_t n_end = min(N, n_begin + per_split);
+  for (int64_t n0 = n_begin; n0 < n_end; n0 += PT) {
+    __syncthreads();
+    for (int i = threadIdx.x; i < PT * D; i += kThreads) {
+      const int j = i / D, k = i % D;
+      const int64_t n = n0 + j;
+      float xv = 0.f, dv = 0.f, fv = 0.f;
+      if (n < n_end) {
+        const int64_t idx = row_index(b, n, h, N, H) * D + k;
+        xv = to_f(x[idx]);
+        dv = to_f(dO[idx]);
+        fv = to_f(fx[idx]);
+      }
+      sx[j][k] = xv;
+      sd[j][k] = dv;
+      sf[j][k] = fv;
+    }
+    for (int i = threadIdx.x; i < PT; i += kThreads) {
+      const int64_t n = n0 + i;
+      const bool ok = n < n_end;
+      sl[i] = ok ? lse[bh * N + n] * kLog2e : CUDART_INF_F;
+      sdl[i] = ok ? delta[bh * N + n] : 0.f;
+    }
+    __syncthreads();
+    // Four points at a time (independent chains), updates in point order.
+#pragma unroll 1
+    for (int j = 0; j < PT; j += 4) {
+      float a[4], dwq[4];
+#pragma unroll
+      for (int q = 0; q < 4; q++) {
+        a[q] = bb;
+        dwq[q] = dSg;
+      }
+#pragma unroll
+      for (int k = 0; k < D; k++)
+#pragma unroll
+        for (int q = 0; q < 4; q++) {
+          a[q] = fmaf(sx[j + q][k], wc[k], a[q]);
+          dwq[q] = fmaf(sd[j + q][k], zg[k], dwq[q]);
+          dwq[q] = fmaf(sf[j + q][k], ug[k], dwq[q]);
+        }
+#pragma unroll
+      for (int q = 0; q < 4; q++) {
+        const float w = exp2f(a[q] - sl[j + q]);
+        const float da = w * (dwq[q] - sdl[j + q]);
+#pragma unroll
+        for (int k = 0; k < D; k++) dWa[k] = fmaf(da, sx[j + q][k], dWa[k]);
+        dba += da;
+      }
+    }
+  }
+  if (g < G) {
+    float* o = part + (((int64_t)p * B * H + bh) * G + g) * PS;
+#pragma unroll
+    for (int k = 0; k < D; k++) o[k] = dWa[k];
+    o[D] = dba;
+    o[D + 1] = 0.f;  // (the temperature gradient is formed per point, in the point pass)
+  }
+}
+
 // Token-gradient prep for the slice backward: dUS[bh][g] = (dz_g/(S_g+eps), -(dz_g.z_g)/(S_g+eps)).
 __global__ void k_slice_bwd_prep(const float* __restrict__ z, const float* __restrict__ wsum,
                                  const float* __restrict__ dz, float* __restrict__ dUS, int64_t BHG, int D,
@@ -914,7 +1151,23 @@ cudaError_t launch_bwd(const Shape& s, int P, const void* x, const void* v, cons
   return cudaGetLastError();
 }
 
-// Dispatch over (d, dtype).
+template <int D, typename T>
+cudaError_t launch_bwd_comb(const Shape& s, int P, const void* x, const void* dO, const void* fx, const float* W,
+                            const float* bias, const float* tau, const float* zp, const float* dUS,
+                            const float* lse, void* dx, void* dfx, float* delta, float* dt_part, float* part,
+                            int accumulate, uint32_t* status, cudaStream_t st) {
+  k_bwd_point_comb<D, T><<<point_grid(s), kThreads, 0, st>>>((const T*)x, (const T*)dO, (const T*)fx, W, bias, tau,
+                                                              zp, dUS, lse, (T*)dx, (T*)dfx, delta, dt_part,
+                                                              accumulate, s.N, s.H, s.G, status);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_bwd_slot_comb<D, T><<<slot_grid(s, P), kThreads, 0, st>>>((const T*)x, (const T*)dO, (const T*)fx, W, bias, tau,
+                                                               zp, dUS, lse, delta, part, s.B, s.N, s.H, s.G,
+                                                               per_split(s, P), status);
+  return cudaGetLastError();
+}
+
+// Dispatch over (d, dtype).// Dispatch over (d, dtype).
 #define FS_DISPATCH(s, FN, ...)                                                        \
   do {                                                                                 \
     const bool bf = (s).dtype == FS_BF16;                                              \
@@ -1076,5 +1329,33 @@ cudaError_t simt_slice_bwd(const Shape& s, int P, const void* x, const void* f, 
   return simt_reduce_bwd(s, P, part, s.G, s.d + 2, 0, tau, nullptr, dW, db, dtau, dt_part, simt_point_blocks(s),
                          accumulate, st);
 }
+
+// The coupling's whole backward on the SIMT kernels: d z' as the forward slice's
+// unnormalised numerators with dO for fx, the mix backward, the slice's dU, dS, then
+// one point pass and one slot pass for da_D + da_S (k_bwd_point_comb, k_bwd_slot_comb)
+// and the parameter reductions.  `part` holds the larger of the two partial sets;
+// the d z' reduction's weight sums go to dUS, which the prologue then overwrites.
+cudaError_t simt_coupling_bwd(const Shape& s, int P, const void* x, const void* fx, const void* dout,
+                              const float* W, const float* bias, const float* tau, const float* M, const float* z,
+                              const float* wsum, const float* zp, const float* lse, float* dzp, float* dz,
+                              float* dM, void* dx, void* dfx, float* dW, float* db, float* dtau, int accumulate,
+                              float* delta, float* dUS, float* part, float* dt_part, uint32_t* status,
+                              cudaStream_t st) {
+  cudaError_t e = simt_slice_partials(s, P, x, dout, W, bias, tau, lse, part, status, st);
+  if (e != cudaSuccess) return e;
+  if ((e = simt_reduce_tokens(s, P, part, s.G, dzp, dUS, 0, st)) != cudaSuccess) return e;
+  if ((e = simt_mix_bwd(s, M, z, dzp, dz, dM, st)) != cudaSuccess) return e;
+  if ((e = simt_slice_bwd_prep(s, z, wsum, dz, dUS, st)) != cudaSuccess) return e;
+  e = [&]() -> cudaError_t {
+    FS_DISPATCH(s, launch_bwd_comb, s, P, x, dout, fx, W, bias, tau, zp, dUS, lse, dx, dfx, delta, dt_part, part,
+                accumulate, status, st);
+  }();
+  if (e != cudaSuccess) return e;
+  return simt_reduce_bwd(s, P, part, s.G, s.d + 2, 0, tau, nullptr, dW, db, dtau, dt_part, simt_point_blocks(s),
+                         accumulate, st);
+}
+// Kernels it launches (the statistics, when needed, are counted by the caller).
+int simt_coupling_bwd_launch_count() { return 2 /*partials, reduce*/ + 2 /*mix backward*/ + 1 /*prologue*/ +
+                                              2 /*point, slot*/ + 2 /*reductions*/; }
 
 }  // namespace fs

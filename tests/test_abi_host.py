@@ -154,11 +154,16 @@ def test_backward_launch_count(fs):
 
 
 def test_coupling_bwd_launch_count_and_overlap_checks(fs):
-    """fs_coupling_bwd: on the SIMT backward it makes the three calls, so it
-    launches what they launch; outputs overlapping M, tokens, tokens_mixed or each
-    other are rejected before any launch (fake aligned addresses, never read)."""
+    """fs_coupling_bwd: on the SIMT backward it makes one fused pass pair (d z' partials
+    and their reduction, the mix backward's two kernels, the dU, dS prologue, the point
+    and slot passes, two reductions: 9 kernels, plus the statistics once when no lse
+    is given) where the three calls make 12; outputs overlapping M, tokens,
+    tokens_mixed or each other are rejected before any launch (fake aligned addresses,
+    never read)."""
     s = fs.make_shape(1, 100, 2, 32, 8, dtype=fs.FS_F32)
-    assert fs.coupling_bwd_launch_count(s, True) == fs.backward_launch_count(s, True)
+    assert fs.coupling_bwd_launch_count(s, True) == 9
+    assert fs.coupling_bwd_launch_count(s, False) == 10
+    assert fs.backward_launch_count(s, True) == 12
     assert fs.coupling_bwd_launch_count(fs.make_shape(1, 100, 2, 48, 8)) == -1
     lib, P = fs._lib, ctypes.c_void_p
     B, N, H, d, G = 1, 100, 2, 32, 8
@@ -167,7 +172,7 @@ def test_coupling_bwd_launch_count_and_overlap_checks(fs):
     addr = [base + i * (1 << 20) for i in range(20)]
     ws = 1 << 30
     nbytes = fs.workspace_bytes(s, fs.FS_OP_COUPLING_BWD)
-    assert nbytes >= max(fs.workspace_bytes(s, fs.FS_OP_DESLICE_BWD), fs.workspace_bytes(s, fs.FS_OP_SLICE_BWD))
+    assert nbytes > 0
     # x, fx, W, bias, tau, M, tokens, wsum, tokens_mixed, lse, dout | dzm, dz, dx, dfx, dW, db, dt, dM
     ins, outs = addr[:11], addr[11:19]
     M, tokens, tokens_mixed = ins[5], ins[6], ins[8]
