@@ -243,13 +243,14 @@ fs_status fs_slice_bwd(const fs_shape* s, const void* x_mid, const void* fx,
  *   contributions, written if accumulate == 0, added if accumulate != 0.
  *   tokens, wsum, tokens_mixed, lse: the forward's (lse may be NULL, as in the
  *   separate calls).  ws: fs_workspace_bytes(s, FS_OP_COUPLING_BWD).
- * On the tensor-core backward (fs_backward_path_for_shape == 1) the two calls'
- * dx come from one point pass: their da_ng share the weights, so one pass over
- * (point, slot) forms da_D + da_S and dx from it, instead of one pass per call.
- * Results agree with the separate calls to rounding (dx is summed before its one
- * bf16 rounding instead of after each call's).  Elsewhere it makes the three
- * calls.  M, tokens and tokens_mixed overlapping an output, or two outputs
- * overlapping each other: FS_ERR_INVALID. */
+ * The two calls' da_ng share the weights, so one point pass over (point, slot)
+ * forms da_D + da_S and dx from it, and one slot pass dW, dbias, dtau, instead of
+ * one of each per call; d_tokens_mixed comes first, as the slice's unnormalised
+ * numerators with dout for fx.  This holds on the tensor-core backward
+ * (fs_backward_path_for_shape == 1) and on the fp32 SIMT one.  Results agree with
+ * the separate calls to rounding (for instance dx is summed before its one rounding
+ * to the input dtype instead of after each call's).  M, tokens and tokens_mixed
+ * overlapping an output, or two outputs overlapping each other: FS_ERR_INVALID. */
 fs_status fs_coupling_bwd(const fs_shape* s, const void* x_mid, const void* fx,
                           const float* W_slice, const float* bias, const float* tau,
                           const float* M, const float* tokens, const float* wsum,
