@@ -53,8 +53,12 @@ def test_small_fp32_problems_keep_the_simt_kernels(lib):
     assert lib.path_for_shape(lib.make_shape(1, 70000, 8, 32, 1025, lib.FS_F32)) == 0
 
 
-def test_fp32_backward_after_tensor_core_forward(lib):
-    wl = make_case(2, 5000, 8, 32, 256, dtype="f32", seed=810, backward=True)
+@pytest.mark.parametrize("G", [256, 512, 1024])
+def test_fp32_backward_after_tensor_core_forward(lib, G):
+    """The fp32 coupling's whole backward (fs_coupling_bwd on the fused SIMT kernels,
+    exact fp32 statistics) after the tensor-core forward, at the fp32 bar."""
+    N = 5000 if G == 256 else 3000
+    wl = make_case(2, N, 8, 32, G, dtype="f32", seed=810 + G, backward=True)
     dev = upload(wl)
     c = lib.Coupling(wl.B, wl.N, wl.H, 32, wl.G, torch.float32, wl.eps, backward=True)
     assert lib.path_for_shape(c.shape) == 1 and lib.backward_path_for_shape(c.shape) == 0
@@ -64,6 +68,7 @@ def test_fp32_backward_after_tensor_core_forward(lib):
     assert c.device_status() == lib.FS_OK
     ref = orc.backward(wl.x_mid, wl.fx, wl.W_slice, wl.bias, wl.tau, wl.M, wl.dout, eps=wl.eps)
     errs = {k: max_rel(host(g[k]), ref[k]) for k in ("dx_mid", "dfx", "dW", "dbias", "dtau", "dM")}
+    print("fp32 backward G={}".format(G), " ".join("{}={:.2e}".format(k, e) for k, e in errs.items()))
     bad = {k: e for k, e in errs.items() if not e <= TOL}
     assert not bad, {k: "{:.2e}".format(e) for k, e in bad.items()}
 
