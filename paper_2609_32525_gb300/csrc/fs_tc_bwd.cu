@@ -104,9 +104,10 @@ __global__ void k_prep_dpx(const float* __restrict__ delta, const float* __restr
 // ---- device pieces -----------------------------------------------------------------------------
 
 // M = 128 x N = 64 product with K = 48 (80 with the residual half, lo_a or lo_b):
-// a0/b0 are the K-major 64B-swizzled 32-channel blocks, ae/be the extra blocks.
+// a0/b0 are the K-major 64B-swizzled 32-channel blocks, ae/be the extra blocks
+// (kExtra = false: K = 32 / 64, no extra block).
 // acc0: add to what d holds (a second chain into the same accumulator).
-template <bool kLoA>
+template <bool kLoA, bool kExtra = true>
 __device__ __forceinline__ void issue_dot64(uint32_t d, uint32_t a, uint32_t b, uint64_t ae, uint64_t be,
                                             uint32_t lo, uint32_t acc0 = 0) {
   constexpr uint32_t idesc = idesc_bf16(128, 64, false, false);
@@ -121,7 +122,7 @@ __device__ __forceinline__ void issue_dot64(uint32_t d, uint32_t a, uint32_t b, 
       mma_ss_w(d, sdesc(a + 32, 16, 512, kSw64), sdesc(lo + 32, 16, 512, kSw64), idesc, 1);
     }
   }
-  mma_ss_w(d, ae, be, idesc, 1);
+  if (kExtra) mma_ss_w(d, ae, be, idesc, 1);
 }
 
 // Point-extra descriptor (no swizzle, 16-byte rows) whose k = 8..15 half is the shared zero block.
@@ -231,8 +232,9 @@ __device__ __forceinline__ bool slot_flush_at(int u) { return ((u >> 1) % kSlotF
 // Two more modes serve fs_coupling_bwd:
 //   MODE 0: the token gradient alone, dZ += w^T dO (no dw chain, no da): part = dZ(32);
 //   MODE 3: da = da_D + da_S as in the combined point pass (dw - delta as two chains:
-//     the deslice's T block against [dO | 1, 1, -delta], the slice's T2 block against
-//     [fx | 1, 1, 0 ...], delta = delta_D + delta_S), written like MODE 2.
+//     the deslice's T block against dO, the slice's T2 block against [fx | 1, 1, -delta]
+//     (its extra block [dS_hi, dS_lo, 1, 1, 1] meets delta's rows), delta = delta_D +
+//     delta_S), written like MODE 2.
 // smem: [W block: hi 8K | extra 4K | lo 8K][T block: same][stages][zero 2K][red 1.5K][bars]
 // TMEM: unit u uses set u % 3: L [128 s, +64), dw [128 s + 64, +64); accumulators
 // dWx_j [384 + 32 j), dZ_j [448 + 32 j).
@@ -254,10 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* s_t = s_w + kWBlockB;     // T block
   uint8_t* s_t2 = s_t + kWBlockB;    // MODE 3: the slice's T block
   uint8_t* s_st = s_t2 + (MODE == 3 ? kWBlockB : 0u);  // stages
-  // MODE 3: point rows [1, 1, 0 ...] (no delta).  Like the stages' point rows it lies
-  // below the zero block, which its descriptor reaches at a positive offset.
-  uint8_t* s_ones = s_st + kNSt * kStgS;
-  uint8_t* s_zero = s_ones + (MODE == 3 ? kPxBytes : 0u);
+  uint8_t* s_zero = s_st + kNSt * kStgS;  // above the stages' point rows (positive LBO)
   float* s_red = reinterpret_cast<float*>(s_zero + kPxZero);  // 3 x 128 floats
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_red + 3 * kGC);
   uint64_t* w_full = bars;
@@ -305,9 +304,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_mbar_init();
   }
   zero_smem(s_zero, kPxZero);
-  if (MODE == 3)
-    for (int r = threadIdx.x; r < kTile; r += blockDim.x)
-      st_shared_v4(smem_u32(s_ones) + (uint32_t)r * 16, 0x3F803F80u, 0u, 0u, 0u);
   fence_proxy_async_smem();
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
@@ -369,12 +365,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t tL = tmem + (uint32_t)bb * kGC;
       issue_dot64<true>(tL, sw, st + rows, sdesc(sw + kGC * 64, 16, 256, kSw32), px_desc(st + kPOff + prow, sz),
                         split ? sw + kGC * 96 : 0u);
-      if (MODE != 0)
+      if (MODE == 1 || MODE == 2)
         issue_dot64<true>(tL + 64, stt, st + kVOff + rows, sdesc(stt + kGC * 64, 16, 256, kSw32),
                           px_desc(st + kDOff + prow, sz), split ? stt + kGC * 96 : 0u);
-      if (MODE == 3)
+      if (MODE == 3) {
+        // The deslice's T has c = 0, so its chain needs no extra block: the slice's
+        // extra block [dS_hi, dS_lo, 1, 1, 1] against delta's rows [1, 1, -delta parts]
+        // adds dS - delta in one K step.
+        issue_dot64<true, false>(tL + 64, stt, st + kVOff + rows, 0ull, 0ull, split ? stt + kGC * 96 : 0u);
         issue_dot64<true>(tL + 64, stt2, st + kBStage + rows, sdesc(stt2 + kGC * 64, 16, 256, kSw32),
-                          px_desc(smem_u32(s_ones) + prow, sz), split ? stt2 + kGC * 96 : 0u, 1u);
+                          px_desc(st + kDOff + prow, sz), split ? stt2 + kGC * 96 : 0u, 1u);
+      }
       mma_commit_w(&s_full[bb]);
       if (half == 1) mma_commit_w(&st_empty[s]);
     }
@@ -561,11 +562,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 //   O_j += da W'^T (B: the W'^T image, channel rows, slots along K).
 // kComb (the whole coupling's backward): da is the sum of the deslice's and the
 // slice's, which share the weights, so one pass serves both: dw - delta is two chains
-// into the same accumulator, [dO | 1, 1, -delta] against the deslice's T image (c = 0)
-// and [fx | 1, 1, 0 ...] (a constant extra block) against the slice's (t = dU, c = dS),
-// with delta = delta_D + delta_S in the point rows.  Each stage also holds the fx tile.
+// into the same accumulator, dO against the deslice's T image (c = 0, so no extra
+// block) and [fx | 1, 1, -delta] against the slice's (t = dU, c = dS): one extra K
+// step adds dS - delta, with delta = delta_D + delta_S in the point rows.  Each stage
+// also holds the fx tile.
 // smem: [W img G x (96 | 160)][T img G x 96][kComb: T2 img G x 96][W'^T img G x 64]
-//       [kComb: constant extra 4K][stages][zero 2K][bars]
+//       [stages][zero 2K][bars]
 // TMEM: sets [0, 384) of (L 64 | dw 64); O_(j, tile parity) at [384 + 32 (2 j + parity)).
 // =========================================================================================
 template <bool split, bool kComb = false>
@@ -584,8 +586,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* s_t = s_w + wbytes;
   uint8_t* s_t2 = s_t + (uint32_t)G * 96;
   uint8_t* s_wt = s_t2 + (kComb ? (uint32_t)G * 96 : 0u);
-  uint8_t* s_ex = s_wt + (uint32_t)G * 64;
-  uint8_t* s_st = s_ex + (kComb ? kExBytes : 0u);
+  uint8_t* s_st = s_wt + (uint32_t)G * 64;
   uint8_t* s_zero = s_st + kDxStages * kStg;
   uint64_t* bars = reinterpret_cast<uint64_t*>(s_zero + kPxZero);
   uint64_t* wz_full = bars;
@@ -629,7 +630,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_mbar_init();
   }
   zero_smem(s_zero, kPxZero);
-  if (kComb) write_const_extra(s_ex);
   fence_proxy_async_smem();
   if (warp == 1) tmem_alloc(tmem_slot, 512);
   tc_fence_before();
@@ -684,11 +684,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         issue_dot64<false>(tL, st, sw + rows, px_desc(st + kPOff, sz),
                            sdesc(sw + (uint32_t)G * 64 + erows, 16, 256, kSw32),
                            hilo ? sw + (uint32_t)G * 96 + rows : 0u);
-        issue_dot64<false>(tL + 64, st + kVOff, stt + rows, px_desc(st + kDOff, sz),
-                           sdesc(stt + (uint32_t)G * 64 + erows, 16, 256, kSw32), 0u);
-        if (kComb)
-          issue_dot64<false>(tL + 64, st + kBStage, stt2 + rows, const_extra_desc(smem_u32(s_ex)),
+        if (kComb) {
+          // As in the slot pass: the deslice's chain without an extra block, the slice's
+          // extra block against delta's rows (dS - delta in one K step).
+          issue_dot64<false, false>(tL + 64, st + kVOff, stt + rows, 0ull, 0ull, 0u);
+          issue_dot64<false>(tL + 64, st + kBStage, stt2 + rows, px_desc(st + kDOff, sz),
                              sdesc(stt2 + (uint32_t)G * 64 + erows, 16, 256, kSw32), 0u, 1u);
+        } else {
+          issue_dot64<false>(tL + 64, st + kVOff, stt + rows, px_desc(st + kDOff, sz),
+                             sdesc(stt + (uint32_t)G * 64 + erows, 16, 256, kSw32), 0u);
+        }
         mma_commit_w(&s_full[bb]);
         if (c == nch - 1) mma_commit_w(&x_empty[s]);
       }
@@ -801,10 +806,10 @@ __global__ void __launch_bounds__(kThreads, 1)
 size_t smem_bwd_slot(int mode = 1) {
   const bool m3 = mode == 3;
   return 1024 + (m3 ? 3 : 2) * (size_t)kWBlockB + (m3 ? kBStages - 1 : kBStages) * (size_t)(kBStage + (m3 ? kXBytes : 0)) +
-         kPxZero + (m3 ? kPxBytes : 0) + 3 * kGC * 4 + 512;
+         kPxZero + 3 * kGC * 4 + 512;
 }
 size_t smem_bwd_dx(int G, bool hilo, bool comb = false) {
-  return 1024 + (size_t)G * ((hilo ? kWRow : 96) + 96 * (comb ? 2 : 1) + 64) + (comb ? kExBytes : 0) +
+  return 1024 + (size_t)G * ((hilo ? kWRow : 96) + 96 * (comb ? 2 : 1) + 64) +
          kDxStages * (size_t)(kBStage + (comb ? kXBytes : 0)) + kPxZero + 512;
 }
 
