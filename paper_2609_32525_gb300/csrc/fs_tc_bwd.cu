@@ -125,6 +125,20 @@ __device__ __forceinline__ void issue_dot64(uint32_t d, uint32_t a, uint32_t b, 
   if (kExtra) mma_ss_w(d, ae, be, idesc, 1);
 }
 
+// The same logits product with the slot side (A) in TMEM: tW holds a slot block's W'
+// image as packed bf16 pairs, K steps of 8 columns: W' (2 steps), its residual (2), the
+// extra block (1).  Only the point side (B) is read from shared memory.
+__device__ __forceinline__ void issue_logits64_ts(uint32_t d, uint32_t tW, uint32_t b, uint64_t be, bool lo) {
+  constexpr uint32_t idesc = idesc_bf16(128, 64, false, false);
+  mma_ts_w(d, tW, sdesc(b, 16, 512, kSw64), idesc, 0u);
+  mma_ts_w(d, tW + 8, sdesc(b + 32, 16, 512, kSw64), idesc, 1u);
+  if (lo) {
+    mma_ts_w(d, tW + 16, sdesc(b, 16, 512, kSw64), idesc, 1u);
+    mma_ts_w(d, tW + 24, sdesc(b + 32, 16, 512, kSw64), idesc, 1u);
+  }
+  mma_ts_w(d, tW + 32, be, idesc, 1u);
+}
+
 // Point-extra descriptor (no swizzle, 16-byte rows) whose k = 8..15 half is the shared zero block.
 __device__ __forceinline__ uint64_t px_desc(uint32_t px_s, uint32_t zero_s) { return sdesc(px_s, zero_s - px_s, 128, 0); }
 
@@ -267,7 +281,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* pv_done = p_ready + 2 * kSBuf;
   uint64_t* acc_full = pv_done + kSBuf;
   uint64_t* acc_done = acc_full + 1;  // [issuer]: products of each of its units complete
-  uint64_t* drain = acc_done + 2;
+  uint64_t* wt_ready = acc_done + 2;  // MODES 2, 3: the W' image is in TMEM
+  uint64_t* drain = wt_ready + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 3);
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
 
@@ -280,6 +295,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   // kSlotFlush of its units after warpgroup j has added the accumulator into
   // registers.  MODE 1 keeps two accumulators per issuer (dW, dZ) and no flushes.
   constexpr bool kFl = MODE != 1;
+  // MODES 2 and 3 keep no dZ accumulator, so its 64 TMEM columns hold the slot block's
+  // W' image (40 columns) and the logits read only their point side from shared memory.
+  constexpr bool kWT = MODE == 2 || MODE == 3;
   constexpr uint32_t kAccW = kSBuf * kGC, kAccZ = kAccW + 64;
   constexpr uint32_t kAccF = MODE == 0 ? kAccZ : kAccW;  // the flushed accumulator
   constexpr uint32_t kVOff = kXBytes, kPOff = 2 * kXBytes, kDOff = 2 * kXBytes + kPxBytes;
@@ -299,6 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(acc_full, 2);
     mbar_init(&acc_done[0], 1);
     mbar_init(&acc_done[1], 1);
+    mbar_init(wt_ready, 4);
     for (int i = 0; i < 3; i++) mbar_init(&drain[i], 1);
     ab->flag = 0;
     fence_mbar_init();
@@ -352,6 +371,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------ logits and dw issuer ------------------------------
     const uint32_t sw = smem_u32(s_w), stt = smem_u32(s_t), stt2 = smem_u32(s_t2), sz = smem_u32(s_zero);
     bool ok = mbar_wait_w(w_full, 0, ab, status);
+    if (kWT && ok) {
+      ok = mbar_wait_w(wt_ready, 0, ab, status);
+      tc_fence_after();
+    }
     for (int u = 0; ok && u < units; u++) {
       const int i = u >> 1, half = u & 1;
       const int s = i % kNSt;
@@ -363,8 +386,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t rows = (uint32_t)half * 64 * 64;     // the unit's 64 points in the 64-byte-row tiles
       const uint32_t prow = (uint32_t)half * 64 * 16;     // ... and in the 16-byte extra rows
       const uint32_t tL = tmem + (uint32_t)bb * kGC;
-      issue_dot64<true>(tL, sw, st + rows, sdesc(sw + kGC * 64, 16, 256, kSw32), px_desc(st + kPOff + prow, sz),
-                        split ? sw + kGC * 96 : 0u);
+      if (kWT)
+        issue_logits64_ts(tL, tmem + kAccZ, st + rows, px_desc(st + kPOff + prow, sz), split);
+      else
+        issue_dot64<true>(tL, sw, st + rows, sdesc(sw + kGC * 64, 16, 256, kSw32), px_desc(st + kPOff + prow, sz),
+                          split ? sw + kGC * 96 : 0u);
       if (MODE == 1 || MODE == 2)
         issue_dot64<true>(tL + 64, stt, st + kVOff + rows, sdesc(stt + kGC * 64, 16, 256, kSw32),
                           px_desc(st + kDOff + prow, sz), split ? stt + kGC * 96 : 0u);
@@ -430,6 +456,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     bool ok = true;
     float dt = 0.f, db = 0.f;
+    if (kWT && wg == 0) {
+      // Slot r's W' row from the block's image in shared memory (64B / 32B swizzled
+      // rows) into TMEM columns [kAccZ, kAccZ + 48) of lane r: packed bf16 pairs of W'
+      // (16), its residual (16), the extra block (8, then 8 zero columns).
+      if ((ok = mbar_wait(w_full, 0, ab, status))) {
+        const uint8_t* wrow = s_w;
+        uint32_t hi[16], lo[16], ex[16];
+#pragma unroll
+        for (int c = 0; c < 16; c++) {
+          hi[c] = *reinterpret_cast<const uint32_t*>(wrow + off_sw64(r, 2 * c));
+          lo[c] = split ? *reinterpret_cast<const uint32_t*>(wrow + kGC * 96 + off_sw64(r, 2 * c)) : 0u;
+          ex[c] = c < 8 ? *reinterpret_cast<const uint32_t*>(wrow + kGC * 64 + off_sw32(r, 2 * c)) : 0u;
+        }
+        const uint32_t tW = tmem + lane_addr + kAccZ;
+        tmem_st16(tW, hi);
+        tmem_st16(tW + 16, lo);
+        tmem_st16(tW + 32, ex);
+        tmem_wait_st();
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(wt_ready);
+    }
     float acc[kD];  // this warpgroup's flushed share of dWx (MODE 0: dZ)
 #pragma unroll
     for (int k = 0; k < kD; k++) acc[k] = 0.f;
