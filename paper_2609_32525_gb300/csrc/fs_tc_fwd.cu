@@ -684,7 +684,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* pv_done = p_ready + 2 * kSBuf;
   uint64_t* acc_full = pv_done + kSBuf;
   uint64_t* acc_done = acc_full + 1;  // [issuer]: products of each of its tiles complete
-  uint64_t* drain = acc_done + 2;  // one per issuing warp
+  uint64_t* wt_ready = acc_done + 2;  // single-level products: the W' image is in TMEM
+  uint64_t* drain = wt_ready + 1;  // one per issuing warp
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 3);
   Abort* ab = reinterpret_cast<Abort*>(tmem_slot + 1);
 
@@ -694,6 +695,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int h = (int)(wk.bh % H);
   constexpr uint32_t kA = kSBuf * kGC;  // TMEM column base of the accumulators
   constexpr uint32_t kFOff = kXBytes, kPOff = kXBytes + 3 * kFBlock;
+  // With single-level products the slot block's W' image (W' and its extra block: 24
+  // columns) fits in the 32 TMEM columns after the accumulators, and the logits read
+  // only their point side from shared memory.
+  constexpr bool kWT = !split && !X3;
+  constexpr uint32_t kTW = kA + 96;
 
   if (threadIdx.x == 0) {
     mbar_init(w_full, 1);
@@ -710,6 +716,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(acc_full, 2);
     mbar_init(&acc_done[0], 1);
     mbar_init(&acc_done[1], 1);
+    mbar_init(wt_ready, 4);
     for (int i = 0; i < 3; i++) mbar_init(&drain[i], 1);
     ab->flag = 0;
     fence_mbar_init();
@@ -775,6 +782,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     {
       const uint32_t sw = smem_u32(s_w), swe = sw + kGC * 64;
       bool ok = mbar_wait_w(w_full, 0, ab, status);
+      if (kWT && ok) {
+        ok = mbar_wait_w(wt_ready, 0, ab, status);
+        tc_fence_after();
+      }
       for (int i = 0; ok && i < wk.ntiles; i++) {
         const int s = i % kNSt;
         const int bb = i % kSBuf;
@@ -782,8 +793,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (i >= kSBuf && !(ok = mbar_wait_w(&pv_done[bb], (uint32_t)(((i / kSBuf) - 1) & 1), ab, status))) break;
         tc_fence_after();
         const uint32_t xs = smem_u32(s_st + s * kStB);
-        issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kPOff), sw, swe, split ? sw + kGC * 96 : 0u,
-                     0, false, X3 ? xs + kXROff : 0u);
+        if (kWT) {
+          constexpr uint32_t idesc = idesc_bf16(128, kGC, false, false);
+          const uint32_t tD = tmem + (uint32_t)bb * kGC;
+          mma_ts_w(tD, tmem + kTW, sdesc(xs, 16, 512, kSw64), idesc, 0u);
+          mma_ts_w(tD, tmem + kTW + 8, sdesc(xs + 32, 16, 512, kSw64), idesc, 1u);
+          mma_ts_w(tD, tmem + kTW + 16, point_extra_desc(xs + kPOff), idesc, 1u);
+        } else {
+          issue_logits(tmem + (uint32_t)bb * kGC, xs, point_extra_desc(xs + kPOff), sw, swe,
+                       split ? sw + kGC * 96 : 0u, 0, false, X3 ? xs + kXROff : 0u);
+        }
         mma_commit_w(&s_full[bb]);
         mma_commit_w(&st_empty[s]);
       }
@@ -835,6 +854,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int r = wq * 32 + lane;  // TMEM lane: slot g_base + r
     const uint32_t lane_addr = (uint32_t)(wq * 32) << 16;
     bool ok = true;
+    if (kWT && wg == 0) {
+      // Slot r's W' row (64B-swizzled) and extra row (32B-swizzled) from the block's image
+      // in shared memory into TMEM columns [kTW, kTW + 24) of lane r (packed bf16 pairs).
+      if ((ok = mbar_wait(w_full, 0, ab, status))) {
+        uint32_t hi[16], ex[16];
+#pragma unroll
+        for (int c = 0; c < 16; c++) {
+          hi[c] = *reinterpret_cast<const uint32_t*>(s_w + off_sw64(r, 2 * c));
+          ex[c] = c < 8 ? *reinterpret_cast<const uint32_t*>(s_w + kGC * 64 + off_sw32(r, 2 * c)) : 0u;
+        }
+        tmem_st16(tmem + lane_addr + kTW, hi);
+        tmem_st16(tmem + lane_addr + kTW + 16, ex);
+        tmem_wait_st();
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(wt_ready);
+    }
     // This warpgroup's share of (U, S) for slot r, moved out of A_wg at every flush.
     float acc[kD + 1];
 #pragma unroll
