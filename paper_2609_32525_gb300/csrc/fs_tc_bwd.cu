@@ -295,9 +295,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   // kSlotFlush of its units after warpgroup j has added the accumulator into
   // registers.  MODE 1 keeps two accumulators per issuer (dW, dZ) and no flushes.
   constexpr bool kFl = MODE != 1;
-  // MODES 2 and 3 keep no dZ accumulator, so its 64 TMEM columns hold the slot block's
-  // W' image (40 columns) and the logits read only their point side from shared memory.
+  // MODES 2 and 3 keep no dZ accumulator, so its 64 TMEM columns hold slot-side images
+  // and those MMAs read only their point side from shared memory: MODE 2 the W' image
+  // (W', its residual, the extra block: 40 columns); MODE 3 W' and its residual (32)
+  // and the deslice's T image and its residual (32), the two extra blocks staying in
+  // shared memory.
   constexpr bool kWT = MODE == 2 || MODE == 3;
+  constexpr bool kTT = MODE == 3;
   constexpr uint32_t kAccW = kSBuf * kGC, kAccZ = kAccW + 64;
   constexpr uint32_t kAccF = MODE == 0 ? kAccZ : kAccW;  // the flushed accumulator
   constexpr uint32_t kVOff = kXBytes, kPOff = 2 * kXBytes, kDOff = 2 * kXBytes + kPxBytes;
@@ -386,7 +390,25 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t rows = (uint32_t)half * 64 * 64;     // the unit's 64 points in the 64-byte-row tiles
       const uint32_t prow = (uint32_t)half * 64 * 16;     // ... and in the 16-byte extra rows
       const uint32_t tL = tmem + (uint32_t)bb * kGC;
-      if (kWT)
+      if (kTT) {
+        constexpr uint32_t idesc = idesc_bf16(128, 64, false, false);
+        const uint32_t tW = tmem + kAccZ, tT = tW + 32;
+        const uint32_t xb = st + rows, vb = st + kVOff + rows;
+        mma_ts_w(tL, tW, sdesc(xb, 16, 512, kSw64), idesc, 0u);
+        mma_ts_w(tL, tW + 8, sdesc(xb + 32, 16, 512, kSw64), idesc, 1u);
+        if (split) {
+          mma_ts_w(tL, tW + 16, sdesc(xb, 16, 512, kSw64), idesc, 1u);
+          mma_ts_w(tL, tW + 24, sdesc(xb + 32, 16, 512, kSw64), idesc, 1u);
+        }
+        mma_ss_w(tL, sdesc(sw + kGC * 64, 16, 256, kSw32), px_desc(st + kPOff + prow, sz), idesc, 1u);
+        // the deslice's chain: T (and its residual) from TMEM against dO, no extra block
+        mma_ts_w(tL + 64, tT, sdesc(vb, 16, 512, kSw64), idesc, 0u);
+        mma_ts_w(tL + 64, tT + 8, sdesc(vb + 32, 16, 512, kSw64), idesc, 1u);
+        if (split) {
+          mma_ts_w(tL + 64, tT + 16, sdesc(vb, 16, 512, kSw64), idesc, 1u);
+          mma_ts_w(tL + 64, tT + 24, sdesc(vb + 32, 16, 512, kSw64), idesc, 1u);
+        }
+      } else if (kWT)
         issue_logits64_ts(tL, tmem + kAccZ, st + rows, px_desc(st + kPOff + prow, sz), split);
       else
         issue_dot64<true>(tL, sw, st + rows, sdesc(sw + kGC * 64, 16, 256, kSw32), px_desc(st + kPOff + prow, sz),
@@ -395,10 +417,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         issue_dot64<true>(tL + 64, stt, st + kVOff + rows, sdesc(stt + kGC * 64, 16, 256, kSw32),
                           px_desc(st + kDOff + prow, sz), split ? stt + kGC * 96 : 0u);
       if (MODE == 3) {
-        // The deslice's T has c = 0, so its chain needs no extra block: the slice's
-        // extra block [dS_hi, dS_lo, 1, 1, 1] against delta's rows [1, 1, -delta parts]
-        // adds dS - delta in one K step.
-        issue_dot64<true, false>(tL + 64, stt, st + kVOff + rows, 0ull, 0ull, split ? stt + kGC * 96 : 0u);
+        // The deslice's T has c = 0, so its chain (issued above from TMEM) needs no extra
+        // block: the slice's extra block [dS_hi, dS_lo, 1, 1, 1] against delta's rows
+        // [1, 1, -delta parts] adds dS - delta in one K step.
         issue_dot64<true>(tL + 64, stt2, st + kBStage + rows, sdesc(stt2 + kGC * 64, 16, 256, kSw32),
                           px_desc(st + kDOff + prow, sz), split ? stt2 + kGC * 96 : 0u, 1u);
       }
@@ -461,18 +482,28 @@ __global__ void __launch_bounds__(kThreads, 1)
       // rows) into TMEM columns [kAccZ, kAccZ + 48) of lane r: packed bf16 pairs of W'
       // (16), its residual (16), the extra block (8, then 8 zero columns).
       if ((ok = mbar_wait(w_full, 0, ab, status))) {
-        const uint8_t* wrow = s_w;
-        uint32_t hi[16], lo[16], ex[16];
-#pragma unroll
-        for (int c = 0; c < 16; c++) {
-          hi[c] = *reinterpret_cast<const uint32_t*>(wrow + off_sw64(r, 2 * c));
-          lo[c] = split ? *reinterpret_cast<const uint32_t*>(wrow + kGC * 96 + off_sw64(r, 2 * c)) : 0u;
-          ex[c] = c < 8 ? *reinterpret_cast<const uint32_t*>(wrow + kGC * 64 + off_sw32(r, 2 * c)) : 0u;
-        }
         const uint32_t tW = tmem + lane_addr + kAccZ;
-        tmem_st16(tW, hi);
-        tmem_st16(tW + 16, lo);
-        tmem_st16(tW + 32, ex);
+        // a slot-block image's row r: bf16 pairs of the main half and of the residual
+        auto copy_rows = [&](const uint8_t* img, uint32_t tdst) {
+          uint32_t hi[16], lo[16];
+#pragma unroll
+          for (int c = 0; c < 16; c++) {
+            hi[c] = *reinterpret_cast<const uint32_t*>(img + off_sw64(r, 2 * c));
+            lo[c] = split ? *reinterpret_cast<const uint32_t*>(img + kGC * 96 + off_sw64(r, 2 * c)) : 0u;
+          }
+          tmem_st16(tdst, hi);
+          tmem_st16(tdst + 16, lo);
+        };
+        copy_rows(s_w, tW);
+        if (kTT) {
+          copy_rows(s_t, tW + 32);
+        } else {
+          uint32_t ex[16];
+#pragma unroll
+          for (int c = 0; c < 16; c++)
+            ex[c] = c < 8 ? *reinterpret_cast<const uint32_t*>(s_w + kGC * 64 + off_sw32(r, 2 * c)) : 0u;
+          tmem_st16(tW + 32, ex);
+        }
         tmem_wait_st();
       }
       tc_fence_before();
