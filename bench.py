@@ -594,7 +594,7 @@ def run_variant(args, wl, dev, world, rank):
         print(json.dumps(line), flush=True)
 
 
-def main():
+def build_parser() -> argparse.ArgumentParser:
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=50)
@@ -618,7 +618,11 @@ def main():
                     help="the workload's recipe at another slot count G (the line says so)")
     ap.add_argument("--dtype", default=None, choices=["bf16", "f32"],
                     help="the workload's recipe with inputs of this dtype (the line says so)")
-    args = ap.parse_args()
+    return ap
+
+
+def main():
+    args = build_parser().parse_args()
     if args.warmup < 3:
         args.warmup = 3
     if args.impl == "reference":

@@ -42,3 +42,49 @@ def test_named_workload_dtype_override():
     assert (a.W_slice == b.W_slice).all() and (a.M == b.M).all()
     with pytest.raises(ValueError):
         make_named("train_bf16", n_override=256, dtype_override="f16")
+
+
+# Values for the placeholders the documentation writes in place of a number or a name.
+_PLACEHOLDER = {"--gpus": "2", "--steps": "1", "--warmup": "3", "--variant": "frozen"}
+
+
+def _documented_bench_commands():
+    """The bench.py argument lists in the fenced code blocks of the README and the
+    profile summaries (up to the first shell operator, comment or closing quote)."""
+    import glob
+    import re
+    import shlex
+
+    files = [os.path.join(ROOT, "README.md")] + sorted(glob.glob(os.path.join(ROOT, "profiles", "*.md")))
+    cmds = []
+    for path in files:
+        fenced = False
+        for line in open(path, encoding="utf-8"):
+            if line.lstrip().startswith("```"):
+                fenced = not fenced
+                continue
+            if not fenced:
+                continue
+            for m in re.finditer(r"bench\.py((?:\s+[^\s\"'`>|&#;)]+)*)", line):
+                argv = shlex.split(m.group(1))
+                cmds.append((os.path.relpath(path, ROOT), [
+                    _PLACEHOLDER.get(argv[i - 1], a) if i and re.fullmatch(r"[A-Z]", a) else a
+                    for i, a in enumerate(argv)]))
+    return cmds
+
+
+def test_documented_bench_commands_parse():
+    """Every bench.py command that the README and profiles/ give parses with the
+    current flags, so the recipes beside the committed numbers still run."""
+    import bench
+    from paper_2609_32525_gb300.workloads import NAMED
+
+    cmds = _documented_bench_commands()
+    assert len(cmds) >= 8
+    parser = bench.build_parser()
+    for path, argv in cmds:
+        try:
+            args = parser.parse_args(argv)
+        except SystemExit:
+            pytest.fail(f"{path}: bench.py {' '.join(argv)} does not parse")
+        assert args.workload in NAMED, f"{path}: unknown workload {args.workload}"
